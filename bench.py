@@ -1,0 +1,352 @@
+"""Benchmark of the SLORR regularizer hot path (forward value + weight gradient
+over a whole weight set, Listing 1 / Alg. 2) on GB300.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload vit_l16]
+                  [--variant hoyer|nuclear] [--compute fp16|bf16|fp32] [--impl ours|reference]
+
+A step is one slorr_reg_forward_backward call over the whole weight set
+(norm, cast, T = 6 Polar Express steps of three grouped GEMMs, dot, combine).
+The default workload is the ViT-L/16-shaped set (96 matrices, 302 M weights,
+1.21 GB of fp32 weights: larger than the 129 MB L2, so no flush is needed).
+
+Printed: one JSON line.  value = algorithmic TFLOP/s of the whole job, using
+the paper's count T * sum_i (4 P_i^2 Q_i + 2 P_i^3) (Sec. 3 "Computational
+cost"); e2e = the same through the C ABI with the weights and grads copied from
+pinned host memory and the grads and loss copied back inside the timed region;
+roofline = the tensor-core GEMM kernel measured live with CUDA events around
+each of its launches on the call's stream; cpu_baseline = the fp64 oracle on a
+bounded sample of the same workload on this host's cores.
+
+With --gpus N > 1 (launched by torchrun) every rank regularizes its own full
+copy of the weight set (weak scaling, no collective on the data path); the
+time is the max over ranks.  --impl reference times the oracle instead.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads  # noqa: E402
+
+METRIC = "regularizer fwd+bwd ms/step & TFLOP/s (% GB300 dense peak) per weight set"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+PROFILE_FILE = os.path.join(ROOT, "profiles", "tc_gemm_vit_l16.txt")
+TC_SOURCE = os.path.join(ROOT, "paper_2607_08754_gb300", "csrc", "kernels_tc.cu")
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", default="vit_l16", choices=list(workloads.WEIGHT_SETS))
+    ap.add_argument("--variant", default="hoyer", choices=["hoyer", "nuclear"])
+    ap.add_argument("--compute", default="fp16", choices=["fp16", "bf16", "fp32"])
+    ap.add_argument("--iters", type=int, default=6)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    try:
+        with open(PEAKS_FILE) as f:
+            d = json.load(f)
+        return {"hbm": float(d["hbm_gbs"]), "bf16": float(d["bf16_tflops"]),
+                "bf16_sustained": float(d["bf16_tflops_sustained"]), "source": "measured"}
+    except Exception:
+        return {"hbm": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "source": "fallback"}
+
+
+def cpu_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:  # pragma: no cover
+        return os.cpu_count() or 1
+
+
+def oracle_sample(name: str, variant: str, iters: int, budget_s: float, max_steps: int = 1):
+    """Times the fp64 oracle on the leading matrices of the weight set until
+    about `budget_s` seconds of work; returns (flops, seconds, description)."""
+    import oracle
+    co = oracle.pe_coefficients(T=iters)
+    shapes = workloads.shapes(name)
+    flops = 0
+    t_total = 0.0
+    used = []
+    for i, (m, n) in enumerate(shapes):
+        W = workloads.generate_one(name, i).astype(np.float64)
+        t0 = time.perf_counter()
+        oracle.reg_forward_backward([W], variant, co, 1.0)
+        t_total += time.perf_counter() - t0
+        flops += oracle.pe_flops(m, n, iters)
+        used.append(f"{m}x{n}")
+        if t_total >= budget_s:
+            break
+    desc = f"first {len(used)} of {len(shapes)} matrices of {name} ({', '.join(used[:4])}" + \
+           (", ..." if len(used) > 4 else "") + f"), fp64 numpy oracle, T={iters}"
+    return flops, t_total, desc
+
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            import tempfile
+            fd, self.path = tempfile.mkstemp(prefix="clocks_", suffix=".csv")
+            os.close(fd)
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.out, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.out.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        reasons = set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            for name, v in zip(names, r[5:9]):
+                if v.strip().lower() == "active":
+                    reasons.add(name)
+        loaded = sorted(sm)[len(sm) // 2:] if sm else []
+        return {"sm_mhz": statistics.median(loaded) if loaded else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons), "samples": len(rows)}
+
+
+def tc_traffic():
+    """dram bytes per launch of the tensor-core GEMM from the committed ncu
+    summary, or None when the kernel source changed since it was taken."""
+    try:
+        src = hashlib.sha256(open(TC_SOURCE, "rb").read()).hexdigest()
+        vals = {}
+        with open(PROFILE_FILE) as f:
+            for line in f:
+                if ":" in line:
+                    k, v = line.split(":", 1)
+                    vals[k.strip()] = v.strip()
+        if vals.get("source_sha256") != src:
+            return None
+        return float(vals["dram_bytes_per_launch_scaled"])
+    except Exception:
+        return None
+
+
+def run_reference(args, rank, world):
+    """--impl reference: the fp64 oracle on this host's cores (rank 0 only)."""
+    if rank != 0:
+        return
+    shapes = workloads.shapes(args.workload)
+    total_flops = sum(__import__("oracle").pe_flops(m, n, args.iters) for m, n in shapes)
+    budget = max(2.0, 120.0 / max(1, args.steps + args.warmup))
+    for _ in range(args.warmup):
+        oracle_sample(args.workload, args.variant, args.iters, budget * 0.25)
+    times = []
+    flops_done = 0
+    desc = ""
+    for _ in range(args.steps):
+        f, t, desc = oracle_sample(args.workload, args.variant, args.iters, budget)
+        flops_done += f
+        times.append(t)
+    secs = sum(times)
+    tflops = flops_done / secs / 1e12
+    ms_full = total_flops / (flops_done / secs) * 1e3
+    line = {"metric": METRIC, "value": tflops, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_full, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": f"{args.workload} {args.variant}, T={args.iters}", "matrices": len(shapes)},
+            "cpu_baseline": {"value": tflops, "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
+                             "sample": f"each step: {desc}; ms_per_step extrapolated to the whole set by FLOPs"},
+            "e2e": {"value": tflops, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", str(args.gpus)))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+
+    import torch
+    import torch.distributed as dist
+
+    import __graft_entry__
+    __graft_entry__.build() if rank == 0 else None
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        dist.barrier()
+    from paper_2607_08754_gb300 import slorr
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    name = args.workload
+    shapes = workloads.shapes(name)
+    reg = slorr.Regularizer(shapes, variant=args.variant, compute=args.compute, iters=args.iters, lam=1.0)
+    W_host = [torch.from_numpy(workloads.generate_one(name, i)) for i in range(len(shapes))]
+    W = [w.to(dev) for w in W_host]
+    G = [torch.zeros_like(w) for w in W]
+    loss = torch.zeros(1, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    flops_step = slorr.slorr_flops(shapes, args.iters)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    # warm-up
+    for _ in range(max(args.warmup, 3)):
+        reg(W, G, loss=loss)
+    barrier()
+    assert reg.status() == 0, "device status word reports an error after warm-up"
+
+    # timed region (device-resident inputs), per-kernel events on the same stream
+    slorr.slorr_set_timing(reg.handle, True)
+    slorr.slorr_read_timing(reg.handle)
+    clocks = ClockSampler(local)
+    clocks.start()
+    barrier()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        reg(W, G, loss=loss)
+    t1.record(stream)
+    barrier()
+    clk = clocks.stop()
+    ms_total = t0.elapsed_time(t1)
+    kt = slorr.slorr_read_timing(reg.handle)
+    slorr.slorr_set_timing(reg.handle, False)
+    ms = torch.tensor([ms_total], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(ms, op=dist.ReduceOp.MAX)
+    ms_step = ms.item() / args.steps
+    value = world * flops_step / (ms_step * 1e-3) / 1e12
+    assert reg.status() == 0, "device status word reports an error in the timed region"
+
+    # e2e: pinned host buffers, copies inside the timed region
+    Wp = [w.pin_memory() for w in W_host]
+    Gp = [torch.zeros_like(w).pin_memory() for w in W_host]
+    Lp = torch.zeros(1, dtype=torch.float32).pin_memory()
+    Wd = [torch.empty_like(w) for w in W]
+    Gd = [torch.empty_like(w) for w in W]
+    h2d = sum(w.numel() * w.element_size() for w in Wp) + sum(g.numel() * g.element_size() for g in Gp)
+    d2h = sum(g.numel() * g.element_size() for g in Gp) + 4
+
+    def e2e_step():
+        for d, h in zip(Wd, Wp):
+            d.copy_(h, non_blocking=True)
+        for d, h in zip(Gd, Gp):
+            d.copy_(h, non_blocking=True)
+        reg(Wd, Gd, loss=loss)
+        for d, h in zip(Gp, Gd):
+            d.copy_(h, non_blocking=True)
+        Lp.copy_(loss, non_blocking=True)
+
+    e2e_step()
+    barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    barrier()
+    ems = torch.tensor([e0.elapsed_time(e1)], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(ems, op=dist.ReduceOp.MAX)
+    e2e_ms = ems.item() / args.e2e_steps
+    e2e_val = world * flops_step / (e2e_ms * 1e-3) / 1e12
+
+    if rank == 0:
+        pk = peaks()
+        gemm_ms = sum(kt[k][0] for k in ("gram", "poly", "update"))
+        gemm_launches = sum(kt[k][1] for k in ("gram", "poly", "update"))
+        launches = sum(v[1] for v in kt.values())
+        per_launch_ms = gemm_ms / max(gemm_launches, 1)
+        flops_per_launch = flops_step / (3 * args.iters)
+        achieved = flops_per_launch / (per_launch_ms * 1e-3) / 1e12
+        peak = pk["bf16"]  # fp16 and bf16 share the dense tensor rate (nominal ratio 1)
+        mem_ms = sum(kt[k][0] for k in ("sumsq", "cast", "dot", "combine")) / args.steps
+        kernel_breakdown = {k: {"ms_per_step": v[0] / args.steps, "launches_per_step": v[1] / args.steps}
+                            for k, v in kt.items()}
+        line = {
+            "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f16" if args.compute == "fp16" else args.compute,
+            "data": "synthetic",
+            "config": {"workload": f"{name} {args.variant}: {len(shapes)} matrices, T={args.iters}, "
+                                   f"{args.compute} operands / fp32 accumulate, fp32 weights and grads",
+                       "matrices": len(shapes), "iters": args.iters, "variant": args.variant,
+                       "gflop_per_step": flops_step / 1e9,
+                       "l2": "inputs larger than L2 (fp32 weights %.2f GB)" %
+                             (sum(w.numel() for w in W) * 4 / 1e9)},
+            "pct_of_dense_peak": value / world / pk["bf16"],
+            "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                         "frac": achieved / peak, "traffic": tc_traffic(),
+                         "kernel": "tc_gemm_kernel (Gram/Poly/Update launches)",
+                         "peak_source": pk["source"] + " bf16 burst (fp16 dense rate equal)"},
+            "memory_phases_ms_per_step": mem_ms,
+            "kernels": kernel_breakdown,
+            "gpu_launches": launches,
+            "e2e": {"value": e2e_val, "unit": "TFLOP/s", "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h},
+            "clocks": clk,
+        }
+        if not args.no_cpu_baseline:
+            f, t, desc = oracle_sample(name, args.variant, args.iters, args.cpu_seconds)
+            line["cpu_baseline"] = {"value": f / t / 1e12, "unit": "TFLOP/s", "cores": cpu_cores(),
+                                    "kind": "oracle", "sample": desc}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,208 @@
+/*
+ * slorr.h -- C ABI of libslorr, the GB300 (sm_103a) implementation of the SLORR
+ * regularizer hot path (SLORR: Simple and Efficient In-Training Low-Rank
+ * Regularization, arXiv 2607.08754).
+ *
+ * For every regularized weight matrix W_i (row-major m_i x n_i; conv kernels in
+ * the (C_out, C_in*k*k) view of App. D.1) one call computes, on the caller's
+ * stream, the SVD-free forward value and weight gradient of
+ *
+ *   SLORR-Hoyer  L = sum_i ||W_i||_*^2 / ||W_i||_F^2      (Sec. 3, Eq. 1)
+ *   SLORR-Nuc    L = sum_i ||W_i||_*                      (Sec. 3, Eq. 1)
+ *
+ * with U V^T replaced by the Polar Express approximation P_hat (Sec. 3
+ * "Computing the polar factor"): X_0 = W / (||W||_F + eps) on the Gram side
+ * (X = W^T when m > n), then T steps of A = X X^T, B = b_t A + c_t A^2,
+ * X <- a_t X + B X; n_hat = sum(W * P_hat) (Sec. 3 "Computing the nuclear and
+ * Frobenius norms"); value and gradient as in Listing 1:
+ *   frob = ||W||_F + eps, reg = n_hat / frob,
+ *   Hoyer: L_i = reg^2,  G_i = 2 reg (P_hat / frob - n_hat / frob^3 W)
+ *   Nuc:   L_i = n_hat,  G_i = P_hat
+ * and the memory-efficient accumulation of Alg. 2 (App. C.3):
+ *   W_i.grad += lambda * grad_scale * G_i,   loss = lambda * sum_i L_i.
+ *
+ * Memory: the caller owns every device buffer (weights, grads, outputs and one
+ * workspace); the library allocates no device memory.  The handle owns only
+ * host memory (the plan and the coefficient table).
+ *
+ * Errors: host-detectable problems (bad arguments, misalignment, a workspace
+ * that is too small) return a non-zero status before anything is launched.
+ * Problems found on the device (a non-finite norm or estimate, an internal
+ * wait that ran out of time) are recorded in a status word inside the
+ * workspace; slorr_get_status() reads it.  A matrix whose norm or estimate is
+ * not finite leaves its gradient untouched.
+ */
+#ifndef SLORR_H
+#define SLORR_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SLORR_API __attribute__((visibility("default")))
+#else
+#define SLORR_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum slorr_status {
+    SLORR_OK = 0,
+    SLORR_ERR_INVALID_ARG = 1,   /* null / misaligned pointer, bad shape or option   */
+    SLORR_ERR_UNSUPPORTED = 2,   /* valid request this build or device cannot serve */
+    SLORR_ERR_CUDA = 3,          /* a CUDA runtime call failed                        */
+    SLORR_ERR_WORKSPACE = 4,     /* workspace missing or smaller than required        */
+    SLORR_ERR_TIMEOUT = 5,       /* a bounded device-side wait gave up (status word)  */
+    SLORR_ERR_NONFINITE = 6      /* non-finite norm or nuclear estimate (status word) */
+} slorr_status;
+
+typedef enum slorr_variant {
+    SLORR_HOYER = 0,             /* squared l1/l2 ratio of singular values (Sec. 3)  */
+    SLORR_NUCLEAR = 1            /* nuclear norm (Sec. 3)                            */
+} slorr_variant;
+
+typedef enum slorr_dtype {       /* storage type of the weights and of their grads   */
+    SLORR_F32 = 0,
+    SLORR_BF16 = 1
+} slorr_dtype;
+
+typedef enum slorr_compute {     /* operand type of the Polar Express matrix products */
+    SLORR_COMPUTE_FP16 = 0,      /* fp16 operands, fp32 accumulation (tensor cores)  */
+    SLORR_COMPUTE_BF16 = 1,      /* bf16 operands, fp32 accumulation (tensor cores)  */
+    SLORR_COMPUTE_FP32 = 2       /* fp32 operands and accumulation (CUDA cores)      */
+} slorr_compute;
+
+typedef struct slorr_shape {
+    int64_t m;                   /* rows    (C_out for a conv kernel)                */
+    int64_t n;                   /* columns (C_in*k_h*k_w for a conv kernel)          */
+} slorr_shape;
+
+typedef struct slorr_options {
+    int32_t variant;             /* slorr_variant                        (HOYER)     */
+    int32_t compute;             /* slorr_compute                        (FP16)      */
+    int32_t dtype;               /* slorr_dtype of weights and grads     (F32)       */
+    int32_t iters;               /* T, Polar Express steps, 1..16        (6)         */
+    double  ell;                 /* lower singular-value bound ell, (0,1) (1e-3)     */
+    double  cushion;             /* cushion ratio; < 0: derived default, 0: off (-1) */
+    double  safety;              /* safety factor s >= 1; 1: off          (1.01)     */
+    float   lambda;              /* regularization strength lambda       (1)         */
+    float   eps;                 /* eps added to ||W||_F, >= 0            (1e-7)      */
+    float   grad_scale;          /* extra factor on the gradient only    (1)         */
+    int32_t flags;               /* SLORR_FLAG_* bits                     (0)         */
+    double  timeout_s;           /* budget of each bounded device wait, s (2.0)      */
+} slorr_options;
+
+/* Flags. */
+#define SLORR_FLAG_SIMT_GEMM    1   /* run the 16-bit products on CUDA cores (debug)  */
+
+/* Fill *opt with the defaults listed beside each field above (App. C.1: T = 6,
+ * ell = 1e-3, degree 5; eps, lambda and grad_scale as in Listing 1 / Alg. 2). */
+SLORR_API void slorr_default_options(slorr_options* opt);
+
+typedef struct slorr_handle slorr_handle;
+
+/* Plan one weight set (Sec. 3; Alg. 2).  shapes: host array of `count` shapes,
+ * copied.  opt: host struct, copied (NULL = defaults).  Builds the Polar Express
+ * coefficient table (Sec. 3, App. C.1) and the tile schedule on the host; makes
+ * no CUDA call.  Returns INVALID_ARG for count < 1, a non-positive dimension, a
+ * dimension above 65536, or an option outside its range. */
+SLORR_API slorr_status slorr_create(slorr_handle** out, const slorr_shape* shapes, int32_t count,
+                          const slorr_options* opt);
+
+/* Bytes of device workspace a call needs (host-only; no CUDA call). */
+SLORR_API slorr_status slorr_workspace_size(const slorr_handle* h, size_t* bytes);
+
+/* One regularizer forward + backward over the whole weight set (Listing 1,
+ * Alg. 2), enqueued on `stream` (a cudaStream_t; NULL = legacy default stream).
+ *   weights[i]      device pointer to W_i, row-major m_i x n_i, 16-byte aligned
+ *   grads[i]        device pointer to W_i.grad, same layout; ACCUMULATED (+=)
+ *   loss_out        device pointer to 1 float, written with lambda * sum_i L_i
+ *   per_matrix_out  device pointer to `count` floats (unweighted L_i), or NULL
+ *   workspace       device buffer of at least slorr_workspace_size() bytes,
+ *                   256-byte aligned; it keeps a plan written on its first use,
+ *                   so do not modify it between calls (pass another buffer, or
+ *                   call slorr_reset_workspace(), to re-plan)
+ * weights/grads are host arrays of `count` device pointers.  The call is
+ * asynchronous; the grads must not alias the weights. */
+SLORR_API slorr_status slorr_reg_forward_backward(slorr_handle* h, const void* const* weights,
+                                        void* const* grads, float* loss_out,
+                                        float* per_matrix_out, void* workspace,
+                                        size_t workspace_bytes, void* stream);
+
+/* Forget which workspace holds the plan; the next call re-writes it. */
+SLORR_API slorr_status slorr_reset_workspace(slorr_handle* h);
+
+/* Synchronize `stream`, read the device status word of `workspace`, clear it,
+ * and return OK, TIMEOUT or NONFINITE (TIMEOUT wins if both were recorded). */
+SLORR_API slorr_status slorr_get_status(slorr_handle* h, const void* workspace, void* stream);
+
+/* Run only the Frobenius norm, the normalisation and the first `steps` Polar
+ * Express steps (0 <= steps <= T) on `stream`, leaving the iterate X_steps in the
+ * workspace (introspection for tests; Sec. 3 "Computing the polar factor"). */
+SLORR_API slorr_status slorr_run_steps(slorr_handle* h, const void* const* weights, void* workspace,
+                             size_t workspace_bytes, int32_t steps, void* stream);
+
+/* Where matrix i's current iterate lives inside `workspace`: a P x Q row-major
+ * array (P = min(m,n), Q = max(m,n); the iterate is W^T-shaped when m > n) of
+ * element type elem (0 fp32, 1 fp16, 2 bf16) with leading dimension ld >= Q.
+ * Also returns device pointers to ||W_i||_F^2 (double) and n_hat_i (double). */
+typedef struct slorr_matrix_view {
+    const void*   x;
+    int64_t       rows, cols, ld;
+    int32_t       elem;
+    int32_t       transposed;
+    const double* frob_sq;
+    const double* n_hat;
+} slorr_matrix_view;
+SLORR_API slorr_status slorr_iterate_view(const slorr_handle* h, const void* workspace, int32_t i,
+                                int32_t after_steps, slorr_matrix_view* out);
+
+/* The handle's (a_t, b_t, c_t) table, t = 1..T, as 3*T doubles (App. C.1). */
+SLORR_API slorr_status slorr_get_coefficients(const slorr_handle* h, double* abc, int32_t capacity);
+
+/* Polar Express schedule without a handle (host-only): greedy minimax odd
+ * quintics on [l_t, u_t], l_{t+1} = p_t(l_t), u_{t+1} = 2 - l_{t+1}, with the
+ * cushion and safety-factor options of slorr_options (Sec. 3, App. C.1).
+ * Writes 3*iters doubles. */
+SLORR_API slorr_status slorr_pe_coefficients(int32_t iters, double ell, double cushion, double safety,
+                                   double* abc);
+
+/* The derived cushion ratio kappa (minimax error 9/11 on [kappa, 1]). */
+SLORR_API double slorr_cushion_ratio(void);
+
+/* Algorithmic FLOPs of one call: T * sum_i (4 P_i^2 Q_i + 2 P_i^3) (Sec. 3
+ * "Computational cost"). */
+SLORR_API int64_t slorr_flops(const slorr_shape* shapes, int32_t count, int32_t iters);
+
+/* Layer partition for data-parallel training (App. F: each rank regularizes a
+ * subset of the layers; set grad_scale = world so the existing gradient
+ * average restores lambda).  Longest-processing-time split of the matrices by
+ * FLOPs; writes the indices owned by `rank` (ascending) to out_indices
+ * (capacity >= count) and their number to *out_count.  Host-only. */
+SLORR_API slorr_status slorr_partition(const slorr_shape* shapes, int32_t count, int32_t world,
+                             int32_t rank, int32_t* out_indices, int32_t* out_count);
+
+/* Per-kernel timing (tracing).  While enabled, every kernel this handle
+ * launches is bracketed by a pair of CUDA events recorded on the caller's
+ * stream (events are created on the host; no device memory is allocated).
+ * slorr_read_timing() waits for the recorded events, adds the elapsed
+ * milliseconds and launch counts per kernel kind into ms[k] / launches[k]
+ * (k < kinds, kinds <= SLORR_NUM_KERNEL_KINDS; kinds are sumsq, cast, gram,
+ * poly, update, dot, combine) and forgets them. */
+#define SLORR_NUM_KERNEL_KINDS 7
+SLORR_API slorr_status slorr_set_timing(slorr_handle* h, int32_t enable);
+SLORR_API slorr_status slorr_read_timing(slorr_handle* h, double* ms, int64_t* launches, int32_t kinds);
+
+SLORR_API void        slorr_destroy(slorr_handle* h);
+SLORR_API const char* slorr_status_string(slorr_status s);
+
+/* Human-readable reason for the last non-OK status returned on this thread. */
+SLORR_API const char* slorr_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SLORR_H */

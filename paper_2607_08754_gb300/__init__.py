@@ -1,0 +1,28 @@
+"""GB300 (sm_103a) implementation of the SLORR regularizer hot path.
+
+The compute lives in ``libslorr.so`` (CUDA kernels behind the C ABI of
+``include/slorr.h``); ``paper_2607_08754_gb300.slorr`` is its ctypes binding.
+"""
+
+from .slorr import (  # noqa: F401
+    Regularizer,
+    SlorrError,
+    load_library,
+    slorr_create,
+    slorr_cushion_ratio,
+    slorr_default_options,
+    slorr_destroy,
+    slorr_flops,
+    slorr_get_coefficients,
+    slorr_get_status,
+    slorr_iterate_view,
+    slorr_partition,
+    slorr_pe_coefficients,
+    slorr_reg_forward_backward,
+    slorr_reset_workspace,
+    slorr_read_timing,
+    slorr_run_steps,
+    slorr_set_timing,
+    slorr_status_string,
+    slorr_workspace_size,
+)

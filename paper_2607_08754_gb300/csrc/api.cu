@@ -1,0 +1,668 @@
+// libslorr C ABI: planning, workspace layout, tensor maps and the launch
+// sequence of one regularizer forward + backward (Listing 1, Alg. 2):
+//   sumsq -> cast -> T x (Gram, Poly, Update) -> dot -> combine
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <numeric>
+#include <string>
+#include <vector>
+
+#include "../../include/slorr.h"
+#include "internal.h"
+
+using namespace slorr;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+slorr_status fail(slorr_status s, const std::string& msg) {
+    g_last_error = msg;
+    return s;
+}
+
+slorr_status cuda_fail(cudaError_t e, const char* what) {
+    g_last_error = std::string(what) + ": " + cudaGetErrorString(e);
+    if (e == cudaErrorNoKernelImageForDevice || e == cudaErrorInvalidDeviceFunction)
+        return SLORR_ERR_UNSUPPORTED;
+    return SLORR_ERR_CUDA;
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+struct Geom {
+    int m, n, P, Q, Ppad, Qpad, transposed;
+    size_t off_x[2], off_a, off_b;
+    int tile_base, tile_count;
+};
+
+}  // namespace
+
+struct slorr_handle {
+    slorr_options opt;
+    std::vector<slorr_shape> shapes;
+    std::vector<Geom> geom;
+    std::vector<double> coeffs;  // 3 * T
+    int elem;                    // Elem of X / A / B
+    int esize;
+    // item lists (host)
+    std::vector<GemmItem> tc_items[3];
+    std::vector<GemmItem> simt_items[3];
+    std::vector<MemItem> w_items;  // tiles of W (sumsq, dot, combine)
+    std::vector<MemItem> x_items;  // tiles of the padded iterate (cast)
+    int total_w_tiles = 0;
+    // workspace layout
+    size_t off_status = 0, off_counters = 0, off_scalars = 0, off_partials = 0, off_tilebase = 0,
+           off_tilecount = 0, off_mats = 0, off_maps = 0, off_tc_items[3] = {}, off_simt_items[3] = {},
+           off_w_items = 0, off_x_items = 0, off_ptrs = 0, off_plan_end = 0, total_bytes = 0;
+    // device state
+    const void* prepared_ws = nullptr;
+    std::vector<const void*> last_ptrs;  // weights then grads last uploaded
+    int num_sms = 0;
+    // tracing
+    bool timing = false;
+    std::vector<cudaEvent_t> ev_pool;
+    struct Mark { int kind; cudaEvent_t start, stop; };
+    std::vector<Mark> marks;
+    ~slorr_handle() {
+        for (auto& m : marks) {
+            cudaEventDestroy(m.start);
+            cudaEventDestroy(m.stop);
+        }
+        for (auto e : ev_pool) cudaEventDestroy(e);
+    }
+};
+
+namespace {
+
+bool valid_options(const slorr_options& o, std::string* why) {
+    if (o.variant != SLORR_HOYER && o.variant != SLORR_NUCLEAR) return *why = "variant", false;
+    if (o.compute < SLORR_COMPUTE_FP16 || o.compute > SLORR_COMPUTE_FP32) return *why = "compute", false;
+    if (o.dtype != SLORR_F32 && o.dtype != SLORR_BF16) return *why = "dtype", false;
+    if (o.iters < 1 || o.iters > kMaxIters) return *why = "iters must be in [1, 16]", false;
+    if (!(o.ell > 0.0 && o.ell < 1.0)) return *why = "ell must be in (0, 1)", false;
+    if (!(o.safety >= 1.0) || !std::isfinite(o.safety)) return *why = "safety must be >= 1", false;
+    if (!std::isfinite(o.cushion) || o.cushion >= 1.0) return *why = "cushion must be < 1", false;
+    if (!(o.eps >= 0.f) || !std::isfinite(o.eps)) return *why = "eps must be >= 0", false;
+    if (!std::isfinite(o.lambda) || !std::isfinite(o.grad_scale)) return *why = "lambda/grad_scale", false;
+    if (!(o.timeout_s > 0.0) || o.timeout_s > 3600.0) return *why = "timeout_s must be in (0, 3600]", false;
+    return true;
+}
+
+void build_plan(slorr_handle* h) {
+    const int count = int(h->shapes.size());
+    h->geom.resize(count);
+    for (int i = 0; i < 3; ++i) {
+        h->tc_items[i].clear();
+        h->simt_items[i].clear();
+    }
+    h->w_items.clear();
+    h->x_items.clear();
+    int tile_base = 0;
+    for (int i = 0; i < count; ++i) {
+        Geom& g = h->geom[i];
+        g.m = int(h->shapes[i].m);
+        g.n = int(h->shapes[i].n);
+        g.transposed = g.m > g.n ? 1 : 0;
+        g.P = std::min(g.m, g.n);
+        g.Q = std::max(g.m, g.n);
+        g.Ppad = int(align_up(size_t(g.P), kPadRows));
+        g.Qpad = int(align_up(size_t(g.Q), kPadCols));
+        const int tr = (g.m + 63) / 64, tc = (g.n + 63) / 64;
+        g.tile_base = tile_base;
+        g.tile_count = tr * tc;
+        int seq = 0;
+        for (int r = 0; r < tr; ++r)
+            for (int c = 0; c < tc; ++c)
+                h->w_items.push_back(MemItem{uint16_t(i), uint16_t(r), uint16_t(c), uint16_t(seq++)});
+        tile_base += g.tile_count;
+        for (int r = 0; r < g.Ppad / 64; ++r)
+            for (int c = 0; c < g.Qpad / 64; ++c)
+                h->x_items.push_back(MemItem{uint16_t(i), uint16_t(r), uint16_t(c), 0});
+        // tensor-core tiles: 128 x nsz, nsz <= 256
+        for (int ph = 0; ph < 3; ++ph) {
+            const int N = ph == kUpdate ? g.Qpad : g.Ppad;
+            for (int tm = 0; tm < g.Ppad / 128; ++tm)
+                for (int tn = 0; tn * 256 < N; ++tn)
+                    h->tc_items[ph].push_back(
+                        GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), uint16_t(std::min(256, N - tn * 256))});
+            for (int tm = 0; tm < g.Ppad / 64; ++tm)
+                for (int tn = 0; tn < N / 64; ++tn)
+                    h->simt_items[ph].push_back(GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), 64});
+        }
+    }
+    h->total_w_tiles = tile_base;
+    // Longest K first (stable: keeps a matrix's tiles together).
+    for (int ph = 0; ph < 3; ++ph) {
+        auto kdim = [&](const GemmItem& it) {
+            const Geom& g = h->geom[it.mat];
+            return ph == kGram ? g.Qpad : g.Ppad;
+        };
+        std::stable_sort(h->tc_items[ph].begin(), h->tc_items[ph].end(),
+                         [&](const GemmItem& a, const GemmItem& b) { return kdim(a) > kdim(b); });
+    }
+
+    // Workspace layout.
+    size_t off = 0;
+    h->off_status = off;
+    off += 256;
+    h->off_counters = off;
+    off = align_up(off + size_t(count + 1) * 4, 256);
+    h->off_scalars = off;
+    off = align_up(off + size_t(count) * sizeof(MatScalars), 256);
+    h->off_partials = off;
+    off = align_up(off + size_t(h->total_w_tiles) * 4, 256);
+    h->off_tilebase = off;
+    off = align_up(off + size_t(count) * 4, 256);
+    h->off_tilecount = off;
+    off = align_up(off + size_t(count) * 4, 256);
+    h->off_mats = off;
+    off = align_up(off + size_t(count) * sizeof(MatDev), 256);
+    h->off_maps = off;
+    off = align_up(off + size_t(count) * 4 * 128, 256);
+    for (int ph = 0; ph < 3; ++ph) {
+        h->off_tc_items[ph] = off;
+        off = align_up(off + h->tc_items[ph].size() * sizeof(GemmItem), 256);
+        h->off_simt_items[ph] = off;
+        off = align_up(off + h->simt_items[ph].size() * sizeof(GemmItem), 256);
+    }
+    h->off_w_items = off;
+    off = align_up(off + h->w_items.size() * sizeof(MemItem), 256);
+    h->off_x_items = off;
+    off = align_up(off + h->x_items.size() * sizeof(MemItem), 256);
+    h->off_ptrs = off;
+    off = align_up(off + size_t(2 * count) * sizeof(void*), 1024);
+    h->off_plan_end = off;
+    for (int i = 0; i < count; ++i) {
+        Geom& g = h->geom[i];
+        const size_t xbytes = size_t(g.Ppad) * g.Qpad * h->esize;
+        const size_t pbytes = size_t(g.Ppad) * g.Ppad * h->esize;
+        g.off_x[0] = off;
+        off = align_up(off + xbytes, 1024);
+        g.off_x[1] = off;
+        off = align_up(off + xbytes, 1024);
+        g.off_a = off;
+        off = align_up(off + pbytes, 1024);
+        g.off_b = off;
+        off = align_up(off + pbytes, 1024);
+    }
+    h->total_bytes = off;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    }
+    return fn;
+}
+
+// Row-major rows x cols 16-bit matrix, 64 x 64 boxes, 128-byte swizzle.
+bool encode_map(CUtensorMap* map, void* base, int rows, int cols, bool bf16) {
+    auto enc = get_encode();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {cuuint64_t(cols), cuuint64_t(rows)};
+    cuuint64_t strides[1] = {cuuint64_t(cols) * 2};
+    cuuint32_t box[2] = {64, 64};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(map, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, base,
+                     dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+template <typename T>
+void put(std::vector<uint8_t>& buf, size_t off, const T* src, size_t n) {
+    if (n) std::memcpy(buf.data() + off, src, n * sizeof(T));
+}
+
+slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
+    if (h->prepared_ws == ws) return SLORR_OK;
+    const int count = int(h->shapes.size());
+    if (h->num_sms == 0) {
+        int dev = 0;
+        cudaError_t e = cudaGetDevice(&dev);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return cuda_fail(e, "device query");
+    }
+    std::vector<uint8_t> plan(h->off_plan_end - h->off_tilebase, 0);
+    const size_t base = h->off_tilebase;
+    std::vector<int32_t> tb(count), tcnt(count);
+    std::vector<MatDev> mats(count);
+    std::vector<uint8_t> maps(size_t(count) * 4 * 128, 0);
+    const bool tc = h->opt.compute != SLORR_COMPUTE_FP32;
+    for (int i = 0; i < count; ++i) {
+        const Geom& g = h->geom[i];
+        tb[i] = g.tile_base;
+        tcnt[i] = g.tile_count;
+        MatDev& md = mats[i];
+        md.x[0] = ws + g.off_x[0];
+        md.x[1] = ws + g.off_x[1];
+        md.a = ws + g.off_a;
+        md.b = ws + g.off_b;
+        md.m = g.m;
+        md.n = g.n;
+        md.P = g.P;
+        md.Q = g.Q;
+        md.Ppad = g.Ppad;
+        md.Qpad = g.Qpad;
+        md.transposed = g.transposed;
+        md.pad_ = 0;
+        if (tc) {
+            const bool bf = h->opt.compute == SLORR_COMPUTE_BF16;
+            CUtensorMap* mp = reinterpret_cast<CUtensorMap*>(maps.data() + size_t(i) * 4 * 128);
+            if (!encode_map(mp + 0, md.x[0], g.Ppad, g.Qpad, bf) || !encode_map(mp + 1, md.x[1], g.Ppad, g.Qpad, bf) ||
+                !encode_map(mp + 2, md.a, g.Ppad, g.Ppad, bf) || !encode_map(mp + 3, md.b, g.Ppad, g.Ppad, bf))
+                return fail(SLORR_ERR_CUDA, "cuTensorMapEncodeTiled failed");
+        }
+    }
+    put(plan, h->off_tilebase - base, tb.data(), tb.size());
+    put(plan, h->off_tilecount - base, tcnt.data(), tcnt.size());
+    put(plan, h->off_mats - base, mats.data(), mats.size());
+    put(plan, h->off_maps - base, maps.data(), maps.size());
+    for (int ph = 0; ph < 3; ++ph) {
+        put(plan, h->off_tc_items[ph] - base, h->tc_items[ph].data(), h->tc_items[ph].size());
+        put(plan, h->off_simt_items[ph] - base, h->simt_items[ph].data(), h->simt_items[ph].size());
+    }
+    put(plan, h->off_w_items - base, h->w_items.data(), h->w_items.size());
+    put(plan, h->off_x_items - base, h->x_items.data(), h->x_items.size());
+    cudaError_t e = cudaMemcpyAsync(ws + base, plan.data(), plan.size(), cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(ws + h->off_status, 0, h->off_tilebase - h->off_status, st);
+    if (e != cudaSuccess) return cuda_fail(e, "plan upload");
+    h->prepared_ws = ws;
+    h->last_ptrs.clear();
+    return SLORR_OK;
+}
+
+slorr_status upload_ptrs(slorr_handle* h, uint8_t* ws, const void* const* weights, void* const* grads,
+                         cudaStream_t st) {
+    const int count = int(h->shapes.size());
+    std::vector<const void*> ptrs(size_t(2 * count));
+    for (int i = 0; i < count; ++i) {
+        ptrs[i] = weights[i];
+        ptrs[count + i] = grads ? grads[i] : nullptr;
+    }
+    if (ptrs == h->last_ptrs) return SLORR_OK;
+    cudaError_t e = cudaMemcpyAsync(ws + h->off_ptrs, ptrs.data(), ptrs.size() * sizeof(void*),
+                                    cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess) return cuda_fail(e, "pointer upload");
+    h->last_ptrs = ptrs;
+    return SLORR_OK;
+}
+
+cudaEvent_t take_event(slorr_handle* h) {
+    if (!h->ev_pool.empty()) {
+        cudaEvent_t e = h->ev_pool.back();
+        h->ev_pool.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    return e;
+}
+
+// Brackets one launch with events when tracing is on.
+struct Traced {
+    slorr_handle* h;
+    cudaStream_t st;
+    int kind;
+    cudaEvent_t start = nullptr;
+    Traced(slorr_handle* h_, int kind_, cudaStream_t st_) : h(h_), st(st_), kind(kind_) {
+        if (h->timing && (start = take_event(h)) != nullptr) cudaEventRecord(start, st);
+    }
+    void done() {
+        if (!start) return;
+        cudaEvent_t stop = take_event(h);
+        if (!stop) {
+            h->ev_pool.push_back(start);
+            return;
+        }
+        cudaEventRecord(stop, st);
+        h->marks.push_back({kind, start, stop});
+        start = nullptr;
+    }
+};
+
+slorr_status check_matrix_ptrs(const slorr_handle* h, const void* const* arr, const char* what) {
+    if (!arr) return fail(SLORR_ERR_INVALID_ARG, std::string(what) + " array is NULL");
+    for (size_t i = 0; i < h->shapes.size(); ++i) {
+        if (!arr[i]) return fail(SLORR_ERR_INVALID_ARG, std::string(what) + " pointer is NULL");
+        if (reinterpret_cast<uintptr_t>(arr[i]) % 16 != 0)
+            return fail(SLORR_ERR_INVALID_ARG, std::string(what) + " pointer is not 16-byte aligned");
+    }
+    return SLORR_OK;
+}
+
+MemLaunch mem_params(slorr_handle* h, uint8_t* ws, float* loss, float* per, int cur) {
+    MemLaunch p{};
+    p.mats = reinterpret_cast<const MatDev*>(ws + h->off_mats);
+    p.scalars = reinterpret_cast<MatScalars*>(ws + h->off_scalars);
+    p.partials = reinterpret_cast<float*>(ws + h->off_partials);
+    p.tile_base = reinterpret_cast<const int32_t*>(ws + h->off_tilebase);
+    p.tile_count = reinterpret_cast<const int32_t*>(ws + h->off_tilecount);
+    p.counters = reinterpret_cast<uint32_t*>(ws + h->off_counters);
+    p.status = reinterpret_cast<uint32_t*>(ws + h->off_status);
+    p.count = int(h->shapes.size());
+    p.cur = cur;
+    p.elem = h->elem;
+    p.wdtype = h->opt.dtype == SLORR_BF16 ? 1 : 0;
+    p.variant = h->opt.variant;
+    p.eps = h->opt.eps;
+    p.lambda = h->opt.lambda;
+    p.grad_scale = h->opt.grad_scale;
+    p.loss_out = loss;
+    p.per_matrix_out = per;
+    p.weights = reinterpret_cast<const void* const*>(ws + h->off_ptrs);
+    p.grads = reinterpret_cast<void* const*>(ws + h->off_ptrs + h->shapes.size() * sizeof(void*));
+    return p;
+}
+
+slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads, float* loss, float* per,
+                 void* workspace, size_t ws_bytes, int steps, bool finish, cudaStream_t st) {
+    if (!h) return fail(SLORR_ERR_INVALID_ARG, "handle is NULL");
+    slorr_status s = check_matrix_ptrs(h, weights, "weight");
+    if (s != SLORR_OK) return s;
+    if (finish) {
+        s = check_matrix_ptrs(h, grads, "grad");
+        if (s != SLORR_OK) return s;
+        if (!loss) return fail(SLORR_ERR_INVALID_ARG, "loss_out is NULL");
+        for (size_t i = 0; i < h->shapes.size(); ++i)
+            if (grads[i] == weights[i]) return fail(SLORR_ERR_INVALID_ARG, "a grad aliases its weight");
+    }
+    if (!workspace) return fail(SLORR_ERR_WORKSPACE, "workspace is NULL");
+    if (reinterpret_cast<uintptr_t>(workspace) % 256 != 0)
+        return fail(SLORR_ERR_WORKSPACE, "workspace is not 256-byte aligned");
+    if (ws_bytes < h->total_bytes) return fail(SLORR_ERR_WORKSPACE, "workspace too small");
+    if (steps < 0 || steps > h->opt.iters) return fail(SLORR_ERR_INVALID_ARG, "steps out of range");
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    s = prepare(h, ws, st);
+    if (s != SLORR_OK) return s;
+    s = upload_ptrs(h, ws, weights, finish ? grads : nullptr, st);
+    if (s != SLORR_OK) return s;
+    cudaError_t e = cudaMemsetAsync(ws + h->off_counters, 0, (h->shapes.size() + 1) * 4, st);
+    if (e != cudaSuccess) return cuda_fail(e, "counter reset");
+
+    MemLaunch mp = mem_params(h, ws, loss, per, 0);
+    mp.items = reinterpret_cast<const MemItem*>(ws + h->off_w_items);
+    mp.num_items = int(h->w_items.size());
+    {
+        Traced tr(h, 0, st);
+        if ((e = launch_sumsq(mp, st)) != cudaSuccess) return cuda_fail(e, "sumsq launch");
+        tr.done();
+    }
+    MemLaunch cp = mp;
+    cp.items = reinterpret_cast<const MemItem*>(ws + h->off_x_items);
+    cp.num_items = int(h->x_items.size());
+    {
+        Traced tr(h, 1, st);
+        if ((e = launch_cast(cp, st)) != cudaSuccess) return cuda_fail(e, "cast launch");
+        tr.done();
+    }
+
+    const bool use_tc = h->opt.compute != SLORR_COMPUTE_FP32 && !(h->opt.flags & SLORR_FLAG_SIMT_GEMM);
+    GemmLaunch g{};
+    g.mats = reinterpret_cast<const MatDev*>(ws + h->off_mats);
+    g.maps = ws + h->off_maps;
+    g.status = reinterpret_cast<uint32_t*>(ws + h->off_status);
+    g.timeout_ns = static_cast<unsigned long long>(h->opt.timeout_s * 1e9);
+    for (int t = 0; t < steps; ++t) {
+        g.cur = t & 1;
+        g.a = float(h->coeffs[3 * t + 0]);
+        g.b = float(h->coeffs[3 * t + 1]);
+        g.c = float(h->coeffs[3 * t + 2]);
+        for (int ph = 0; ph < 3; ++ph) {
+            g.phase = ph;
+            Traced tr(h, 2 + ph, st);
+            if (use_tc) {
+                g.items = reinterpret_cast<const GemmItem*>(ws + h->off_tc_items[ph]);
+                g.num_items = int(h->tc_items[ph].size());
+                e = launch_gemm_tc(g, h->elem, h->num_sms, st);
+            } else {
+                g.items = reinterpret_cast<const GemmItem*>(ws + h->off_simt_items[ph]);
+                g.num_items = int(h->simt_items[ph].size());
+                e = launch_gemm_simt(g, h->elem, st);
+            }
+            if (e != cudaSuccess) return cuda_fail(e, "gemm launch");
+            tr.done();
+        }
+    }
+    if (!finish) return SLORR_OK;
+    MemLaunch dp = mem_params(h, ws, loss, per, steps & 1);
+    dp.items = reinterpret_cast<const MemItem*>(ws + h->off_w_items);
+    dp.num_items = int(h->w_items.size());
+    {
+        Traced tr(h, 5, st);
+        if ((e = launch_dot(dp, st)) != cudaSuccess) return cuda_fail(e, "dot launch");
+        tr.done();
+    }
+    {
+        Traced tr(h, 6, st);
+        if ((e = launch_combine(dp, st)) != cudaSuccess) return cuda_fail(e, "combine launch");
+        tr.done();
+    }
+    return SLORR_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+void slorr_default_options(slorr_options* o) {
+    if (!o) return;
+    std::memset(o, 0, sizeof(*o));
+    o->variant = SLORR_HOYER;
+    o->compute = SLORR_COMPUTE_FP16;
+    o->dtype = SLORR_F32;
+    o->iters = 6;
+    o->ell = 1e-3;
+    o->cushion = -1.0;
+    o->safety = 1.01;
+    o->lambda = 1.0f;
+    o->eps = 1e-7f;
+    o->grad_scale = 1.0f;
+    o->flags = 0;
+    o->timeout_s = 2.0;
+}
+
+slorr_status slorr_create(slorr_handle** out, const slorr_shape* shapes, int32_t count, const slorr_options* opt) {
+    if (!out) return fail(SLORR_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    if (!shapes) return fail(SLORR_ERR_INVALID_ARG, "shapes is NULL");
+    if (count < 1 || count > kMaxMatrices) return fail(SLORR_ERR_INVALID_ARG, "count must be in [1, 4096]");
+    slorr_options o;
+    if (opt)
+        o = *opt;
+    else
+        slorr_default_options(&o);
+    std::string why;
+    if (!valid_options(o, &why)) return fail(SLORR_ERR_INVALID_ARG, "bad option: " + why);
+    for (int i = 0; i < count; ++i)
+        if (shapes[i].m < 1 || shapes[i].n < 1 || shapes[i].m > 65536 || shapes[i].n > 65536)
+            return fail(SLORR_ERR_INVALID_ARG, "matrix dimensions must be in [1, 65536]");
+    auto* h = new slorr_handle();
+    h->opt = o;
+    h->shapes.assign(shapes, shapes + count);
+    h->coeffs.resize(size_t(3) * o.iters);
+    if (!host::pe_schedule(o.iters, o.ell, o.cushion, o.safety, h->coeffs.data())) {
+        delete h;
+        return fail(SLORR_ERR_INVALID_ARG, "Polar Express schedule could not be built");
+    }
+    if (o.compute == SLORR_COMPUTE_FP32) {
+        h->elem = kF32;
+        h->esize = 4;
+    } else {
+        h->elem = o.compute == SLORR_COMPUTE_BF16 ? kBF16 : kF16;
+        h->esize = 2;
+    }
+    build_plan(h);
+    *out = h;
+    return SLORR_OK;
+}
+
+slorr_status slorr_workspace_size(const slorr_handle* h, size_t* bytes) {
+    if (!h || !bytes) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
+    *bytes = h->total_bytes;
+    return SLORR_OK;
+}
+
+slorr_status slorr_reg_forward_backward(slorr_handle* h, const void* const* weights, void* const* grads,
+                                        float* loss_out, float* per_matrix_out, void* workspace,
+                                        size_t workspace_bytes, void* stream) {
+    if (!h) return fail(SLORR_ERR_INVALID_ARG, "handle is NULL");
+    return run(h, weights, grads, loss_out, per_matrix_out, workspace, workspace_bytes, h->opt.iters, true,
+               static_cast<cudaStream_t>(stream));
+}
+
+slorr_status slorr_reset_workspace(slorr_handle* h) {
+    if (!h) return fail(SLORR_ERR_INVALID_ARG, "handle is NULL");
+    h->prepared_ws = nullptr;
+    h->last_ptrs.clear();
+    return SLORR_OK;
+}
+
+slorr_status slorr_get_status(slorr_handle* h, const void* workspace, void* stream) {
+    if (!h || !workspace) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+    uint32_t word = 0;
+    uint8_t* ws = static_cast<uint8_t*>(const_cast<void*>(workspace));
+    e = cudaMemcpy(&word, ws + h->off_status, 4, cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess) e = cudaMemset(ws + h->off_status, 0, 4);
+    if (e != cudaSuccess) return cuda_fail(e, "status read");
+    if (word & kStatusTimeout) return fail(SLORR_ERR_TIMEOUT, "a device-side wait timed out");
+    if (word & kStatusNonFinite) return fail(SLORR_ERR_NONFINITE, "non-finite norm or estimate");
+    return SLORR_OK;
+}
+
+slorr_status slorr_run_steps(slorr_handle* h, const void* const* weights, void* workspace, size_t workspace_bytes,
+                             int32_t steps, void* stream) {
+    return run(h, weights, nullptr, nullptr, nullptr, workspace, workspace_bytes, steps, false,
+               static_cast<cudaStream_t>(stream));
+}
+
+slorr_status slorr_iterate_view(const slorr_handle* h, const void* workspace, int32_t i, int32_t after_steps,
+                                slorr_matrix_view* out) {
+    if (!h || !workspace || !out) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
+    if (i < 0 || i >= int(h->shapes.size())) return fail(SLORR_ERR_INVALID_ARG, "matrix index out of range");
+    if (after_steps < 0 || after_steps > h->opt.iters) return fail(SLORR_ERR_INVALID_ARG, "steps out of range");
+    const Geom& g = h->geom[i];
+    const uint8_t* ws = static_cast<const uint8_t*>(workspace);
+    out->x = ws + g.off_x[after_steps & 1];
+    out->rows = g.P;
+    out->cols = g.Q;
+    out->ld = g.Qpad;
+    out->elem = h->elem;
+    out->transposed = g.transposed;
+    const MatScalars* sc = reinterpret_cast<const MatScalars*>(ws + h->off_scalars) + i;
+    out->frob_sq = &sc->frob_sq;
+    out->n_hat = &sc->n_hat;
+    return SLORR_OK;
+}
+
+slorr_status slorr_get_coefficients(const slorr_handle* h, double* abc, int32_t capacity) {
+    if (!h || !abc) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
+    if (capacity < int(h->coeffs.size())) return fail(SLORR_ERR_INVALID_ARG, "capacity too small");
+    std::copy(h->coeffs.begin(), h->coeffs.end(), abc);
+    return SLORR_OK;
+}
+
+slorr_status slorr_pe_coefficients(int32_t iters, double ell, double cushion, double safety, double* abc) {
+    if (!abc) return fail(SLORR_ERR_INVALID_ARG, "abc is NULL");
+    if (iters < 1 || iters > kMaxIters) return fail(SLORR_ERR_INVALID_ARG, "iters must be in [1, 16]");
+    if (!host::pe_schedule(iters, ell, cushion, safety, abc))
+        return fail(SLORR_ERR_INVALID_ARG, "Polar Express schedule could not be built");
+    return SLORR_OK;
+}
+
+double slorr_cushion_ratio(void) { return host::cushion_ratio(); }
+
+int64_t slorr_flops(const slorr_shape* shapes, int32_t count, int32_t iters) {
+    if (!shapes || count < 0 || iters < 0) return -1;
+    int64_t total = 0;
+    for (int i = 0; i < count; ++i) {
+        const int64_t P = std::min(shapes[i].m, shapes[i].n), Q = std::max(shapes[i].m, shapes[i].n);
+        total += 4 * P * P * Q + 2 * P * P * P;
+    }
+    return total * iters;
+}
+
+slorr_status slorr_partition(const slorr_shape* shapes, int32_t count, int32_t world, int32_t rank,
+                             int32_t* out_indices, int32_t* out_count) {
+    if (!shapes || !out_indices || !out_count || count < 0) return fail(SLORR_ERR_INVALID_ARG, "bad argument");
+    if (world < 1 || rank < 0 || rank >= world) return fail(SLORR_ERR_INVALID_ARG, "bad world/rank");
+    std::vector<int> order(count);
+    std::iota(order.begin(), order.end(), 0);
+    auto cost = [&](int i) { return slorr_flops(&shapes[i], 1, 1); };
+    std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return cost(a) > cost(b); });
+    std::vector<int64_t> load(world, 0);
+    std::vector<int> owner(count, 0);
+    for (int i : order) {
+        int best = 0;
+        for (int r = 1; r < world; ++r)
+            if (load[r] < load[best]) best = r;
+        owner[i] = best;
+        load[best] += cost(i);
+    }
+    int k = 0;
+    for (int i = 0; i < count; ++i)
+        if (owner[i] == rank) out_indices[k++] = i;
+    *out_count = k;
+    return SLORR_OK;
+}
+
+slorr_status slorr_set_timing(slorr_handle* h, int32_t enable) {
+    if (!h) return fail(SLORR_ERR_INVALID_ARG, "handle is NULL");
+    h->timing = enable != 0;
+    return SLORR_OK;
+}
+
+slorr_status slorr_read_timing(slorr_handle* h, double* ms, int64_t* launches, int32_t kinds) {
+    if (!h || !ms || !launches || kinds < 1 || kinds > SLORR_NUM_KERNEL_KINDS)
+        return fail(SLORR_ERR_INVALID_ARG, "bad argument");
+    slorr_status s = SLORR_OK;
+    for (auto& m : h->marks) {
+        float t = 0.f;
+        cudaError_t e = cudaEventSynchronize(m.stop);
+        if (e == cudaSuccess) e = cudaEventElapsedTime(&t, m.start, m.stop);
+        if (e != cudaSuccess && s == SLORR_OK) s = cuda_fail(e, "event timing");
+        if (m.kind < kinds) {
+            ms[m.kind] += double(t);
+            launches[m.kind] += 1;
+        }
+        h->ev_pool.push_back(m.start);
+        h->ev_pool.push_back(m.stop);
+    }
+    h->marks.clear();
+    return s;
+}
+
+void slorr_destroy(slorr_handle* h) { delete h; }
+
+const char* slorr_status_string(slorr_status s) {
+    switch (s) {
+        case SLORR_OK: return "ok";
+        case SLORR_ERR_INVALID_ARG: return "invalid argument";
+        case SLORR_ERR_UNSUPPORTED: return "unsupported";
+        case SLORR_ERR_CUDA: return "CUDA error";
+        case SLORR_ERR_WORKSPACE: return "workspace missing or too small";
+        case SLORR_ERR_TIMEOUT: return "device wait timed out";
+        case SLORR_ERR_NONFINITE: return "non-finite value";
+    }
+    return "unknown status";
+}
+
+const char* slorr_last_error(void) { return g_last_error.c_str(); }
+
+}  // extern "C"

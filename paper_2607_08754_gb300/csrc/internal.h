@@ -1,0 +1,117 @@
+// Internal declarations shared by libslorr's translation units.
+//
+// Device-side plan: for each weight matrix W_i (m x n) the Polar Express
+// iterate X is P x Q with P = min(m, n), Q = max(m, n) (Sec. 3 "Computational
+// cost": the Gram matrix is formed on the min side), stored row-major and
+// zero-padded to Ppad x Qpad (Ppad a multiple of 128, Qpad a multiple of 64).
+// Zero padding is exact: zero rows/columns of X give zero rows/columns of
+// A = X X^T and B = b A + c A^2, and the odd polynomial maps zero to zero
+// (App. B, "zero singular values stay zero").
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+namespace slorr {
+
+constexpr int kMaxMatrices = 4096;
+constexpr int kMaxIters = 16;
+constexpr int kPadRows = 128;   // Ppad granularity (tcgen05 tile M)
+constexpr int kPadCols = 64;    // Qpad granularity (one 128-byte swizzle row of 16-bit)
+
+// Element type of the iterate buffers X, A, B.
+enum Elem : int32_t { kF32 = 0, kF16 = 1, kBF16 = 2 };
+
+// Status bits written by kernels into the workspace status word.
+enum StatusBits : uint32_t { kStatusTimeout = 1u, kStatusNonFinite = 2u };
+
+// Per-matrix device descriptor (lives in the workspace).
+struct MatDev {
+    void* x[2];        // ping-pong iterate buffers, Ppad x Qpad
+    void* a;           // A = X X^T, Ppad x Ppad
+    void* b;           // B = b A + c A^2, Ppad x Ppad
+    int32_t m, n;      // shape of W
+    int32_t P, Q;      // min / max
+    int32_t Ppad, Qpad;
+    int32_t transposed;  // 1 when m > n (X = W^T)
+    int32_t pad_;
+};
+
+// Per-matrix scalars (workspace).
+struct MatScalars {
+    double frob_sq;    // ||W||_F^2
+    double n_hat;      // sum(W * P_hat)
+};
+
+// One output tile of a grouped GEMM phase.
+struct GemmItem {
+    uint16_t mat;
+    uint16_t tm;       // row tile index (tile rows = 128 for tcgen05, 64 for SIMT)
+    uint16_t tn;       // column tile index
+    uint16_t nsz;      // columns in this tile
+};
+
+// One chunk of a memory-bound pass over a weight matrix: a 2-D tile of W.
+struct MemItem {
+    uint16_t mat;
+    uint16_t tile_r;   // tile row index over W (64 rows)
+    uint16_t tile_c;   // tile column index over W (64 cols)
+    uint16_t seq;      // index of this tile within its matrix
+};
+
+// Phases of one Polar Express step.
+enum Phase : int32_t { kGram = 0, kPoly = 1, kUpdate = 2 };
+
+struct GemmLaunch {
+    const GemmItem* items;
+    int32_t num_items;
+    int32_t phase;
+    int32_t cur;               // index of the current iterate buffer (0/1)
+    float a, b, c;             // step coefficients (a_t, b_t, c_t)
+    const MatDev* mats;
+    const void* maps;          // CUtensorMap array, 4 per matrix (X0, X1, A, B)
+    uint32_t* status;
+    unsigned long long timeout_ns;
+};
+
+struct MemLaunch {
+    const MemItem* items;
+    int32_t num_items;
+    const MatDev* mats;
+    MatScalars* scalars;
+    float* partials;           // one float per (matrix, tile)
+    const int32_t* tile_base;  // first partial index of each matrix
+    const int32_t* tile_count; // tiles per matrix
+    uint32_t* counters;        // per-matrix completion counters
+    uint32_t* status;
+    int32_t count;             // matrices
+    int32_t cur;               // iterate buffer holding X_0 (cast) or X_T (dot/combine)
+    int32_t elem;              // Elem of the iterate
+    int32_t wdtype;            // 0 fp32, 1 bf16 weights/grads
+    int32_t variant;           // 0 Hoyer, 1 Nuc
+    float eps, lambda, grad_scale;
+    float* loss_out;
+    float* per_matrix_out;
+    const void* const* weights;  // device array of weight pointers
+    void* const* grads;          // device array of grad pointers
+};
+
+// Launchers (return cudaGetLastError() of the launch).
+cudaError_t launch_sumsq(const MemLaunch& p, cudaStream_t s);
+cudaError_t launch_cast(const MemLaunch& p, cudaStream_t s);
+cudaError_t launch_dot(const MemLaunch& p, cudaStream_t s);
+cudaError_t launch_combine(const MemLaunch& p, cudaStream_t s);
+cudaError_t launch_gemm_simt(const GemmLaunch& p, int elem, cudaStream_t s);
+cudaError_t launch_gemm_tc(const GemmLaunch& p, int elem, int grid, cudaStream_t s);
+int tc_smem_bytes();
+
+// Host Polar Express schedule (schedule.cpp).
+namespace host {
+bool minimax_quintic(double lo, double hi, double out[4]);
+double cushion_ratio();
+bool pe_schedule(int T, double ell, double cushion, double safety, double* abc);
+}  // namespace host
+
+}  // namespace slorr

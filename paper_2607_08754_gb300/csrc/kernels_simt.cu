@@ -1,0 +1,121 @@
+// Grouped SIMT (CUDA-core) GEMM for the three phases of a Polar Express step
+// (Sec. 3 "Computational cost": A = X X^T, B = b A + c A^2, X <- a X + B X on
+// the P x Q Gram side).  Used for the fp32 compute mode, whose operands and
+// accumulation are fp32, and, with 16-bit storage, as a CUDA-core check of the
+// tensor-core kernel.  64 x 64 output tile per block, 256 threads, 4 x 4 per
+// thread, K staged 16 at a time through shared memory.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include "internal.h"
+
+namespace slorr {
+namespace {
+
+constexpr int kBM = 64, kBN = 64, kBK = 16;
+
+template <typename T>
+__device__ __forceinline__ float ld_f(const T* p);
+template <>
+__device__ __forceinline__ float ld_f<float>(const float* p) { return *p; }
+template <>
+__device__ __forceinline__ float ld_f<__half>(const __half* p) { return __half2float(*p); }
+template <>
+__device__ __forceinline__ float ld_f<__nv_bfloat16>(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+
+template <typename T>
+__device__ __forceinline__ void st_f(T* p, float v);
+template <>
+__device__ __forceinline__ void st_f<float>(float* p, float v) { *p = v; }
+template <>
+__device__ __forceinline__ void st_f<__half>(__half* p, float v) { *p = __float2half_rn(v); }
+template <>
+__device__ __forceinline__ void st_f<__nv_bfloat16>(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
+
+template <typename T>
+__global__ void __launch_bounds__(256) simt_gemm_kernel(const GemmLaunch p) {
+    __shared__ float As[kBK][kBM + 4];
+    __shared__ float Bs[kBK][kBN + 4];
+    const GemmItem it = p.items[blockIdx.x];
+    const MatDev md = p.mats[it.mat];
+    const T* X = reinterpret_cast<const T*>(md.x[p.cur]);
+    const T* Am = reinterpret_cast<const T*>(md.a);
+    const T* Bm = reinterpret_cast<const T*>(md.b);
+    // Operand addressing: Aop(i, k) = opA[i * lda + k]; Bop(k, j) = opB[j * ldb_j + k * ldb_k].
+    const T* opA;
+    const T* opB;
+    int64_t lda, ldb_j, ldb_k;
+    int K;
+    if (p.phase == kGram) {
+        opA = X; lda = md.Qpad; opB = X; ldb_j = md.Qpad; ldb_k = 1; K = md.Qpad;
+    } else if (p.phase == kPoly) {
+        opA = Am; lda = md.Ppad; opB = Am; ldb_j = md.Ppad; ldb_k = 1; K = md.Ppad;
+    } else {
+        opA = Bm; lda = md.Ppad; opB = X; ldb_j = 1; ldb_k = md.Qpad; K = md.Ppad;
+    }
+    const int m0 = it.tm * kBM, n0 = it.tn * kBN;
+    const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
+    float acc[4][4] = {};
+    for (int k0 = 0; k0 < K; k0 += kBK) {
+        // 64 x 16 of each operand: 1024 values, 4 per thread.
+        for (int e = threadIdx.x; e < kBM * kBK; e += 256) {
+            const int i = e / kBK, k = e % kBK;
+            As[k][i] = ld_f<T>(opA + static_cast<int64_t>(m0 + i) * lda + (k0 + k));
+        }
+        for (int e = threadIdx.x; e < kBN * kBK; e += 256) {
+            int j, k;
+            if (ldb_k == 1) { j = e / kBK; k = e % kBK; } else { k = e / kBN; j = e % kBN; }
+            Bs[k][j] = ld_f<T>(opB + static_cast<int64_t>(n0 + j) * ldb_j + static_cast<int64_t>(k0 + k) * ldb_k);
+        }
+        __syncthreads();
+#pragma unroll
+        for (int k = 0; k < kBK; ++k) {
+            float a[4], b[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) a[u] = As[k][ty * 4 + u];
+#pragma unroll
+            for (int v = 0; v < 4; ++v) b[v] = Bs[k][tx * 4 + v];
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(a[u], b[v], acc[u][v]);
+        }
+        __syncthreads();
+    }
+    T* out;
+    const T* extra;
+    int64_t ldo;
+    float ce, cacc;
+    if (p.phase == kGram) {
+        out = reinterpret_cast<T*>(md.a); extra = nullptr; ldo = md.Ppad; ce = 0.f; cacc = 1.f;
+    } else if (p.phase == kPoly) {
+        out = reinterpret_cast<T*>(md.b); extra = Am; ldo = md.Ppad; ce = p.b; cacc = p.c;
+    } else {
+        out = reinterpret_cast<T*>(md.x[p.cur ^ 1]); extra = X; ldo = md.Qpad; ce = p.a; cacc = 1.f;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            const int64_t idx = static_cast<int64_t>(m0 + ty * 4 + u) * ldo + (n0 + tx * 4 + v);
+            float val = cacc * acc[u][v];
+            if (extra) val = fmaf(ce, ld_f<T>(extra + idx), val);
+            st_f<T>(out + idx, val);
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_gemm_simt(const GemmLaunch& p, int elem, cudaStream_t s) {
+    if (p.num_items == 0) return cudaSuccess;
+    if (elem == kF32)
+        simt_gemm_kernel<float><<<p.num_items, 256, 0, s>>>(p);
+    else if (elem == kF16)
+        simt_gemm_kernel<__half><<<p.num_items, 256, 0, s>>>(p);
+    else
+        simt_gemm_kernel<__nv_bfloat16><<<p.num_items, 256, 0, s>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace slorr

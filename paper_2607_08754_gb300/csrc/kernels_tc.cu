@@ -1,0 +1,371 @@
+// Grouped persistent tensor-core GEMM for one phase of a Polar Express step
+// (Sec. 3 "Computing the polar factor" / "Computational cost"):
+//   Gram    A  = X X^T            M = Ppad, N = Ppad, K = Qpad   (both operands K-major)
+//   Poly    B  = b A + c A A      M = Ppad, N = Ppad, K = Ppad   (A symmetric: both K-major)
+//   Update  X' = a X + B X        M = Ppad, N = Qpad, K = Ppad   (X is the MN-major operand)
+// over every matrix of the weight set in one launch.  Operands are fp16 or
+// bf16, accumulation fp32 in tensor memory.
+//
+// One CTA per SM (192 threads):
+//   warp 0      TMA producer: 128 x 64 A-operand and nsz x 64 B-operand boxes
+//               (128-byte swizzle) into a 4-stage shared-memory ring;
+//   warp 1      allocates 512 TMEM columns; lane 0 issues tcgen05.mma
+//               (M = 128, N = nsz <= 256, K = 16) into one of two 256-column
+//               fp32 accumulators and commits stage releases / tile completion;
+//   warps 2..5  epilogue: tcgen05.ld 32 columns at a time, combine with the
+//               a X or b A term in fp32, round to 16 bit, store to global.
+// Output tiles are 128 x nsz with nsz a multiple of 64, taken round-robin from
+// a host-built list; accumulator double-buffering overlaps a tile's epilogue
+// with the next tile's main loop.  Every wait is bounded; on a timeout the CTA
+// records it in the status word, drains its in-flight copies and MMAs and
+// returns.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace slorr {
+namespace {
+
+constexpr int kBM = 128;
+constexpr int kBNMax = 256;
+constexpr int kBK = 64;  // 64 x 16-bit = one 128-byte swizzle row
+constexpr int kStages = 4;
+constexpr int kABytes = kBM * kBK * 2;      // 16 KB
+constexpr int kBBytes = kBNMax * kBK * 2;   // 32 KB
+constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kBoxBytes = 64 * kBK * 2;     // one 64-row box, 8 KB
+constexpr int kTmemCols = 512;
+constexpr int kAccCols = 256;
+constexpr int kThreads = 192;
+constexpr int kEpiWarps = 4;
+constexpr size_t kSmemBytes = size_t(kStages) * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+
+template <bool BF16>
+__device__ __forceinline__ uint32_t pack2(float lo, float hi) {
+    if constexpr (BF16) {
+        __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+        return *reinterpret_cast<uint32_t*>(&v);
+    } else {
+        __half2 v = __floats2half2_rn(lo, hi);
+        return *reinterpret_cast<uint32_t*>(&v);
+    }
+}
+
+template <bool BF16>
+__device__ __forceinline__ float2 unpack2(uint32_t u) {
+    if constexpr (BF16) {
+        __nv_bfloat162 v = *reinterpret_cast<__nv_bfloat162*>(&u);
+        return __bfloat1622float2(v);
+    } else {
+        __half2 v = *reinterpret_cast<__half2*>(&u);
+        return __half22float2(v);
+    }
+}
+
+struct Smem {
+    uint8_t* stages;
+    uint64_t* full;
+    uint64_t* empty;
+    uint64_t* tfull;
+    uint64_t* tempty;
+    uint64_t* drain;
+    uint32_t* tmem_slot;
+    volatile int* abort;
+    volatile int* never;  // stays 0: drain waits ignore the abort flag
+};
+
+__device__ __forceinline__ void record_timeout(const GemmLaunch& p, const Smem& s) {
+    *s.abort = 1;
+    atomicOr(p.status, kStatusTimeout);
+}
+
+struct PhaseInfo {
+    const void* mapA;
+    const void* mapB;
+    int nkb;
+    bool b_mn;
+};
+
+__device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmItem& it) {
+    const MatDev& md = p.mats[it.mat];
+    const uint8_t* maps = reinterpret_cast<const uint8_t*>(p.maps) + size_t(it.mat) * 4 * 128;
+    PhaseInfo pi;
+    if (p.phase == kGram) {
+        pi.mapA = maps + p.cur * 128;
+        pi.mapB = pi.mapA;
+        pi.nkb = md.Qpad / kBK;
+        pi.b_mn = false;
+    } else if (p.phase == kPoly) {
+        pi.mapA = maps + 2 * 128;
+        pi.mapB = pi.mapA;
+        pi.nkb = md.Ppad / kBK;
+        pi.b_mn = false;
+    } else {
+        pi.mapA = maps + 3 * 128;
+        pi.mapB = maps + p.cur * 128;
+        pi.nkb = md.Ppad / kBK;
+        pi.b_mn = true;
+    }
+    return pi;
+}
+
+__device__ void producer(const GemmLaunch& p, const Smem& s) {
+    int stage = 0;
+    uint32_t phase = 0;
+    int issued_parity[kStages];
+#pragma unroll
+    for (int i = 0; i < kStages; ++i) issued_parity[i] = -1;
+    bool ok = true;
+    for (int idx = blockIdx.x; idx < p.num_items && ok; idx += gridDim.x) {
+        const GemmItem it = p.items[idx];
+        const PhaseInfo pi = phase_info(p, it);
+        const uint32_t bytes = kABytes + uint32_t(it.nsz) * kBK * 2;
+        const int nboxes = it.nsz / 64;
+        for (int kb = 0; kb < pi.nkb; ++kb) {
+            if (!ptx::mbar_wait(&s.empty[stage], phase ^ 1u, s.abort, p.timeout_ns)) {
+                record_timeout(p, s);
+                ok = false;
+                break;
+            }
+            uint8_t* sa = s.stages + size_t(stage) * kStageBytes;
+            uint8_t* sb = sa + kABytes;
+            ptx::mbar_arrive_expect_tx(&s.full[stage], bytes);
+            ptx::tma_load_2d(sa, pi.mapA, &s.full[stage], kb * kBK, it.tm * kBM);
+            ptx::tma_load_2d(sa + kBoxBytes, pi.mapA, &s.full[stage], kb * kBK, it.tm * kBM + 64);
+            for (int j = 0; j < nboxes; ++j) {
+                if (pi.b_mn)
+                    ptx::tma_load_2d(sb + j * kBoxBytes, pi.mapB, &s.full[stage],
+                                     it.tn * kBNMax + j * 64, kb * kBK);
+                else
+                    ptx::tma_load_2d(sb + j * kBoxBytes, pi.mapB, &s.full[stage], kb * kBK,
+                                     it.tn * kBNMax + j * 64);
+            }
+            issued_parity[stage] = int(phase);
+            if (++stage == kStages) {
+                stage = 0;
+                phase ^= 1u;
+            }
+        }
+    }
+    if (!ok) {
+        // Wait (bounded) for every copy this thread issued to land before exit.
+        for (int i = 0; i < kStages; ++i)
+            if (issued_parity[i] >= 0)
+                ptx::mbar_wait(&s.full[i], uint32_t(issued_parity[i]), s.never, p.timeout_ns);
+    }
+}
+
+template <bool BF16>
+__device__ void mma_issuer(const GemmLaunch& p, const Smem& s, uint32_t tmem_base) {
+    int stage = 0;
+    uint32_t phase = 0;
+    int local = 0;
+    bool ok = true;
+    bool issued_any = false;
+    for (int idx = blockIdx.x; idx < p.num_items && ok; idx += gridDim.x, ++local) {
+        const GemmItem it = p.items[idx];
+        const PhaseInfo pi = phase_info(p, it);
+        const uint32_t idesc = ptx::idesc_f16(kBM, it.nsz, BF16, pi.b_mn);
+        const int buf = local & 1;
+        const uint32_t tphase = (uint32_t(local) >> 1) & 1u;
+        if (!ptx::mbar_wait(&s.tempty[buf], tphase ^ 1u, s.abort, p.timeout_ns)) {
+            record_timeout(p, s);
+            ok = false;
+            break;
+        }
+        ptx::tc_fence_after();
+        const uint32_t d_tmem = tmem_base + uint32_t(buf * kAccCols);
+        for (int kb = 0; kb < pi.nkb; ++kb) {
+            if (!ptx::mbar_wait(&s.full[stage], phase, s.abort, p.timeout_ns)) {
+                record_timeout(p, s);
+                ok = false;
+                break;
+            }
+            ptx::tc_fence_after();
+            const uint32_t a0 = ptx::smem_u32(s.stages + size_t(stage) * kStageBytes);
+            const uint32_t b0 = a0 + kABytes;
+#pragma unroll
+            for (int kk = 0; kk < kBK / 16; ++kk) {
+                const uint64_t ad = ptx::sdesc_sw128(a0 + kk * 32, 16, 1024);
+                const uint64_t bd = pi.b_mn ? ptx::sdesc_sw128(b0 + kk * 16 * 128, 8192, 1024)
+                                            : ptx::sdesc_sw128(b0 + kk * 32, 16, 1024);
+                ptx::umma_f16(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
+            }
+            issued_any = true;
+            ptx::umma_commit(&s.empty[stage]);
+            if (++stage == kStages) {
+                stage = 0;
+                phase ^= 1u;
+            }
+        }
+        if (!ok) break;
+        ptx::umma_commit(&s.tfull[buf]);
+    }
+    if (!ok && issued_any) {
+        // Make sure no MMA is still writing TMEM before it is released.
+        ptx::umma_commit(s.drain);
+        ptx::mbar_wait(s.drain, 0u, s.never, p.timeout_ns);
+    }
+}
+
+template <bool BF16>
+__device__ void epilogue(const GemmLaunch& p, const Smem& s, uint32_t tmem_base, int warp,
+                         int lane) {
+    const int quad = warp & 3;  // TMEM lanes [32 quad, 32 quad + 32)
+    int local = 0;
+    for (int idx = blockIdx.x; idx < p.num_items; idx += gridDim.x, ++local) {
+        const GemmItem it = p.items[idx];
+        const MatDev& md = p.mats[it.mat];
+        const int buf = local & 1;
+        const uint32_t tphase = (uint32_t(local) >> 1) & 1u;
+        int ok = 1;
+        if (lane == 0) ok = ptx::mbar_wait(&s.tfull[buf], tphase, s.abort, p.timeout_ns) ? 1 : 0;
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok) {
+            if (lane == 0) record_timeout(p, s);
+            break;
+        }
+        ptx::tc_fence_after();
+        const int row = it.tm * kBM + quad * 32 + lane;
+        uint16_t* out;
+        const uint16_t* extra;
+        int64_t ld;
+        float ce, cacc;
+        if (p.phase == kGram) {
+            out = reinterpret_cast<uint16_t*>(md.a); extra = nullptr; ld = md.Ppad; ce = 0.f; cacc = 1.f;
+        } else if (p.phase == kPoly) {
+            out = reinterpret_cast<uint16_t*>(md.b);
+            extra = reinterpret_cast<const uint16_t*>(md.a);
+            ld = md.Ppad; ce = p.b; cacc = p.c;
+        } else {
+            out = reinterpret_cast<uint16_t*>(md.x[p.cur ^ 1]);
+            extra = reinterpret_cast<const uint16_t*>(md.x[p.cur]);
+            ld = md.Qpad; ce = p.a; cacc = 1.f;
+        }
+        const uint32_t t_row = tmem_base + (uint32_t(quad * 32) << 16) + uint32_t(buf * kAccCols);
+        for (int ch = 0; ch < it.nsz / 32; ++ch) {
+            uint32_t r[32];
+            ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
+            ptx::tmem_ld_wait();
+            const int64_t off = int64_t(row) * ld + int64_t(it.tn) * kBNMax + ch * 32;
+            uint4 o[4];
+            uint32_t* ow = reinterpret_cast<uint32_t*>(o);
+            if (extra) {
+                uint4 e[4];
+                const uint4* src = reinterpret_cast<const uint4*>(extra + off);
+#pragma unroll
+                for (int v = 0; v < 4; ++v) e[v] = src[v];
+                const uint32_t* ew = reinterpret_cast<const uint32_t*>(e);
+#pragma unroll
+                for (int j = 0; j < 16; ++j) {
+                    const float2 x = unpack2<BF16>(ew[j]);
+                    const float lo = fmaf(ce, x.x, cacc * __uint_as_float(r[2 * j]));
+                    const float hi = fmaf(ce, x.y, cacc * __uint_as_float(r[2 * j + 1]));
+                    ow[j] = pack2<BF16>(lo, hi);
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                    ow[j] = pack2<BF16>(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
+            }
+            uint4* dst = reinterpret_cast<uint4*>(out + off);
+#pragma unroll
+            for (int v = 0; v < 4; ++v) dst[v] = o[v];
+        }
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(&s.tempty[buf]);
+    }
+}
+
+template <bool BF16>
+__global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ GemmLaunch p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* base = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    Smem s;
+    s.stages = base;
+    s.full = reinterpret_cast<uint64_t*>(base + size_t(kStages) * kStageBytes);
+    s.empty = s.full + kStages;
+    s.tfull = s.empty + kStages;
+    s.tempty = s.tfull + 2;
+    s.drain = s.tempty + 2;
+    s.tmem_slot = reinterpret_cast<uint32_t*>(s.drain + 1);
+    s.abort = reinterpret_cast<volatile int*>(s.tmem_slot + 1);
+    s.never = s.abort + 1;
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kStages; ++i) {
+            ptx::mbar_init(&s.full[i], 1);
+            ptx::mbar_init(&s.empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            ptx::mbar_init(&s.tfull[i], 1);
+            ptx::mbar_init(&s.tempty[i], kEpiWarps);
+        }
+        ptx::mbar_init(s.drain, 1);
+        *s.abort = 0;
+        *s.never = 0;
+        ptx::fence_mbar_init();
+    }
+    if (warp == 0 && lane == 0) {
+        // Warm the descriptors of the first item.
+        if (blockIdx.x < p.num_items) {
+            const PhaseInfo pi = phase_info(p, p.items[blockIdx.x]);
+            ptx::prefetch_tmap(pi.mapA);
+            ptx::prefetch_tmap(pi.mapB);
+        }
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(s.tmem_slot, kTmemCols);
+        ptx::tmem_relinquish();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem_base = *s.tmem_slot;
+
+    if (warp == 0) {
+        if (lane == 0) producer(p, s);
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0) mma_issuer<BF16>(p, s, tmem_base);
+        __syncwarp();
+    } else {
+        epilogue<BF16>(p, s, tmem_base, warp, lane);
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem_base, kTmemCols);
+    }
+}
+
+}  // namespace
+
+int tc_smem_bytes() { return int(kSmemBytes); }
+
+cudaError_t launch_gemm_tc(const GemmLaunch& p, int elem, int grid, cudaStream_t st) {
+    if (p.num_items == 0) return cudaSuccess;
+    static bool attr_set[2] = {false, false};
+    const int which = elem == kBF16 ? 1 : 0;
+    cudaError_t e;
+    if (!attr_set[which]) {
+        e = which ? cudaFuncSetAttribute(tc_gemm_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kSmemBytes))
+                  : cudaFuncSetAttribute(tc_gemm_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kSmemBytes));
+        if (e != cudaSuccess) return e;
+        attr_set[which] = true;
+    }
+    if (grid > p.num_items) grid = p.num_items;
+    if (which)
+        tc_gemm_kernel<true><<<grid, kThreads, kSmemBytes, st>>>(p);
+    else
+        tc_gemm_kernel<false><<<grid, kThreads, kSmemBytes, st>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace slorr

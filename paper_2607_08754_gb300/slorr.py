@@ -1,0 +1,326 @@
+"""ctypes binding of libslorr (include/slorr.h): argument marshalling only.
+
+Every step of the regularizer runs inside libslorr's CUDA kernels; this module
+only converts Python values into the C ABI's structs and pointers.  PyTorch is
+used (by ``Regularizer``) for device memory and the current stream.  There is
+no fallback: if libslorr.so is missing, loading raises.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libslorr.so")
+HEADER = os.path.join(os.path.dirname(HERE), "include", "slorr.h")
+
+SLORR_OK = 0
+STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "CUDA", 4: "WORKSPACE",
+                5: "TIMEOUT", 6: "NONFINITE"}
+VARIANTS = {"hoyer": 0, "nuclear": 1}
+COMPUTES = {"fp16": 0, "bf16": 1, "fp32": 2}
+DTYPES = {"f32": 0, "bf16": 1}
+FLAG_SIMT_GEMM = 1
+
+
+class SlorrError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        self.status = status
+        super().__init__(f"libslorr: {STATUS_NAMES.get(status, status)}: {message}")
+
+
+class Shape(ctypes.Structure):
+    _fields_ = [("m", ctypes.c_int64), ("n", ctypes.c_int64)]
+
+
+class Options(ctypes.Structure):
+    _fields_ = [("variant", ctypes.c_int32), ("compute", ctypes.c_int32), ("dtype", ctypes.c_int32),
+                ("iters", ctypes.c_int32), ("ell", ctypes.c_double), ("cushion", ctypes.c_double),
+                ("safety", ctypes.c_double), ("lambda_", ctypes.c_float), ("eps", ctypes.c_float),
+                ("grad_scale", ctypes.c_float), ("flags", ctypes.c_int32), ("timeout_s", ctypes.c_double)]
+
+
+class MatrixView(ctypes.Structure):
+    _fields_ = [("x", ctypes.c_void_p), ("rows", ctypes.c_int64), ("cols", ctypes.c_int64),
+                ("ld", ctypes.c_int64), ("elem", ctypes.c_int32), ("transposed", ctypes.c_int32),
+                ("frob_sq", ctypes.c_void_p), ("n_hat", ctypes.c_void_p)]
+
+
+_lib = None
+
+
+def load_library(path: str | None = None) -> ctypes.CDLL:
+    """Load libslorr.so (built in-tree by ``paper_2607_08754_gb300.build``)."""
+    global _lib
+    if _lib is not None and path is None:
+        return _lib
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise ImportError(f"libslorr.so not found at {p}: run __graft_entry__.build() first")
+    lib = ctypes.CDLL(p)
+    vp, i32, i64, dbl = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_double
+    sig = {
+        "slorr_default_options": (None, [ctypes.POINTER(Options)]),
+        "slorr_create": (i32, [ctypes.POINTER(vp), ctypes.POINTER(Shape), i32, ctypes.POINTER(Options)]),
+        "slorr_workspace_size": (i32, [vp, ctypes.POINTER(ctypes.c_size_t)]),
+        "slorr_reg_forward_backward": (i32, [vp, ctypes.POINTER(vp), ctypes.POINTER(vp), vp, vp, vp,
+                                             ctypes.c_size_t, vp]),
+        "slorr_reset_workspace": (i32, [vp]),
+        "slorr_get_status": (i32, [vp, vp, vp]),
+        "slorr_run_steps": (i32, [vp, ctypes.POINTER(vp), vp, ctypes.c_size_t, i32, vp]),
+        "slorr_iterate_view": (i32, [vp, vp, i32, i32, ctypes.POINTER(MatrixView)]),
+        "slorr_get_coefficients": (i32, [vp, ctypes.POINTER(dbl), i32]),
+        "slorr_pe_coefficients": (i32, [i32, dbl, dbl, dbl, ctypes.POINTER(dbl)]),
+        "slorr_cushion_ratio": (dbl, []),
+        "slorr_flops": (i64, [ctypes.POINTER(Shape), i32, i32]),
+        "slorr_partition": (i32, [ctypes.POINTER(Shape), i32, i32, i32, ctypes.POINTER(i32),
+                                  ctypes.POINTER(i32)]),
+        "slorr_set_timing": (i32, [vp, i32]),
+        "slorr_read_timing": (i32, [vp, ctypes.POINTER(dbl), ctypes.POINTER(i64), i32]),
+        "slorr_destroy": (None, [vp]),
+        "slorr_status_string": (ctypes.c_char_p, [i32]),
+        "slorr_last_error": (ctypes.c_char_p, []),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    if path is None:
+        _lib = lib
+    return lib
+
+
+def declared_symbols(header: str = HEADER) -> list[str]:
+    """Names of the functions include/slorr.h declares."""
+    text = open(header).read()
+    return sorted(set(re.findall(r"SLORR_API[^;(]*?\b(slorr_\w+)\s*\(", text)))
+
+
+def _check(status: int) -> None:
+    if status != SLORR_OK:
+        msg = load_library().slorr_last_error()
+        raise SlorrError(status, msg.decode() if msg else "")
+
+
+def _shapes(shapes) -> tuple[ctypes.Array, int]:
+    arr = (Shape * len(shapes))(*[Shape(int(m), int(n)) for m, n in shapes])
+    return arr, len(shapes)
+
+
+def _ptr_array(ptrs) -> ctypes.Array:
+    return (ctypes.c_void_p * len(ptrs))(*[ctypes.c_void_p(int(p)) for p in ptrs])
+
+
+# ---- functions with the C ABI's names ------------------------------------------
+
+def slorr_default_options() -> Options:
+    o = Options()
+    load_library().slorr_default_options(ctypes.byref(o))
+    return o
+
+
+def slorr_create(shapes, options: Options | None = None) -> ctypes.c_void_p:
+    arr, n = _shapes(shapes)
+    h = ctypes.c_void_p()
+    _check(load_library().slorr_create(ctypes.byref(h), arr, n,
+                                       ctypes.byref(options) if options is not None else None))
+    return h
+
+
+def slorr_workspace_size(handle) -> int:
+    out = ctypes.c_size_t()
+    _check(load_library().slorr_workspace_size(handle, ctypes.byref(out)))
+    return out.value
+
+
+def slorr_reg_forward_backward(handle, weight_ptrs, grad_ptrs, loss_ptr, per_matrix_ptr, workspace_ptr,
+                               workspace_bytes, stream) -> None:
+    _check(load_library().slorr_reg_forward_backward(
+        handle, _ptr_array(weight_ptrs), _ptr_array(grad_ptrs), ctypes.c_void_p(loss_ptr),
+        ctypes.c_void_p(per_matrix_ptr or 0), ctypes.c_void_p(workspace_ptr), workspace_bytes,
+        ctypes.c_void_p(stream or 0)))
+
+
+def slorr_reset_workspace(handle) -> None:
+    _check(load_library().slorr_reset_workspace(handle))
+
+
+def slorr_get_status(handle, workspace_ptr, stream) -> int:
+    """Returns the status code (does not raise for device-side errors)."""
+    return int(load_library().slorr_get_status(handle, ctypes.c_void_p(workspace_ptr),
+                                               ctypes.c_void_p(stream or 0)))
+
+
+def slorr_run_steps(handle, weight_ptrs, workspace_ptr, workspace_bytes, steps, stream) -> None:
+    _check(load_library().slorr_run_steps(handle, _ptr_array(weight_ptrs), ctypes.c_void_p(workspace_ptr),
+                                          workspace_bytes, int(steps), ctypes.c_void_p(stream or 0)))
+
+
+def slorr_iterate_view(handle, workspace_ptr, i, after_steps) -> MatrixView:
+    v = MatrixView()
+    _check(load_library().slorr_iterate_view(handle, ctypes.c_void_p(workspace_ptr), int(i),
+                                             int(after_steps), ctypes.byref(v)))
+    return v
+
+
+def slorr_get_coefficients(handle, iters: int) -> np.ndarray:
+    buf = (ctypes.c_double * (3 * iters))()
+    _check(load_library().slorr_get_coefficients(handle, buf, 3 * iters))
+    return np.array(buf, dtype=np.float64).reshape(iters, 3)
+
+
+def slorr_pe_coefficients(iters: int = 6, ell: float = 1e-3, cushion: float = -1.0,
+                          safety: float = 1.01) -> np.ndarray:
+    buf = (ctypes.c_double * (3 * iters))()
+    _check(load_library().slorr_pe_coefficients(int(iters), float(ell), float(cushion), float(safety), buf))
+    return np.array(buf, dtype=np.float64).reshape(iters, 3)
+
+
+def slorr_cushion_ratio() -> float:
+    return float(load_library().slorr_cushion_ratio())
+
+
+def slorr_flops(shapes, iters: int = 6) -> int:
+    arr, n = _shapes(shapes)
+    return int(load_library().slorr_flops(arr, n, int(iters)))
+
+
+def slorr_partition(shapes, world: int, rank: int) -> list[int]:
+    arr, n = _shapes(shapes)
+    out = (ctypes.c_int32 * max(n, 1))()
+    cnt = ctypes.c_int32()
+    _check(load_library().slorr_partition(arr, n, int(world), int(rank), out, ctypes.byref(cnt)))
+    return [int(out[i]) for i in range(cnt.value)]
+
+
+KERNEL_KINDS = ("sumsq", "cast", "gram", "poly", "update", "dot", "combine")
+
+
+def slorr_set_timing(handle, enable: bool) -> None:
+    _check(load_library().slorr_set_timing(handle, 1 if enable else 0))
+
+
+def slorr_read_timing(handle) -> dict:
+    """{kind: (milliseconds, launches)} accumulated since the last read."""
+    n = len(KERNEL_KINDS)
+    ms = (ctypes.c_double * n)()
+    cnt = (ctypes.c_int64 * n)()
+    _check(load_library().slorr_read_timing(handle, ms, cnt, n))
+    return {k: (float(ms[i]), int(cnt[i])) for i, k in enumerate(KERNEL_KINDS)}
+
+
+def slorr_destroy(handle) -> None:
+    load_library().slorr_destroy(handle)
+
+
+def slorr_status_string(status: int) -> str:
+    return load_library().slorr_status_string(int(status)).decode()
+
+
+# ---- torch-facing convenience ----------------------------------------------------
+
+class Regularizer:
+    """One planned weight set.  Holds the handle and a torch-allocated workspace.
+
+    ``reg(weights, grads)`` enqueues the forward value and gradient of every
+    matrix on the current CUDA stream, accumulating lambda * grad into
+    ``grads`` and returning the device loss tensor (lambda * sum_i L_i)."""
+
+    def __init__(self, shapes, variant: str = "hoyer", compute: str = "fp16", dtype: str = "f32",
+                 iters: int = 6, lam: float = 1.0, eps: float = 1e-7, grad_scale: float = 1.0,
+                 ell: float = 1e-3, cushion: float = -1.0, safety: float = 1.01, flags: int = 0,
+                 timeout_s: float = 2.0):
+        o = slorr_default_options()
+        o.variant = VARIANTS[variant]
+        o.compute = COMPUTES[compute]
+        o.dtype = DTYPES[dtype]
+        o.iters = int(iters)
+        o.lambda_ = float(lam)
+        o.eps = float(eps)
+        o.grad_scale = float(grad_scale)
+        o.ell = float(ell)
+        o.cushion = float(cushion)
+        o.safety = float(safety)
+        o.flags = int(flags)
+        o.timeout_s = float(timeout_s)
+        self.shapes = [(int(m), int(n)) for m, n in shapes]
+        self.iters = int(iters)
+        self.options = o
+        self.handle = slorr_create(self.shapes, o)
+        self.workspace_bytes = slorr_workspace_size(self.handle)
+        self._ws = None
+
+    def __del__(self):
+        h = getattr(self, "handle", None)
+        if h is not None and _lib is not None:
+            slorr_destroy(h)
+            self.handle = None
+
+    def workspace(self, device):
+        import torch
+        if self._ws is None or self._ws.device != torch.device(device):
+            self._ws = torch.empty(self.workspace_bytes + 256, dtype=torch.uint8, device=device)
+        base = self._ws.data_ptr()
+        return base + (-base) % 256
+
+    def coefficients(self) -> np.ndarray:
+        return slorr_get_coefficients(self.handle, self.iters)
+
+    def __call__(self, weights, grads, loss=None, per_matrix=None, stream=None):
+        import torch
+        dev = weights[0].device
+        ws = self.workspace(dev)
+        if loss is None:
+            loss = torch.empty(1, dtype=torch.float32, device=dev)
+        s = stream if stream is not None else torch.cuda.current_stream(dev).cuda_stream
+        slorr_reg_forward_backward(self.handle, [w.data_ptr() for w in weights], [g.data_ptr() for g in grads],
+                                   loss.data_ptr(), per_matrix.data_ptr() if per_matrix is not None else 0,
+                                   ws, self.workspace_bytes, s)
+        return loss
+
+    def run_steps(self, weights, steps: int, stream=None):
+        import torch
+        dev = weights[0].device
+        ws = self.workspace(dev)
+        s = stream if stream is not None else torch.cuda.current_stream(dev).cuda_stream
+        slorr_run_steps(self.handle, [w.data_ptr() for w in weights], ws, self.workspace_bytes, steps, s)
+
+    def iterate(self, i: int, after_steps: int):
+        """Copy of matrix i's iterate after `after_steps` steps as a P x Q fp32 tensor."""
+        import torch
+        dev = self._ws.device
+        v = slorr_iterate_view(self.handle, self.workspace(dev), i, after_steps)
+        typestr = {0: "<f4", 1: "<f2", 2: "<u2"}[v.elem]
+        raw = device_view(v.x, (v.rows, v.ld), typestr, dev).clone()
+        if v.elem == 2:
+            raw = raw.view(torch.bfloat16)
+        return raw[:, : v.cols].float()
+
+    def scalars(self, i: int):
+        """(||W_i||_F^2, n_hat_i) read back from the workspace."""
+        dev = self._ws.device
+        v = slorr_iterate_view(self.handle, self.workspace(dev), i, 0)
+        out = device_view(v.frob_sq, (2,), "<f8", dev).clone().cpu()
+        return float(out[0]), float(out[1])
+
+    def status(self, stream=None) -> int:
+        import torch
+        dev = self._ws.device
+        s = stream if stream is not None else torch.cuda.current_stream(dev).cuda_stream
+        return slorr_get_status(self.handle, self.workspace(dev), s)
+
+
+class _DeviceArray:
+    def __init__(self, ptr: int, shape, typestr: str):
+        self.__cuda_array_interface__ = {"shape": tuple(int(d) for d in shape), "typestr": typestr,
+                                         "data": (int(ptr), True), "version": 2, "strides": None}
+
+
+def device_view(ptr: int, shape, typestr: str, device):
+    """A torch tensor aliasing device memory at `ptr` (test introspection only)."""
+    import torch
+    return torch.as_tensor(_DeviceArray(ptr, shape, typestr), device=device)

@@ -1,0 +1,217 @@
+"""GPU parity: libslorr through its C ABI against the fp64 oracle on the same
+seeded inputs (Sec. 3, Eq. 1, Listing 1, Alg. 2).
+
+Tolerances (relative, on the loss and on each matrix's gradient in Frobenius
+norm):
+* fp32 compute mode: 1e-5;
+* fp16-operand mode (tensor cores, the default): 2e-2;
+* bf16-operand mode: 2e-2 on the loss, 5e-2 on the gradient.  bf16 keeps 8
+  significand bits against fp16's 11, and the measured fp16 gradient errors on
+  the paper-shaped sets stay below 4.5e-3, so 8 x that bound (3.6e-2) plus
+  margin gives 5e-2; the loss is a smooth trace and stays within 2e-2.
+"""
+
+import numpy as np
+import pytest
+
+import oracle
+import workloads
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+TOL = {"fp32": (1e-5, 1e-5), "fp16": (2e-2, 2e-2), "bf16": (2e-2, 5e-2)}
+EPS = 1e-7
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _need_gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2607_08754_gb300 import slorr
+    slorr.load_library()   # raises if the extension is missing: no fallback
+
+
+def run_gpu(Ws, variant="hoyer", compute="fp16", lam=1.0, grad_scale=1.0, dtype="f32", iters=6,
+            grads0=None, flags=0, reg=None):
+    from paper_2607_08754_gb300.slorr import Regularizer
+    if reg is None:
+        reg = Regularizer([W.shape for W in Ws], variant=variant, compute=compute, dtype=dtype,
+                          iters=iters, lam=lam, grad_scale=grad_scale, flags=flags)
+    tdt = torch.float32 if dtype == "f32" else torch.bfloat16
+    w = [torch.from_numpy(np.ascontiguousarray(W, dtype=np.float32)).to("cuda").to(tdt) for W in Ws]
+    if grads0 is None:
+        g = [torch.zeros_like(x) for x in w]
+    else:
+        g = [torch.from_numpy(np.ascontiguousarray(G, dtype=np.float32)).to("cuda").to(tdt) for G in grads0]
+    per = torch.full((len(Ws),), float("nan"), device="cuda")
+    loss = reg(w, g, per_matrix=per)
+    torch.cuda.synchronize()
+    status = reg.status()
+    return (loss.item(), per.cpu().double().numpy(), [x.double().cpu().numpy() for x in g], status, reg,
+            [x.double().cpu().numpy() for x in w])
+
+
+def rel(a, b):
+    nb = np.linalg.norm(b)
+    return np.linalg.norm(a - b) / nb if nb > 0 else np.linalg.norm(a - b)
+
+
+def check(Ws, variant, compute, lam=1.0, grad_scale=1.0, dtype="f32", iters=6, grads0=None, flags=0):
+    loss, per, grads, status, reg, w_used = run_gpu(Ws, variant, compute, lam, grad_scale, dtype, iters,
+                                                    grads0, flags)
+    assert status == 0
+    co = oracle.pe_coefficients(T=iters)
+    ref_loss, ref_per, ref_inc = oracle.reg_forward_backward(w_used, variant, co, lam, EPS, grad_scale)
+    tl, tg = TOL[compute]
+    assert abs(loss - ref_loss) <= tl * abs(ref_loss) + 1e-6, (loss, ref_loss)
+    for i in range(len(Ws)):
+        assert abs(per[i] - ref_per[i]) <= tl * abs(ref_per[i]) + 1e-6, (i, per[i], ref_per[i])
+        base = grads0[i] if grads0 is not None else 0.0
+        ref_g = base + ref_inc[i]
+        if dtype == "bf16":
+            # the accumulated gradient is stored in bf16: one extra rounding
+            assert rel(grads[i] - base, ref_inc[i]) <= tg + 8e-3, i
+        else:
+            assert rel(grads[i] - base, ref_inc[i]) <= tg, (i, rel(grads[i] - base, ref_inc[i]))
+            assert np.all(np.isfinite(grads[i])) and grads[i].shape == ref_g.shape
+    return loss, per, grads, reg
+
+
+# ---- cfg1: 8 x 256 x 256, N(0, 1/256), fp32 mode --------------------------------
+
+def test_cfg1_fp32_hoyer():
+    Ws = workloads.generate("cfg1")
+    check(Ws, "hoyer", "fp32")
+
+
+def test_cfg1_fp32_iterates_match_every_step():
+    from paper_2607_08754_gb300.slorr import Regularizer
+    Ws = workloads.generate("cfg1", [0, 1])
+    reg = Regularizer([W.shape for W in Ws], compute="fp32")
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    co = oracle.pe_coefficients(6)
+    for k in range(7):
+        reg.run_steps(w, k)
+        torch.cuda.synchronize()
+        for i, W in enumerate(Ws):
+            ref_steps, tr = oracle.polar_express_steps(W.astype(np.float64), co, EPS)
+            got = reg.iterate(i, k).double().cpu().numpy()
+            assert rel(got, ref_steps[k]) <= 1e-5, (k, i, rel(got, ref_steps[k]))
+        fsq, _ = reg.scalars(0)
+        assert fsq == pytest.approx(float(np.sum(Ws[0].astype(np.float64) ** 2)), rel=1e-6)
+
+
+@pytest.mark.parametrize("compute", ["fp32", "fp16", "bf16"])
+@pytest.mark.parametrize("variant", ["hoyer", "nuclear"])
+def test_ragged_shapes(compute, variant):
+    shapes = [(1, 1), (1, 7), (9, 1), (3, 5), (5, 3), (64, 147), (130, 70), (200, 333), (320, 1280),
+              (1000, 512), (129, 129)]
+    Ws = [workloads.random_matrix(s, seed=10 + i, std=0.05) for i, s in enumerate(shapes)]
+    check(Ws, variant, compute, lam=0.7, grad_scale=2.0)
+
+
+@pytest.mark.parametrize("compute", ["fp16", "bf16"])
+@pytest.mark.parametrize("variant", ["hoyer", "nuclear"])
+def test_resnet18_weight_set(compute, variant):
+    check(workloads.generate("resnet18"), variant, compute)
+
+
+def test_vit_b16_block_fp16():
+    check(workloads.generate("vit_b16", range(4)), "hoyer", "fp16")
+
+
+def test_decoder_560m_layer_fp16():
+    check(workloads.generate("decoder_560m", range(7)), "hoyer", "fp16")
+
+
+# ---- tensor cores vs CUDA cores on the same 16-bit arithmetic -------------------
+
+@pytest.mark.parametrize("compute", ["fp16", "bf16"])
+def test_tensor_core_iterates_match_simt(compute):
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_SIMT_GEMM
+    shapes = [(256, 768), (768, 256), (320, 1280), (384, 384)]
+    Ws = [workloads.random_matrix(s, seed=70 + i, std=0.02) for i, s in enumerate(shapes)]
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    tc = Regularizer(shapes, compute=compute)
+    st = Regularizer(shapes, compute=compute, flags=FLAG_SIMT_GEMM)
+    ulp = 2.0 ** -10 if compute == "fp16" else 2.0 ** -7
+    for k in (1, 2, 6):
+        tc.run_steps(w, k)
+        st.run_steps(w, k)
+        torch.cuda.synchronize()
+        assert tc.status() == 0 and st.status() == 0
+        for i in range(len(shapes)):
+            a = tc.iterate(i, k).double().cpu().numpy()
+            b = st.iterate(i, k).double().cpu().numpy()
+            assert rel(a, b) <= 4 * ulp * (k if k < 6 else 6), (k, i, rel(a, b))
+
+
+# ---- edge cases -------------------------------------------------------------------
+
+@pytest.mark.parametrize("compute", ["fp32", "fp16"])
+def test_zero_matrix_and_accumulation(compute):
+    Ws = [np.zeros((40, 70), np.float32), workloads.random_matrix((70, 40), 3, 0.1)]
+    rng = np.random.default_rng(4)
+    g0 = [rng.normal(size=W.shape).astype(np.float32) for W in Ws]
+    loss, per, grads, reg = check(Ws, "hoyer", compute, grads0=g0)
+    assert per[0] == 0.0
+    assert np.array_equal(grads[0], g0[0].astype(np.float64))   # zero matrix: gradient 0, grad untouched
+
+
+def test_two_calls_reuse_workspace_and_accumulate():
+    from paper_2607_08754_gb300.slorr import Regularizer
+    Ws = [workloads.random_matrix((96, 200), 5, 0.05), workloads.random_matrix((300, 64), 6, 0.05)]
+    reg = Regularizer([W.shape for W in Ws], lam=0.5)
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    g = [torch.zeros_like(x) for x in w]
+    l1 = reg(w, g).item()
+    once = [x.clone() for x in g]
+    l2 = reg(w, g).item()
+    torch.cuda.synchronize()
+    assert reg.status() == 0
+    assert l1 == l2                                    # deterministic
+    for a, b in zip(g, once):
+        assert torch.equal(a, 2 * b) or torch.allclose(a, 2 * b, rtol=1e-6, atol=0)
+
+
+def test_bf16_weights_and_grads():
+    Ws = [workloads.random_matrix((128, 300), 8, 0.05), workloads.random_matrix((257, 100), 9, 0.05)]
+    check(Ws, "hoyer", "fp16", dtype="bf16")
+
+
+def test_nonfinite_weight_reports_status_and_leaves_grad():
+    from paper_2607_08754_gb300.slorr import Regularizer
+    W = workloads.random_matrix((64, 64), 11, 0.1)
+    W[3, 5] = np.inf
+    reg = Regularizer([W.shape, (32, 32)])
+    w = [torch.from_numpy(W).cuda(), torch.from_numpy(workloads.random_matrix((32, 32), 12)).cuda()]
+    g = [torch.ones_like(x) for x in w]
+    reg(w, g)
+    torch.cuda.synchronize()
+    assert reg.status() == 6            # SLORR_ERR_NONFINITE
+    assert torch.all(g[0] == 1.0)       # untouched
+    assert reg.status() == 0            # reading clears it
+
+
+# ---- full-size ViT-L/16 weight set in the benchmark configuration, sampled --------
+
+def test_vit_l16_full_size_sampled():
+    from paper_2607_08754_gb300.slorr import Regularizer
+    name = "vit_l16"
+    shapes = workloads.shapes(name)
+    reg = Regularizer(shapes, compute="fp16", lam=1.0)
+    w = [torch.from_numpy(workloads.generate_one(name, i)).cuda() for i in range(len(shapes))]
+    g = [torch.zeros_like(x) for x in w]
+    per = torch.empty(len(shapes), device="cuda")
+    loss = reg(w, g, per_matrix=per).item()
+    torch.cuda.synchronize()
+    assert reg.status() == 0
+    per = per.double().cpu().numpy()
+    assert loss == pytest.approx(per.sum(), rel=1e-6)
+    co = oracle.pe_coefficients(6)
+    for i in (0, 1, 2, 3, 94):
+        W = workloads.generate_one(name, i).astype(np.float64)
+        L, G, _, _ = oracle.reg_single(W, "hoyer", co, EPS)
+        assert abs(per[i] - L) <= 2e-2 * L
+        assert rel(g[i].double().cpu().numpy(), G) <= 2e-2

@@ -1,0 +1,169 @@
+"""Host-side checks of libslorr (no GPU): the library loads and exports every
+symbol include/slorr.h declares, its Polar Express schedule agrees with the
+oracle's independently written generator, argument validation rejects bad
+requests before any CUDA call, and the App. F layer partition reproduces the
+single-rank gradient under a 2-rank gloo all-reduce."""
+
+import os
+import socket
+
+import numpy as np
+import pytest
+
+import oracle
+import workloads
+
+slorr = pytest.importorskip("paper_2607_08754_gb300.slorr")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    try:
+        return slorr.load_library()
+    except ImportError as e:  # pragma: no cover - the build step makes it
+        pytest.fail(str(e))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = slorr.declared_symbols()
+    assert len(names) >= 16
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+@pytest.mark.parametrize("T", [1, 2, 4, 6, 8, 10])
+def test_schedule_matches_oracle(lib, T):
+    got = slorr.slorr_pe_coefficients(T)
+    ref = oracle.pe_coefficients(T=T)
+    assert np.allclose(got, ref, rtol=1e-9, atol=1e-12)
+
+
+@pytest.mark.parametrize("cushion,safety", [(0.0, 1.0), (0.0, 1.01), (-1.0, 1.0), (0.05, 1.02)])
+def test_schedule_options_match_oracle(lib, cushion, safety):
+    got = slorr.slorr_pe_coefficients(6, 1e-3, cushion, safety)
+    ref = oracle.pe_coefficients(T=6, cushion=None if cushion < 0 else cushion, safety=safety)
+    assert np.allclose(got, ref, rtol=1e-10)
+
+
+def test_cushion_ratio(lib):
+    assert slorr.slorr_cushion_ratio() == pytest.approx(oracle.cushion_ratio(), rel=1e-12)
+
+
+def test_handle_coefficients_and_flops(lib):
+    shapes = workloads.shapes("vit_l16")
+    r = slorr.Regularizer(shapes)
+    assert np.allclose(r.coefficients(), oracle.pe_coefficients(6), rtol=1e-9)
+    assert slorr.slorr_flops(shapes, 6) == oracle.weight_set_flops(shapes, 6)
+    # ViT-L/16: 8659 GFLOP per step at T = 6 (paper's count, Sec. 3)
+    assert slorr.slorr_flops(shapes, 6) / 1e9 == pytest.approx(8659.0, rel=1e-3)
+
+
+def test_validation_rejects_bad_requests(lib):
+    with pytest.raises(slorr.SlorrError) as e:
+        slorr.slorr_create([(0, 3)])
+    assert e.value.status == 1
+    with pytest.raises(slorr.SlorrError):
+        slorr.slorr_create([(3, 70000)])
+    for field, bad in [("iters", 0), ("iters", 17), ("ell", 0.0), ("ell", 1.0), ("safety", 0.5),
+                       ("eps", -1.0), ("variant", 5), ("compute", 9), ("dtype", 3), ("timeout_s", 0.0)]:
+        o = slorr.slorr_default_options()
+        setattr(o, field, bad)
+        with pytest.raises(slorr.SlorrError) as e:
+            slorr.slorr_create([(4, 4)], o)
+        assert e.value.status == 1, field
+    h = slorr.slorr_create([(4, 4)])
+    ws = slorr.slorr_workspace_size(h)
+    # NULL / misaligned pointers and a short workspace are rejected before any launch
+    with pytest.raises(slorr.SlorrError) as e:
+        slorr.slorr_reg_forward_backward(h, [0], [256], 512, 0, 1024, ws, 0)
+    assert e.value.status == 1
+    with pytest.raises(slorr.SlorrError) as e:
+        slorr.slorr_reg_forward_backward(h, [8], [256], 512, 0, 1024, ws, 0)
+    assert e.value.status == 1
+    with pytest.raises(slorr.SlorrError) as e:
+        slorr.slorr_reg_forward_backward(h, [256], [256], 512, 0, 1024, ws, 0)
+    assert e.value.status == 1       # grad aliases weight
+    with pytest.raises(slorr.SlorrError) as e:
+        slorr.slorr_reg_forward_backward(h, [256], [512], 768, 0, 1024, ws - 1, 0)
+    assert e.value.status == 4
+    with pytest.raises(slorr.SlorrError) as e:
+        slorr.slorr_reg_forward_backward(h, [256], [512], 768, 0, 1030, ws, 0)
+    assert e.value.status == 4       # misaligned workspace
+    slorr.slorr_destroy(h)
+
+
+def test_workspace_size_grows_with_the_set(lib):
+    small = slorr.Regularizer([(64, 64)]).workspace_bytes
+    big = slorr.Regularizer([(64, 64), (1000, 512)]).workspace_bytes
+    fp32 = slorr.Regularizer([(64, 64), (1000, 512)], compute="fp32").workspace_bytes
+    assert small < big < fp32
+    # X0, X1 (Ppad x Qpad) and A, B (Ppad x Ppad) of 1000x512 in fp16 alone:
+    assert big - small >= 2 * (512 * 1024 * 2) + 2 * (512 * 512 * 2)
+
+
+def test_partition_is_a_balanced_cover(lib):
+    shapes = workloads.shapes("decoder_560m")
+    for world in (1, 2, 3, 8):
+        parts = [slorr.slorr_partition(shapes, world, r) for r in range(world)]
+        flat = sorted(i for p in parts for i in p)
+        assert flat == list(range(len(shapes)))
+        loads = [sum(oracle.pe_flops(*shapes[i]) for i in p) for p in parts]
+        assert max(loads) <= min(loads) + max(oracle.pe_flops(*s) for s in shapes)
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def _partition_worker(rank, world, port, shapes, q):
+    import torch
+    import torch.distributed as dist
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    from paper_2607_08754_gb300 import slorr as sl
+    mine = sl.slorr_partition(shapes, world, rank)
+    co = oracle.pe_coefficients(6)
+    Ws = [np.random.default_rng(50 + i).normal(size=s) for i, s in enumerate(shapes)]
+    grads = [torch.zeros(s, dtype=torch.float64) for s in shapes]
+    loss = torch.zeros(1, dtype=torch.float64)
+    sub = [Ws[i] for i in mine]
+    l, _, incs = oracle.reg_forward_backward(sub, "hoyer", co, lam=0.3, grad_scale=float(world))
+    for i, g in zip(mine, incs):
+        grads[i] += torch.from_numpy(g)
+    loss += l
+    for g in grads:                      # the data-parallel gradient average
+        dist.all_reduce(g)
+        g /= world
+    dist.all_reduce(loss)                # logged loss: plain sum
+    if rank == 0:
+        q.put((loss.item(), [g.numpy() for g in grads]))
+    dist.barrier()
+    dist.destroy_process_group()
+
+
+def test_layer_partition_two_ranks_gloo(lib):
+    """App. F: each rank regularizes its layers with grad_scale = world; the
+    data-parallel average then equals the single-rank gradient."""
+    import torch.multiprocessing as mp
+    shapes = [(6, 9), (12, 5), (7, 7), (3, 11), (10, 4)]
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_partition_worker, args=(r, 2, port, shapes, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    loss, grads = q.get(timeout=120)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    co = oracle.pe_coefficients(6)
+    Ws = [np.random.default_rng(50 + i).normal(size=s) for i, s in enumerate(shapes)]
+    ref_loss, _, ref = oracle.reg_forward_backward(Ws, "hoyer", co, lam=0.3)
+    assert loss == pytest.approx(ref_loss, rel=1e-12)
+    for g, r in zip(grads, ref):
+        assert np.allclose(g, r, rtol=1e-12, atol=1e-15)
