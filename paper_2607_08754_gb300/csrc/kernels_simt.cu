@@ -1,9 +1,18 @@
 // Grouped SIMT (CUDA-core) GEMM for the three phases of a Polar Express step
 // (Sec. 3 "Computational cost": A = X X^T, B = b A + c A^2, X <- a X + B X on
-// the P x Q Gram side).  Used for the fp32 compute mode, whose operands and
-// accumulation are fp32, and, with 16-bit storage, as a CUDA-core check of the
-// tensor-core kernel.  64 x 64 output tile per block, 256 threads, 4 x 4 per
-// thread, K staged 16 at a time through shared memory.
+// the P x Q Gram side).  Used for the fp32 compute mode and, with 16-bit
+// storage, as a CUDA-core check of the tensor-core kernel.  64 x 64 output
+// tile per block, 256 threads, 4 x 4 per thread, K staged 16 at a time through
+// shared memory.
+//
+// In fp32 mode the dot products are compensated (Ogita-Rump-Oishi "Dot2":
+// each product is split exactly with an FMA, each addition with Knuth's
+// two-sum, and the error terms are summed separately), so a result is as
+// accurate as if it had been accumulated in twice the working precision and
+// only the fp32 storage of X, A and B rounds.  Plain fp32 accumulation of the
+// K <= 4608 long sums loses up to ~1e-5 on the Hoyer gradient of wide,
+// near-full-rank matrices; the compensated sums stay near 4e-7.  The 16-bit
+// check path keeps plain fp32 FMA accumulation, like the tensor cores.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -55,7 +64,9 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const GemmLaunch p) {
     }
     const int m0 = it.tm * kBM, n0 = it.tn * kBN;
     const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
+    constexpr bool kDot2 = sizeof(T) == 4;
     float acc[4][4] = {};
+    float cmp[4][4] = {};
     for (int k0 = 0; k0 < K; k0 += kBK) {
         // 64 x 16 of each operand: 1024 values, 4 per thread.
         for (int e = threadIdx.x; e < kBM * kBK; e += 256) {
@@ -78,7 +89,19 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const GemmLaunch p) {
 #pragma unroll
             for (int u = 0; u < 4; ++u)
 #pragma unroll
-                for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(a[u], b[v], acc[u][v]);
+                for (int v = 0; v < 4; ++v) {
+                    if constexpr (kDot2) {
+                        const float pr = a[u] * b[v];
+                        const float pe = fmaf(a[u], b[v], -pr);   // a b = pr + pe exactly
+                        const float s = acc[u][v] + pr;
+                        const float z = s - acc[u][v];
+                        const float se = (acc[u][v] - (s - z)) + (pr - z);  // two-sum error
+                        acc[u][v] = s;
+                        cmp[u][v] += pe + se;
+                    } else {
+                        acc[u][v] = fmaf(a[u], b[v], acc[u][v]);
+                    }
+                }
         }
         __syncthreads();
     }
@@ -98,7 +121,7 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const GemmLaunch p) {
 #pragma unroll
         for (int v = 0; v < 4; ++v) {
             const int64_t idx = static_cast<int64_t>(m0 + ty * 4 + u) * ldo + (n0 + tx * 4 + v);
-            float val = cacc * acc[u][v];
+            float val = cacc * (acc[u][v] + cmp[u][v]);
             if (extra) val = fmaf(ce, ld_f<T>(extra + idx), val);
             st_f<T>(out + idx, val);
         }

@@ -317,7 +317,7 @@ class Regularizer:
 class _DeviceArray:
     def __init__(self, ptr: int, shape, typestr: str):
         self.__cuda_array_interface__ = {"shape": tuple(int(d) for d in shape), "typestr": typestr,
-                                         "data": (int(ptr), True), "version": 2, "strides": None}
+                                         "data": (int(ptr), False), "version": 2, "strides": None}
 
 
 def device_view(ptr: int, shape, typestr: str, device):

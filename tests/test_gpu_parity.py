@@ -9,6 +9,12 @@ norm):
   significand bits against fp16's 11, and the measured fp16 gradient errors on
   the paper-shaped sets stay below 4.5e-3, so 8 x that bound (3.6e-2) plus
   margin gives 5e-2; the loss is a smooth trace and stays within 2e-2.
+
+The Hoyer gradient is the difference of two terms, 2 reg P_hat / frob and
+2 reg n_hat W / frob^3 (Listing 1).  When they cancel almost completely (rank
+one, equal singular values: the exact gradient is zero) a relative error only
+measures rounding of that cancellation, so for matrices whose gradient norm is
+below 5% of the first term's norm the error is taken relative to that term.
 """
 
 import numpy as np
@@ -57,6 +63,19 @@ def rel(a, b):
     return np.linalg.norm(a - b) / nb if nb > 0 else np.linalg.norm(a - b)
 
 
+def grad_err(got, ref, W, variant, lam, grad_scale):
+    """Relative gradient error, against the first term's scale when the
+    Hoyer terms cancel (see the module docstring)."""
+    nr = np.linalg.norm(ref)
+    if variant == "hoyer":
+        co = oracle.pe_coefficients(6)
+        L, _, n_hat, frob = oracle.reg_single(W, "hoyer", co, EPS)
+        term = abs(lam * grad_scale) * 2.0 * (n_hat / frob) / frob * np.sqrt(min(W.shape))
+        if nr < 0.05 * term:
+            return np.linalg.norm(got - ref) / term
+    return np.linalg.norm(got - ref) / nr if nr > 0 else np.linalg.norm(got - ref)
+
+
 def check(Ws, variant, compute, lam=1.0, grad_scale=1.0, dtype="f32", iters=6, grads0=None, flags=0):
     loss, per, grads, status, reg, w_used = run_gpu(Ws, variant, compute, lam, grad_scale, dtype, iters,
                                                     grads0, flags)
@@ -69,11 +88,12 @@ def check(Ws, variant, compute, lam=1.0, grad_scale=1.0, dtype="f32", iters=6, g
         assert abs(per[i] - ref_per[i]) <= tl * abs(ref_per[i]) + 1e-6, (i, per[i], ref_per[i])
         base = grads0[i] if grads0 is not None else 0.0
         ref_g = base + ref_inc[i]
+        err = grad_err(grads[i] - base, ref_inc[i], w_used[i], variant, lam, grad_scale)
         if dtype == "bf16":
             # the accumulated gradient is stored in bf16: one extra rounding
-            assert rel(grads[i] - base, ref_inc[i]) <= tg + 8e-3, i
+            assert err <= tg + 8e-3, (i, err)
         else:
-            assert rel(grads[i] - base, ref_inc[i]) <= tg, (i, rel(grads[i] - base, ref_inc[i]))
+            assert err <= tg, (i, err)
             assert np.all(np.isfinite(grads[i])) and grads[i].shape == ref_g.shape
     return loss, per, grads, reg
 
