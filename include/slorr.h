@@ -144,10 +144,12 @@ SLORR_API slorr_status slorr_get_status(slorr_handle* h, const void* workspace, 
 SLORR_API slorr_status slorr_run_steps(slorr_handle* h, const void* const* weights, void* workspace,
                              size_t workspace_bytes, int32_t steps, void* stream);
 
-/* Where matrix i's current iterate lives inside `workspace`: a P x Q row-major
- * array (P = min(m,n), Q = max(m,n); the iterate is W^T-shaped when m > n) of
- * element type elem (0 fp32, 1 fp16, 2 bf16) with leading dimension ld >= Q.
- * Also returns device pointers to ||W_i||_F^2 (double) and n_hat_i (double). */
+/* Where matrix i's iterate after `after_steps` steps lives inside `workspace`:
+ * an array in W's orientation -- rows x cols = m x n, row-major with leading
+ * dimension ld >= n -- of element type elem (0 fp32, 1 fp16, 2 bf16).  The
+ * Polar Express iterate X (P x Q, P = min(m,n)) is this array when m <= n and
+ * its transpose when m > n (transposed = 1).  Also returns device pointers to
+ * ||W_i||_F^2 (double) and n_hat_i (double). */
 typedef struct slorr_matrix_view {
     const void*   x;
     int64_t       rows, cols, ld;

@@ -37,7 +37,7 @@ slorr_status cuda_fail(cudaError_t e, const char* what) {
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct Geom {
-    int m, n, P, Q, Ppad, Qpad, transposed;
+    int m, n, P, Q, Ppad, Qpad, transposed, rows, ld;
     size_t off_x[2], off_a, off_b;
     int tile_base, tile_count;
 };
@@ -114,7 +114,10 @@ void build_plan(slorr_handle* h) {
         g.Q = std::max(g.m, g.n);
         g.Ppad = int(align_up(size_t(g.P), kPadRows));
         g.Qpad = int(align_up(size_t(g.Q), kPadCols));
-        const int tr = (g.m + 63) / 64, tc = (g.n + 63) / 64;
+        // iterate buffer in W's orientation
+        g.rows = g.transposed ? g.Qpad : g.Ppad;
+        g.ld = g.transposed ? g.Ppad : g.Qpad;
+        const int tr = (g.m + kMemRows - 1) / kMemRows, tc = (g.n + kMemCols - 1) / kMemCols;
         g.tile_base = tile_base;
         g.tile_count = tr * tc;
         int seq = 0;
@@ -122,8 +125,8 @@ void build_plan(slorr_handle* h) {
             for (int c = 0; c < tc; ++c)
                 h->w_items.push_back(MemItem{uint16_t(i), uint16_t(r), uint16_t(c), uint16_t(seq++)});
         tile_base += g.tile_count;
-        for (int r = 0; r < g.Ppad / 64; ++r)
-            for (int c = 0; c < g.Qpad / 64; ++c)
+        for (int r = 0; r < (g.rows + kMemRows - 1) / kMemRows; ++r)
+            for (int c = 0; c < (g.ld + kMemCols - 1) / kMemCols; ++c)
                 h->x_items.push_back(MemItem{uint16_t(i), uint16_t(r), uint16_t(c), 0});
         // tensor-core tiles: 128 x nsz, nsz <= 256
         for (int ph = 0; ph < 3; ++ph) {
@@ -181,7 +184,7 @@ void build_plan(slorr_handle* h) {
     h->off_plan_end = off;
     for (int i = 0; i < count; ++i) {
         Geom& g = h->geom[i];
-        const size_t xbytes = size_t(g.Ppad) * g.Qpad * h->esize;
+        const size_t xbytes = size_t(g.rows) * g.ld * h->esize;
         const size_t pbytes = size_t(g.Ppad) * g.Ppad * h->esize;
         g.off_x[0] = off;
         off = align_up(off + xbytes, 1024);
@@ -258,11 +261,13 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
         md.Ppad = g.Ppad;
         md.Qpad = g.Qpad;
         md.transposed = g.transposed;
+        md.rows = g.rows;
+        md.ld = g.ld;
         md.pad_ = 0;
         if (tc) {
             const bool bf = h->opt.compute == SLORR_COMPUTE_BF16;
             CUtensorMap* mp = reinterpret_cast<CUtensorMap*>(maps.data() + size_t(i) * 4 * 128);
-            if (!encode_map(mp + 0, md.x[0], g.Ppad, g.Qpad, bf) || !encode_map(mp + 1, md.x[1], g.Ppad, g.Qpad, bf) ||
+            if (!encode_map(mp + 0, md.x[0], g.rows, g.ld, bf) || !encode_map(mp + 1, md.x[1], g.rows, g.ld, bf) ||
                 !encode_map(mp + 2, md.a, g.Ppad, g.Ppad, bf) || !encode_map(mp + 3, md.b, g.Ppad, g.Ppad, bf))
                 return fail(SLORR_ERR_CUDA, "cuTensorMapEncodeTiled failed");
         }
@@ -560,9 +565,9 @@ slorr_status slorr_iterate_view(const slorr_handle* h, const void* workspace, in
     const Geom& g = h->geom[i];
     const uint8_t* ws = static_cast<const uint8_t*>(workspace);
     out->x = ws + g.off_x[after_steps & 1];
-    out->rows = g.P;
-    out->cols = g.Q;
-    out->ld = g.Qpad;
+    out->rows = g.m;
+    out->cols = g.n;
+    out->ld = g.ld;
     out->elem = h->elem;
     out->transposed = g.transposed;
     const MatScalars* sc = reinterpret_cast<const MatScalars*>(ws + h->off_scalars) + i;

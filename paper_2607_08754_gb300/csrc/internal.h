@@ -2,10 +2,14 @@
 //
 // Device-side plan: for each weight matrix W_i (m x n) the Polar Express
 // iterate X is P x Q with P = min(m, n), Q = max(m, n) (Sec. 3 "Computational
-// cost": the Gram matrix is formed on the min side), stored row-major and
-// zero-padded to Ppad x Qpad (Ppad a multiple of 128, Qpad a multiple of 64).
-// Zero padding is exact: zero rows/columns of X give zero rows/columns of
-// A = X X^T and B = b A + c A^2, and the odd polynomial maps zero to zero
+// cost": the Gram matrix is formed on the min side).  It is stored in W's own
+// orientation -- row-major [m][n], i.e. as X^T when m > n -- so that the norm,
+// cast, dot and gradient passes are elementwise; the tensor-core kernel reads
+// it as a K-major or MN-major operand as each phase needs.  Both dimensions
+// are zero-padded: P to Ppad (a multiple of 128) and Q to Qpad (a multiple of
+// 64).  Zero padding is exact: zero rows/columns of X give zero rows/columns
+// of A = X X^T; M = a I + b A + c A^2 is a I on the padded block, which only
+// ever multiplies zero rows of X; and the odd polynomial maps zero to zero
 // (App. B, "zero singular values stay zero").
 #pragma once
 
@@ -29,13 +33,15 @@ enum StatusBits : uint32_t { kStatusTimeout = 1u, kStatusNonFinite = 2u };
 
 // Per-matrix device descriptor (lives in the workspace).
 struct MatDev {
-    void* x[2];        // ping-pong iterate buffers, Ppad x Qpad
+    void* x[2];        // ping-pong iterate buffers, rows x ld in W's orientation
     void* a;           // A = X X^T, Ppad x Ppad
-    void* b;           // B = b A + c A^2, Ppad x Ppad
+    void* b;           // M = a I + b A + c A^2, Ppad x Ppad
     int32_t m, n;      // shape of W
     int32_t P, Q;      // min / max
     int32_t Ppad, Qpad;
-    int32_t transposed;  // 1 when m > n (X = W^T)
+    int32_t transposed;  // 1 when m > n: the buffer holds X^T (Qpad x Ppad)
+    int32_t rows;      // buffer rows: Ppad, or Qpad when transposed
+    int32_t ld;        // buffer row length: Qpad, or Ppad when transposed
     int32_t pad_;
 };
 
@@ -53,15 +59,19 @@ struct GemmItem {
     uint16_t nsz;      // columns in this tile
 };
 
-// One chunk of a memory-bound pass over a weight matrix: a 2-D tile of W.
+// One chunk of a memory-bound pass: a kMemRows x kMemCols tile of W (or of
+// the padded iterate buffer for the cast).
+constexpr int kMemRows = 16;
+constexpr int kMemCols = 512;
 struct MemItem {
     uint16_t mat;
-    uint16_t tile_r;   // tile row index over W (64 rows)
-    uint16_t tile_c;   // tile column index over W (64 cols)
+    uint16_t tile_r;   // tile row index (kMemRows rows)
+    uint16_t tile_c;   // tile column index (kMemCols cols)
     uint16_t seq;      // index of this tile within its matrix
 };
 
-// Phases of one Polar Express step.
+// Phases of one Polar Express step (the step's polynomial is applied as
+// X <- M X with M = a I + b A + c A^2, the same product as a X + (b A + c A^2) X).
 enum Phase : int32_t { kGram = 0, kPoly = 1, kUpdate = 2 };
 
 struct GemmLaunch {

@@ -1,13 +1,16 @@
 // Memory-bound passes of the SLORR hot path, grouped over all weight matrices:
 //   sumsq   ||W_i||_F^2                                  (Listing 1, frob)
-//   cast    X_0 = W_i / (||W_i||_F + eps), Gram-side orientation, zero padded
-//                                                        (Sec. 3 "Computing the polar factor")
+//   cast    X_0 = W_i / (||W_i||_F + eps), zero padded    (Sec. 3 "Computing the polar factor")
 //   dot     n_hat_i = sum(W_i * P_hat_i), values L_i and the loss
 //                                                        (Sec. 3 "Computing the nuclear ...", Listing 1)
 //   combine W_i.grad += lambda * grad_scale * G_i       (Listing 1 backward, Alg. 2)
-// Each block handles one 64 x 64 tile.  Cross-tile sums are deterministic: a
-// block writes its partial, the last block of a matrix (per-matrix counter)
-// adds the partials in index order in double precision.
+// The iterates are stored in W's orientation (row-major, row length `ld`), so
+// every pass is elementwise.  A block handles one kMemRows x kMemCols tile:
+// each of its 256 threads owns 4 consecutive columns of 8 rows and issues all
+// eight 128-bit loads before using them (64-bit for 16-bit data).  Rows whose
+// length is not a multiple of 4 take a scalar path.  Cross-tile sums are
+// deterministic: each block writes a partial; the last block of a matrix (per-
+// matrix counter) adds the partials in index order in double precision.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -16,27 +19,99 @@
 namespace slorr {
 namespace {
 
-constexpr int kTile = 64;
 constexpr int kThreads = 256;
-constexpr int kRowsPerPass = kThreads / kTile;  // 4
+constexpr int kVecPerRow = kMemCols / 4;             // 128 threads per tile row
+constexpr int kRowsPerPass = kThreads / kVecPerRow;  // 2
+constexpr int kPasses = kMemRows / kRowsPerPass;     // 8
 
-template <typename T>
-__device__ __forceinline__ float to_f(T v);
-template <>
-__device__ __forceinline__ float to_f<float>(float v) { return v; }
-template <>
-__device__ __forceinline__ float to_f<__half>(__half v) { return __half2float(v); }
-template <>
-__device__ __forceinline__ float to_f<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
+__device__ __forceinline__ float bf2f(uint16_t u) { return __uint_as_float(uint32_t(u) << 16); }
 
-template <typename T>
-__device__ __forceinline__ T from_f(float v);
-template <>
-__device__ __forceinline__ float from_f<float>(float v) { return v; }
-template <>
-__device__ __forceinline__ __half from_f<__half>(float v) { return __float2half_rn(v); }
-template <>
-__device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
+// ---- 4-element loads and stores ------------------------------------------------
+
+// W (fp32 or bf16) elements (r, c .. c+3) of an m x n row-major matrix, zero
+// outside.  vec: n % 4 == 0, so the four are either all inside or all outside.
+template <typename TW>
+__device__ __forceinline__ float4 load_w4(const TW* W, int m, int n, int r, int c, bool vec) {
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (r >= m || c >= n) return v;
+    const int64_t idx = int64_t(r) * n + c;
+    if (vec) {
+        if constexpr (sizeof(TW) == 4) {
+            v = *reinterpret_cast<const float4*>(W + idx);
+        } else {
+            const uint2 u = *reinterpret_cast<const uint2*>(W + idx);
+            v = make_float4(bf2f(u.x & 0xffff), bf2f(u.x >> 16), bf2f(u.y & 0xffff), bf2f(u.y >> 16));
+        }
+    } else {
+        float t[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int e = 0; e < 4 && c + e < n; ++e) {
+            if constexpr (sizeof(TW) == 4)
+                t[e] = reinterpret_cast<const float*>(W)[idx + e];
+            else
+                t[e] = bf2f(reinterpret_cast<const uint16_t*>(W)[idx + e]);
+        }
+        v = make_float4(t[0], t[1], t[2], t[3]);
+    }
+    return v;
+}
+
+template <typename TW>
+__device__ __forceinline__ void store_w4(TW* W, int n, int r, int c, bool vec, float4 v) {
+    const int64_t idx = int64_t(r) * n + c;
+    if (vec) {
+        if constexpr (sizeof(TW) == 4) {
+            *reinterpret_cast<float4*>(W + idx) = v;
+        } else {
+            const uint32_t lo = __bfloat16_as_ushort(__float2bfloat16_rn(v.x)) |
+                                (uint32_t(__bfloat16_as_ushort(__float2bfloat16_rn(v.y))) << 16);
+            const uint32_t hi = __bfloat16_as_ushort(__float2bfloat16_rn(v.z)) |
+                                (uint32_t(__bfloat16_as_ushort(__float2bfloat16_rn(v.w))) << 16);
+            *reinterpret_cast<uint2*>(W + idx) = make_uint2(lo, hi);
+        }
+    } else {
+        const float t[4] = {v.x, v.y, v.z, v.w};
+        for (int e = 0; e < 4 && c + e < n; ++e) {
+            if constexpr (sizeof(TW) == 4)
+                reinterpret_cast<float*>(W)[idx + e] = t[e];
+            else
+                reinterpret_cast<__nv_bfloat16*>(W)[idx + e] = __float2bfloat16_rn(t[e]);
+        }
+    }
+}
+
+// Iterate buffer elements [off .. off+3] (aligned: ld is a multiple of 64).
+template <typename TX>
+__device__ __forceinline__ float4 load_x4(const void* X, int64_t off) {
+    if constexpr (sizeof(TX) == 4) {
+        return *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(X) + off);
+    } else {
+        const uint2 u = *reinterpret_cast<const uint2*>(reinterpret_cast<const uint16_t*>(X) + off);
+        if constexpr (std::is_same<TX, __half>::value) {
+            const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&u.x));
+            const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&u.y));
+            return make_float4(a.x, a.y, b.x, b.y);
+        } else {
+            return make_float4(bf2f(u.x & 0xffff), bf2f(u.x >> 16), bf2f(u.y & 0xffff), bf2f(u.y >> 16));
+        }
+    }
+}
+
+template <typename TX>
+__device__ __forceinline__ void store_x4(void* X, int64_t off, float4 v) {
+    if constexpr (sizeof(TX) == 4) {
+        *reinterpret_cast<float4*>(reinterpret_cast<float*>(X) + off) = v;
+    } else if constexpr (std::is_same<TX, __half>::value) {
+        __half2 a = __floats2half2_rn(v.x, v.y), b = __floats2half2_rn(v.z, v.w);
+        *reinterpret_cast<uint2*>(reinterpret_cast<uint16_t*>(X) + off) =
+            make_uint2(*reinterpret_cast<uint32_t*>(&a), *reinterpret_cast<uint32_t*>(&b));
+    } else {
+        __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+        *reinterpret_cast<uint2*>(reinterpret_cast<uint16_t*>(X) + off) =
+            make_uint2(*reinterpret_cast<uint32_t*>(&a), *reinterpret_cast<uint32_t*>(&b));
+    }
+}
+
+// ---- reductions ----------------------------------------------------------------
 
 __device__ __forceinline__ float block_sum(float v, float* red) {
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -60,8 +135,8 @@ __device__ __forceinline__ double sum_partials(const float* partials, int base, 
     return s;
 }
 
-// Publishes this block's partial and returns true in the block that completed
-// the matrix (all threads see the result).
+// Publishes this block's partial; true (in every thread) in the block that
+// completed the matrix.
 __device__ __forceinline__ bool finish_tile(const MemLaunch& p, int mat, int seq, float part,
                                             int* flag_smem) {
     if (threadIdx.x == 0) {
@@ -79,12 +154,18 @@ __device__ __forceinline__ bool finish_tile(const MemLaunch& p, int mat, int seq
     return *flag_smem != 0;
 }
 
-template <typename TW>
-__device__ __forceinline__ float load_w(const void* base, int64_t idx) {
-    return to_f<TW>(reinterpret_cast<const TW*>(base)[idx]);
+struct TileCoord {
+    int r0, c;  // first row of this thread, its first column
+};
+
+__device__ __forceinline__ TileCoord tile_coord(const MemItem& it) {
+    TileCoord t;
+    t.r0 = it.tile_r * kMemRows + int(threadIdx.x) / kVecPerRow;
+    t.c = it.tile_c * kMemCols + (int(threadIdx.x) % kVecPerRow) * 4;
+    return t;
 }
 
-// ---- sumsq ----------------------------------------------------------------------
+// ---- kernels ---------------------------------------------------------------------
 
 template <typename TW>
 __global__ void __launch_bounds__(kThreads) sumsq_kernel(const MemLaunch p) {
@@ -92,19 +173,19 @@ __global__ void __launch_bounds__(kThreads) sumsq_kernel(const MemLaunch p) {
     __shared__ int flag;
     const MemItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
-    const void* W = p.weights[it.mat];
-    const int c = it.tile_c * kTile + (threadIdx.x % kTile);
-    const int r0 = it.tile_r * kTile + (threadIdx.x / kTile);
+    const TW* W = reinterpret_cast<const TW*>(p.weights[it.mat]);
+    const bool vec = (md.n & 3) == 0;
+    const TileCoord tc = tile_coord(it);
+    float4 w[kPasses];
+#pragma unroll
+    for (int k = 0; k < kPasses; ++k) w[k] = load_w4<TW>(W, md.m, md.n, tc.r0 + k * kRowsPerPass, tc.c, vec);
     float acc = 0.f;
-    if (c < md.n) {
-#pragma unroll 4
-        for (int k = 0; k < kTile / kRowsPerPass; ++k) {
-            const int r = r0 + k * kRowsPerPass;
-            if (r < md.m) {
-                const float w = load_w<TW>(W, static_cast<int64_t>(r) * md.n + c);
-                acc = fmaf(w, w, acc);
-            }
-        }
+#pragma unroll
+    for (int k = 0; k < kPasses; ++k) {
+        acc = fmaf(w[k].x, w[k].x, acc);
+        acc = fmaf(w[k].y, w[k].y, acc);
+        acc = fmaf(w[k].z, w[k].z, acc);
+        acc = fmaf(w[k].w, w[k].w, acc);
     }
     const float part = block_sum(acc, red);
     if (finish_tile(p, it.mat, it.seq, part, &flag) && threadIdx.x < 32) {
@@ -116,93 +197,56 @@ __global__ void __launch_bounds__(kThreads) sumsq_kernel(const MemLaunch p) {
     }
 }
 
-// ---- cast -----------------------------------------------------------------------
-
-// Items tile the padded iterate (Ppad x Qpad); writes X_0 including zeros in
-// the padding.
+// Items tile the padded buffer (rows x ld); zeros are written to the padding.
 template <typename TW, typename TX>
 __global__ void __launch_bounds__(kThreads) cast_kernel(const MemLaunch p) {
-    __shared__ float tile[kTile][kTile + 1];
     const MemItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
-    const void* W = p.weights[it.mat];
+    const TW* W = reinterpret_cast<const TW*>(p.weights[it.mat]);
     const double f = sqrt(p.scalars[it.mat].frob_sq);
     const float scale = static_cast<float>(1.0 / (f + static_cast<double>(p.eps)));
-    TX* X = reinterpret_cast<TX*>(md.x[p.cur]);
-    const int p0 = it.tile_r * kTile, q0 = it.tile_c * kTile;
-    const int lx = threadIdx.x % kTile, ly = threadIdx.x / kTile;
-    if (!md.transposed) {
-        // X[p][q] = W[p][q]
-        for (int k = 0; k < kTile / kRowsPerPass; ++k) {
-            const int pp = p0 + ly + k * kRowsPerPass, qq = q0 + lx;
-            float v = 0.f;
-            if (pp < md.P && qq < md.Q) v = load_w<TW>(W, static_cast<int64_t>(pp) * md.n + qq) * scale;
-            X[static_cast<int64_t>(pp) * md.Qpad + qq] = from_f<TX>(v);
-        }
-    } else {
-        // X[p][q] = W[q][p]: read W rows q (contiguous in p), write X rows p.
-        for (int k = 0; k < kTile / kRowsPerPass; ++k) {
-            const int qq = q0 + ly + k * kRowsPerPass, pp = p0 + lx;
-            float v = 0.f;
-            if (pp < md.P && qq < md.Q) v = load_w<TW>(W, static_cast<int64_t>(qq) * md.n + pp);
-            tile[ly + k * kRowsPerPass][lx] = v;
-        }
-        __syncthreads();
-        for (int k = 0; k < kTile / kRowsPerPass; ++k) {
-            const int pl = ly + k * kRowsPerPass;
-            const int pp = p0 + pl, qq = q0 + lx;
-            X[static_cast<int64_t>(pp) * md.Qpad + qq] = from_f<TX>(tile[lx][pl] * scale);
-        }
-    }
-}
-
-// ---- W-tile traversal with the final iterate in W's orientation ---------------
-
-// Loads, for this thread's 16 elements (rows r0 + ly + 4k, column c), the value
-// of P_hat = X_T in W's orientation into xv[k].
-template <typename TX>
-__device__ __forceinline__ void load_phat(const MatDev& md, const TX* X, int r_base, int c_base,
-                                          float (*tile)[kTile + 1], float xv[16]) {
-    const int lx = threadIdx.x % kTile, ly = threadIdx.x / kTile;
-    if (!md.transposed) {
-        const int c = c_base + lx;
+    void* X = md.x[p.cur];
+    const bool vec = (md.n & 3) == 0;
+    const TileCoord tc = tile_coord(it);
+    if (tc.c >= md.ld) return;
+    float4 w[kPasses];
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
-            const int r = r_base + ly + k * kRowsPerPass;
-            xv[k] = (r < md.m && c < md.n) ? to_f<TX>(X[static_cast<int64_t>(r) * md.Qpad + c]) : 0.f;
-        }
-    } else {
-        // W(r, c) = X[c][r]: stage X rows c (contiguous in r) through shared memory.
+    for (int k = 0; k < kPasses; ++k) w[k] = load_w4<TW>(W, md.m, md.n, tc.r0 + k * kRowsPerPass, tc.c, vec);
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
-            const int cl = ly + k * kRowsPerPass;
-            const int c = c_base + cl, r = r_base + lx;
-            tile[cl][lx] = (r < md.m && c < md.n) ? to_f<TX>(X[static_cast<int64_t>(c) * md.Qpad + r]) : 0.f;
+    for (int k = 0; k < kPasses; ++k) {
+        const int r = tc.r0 + k * kRowsPerPass;
+        if (r < md.rows) {
+            const float4 v = make_float4(w[k].x * scale, w[k].y * scale, w[k].z * scale, w[k].w * scale);
+            store_x4<TX>(X, int64_t(r) * md.ld + tc.c, v);
         }
-        __syncthreads();
-#pragma unroll
-        for (int k = 0; k < 16; ++k) xv[k] = tile[lx][ly + k * kRowsPerPass];
     }
 }
 
 template <typename TW, typename TX>
 __global__ void __launch_bounds__(kThreads) dot_kernel(const MemLaunch p) {
-    __shared__ float tile[kTile][kTile + 1];
     __shared__ float red[kThreads / 32];
     __shared__ int flag;
     const MemItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
-    const void* W = p.weights[it.mat];
-    const TX* X = reinterpret_cast<const TX*>(md.x[p.cur]);
-    const int r_base = it.tile_r * kTile, c_base = it.tile_c * kTile;
-    float xv[16];
-    load_phat<TX>(md, X, r_base, c_base, tile, xv);
-    const int c = c_base + threadIdx.x % kTile;
+    const TW* W = reinterpret_cast<const TW*>(p.weights[it.mat]);
+    const void* X = md.x[p.cur];
+    const bool vec = (md.n & 3) == 0;
+    const TileCoord tc = tile_coord(it);
+    float4 w[kPasses], x[kPasses];
+#pragma unroll
+    for (int k = 0; k < kPasses; ++k) {
+        const int r = tc.r0 + k * kRowsPerPass;
+        w[k] = load_w4<TW>(W, md.m, md.n, r, tc.c, vec);
+        x[k] = (r < md.m && tc.c < md.n) ? load_x4<TX>(X, int64_t(r) * md.ld + tc.c)
+                                          : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
     float acc = 0.f;
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
-        const int r = r_base + threadIdx.x / kTile + k * kRowsPerPass;
-        if (r < md.m && c < md.n) acc = fmaf(load_w<TW>(W, static_cast<int64_t>(r) * md.n + c), xv[k], acc);
+    for (int k = 0; k < kPasses; ++k) {
+        acc = fmaf(w[k].x, x[k].x, acc);
+        acc = fmaf(w[k].y, x[k].y, acc);
+        acc = fmaf(w[k].z, x[k].z, acc);
+        acc = fmaf(w[k].w, x[k].w, acc);
     }
     const float part = block_sum(acc, red);
     if (!finish_tile(p, it.mat, it.seq, part, &flag)) return;
@@ -211,7 +255,7 @@ __global__ void __launch_bounds__(kThreads) dot_kernel(const MemLaunch p) {
     if (threadIdx.x == 0) {
         p.scalars[it.mat].n_hat = nh;
         if (!isfinite(nh)) atomicOr(p.status, kStatusNonFinite);
-        // Last matrix to finish writes the values and the loss in index order.
+        // The last matrix to finish writes the values and the loss in index order.
         __threadfence();
         const uint32_t done = atomicAdd(p.counters + p.count, 1u);
         if (done == static_cast<uint32_t>(p.count - 1)) {
@@ -238,21 +282,20 @@ __global__ void __launch_bounds__(kThreads) dot_kernel(const MemLaunch p) {
 
 template <typename TW, typename TX>
 __global__ void __launch_bounds__(kThreads) combine_kernel(const MemLaunch p) {
-    __shared__ float tile[kTile][kTile + 1];
     const MemItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
-    const void* W = p.weights[it.mat];
-    void* G = p.grads[it.mat];
-    const TX* X = reinterpret_cast<const TX*>(md.x[p.cur]);
+    const TW* W = reinterpret_cast<const TW*>(p.weights[it.mat]);
+    TW* G = reinterpret_cast<TW*>(p.grads[it.mat]);
+    const void* X = md.x[p.cur];
     const double nh = p.scalars[it.mat].n_hat;
     const double frob = sqrt(p.scalars[it.mat].frob_sq) + static_cast<double>(p.eps);
     const double lg = static_cast<double>(p.lambda) * static_cast<double>(p.grad_scale);
     double alpha, beta;
-    if (p.variant == 0) {
+    if (p.variant == 0) {  // 2 reg (P_hat / frob - n_hat / frob^3 W)
         const double reg = nh / frob;
         alpha = lg * 2.0 * reg / frob;
         beta = lg * 2.0 * reg * nh / (frob * frob * frob);
-    } else {
+    } else {               // P_hat
         alpha = lg;
         beta = 0.0;
     }
@@ -261,24 +304,29 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const MemLaunch p) {
         return;  // leave this matrix's gradient untouched
     }
     const float fa = static_cast<float>(alpha), fb = static_cast<float>(beta);
-    const int r_base = it.tile_r * kTile, c_base = it.tile_c * kTile;
-    float xv[16];
-    load_phat<TX>(md, X, r_base, c_base, tile, xv);
-    const int c = c_base + threadIdx.x % kTile;
-    if (c >= md.n) return;
+    const bool vec = (md.n & 3) == 0;
+    const TileCoord tc = tile_coord(it);
+    if (tc.c >= md.n) return;
+    float4 w[kPasses], x[kPasses], g[kPasses];
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
-        const int r = r_base + threadIdx.x / kTile + k * kRowsPerPass;
+    for (int k = 0; k < kPasses; ++k) {
+        const int r = tc.r0 + k * kRowsPerPass;
+        w[k] = load_w4<TW>(W, md.m, md.n, r, tc.c, vec);
+        g[k] = load_w4<TW>(G, md.m, md.n, r, tc.c, vec);
+        x[k] = r < md.m ? load_x4<TX>(X, int64_t(r) * md.ld + tc.c) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int k = 0; k < kPasses; ++k) {
+        const int r = tc.r0 + k * kRowsPerPass;
         if (r >= md.m) continue;
-        const int64_t idx = static_cast<int64_t>(r) * md.n + c;
-        const float w = load_w<TW>(W, idx);
-        TW* g = reinterpret_cast<TW*>(G) + idx;
-        *g = from_f<TW>(to_f<TW>(*g) + (fa * xv[k] - fb * w));
+        float4 o;
+        o.x = g[k].x + (fa * x[k].x - fb * w[k].x);
+        o.y = g[k].y + (fa * x[k].y - fb * w[k].y);
+        o.z = g[k].z + (fa * x[k].z - fb * w[k].z);
+        o.w = g[k].w + (fa * x[k].w - fb * w[k].w);
+        store_w4<TW>(G, md.n, r, tc.c, vec, o);
     }
 }
-
-template <template <typename, typename> class K>
-struct Dummy;
 
 }  // namespace
 
@@ -291,17 +339,17 @@ cudaError_t launch_sumsq(const MemLaunch& p, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-#define SLORR_DISPATCH_WX(KERNEL)                                                         \
-    do {                                                                                  \
-        if (p.wdtype == 0) {                                                              \
-            if (p.elem == kF32) KERNEL<float, float><<<p.num_items, kThreads, 0, s>>>(p); \
-            else if (p.elem == kF16) KERNEL<float, __half><<<p.num_items, kThreads, 0, s>>>(p); \
-            else KERNEL<float, __nv_bfloat16><<<p.num_items, kThreads, 0, s>>>(p);       \
-        } else {                                                                          \
-            if (p.elem == kF32) KERNEL<__nv_bfloat16, float><<<p.num_items, kThreads, 0, s>>>(p); \
+#define SLORR_DISPATCH_WX(KERNEL)                                                                  \
+    do {                                                                                           \
+        if (p.wdtype == 0) {                                                                       \
+            if (p.elem == kF32) KERNEL<float, float><<<p.num_items, kThreads, 0, s>>>(p);          \
+            else if (p.elem == kF16) KERNEL<float, __half><<<p.num_items, kThreads, 0, s>>>(p);    \
+            else KERNEL<float, __nv_bfloat16><<<p.num_items, kThreads, 0, s>>>(p);                \
+        } else {                                                                                   \
+            if (p.elem == kF32) KERNEL<__nv_bfloat16, float><<<p.num_items, kThreads, 0, s>>>(p);  \
             else if (p.elem == kF16) KERNEL<__nv_bfloat16, __half><<<p.num_items, kThreads, 0, s>>>(p); \
-            else KERNEL<__nv_bfloat16, __nv_bfloat16><<<p.num_items, kThreads, 0, s>>>(p); \
-        }                                                                                 \
+            else KERNEL<__nv_bfloat16, __nv_bfloat16><<<p.num_items, kThreads, 0, s>>>(p);        \
+        }                                                                                          \
     } while (0)
 
 cudaError_t launch_cast(const MemLaunch& p, cudaStream_t s) {

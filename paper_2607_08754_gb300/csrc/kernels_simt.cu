@@ -1,6 +1,6 @@
 // Grouped SIMT (CUDA-core) GEMM for the three phases of a Polar Express step
-// (Sec. 3 "Computational cost": A = X X^T, B = b A + c A^2, X <- a X + B X on
-// the P x Q Gram side).  Used for the fp32 compute mode and, with 16-bit
+// (Sec. 3 "Computational cost": A = X X^T, M = a I + b A + c A^2, X <- M X on
+// the P x Q Gram side; M X is the step's a X + (b A + c A^2) X).  Used for the fp32 compute mode and, with 16-bit
 // storage, as a CUDA-core check of the tensor-core kernel.  64 x 64 output
 // tile per block, 256 threads, 4 x 4 per thread, K staged 16 at a time through
 // shared memory.
@@ -50,17 +50,19 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const GemmLaunch p) {
     const T* X = reinterpret_cast<const T*>(md.x[p.cur]);
     const T* Am = reinterpret_cast<const T*>(md.a);
     const T* Bm = reinterpret_cast<const T*>(md.b);
-    // Operand addressing: Aop(i, k) = opA[i * lda + k]; Bop(k, j) = opB[j * ldb_j + k * ldb_k].
+    // X(p, q) lives at xb[p * sp + q * sq] (the buffer is in W's orientation).
+    const int64_t sp = md.transposed ? 1 : md.ld, sq = md.transposed ? md.ld : 1;
+    // Operands: Aop(i, k) = opA[i * sa_i + k * sa_k]; Bop(k, j) = opB[j * sb_j + k * sb_k].
     const T* opA;
     const T* opB;
-    int64_t lda, ldb_j, ldb_k;
+    int64_t sa_i, sa_k, sb_j, sb_k;
     int K;
-    if (p.phase == kGram) {
-        opA = X; lda = md.Qpad; opB = X; ldb_j = md.Qpad; ldb_k = 1; K = md.Qpad;
-    } else if (p.phase == kPoly) {
-        opA = Am; lda = md.Ppad; opB = Am; ldb_j = md.Ppad; ldb_k = 1; K = md.Ppad;
-    } else {
-        opA = Bm; lda = md.Ppad; opB = X; ldb_j = 1; ldb_k = md.Qpad; K = md.Ppad;
+    if (p.phase == kGram) {          // A = X X^T
+        opA = X; sa_i = sp; sa_k = sq; opB = X; sb_j = sp; sb_k = sq; K = md.Qpad;
+    } else if (p.phase == kPoly) {   // A A
+        opA = Am; sa_i = md.Ppad; sa_k = 1; opB = Am; sb_j = md.Ppad; sb_k = 1; K = md.Ppad;
+    } else {                         // M X
+        opA = Bm; sa_i = md.Ppad; sa_k = 1; opB = X; sb_j = sq; sb_k = sp; K = md.Ppad;
     }
     const int m0 = it.tm * kBM, n0 = it.tn * kBN;
     const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
@@ -70,13 +72,14 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const GemmLaunch p) {
     for (int k0 = 0; k0 < K; k0 += kBK) {
         // 64 x 16 of each operand: 1024 values, 4 per thread.
         for (int e = threadIdx.x; e < kBM * kBK; e += 256) {
-            const int i = e / kBK, k = e % kBK;
-            As[k][i] = ld_f<T>(opA + static_cast<int64_t>(m0 + i) * lda + (k0 + k));
+            int i, k;
+            if (sa_k == 1) { i = e / kBK; k = e % kBK; } else { k = e / kBM; i = e % kBM; }
+            As[k][i] = ld_f<T>(opA + static_cast<int64_t>(m0 + i) * sa_i + static_cast<int64_t>(k0 + k) * sa_k);
         }
         for (int e = threadIdx.x; e < kBN * kBK; e += 256) {
             int j, k;
-            if (ldb_k == 1) { j = e / kBK; k = e % kBK; } else { k = e / kBN; j = e % kBN; }
-            Bs[k][j] = ld_f<T>(opB + static_cast<int64_t>(n0 + j) * ldb_j + static_cast<int64_t>(k0 + k) * ldb_k);
+            if (sb_k == 1) { j = e / kBK; k = e % kBK; } else { k = e / kBN; j = e % kBN; }
+            Bs[k][j] = ld_f<T>(opB + static_cast<int64_t>(n0 + j) * sb_j + static_cast<int64_t>(k0 + k) * sb_k);
         }
         __syncthreads();
 #pragma unroll
@@ -105,25 +108,23 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const GemmLaunch p) {
         }
         __syncthreads();
     }
-    T* out;
-    const T* extra;
-    int64_t ldo;
-    float ce, cacc;
-    if (p.phase == kGram) {
-        out = reinterpret_cast<T*>(md.a); extra = nullptr; ldo = md.Ppad; ce = 0.f; cacc = 1.f;
-    } else if (p.phase == kPoly) {
-        out = reinterpret_cast<T*>(md.b); extra = Am; ldo = md.Ppad; ce = p.b; cacc = p.c;
-    } else {
-        out = reinterpret_cast<T*>(md.x[p.cur ^ 1]); extra = X; ldo = md.Qpad; ce = p.a; cacc = 1.f;
-    }
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
 #pragma unroll
         for (int v = 0; v < 4; ++v) {
-            const int64_t idx = static_cast<int64_t>(m0 + ty * 4 + u) * ldo + (n0 + tx * 4 + v);
-            float val = cacc * (acc[u][v] + cmp[u][v]);
-            if (extra) val = fmaf(ce, ld_f<T>(extra + idx), val);
-            st_f<T>(out + idx, val);
+            const int i = m0 + ty * 4 + u, j = n0 + tx * 4 + v;
+            const float acc_uv = acc[u][v] + cmp[u][v];
+            if (p.phase == kGram) {
+                st_f<T>(reinterpret_cast<T*>(md.a) + static_cast<int64_t>(i) * md.Ppad + j, acc_uv);
+            } else if (p.phase == kPoly) {      // M = c A^2 + b A + a I
+                const int64_t idx = static_cast<int64_t>(i) * md.Ppad + j;
+                float val = fmaf(p.b, ld_f<T>(Am + idx), p.c * acc_uv);
+                if (i == j) val += p.a;
+                st_f<T>(reinterpret_cast<T*>(md.b) + idx, val);
+            } else {                            // X' = M X
+                st_f<T>(reinterpret_cast<T*>(md.x[p.cur ^ 1]) + static_cast<int64_t>(i) * sp +
+                            static_cast<int64_t>(j) * sq, acc_uv);
+            }
         }
     }
 }

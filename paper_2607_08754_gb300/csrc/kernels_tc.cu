@@ -1,9 +1,13 @@
 // Grouped persistent tensor-core GEMM for one phase of a Polar Express step
 // (Sec. 3 "Computing the polar factor" / "Computational cost"):
-//   Gram    A  = X X^T            M = Ppad, N = Ppad, K = Qpad   (both operands K-major)
-//   Poly    B  = b A + c A A      M = Ppad, N = Ppad, K = Ppad   (A symmetric: both K-major)
-//   Update  X' = a X + B X        M = Ppad, N = Qpad, K = Ppad   (X is the MN-major operand)
-// over every matrix of the weight set in one launch.  Operands are fp16 or
+//   Gram    A  = X X^T                 M = Ppad, N = Ppad, K = Qpad
+//   Poly    M  = a I + b A + c A A     M = Ppad, N = Ppad, K = Ppad   (A symmetric)
+//   Update  X' = M X                   M = Ppad, N = Qpad, K = Ppad
+// over every matrix of the weight set in one launch; M X equals the step's
+// a X + (b A + c A^2) X.  The iterate X is stored in W's orientation, so for
+// m <= n it is a K-major operand of the Gram product and an MN-major one of
+// the update, and the other way round for m > n; the UMMA descriptors take
+// either form, so no transpose is ever materialised.  Operands are fp16 or
 // bf16, accumulation fp32 in tensor memory.
 //
 // One CTA per SM (192 threads):
@@ -12,8 +16,9 @@
 //   warp 1      allocates 512 TMEM columns; lane 0 issues tcgen05.mma
 //               (M = 128, N = nsz <= 256, K = 16) into one of two 256-column
 //               fp32 accumulators and commits stage releases / tile completion;
-//   warps 2..5  epilogue: tcgen05.ld 32 columns at a time, combine with the
-//               a X or b A term in fp32, round to 16 bit, store to global.
+//   warps 2..5  epilogue: tcgen05.ld 32 columns at a time, add b A + a I
+//               (Poly only) in fp32, round to 16 bit, store to global (the
+//               update of an m > n matrix stores its tile transposed).
 // Output tiles are 128 x nsz with nsz a multiple of 64, taken round-robin from
 // a host-built list; accumulator double-buffering overlaps a tile's epilogue
 // with the next tile's main loop.  Every wait is bounded; on a timeout the CTA
@@ -54,6 +59,14 @@ __device__ __forceinline__ uint32_t pack2(float lo, float hi) {
 }
 
 template <bool BF16>
+__device__ __forceinline__ uint16_t to16(float x) {
+    if constexpr (BF16)
+        return __bfloat16_as_ushort(__float2bfloat16_rn(x));
+    else
+        return __half_as_ushort(__float2half_rn(x));
+}
+
+template <bool BF16>
 __device__ __forceinline__ float2 unpack2(uint32_t u) {
     if constexpr (BF16) {
         __nv_bfloat162 v = *reinterpret_cast<__nv_bfloat162*>(&u);
@@ -85,30 +98,44 @@ struct PhaseInfo {
     const void* mapA;
     const void* mapB;
     int nkb;
-    bool b_mn;
+    bool a_mn;   // A operand MN-major (else K-major)
+    bool b_mn;   // B operand MN-major (else K-major)
 };
 
 __device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmItem& it) {
     const MatDev& md = p.mats[it.mat];
     const uint8_t* maps = reinterpret_cast<const uint8_t*>(p.maps) + size_t(it.mat) * 4 * 128;
+    const bool tr = md.transposed != 0;
     PhaseInfo pi;
     if (p.phase == kGram) {
         pi.mapA = maps + p.cur * 128;
         pi.mapB = pi.mapA;
         pi.nkb = md.Qpad / kBK;
-        pi.b_mn = false;
+        pi.a_mn = tr;
+        pi.b_mn = tr;
     } else if (p.phase == kPoly) {
         pi.mapA = maps + 2 * 128;
         pi.mapB = pi.mapA;
         pi.nkb = md.Ppad / kBK;
+        pi.a_mn = false;
         pi.b_mn = false;
     } else {
         pi.mapA = maps + 3 * 128;
         pi.mapB = maps + p.cur * 128;
         pi.nkb = md.Ppad / kBK;
-        pi.b_mn = true;
+        pi.a_mn = false;
+        pi.b_mn = !tr;
     }
     return pi;
+}
+
+// Shared-memory descriptor of one K = 16 slice (kk) of a 64-wide K block:
+// K-major: rows of 128 bytes, slice kk starts 32 bytes further in the swizzle
+// atom; MN-major: 64-element MN chunks 8 KB apart (LBO), 8-row K groups 1 KB
+// apart (SBO), slice kk starts 16 rows = 2 KB further.
+__device__ __forceinline__ uint64_t operand_desc(uint32_t base, int kk, bool mn) {
+    return mn ? ptx::sdesc_sw128(base + kk * 16 * 128, kBoxBytes, 1024)
+              : ptx::sdesc_sw128(base + kk * 32, 16, 1024);
 }
 
 __device__ void producer(const GemmLaunch& p, const Smem& s) {
@@ -132,15 +159,16 @@ __device__ void producer(const GemmLaunch& p, const Smem& s) {
             uint8_t* sa = s.stages + size_t(stage) * kStageBytes;
             uint8_t* sb = sa + kABytes;
             ptx::mbar_arrive_expect_tx(&s.full[stage], bytes);
-            ptx::tma_load_2d(sa, pi.mapA, &s.full[stage], kb * kBK, it.tm * kBM);
-            ptx::tma_load_2d(sa + kBoxBytes, pi.mapA, &s.full[stage], kb * kBK, it.tm * kBM + 64);
+            // box coordinates are (inner, outer): (k, mn) for K-major, (mn, k) for MN-major
+            for (int h = 0; h < 2; ++h) {
+                const int mn = it.tm * kBM + h * 64, k = kb * kBK;
+                ptx::tma_load_2d(sa + h * kBoxBytes, pi.mapA, &s.full[stage], pi.a_mn ? mn : k,
+                                 pi.a_mn ? k : mn);
+            }
             for (int j = 0; j < nboxes; ++j) {
-                if (pi.b_mn)
-                    ptx::tma_load_2d(sb + j * kBoxBytes, pi.mapB, &s.full[stage],
-                                     it.tn * kBNMax + j * 64, kb * kBK);
-                else
-                    ptx::tma_load_2d(sb + j * kBoxBytes, pi.mapB, &s.full[stage], kb * kBK,
-                                     it.tn * kBNMax + j * 64);
+                const int mn = it.tn * kBNMax + j * 64, k = kb * kBK;
+                ptx::tma_load_2d(sb + j * kBoxBytes, pi.mapB, &s.full[stage], pi.b_mn ? mn : k,
+                                 pi.b_mn ? k : mn);
             }
             issued_parity[stage] = int(phase);
             if (++stage == kStages) {
@@ -167,7 +195,7 @@ __device__ void mma_issuer(const GemmLaunch& p, const Smem& s, uint32_t tmem_bas
     for (int idx = blockIdx.x; idx < p.num_items && ok; idx += gridDim.x, ++local) {
         const GemmItem it = p.items[idx];
         const PhaseInfo pi = phase_info(p, it);
-        const uint32_t idesc = ptx::idesc_f16(kBM, it.nsz, BF16, pi.b_mn);
+        const uint32_t idesc = ptx::idesc_f16(kBM, it.nsz, BF16, pi.a_mn, pi.b_mn);
         const int buf = local & 1;
         const uint32_t tphase = (uint32_t(local) >> 1) & 1u;
         if (!ptx::mbar_wait(&s.tempty[buf], tphase ^ 1u, s.abort, p.timeout_ns)) {
@@ -188,10 +216,8 @@ __device__ void mma_issuer(const GemmLaunch& p, const Smem& s, uint32_t tmem_bas
             const uint32_t b0 = a0 + kABytes;
 #pragma unroll
             for (int kk = 0; kk < kBK / 16; ++kk) {
-                const uint64_t ad = ptx::sdesc_sw128(a0 + kk * 32, 16, 1024);
-                const uint64_t bd = pi.b_mn ? ptx::sdesc_sw128(b0 + kk * 16 * 128, 8192, 1024)
-                                            : ptx::sdesc_sw128(b0 + kk * 32, 16, 1024);
-                ptx::umma_f16(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
+                ptx::umma_f16(d_tmem, operand_desc(a0, kk, pi.a_mn), operand_desc(b0, kk, pi.b_mn), idesc,
+                              (kb | kk) != 0 ? 1u : 0u);
             }
             issued_any = true;
             ptx::umma_commit(&s.empty[stage]);
@@ -229,50 +255,72 @@ __device__ void epilogue(const GemmLaunch& p, const Smem& s, uint32_t tmem_base,
         }
         ptx::tc_fence_after();
         const int row = it.tm * kBM + quad * 32 + lane;
-        uint16_t* out;
-        const uint16_t* extra;
-        int64_t ld;
-        float ce, cacc;
-        if (p.phase == kGram) {
-            out = reinterpret_cast<uint16_t*>(md.a); extra = nullptr; ld = md.Ppad; ce = 0.f; cacc = 1.f;
-        } else if (p.phase == kPoly) {
-            out = reinterpret_cast<uint16_t*>(md.b);
-            extra = reinterpret_cast<const uint16_t*>(md.a);
-            ld = md.Ppad; ce = p.b; cacc = p.c;
-        } else {
-            out = reinterpret_cast<uint16_t*>(md.x[p.cur ^ 1]);
-            extra = reinterpret_cast<const uint16_t*>(md.x[p.cur]);
-            ld = md.Qpad; ce = p.a; cacc = 1.f;
-        }
         const uint32_t t_row = tmem_base + (uint32_t(quad * 32) << 16) + uint32_t(buf * kAccCols);
-        for (int ch = 0; ch < it.nsz / 32; ++ch) {
-            uint32_t r[32];
-            ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
-            ptx::tmem_ld_wait();
-            const int64_t off = int64_t(row) * ld + int64_t(it.tn) * kBNMax + ch * 32;
-            uint4 o[4];
-            uint32_t* ow = reinterpret_cast<uint32_t*>(o);
-            if (extra) {
-                uint4 e[4];
-                const uint4* src = reinterpret_cast<const uint4*>(extra + off);
+        if (p.phase == kUpdate) {
+            uint16_t* out = reinterpret_cast<uint16_t*>(md.x[p.cur ^ 1]);
+            const int64_t ld = md.ld;
+            for (int ch = 0; ch < it.nsz / 32; ++ch) {
+                uint32_t r[32];
+                ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
+                ptx::tmem_ld_wait();
+                const int col0 = it.tn * kBNMax + ch * 32;
+                if (md.transposed) {
+                    // X^T[q][p]: for each column the warp's 32 rows are contiguous
+                    uint16_t* dst = out + int64_t(col0) * ld + row;
 #pragma unroll
-                for (int v = 0; v < 4; ++v) e[v] = src[v];
-                const uint32_t* ew = reinterpret_cast<const uint32_t*>(e);
+                    for (int j = 0; j < 32; ++j) dst[int64_t(j) * ld] = to16<BF16>(__uint_as_float(r[j]));
+                } else {
+                    uint4 o[4];
+                    uint32_t* ow = reinterpret_cast<uint32_t*>(o);
 #pragma unroll
-                for (int j = 0; j < 16; ++j) {
-                    const float2 x = unpack2<BF16>(ew[j]);
-                    const float lo = fmaf(ce, x.x, cacc * __uint_as_float(r[2 * j]));
-                    const float hi = fmaf(ce, x.y, cacc * __uint_as_float(r[2 * j + 1]));
-                    ow[j] = pack2<BF16>(lo, hi);
+                    for (int j = 0; j < 16; ++j)
+                        ow[j] = pack2<BF16>(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
+                    uint4* dst = reinterpret_cast<uint4*>(out + int64_t(row) * ld + col0);
+#pragma unroll
+                    for (int v = 0; v < 4; ++v) dst[v] = o[v];
                 }
-            } else {
-#pragma unroll
-                for (int j = 0; j < 16; ++j)
-                    ow[j] = pack2<BF16>(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
             }
-            uint4* dst = reinterpret_cast<uint4*>(out + off);
+        } else {
+            uint16_t* out = reinterpret_cast<uint16_t*>(p.phase == kGram ? md.a : md.b);
+            const uint16_t* amat = reinterpret_cast<const uint16_t*>(md.a);
+            const int64_t ld = md.Ppad;
+            const bool poly = p.phase == kPoly;
+            const float cacc = poly ? p.c : 1.f;
+            for (int ch = 0; ch < it.nsz / 32; ++ch) {
+                uint32_t r[32];
+                ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
+                ptx::tmem_ld_wait();
+                const int col0 = it.tn * kBNMax + ch * 32;
+                const int64_t off = int64_t(row) * ld + col0;
+                float v[32];
 #pragma unroll
-            for (int v = 0; v < 4; ++v) dst[v] = o[v];
+                for (int j = 0; j < 32; ++j) v[j] = cacc * __uint_as_float(r[j]);
+                if (poly) {
+                    // M = c A^2 + b A + a I
+                    uint4 e[4];
+                    const uint4* src = reinterpret_cast<const uint4*>(amat + off);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) e[q] = src[q];
+                    const uint32_t* ew = reinterpret_cast<const uint32_t*>(e);
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) {
+                        const float2 x = unpack2<BF16>(ew[j]);
+                        v[2 * j] = fmaf(p.b, x.x, v[2 * j]);
+                        v[2 * j + 1] = fmaf(p.b, x.y, v[2 * j + 1]);
+                    }
+                    const int d = row - col0;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        if (j == d) v[j] += p.a;
+                }
+                uint4 o[4];
+                uint32_t* ow = reinterpret_cast<uint32_t*>(o);
+#pragma unroll
+                for (int j = 0; j < 16; ++j) ow[j] = pack2<BF16>(v[2 * j], v[2 * j + 1]);
+                uint4* dst = reinterpret_cast<uint4*>(out + off);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) dst[q] = o[q];
+            }
         }
         ptx::tc_fence_before();
         __syncwarp();

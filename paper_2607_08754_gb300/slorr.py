@@ -290,7 +290,7 @@ class Regularizer:
         slorr_run_steps(self.handle, [w.data_ptr() for w in weights], ws, self.workspace_bytes, steps, s)
 
     def iterate(self, i: int, after_steps: int):
-        """Copy of matrix i's iterate after `after_steps` steps as a P x Q fp32 tensor."""
+        """Copy of matrix i's Polar Express iterate X (P x Q) after `after_steps` steps, fp32."""
         import torch
         dev = self._ws.device
         v = slorr_iterate_view(self.handle, self.workspace(dev), i, after_steps)
@@ -298,7 +298,8 @@ class Regularizer:
         raw = device_view(v.x, (v.rows, v.ld), typestr, dev).clone()
         if v.elem == 2:
             raw = raw.view(torch.bfloat16)
-        return raw[:, : v.cols].float()
+        x = raw[:, : v.cols].float()
+        return x.t().contiguous() if v.transposed else x
 
     def scalars(self, i: int):
         """(||W_i||_F^2, n_hat_i) read back from the workspace."""
