@@ -59,6 +59,7 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--flags", type=int, default=0, help="slorr_options.flags (tuning / debug)")
     return ap.parse_args()
 
 
@@ -226,7 +227,8 @@ def main():
     dev = torch.device("cuda", local)
     name = args.workload
     shapes = workloads.shapes(name)
-    reg = slorr.Regularizer(shapes, variant=args.variant, compute=args.compute, iters=args.iters, lam=1.0)
+    reg = slorr.Regularizer(shapes, variant=args.variant, compute=args.compute, iters=args.iters, lam=1.0,
+                            flags=args.flags)
     W_host = [torch.from_numpy(workloads.generate_one(name, i)) for i in range(len(shapes))]
     W = [w.to(dev) for w in W_host]
     G = [torch.zeros_like(w) for w in W]

@@ -96,6 +96,7 @@ typedef struct slorr_options {
 
 /* Flags. */
 #define SLORR_FLAG_SIMT_GEMM    1   /* run the 16-bit products on CUDA cores (debug)  */
+#define SLORR_FLAG_L2_PREFETCH  2   /* tensor-core producer also warms L2 ahead (tuning) */
 
 /* Fill *opt with the defaults listed beside each field above (App. C.1: T = 6,
  * ell = 1e-3, degree 5; eps, lambda and grad_scale as in Listing 1 / Alg. 2). */

@@ -128,13 +128,17 @@ void build_plan(slorr_handle* h) {
         for (int r = 0; r < (g.rows + kMemRows - 1) / kMemRows; ++r)
             for (int c = 0; c < (g.ld + kMemCols - 1) / kMemCols; ++c)
                 h->x_items.push_back(MemItem{uint16_t(i), uint16_t(r), uint16_t(c), 0});
-        // tensor-core tiles: 128 x nsz, nsz <= 256
+        // tensor-core tiles: 128 x nsz, nsz <= 256.  The Gram and Poly outputs
+        // are symmetric: tiles lying strictly below the diagonal (in 128 x 128
+        // blocks) are skipped; the kernel mirrors the blocks they need.
         for (int ph = 0; ph < 3; ++ph) {
             const int N = ph == kUpdate ? g.Qpad : g.Ppad;
             for (int tm = 0; tm < g.Ppad / 128; ++tm)
-                for (int tn = 0; tn * 256 < N; ++tn)
-                    h->tc_items[ph].push_back(
-                        GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), uint16_t(std::min(256, N - tn * 256))});
+                for (int tn = 0; tn * 256 < N; ++tn) {
+                    const int nsz = std::min(256, N - tn * 256);
+                    if (ph != kUpdate && (2 * tn + nsz / 128 - 1) < tm) continue;
+                    h->tc_items[ph].push_back(GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), uint16_t(nsz)});
+                }
             for (int tm = 0; tm < g.Ppad / 64; ++tm)
                 for (int tn = 0; tn < N / 64; ++tn)
                     h->simt_items[ph].push_back(GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), 64});
@@ -404,6 +408,7 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
     {
         Traced tr(h, 0, st);
         if ((e = launch_sumsq(mp, st)) != cudaSuccess) return cuda_fail(e, "sumsq launch");
+        if ((e = launch_finalize(mp, 0, st)) != cudaSuccess) return cuda_fail(e, "finalize launch");
         tr.done();
     }
     MemLaunch cp = mp;
@@ -421,6 +426,7 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
     g.maps = ws + h->off_maps;
     g.status = reinterpret_cast<uint32_t*>(ws + h->off_status);
     g.timeout_ns = static_cast<unsigned long long>(h->opt.timeout_s * 1e9);
+    g.prefetch = (h->opt.flags & SLORR_FLAG_L2_PREFETCH) ? 8 : 0;
     for (int t = 0; t < steps; ++t) {
         g.cur = t & 1;
         g.a = float(h->coeffs[3 * t + 0]);
@@ -449,6 +455,7 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
     {
         Traced tr(h, 5, st);
         if ((e = launch_dot(dp, st)) != cudaSuccess) return cuda_fail(e, "dot launch");
+        if ((e = launch_finalize(dp, 1, st)) != cudaSuccess) return cuda_fail(e, "finalize launch");
         tr.done();
     }
     {

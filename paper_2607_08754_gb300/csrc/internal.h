@@ -49,6 +49,10 @@ struct MatDev {
 struct MatScalars {
     double frob_sq;    // ||W||_F^2
     double n_hat;      // sum(W * P_hat)
+    float scale;       // 1 / (||W||_F + eps): the normalisation of X_0
+    float alpha;       // gradient = alpha * P_hat - beta * W (lambda, grad_scale included)
+    float beta;
+    int32_t skip;      // non-finite norm or estimate: leave the gradient untouched
 };
 
 // One output tile of a grouped GEMM phase.
@@ -63,6 +67,7 @@ struct GemmItem {
 // the padded iterate buffer for the cast).
 constexpr int kMemRows = 16;
 constexpr int kMemCols = 512;
+constexpr int kMemVec = 8;      // consecutive columns per thread
 struct MemItem {
     uint16_t mat;
     uint16_t tile_r;   // tile row index (kMemRows rows)
@@ -84,6 +89,7 @@ struct GemmLaunch {
     const void* maps;          // CUtensorMap array, 4 per matrix (X0, X1, A, B)
     uint32_t* status;
     unsigned long long timeout_ns;
+    int32_t prefetch;          // k blocks of L2 prefetch lookahead (0 = off)
 };
 
 struct MemLaunch {
@@ -112,6 +118,7 @@ struct MemLaunch {
 cudaError_t launch_sumsq(const MemLaunch& p, cudaStream_t s);
 cudaError_t launch_cast(const MemLaunch& p, cudaStream_t s);
 cudaError_t launch_dot(const MemLaunch& p, cudaStream_t s);
+cudaError_t launch_finalize(const MemLaunch& p, int which, cudaStream_t s);
 cudaError_t launch_combine(const MemLaunch& p, cudaStream_t s);
 cudaError_t launch_gemm_simt(const GemmLaunch& p, int elem, cudaStream_t s);
 cudaError_t launch_gemm_tc(const GemmLaunch& p, int elem, int grid, cudaStream_t s);

@@ -6,11 +6,14 @@
 //   combine W_i.grad += lambda * grad_scale * G_i       (Listing 1 backward, Alg. 2)
 // The iterates are stored in W's orientation (row-major, row length `ld`), so
 // every pass is elementwise.  A block handles one kMemRows x kMemCols tile:
-// each of its 256 threads owns 4 consecutive columns of 8 rows and issues all
-// eight 128-bit loads before using them (64-bit for 16-bit data).  Rows whose
-// length is not a multiple of 4 take a scalar path.  Cross-tile sums are
-// deterministic: each block writes a partial; the last block of a matrix (per-
-// matrix counter) adds the partials in index order in double precision.
+// each of its 256 threads owns 8 consecutive columns of 4 rows and issues all
+// its 128-bit loads before using them.  Rows whose length is not a multiple
+// of 8 take a scalar path.  Per-matrix coefficients (the cast scale, the
+// gradient's alpha and beta) are computed once by the finalize kernels, in
+// double precision, and read as floats by the streaming passes.  Cross-tile sums are
+// deterministic: each streaming block writes one partial per tile and exits;
+// a finalize kernel (one block per matrix) adds a matrix's partials in index
+// order in double precision.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -20,57 +23,74 @@ namespace slorr {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kVecPerRow = kMemCols / 4;             // 128 threads per tile row
-constexpr int kRowsPerPass = kThreads / kVecPerRow;  // 2
-constexpr int kPasses = kMemRows / kRowsPerPass;     // 8
+constexpr int kVecPerRow = kMemCols / kMemVec;       // 64 threads per tile row
+constexpr int kRowsPerPass = kThreads / kVecPerRow;  // 4
+constexpr int kPasses = kMemRows / kRowsPerPass;     // 4
 
-__device__ __forceinline__ float bf2f(uint16_t u) { return __uint_as_float(uint32_t(u) << 16); }
+struct F8 {
+    float4 lo, hi;
+};
 
-// ---- 4-element loads and stores ------------------------------------------------
+__device__ __forceinline__ float bf2f(uint32_t u16) { return __uint_as_float(u16 << 16); }
 
-// W (fp32 or bf16) elements (r, c .. c+3) of an m x n row-major matrix, zero
-// outside.  vec: n % 4 == 0, so the four are either all inside or all outside.
+__device__ __forceinline__ F8 zero8() {
+    F8 z;
+    z.lo = make_float4(0.f, 0.f, 0.f, 0.f);
+    z.hi = z.lo;
+    return z;
+}
+
+// ---- 8-element loads and stores ------------------------------------------------
+
+// W (fp32 or bf16) elements (r, c .. c+7) of an m x n row-major matrix, zero
+// outside.  vec: n % 8 == 0, so the eight are either all inside or all outside.
 template <typename TW>
-__device__ __forceinline__ float4 load_w4(const TW* W, int m, int n, int r, int c, bool vec) {
-    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+__device__ __forceinline__ F8 load_w8(const TW* W, int m, int n, int r, int c, bool vec) {
+    F8 v = zero8();
     if (r >= m || c >= n) return v;
     const int64_t idx = int64_t(r) * n + c;
     if (vec) {
         if constexpr (sizeof(TW) == 4) {
-            v = *reinterpret_cast<const float4*>(W + idx);
+            v.lo = *reinterpret_cast<const float4*>(W + idx);
+            v.hi = *reinterpret_cast<const float4*>(W + idx + 4);
         } else {
-            const uint2 u = *reinterpret_cast<const uint2*>(W + idx);
-            v = make_float4(bf2f(u.x & 0xffff), bf2f(u.x >> 16), bf2f(u.y & 0xffff), bf2f(u.y >> 16));
+            const uint4 u = *reinterpret_cast<const uint4*>(W + idx);
+            v.lo = make_float4(bf2f(u.x & 0xffff), bf2f(u.x >> 16), bf2f(u.y & 0xffff), bf2f(u.y >> 16));
+            v.hi = make_float4(bf2f(u.z & 0xffff), bf2f(u.z >> 16), bf2f(u.w & 0xffff), bf2f(u.w >> 16));
         }
     } else {
-        float t[4] = {0.f, 0.f, 0.f, 0.f};
-        for (int e = 0; e < 4 && c + e < n; ++e) {
+        float t[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        for (int e = 0; e < 8 && c + e < n; ++e) {
             if constexpr (sizeof(TW) == 4)
                 t[e] = reinterpret_cast<const float*>(W)[idx + e];
             else
                 t[e] = bf2f(reinterpret_cast<const uint16_t*>(W)[idx + e]);
         }
-        v = make_float4(t[0], t[1], t[2], t[3]);
+        v.lo = make_float4(t[0], t[1], t[2], t[3]);
+        v.hi = make_float4(t[4], t[5], t[6], t[7]);
     }
     return v;
 }
 
+__device__ __forceinline__ uint32_t pack_bf2(float a, float b) {
+    return uint32_t(__bfloat16_as_ushort(__float2bfloat16_rn(a))) |
+           (uint32_t(__bfloat16_as_ushort(__float2bfloat16_rn(b))) << 16);
+}
+
 template <typename TW>
-__device__ __forceinline__ void store_w4(TW* W, int n, int r, int c, bool vec, float4 v) {
+__device__ __forceinline__ void store_w8(TW* W, int n, int r, int c, bool vec, const F8& v) {
     const int64_t idx = int64_t(r) * n + c;
     if (vec) {
         if constexpr (sizeof(TW) == 4) {
-            *reinterpret_cast<float4*>(W + idx) = v;
+            *reinterpret_cast<float4*>(W + idx) = v.lo;
+            *reinterpret_cast<float4*>(W + idx + 4) = v.hi;
         } else {
-            const uint32_t lo = __bfloat16_as_ushort(__float2bfloat16_rn(v.x)) |
-                                (uint32_t(__bfloat16_as_ushort(__float2bfloat16_rn(v.y))) << 16);
-            const uint32_t hi = __bfloat16_as_ushort(__float2bfloat16_rn(v.z)) |
-                                (uint32_t(__bfloat16_as_ushort(__float2bfloat16_rn(v.w))) << 16);
-            *reinterpret_cast<uint2*>(W + idx) = make_uint2(lo, hi);
+            *reinterpret_cast<uint4*>(W + idx) = make_uint4(pack_bf2(v.lo.x, v.lo.y), pack_bf2(v.lo.z, v.lo.w),
+                                                            pack_bf2(v.hi.x, v.hi.y), pack_bf2(v.hi.z, v.hi.w));
         }
     } else {
-        const float t[4] = {v.x, v.y, v.z, v.w};
-        for (int e = 0; e < 4 && c + e < n; ++e) {
+        const float t[8] = {v.lo.x, v.lo.y, v.lo.z, v.lo.w, v.hi.x, v.hi.y, v.hi.z, v.hi.w};
+        for (int e = 0; e < 8 && c + e < n; ++e) {
             if constexpr (sizeof(TW) == 4)
                 reinterpret_cast<float*>(W)[idx + e] = t[e];
             else
@@ -79,36 +99,64 @@ __device__ __forceinline__ void store_w4(TW* W, int n, int r, int c, bool vec, f
     }
 }
 
-// Iterate buffer elements [off .. off+3] (aligned: ld is a multiple of 64).
+// Iterate buffer elements [off .. off+7] (aligned: ld is a multiple of 64).
 template <typename TX>
-__device__ __forceinline__ float4 load_x4(const void* X, int64_t off) {
+__device__ __forceinline__ F8 load_x8(const void* X, int64_t off) {
+    F8 v;
     if constexpr (sizeof(TX) == 4) {
-        return *reinterpret_cast<const float4*>(reinterpret_cast<const float*>(X) + off);
+        const float* x = reinterpret_cast<const float*>(X) + off;
+        v.lo = *reinterpret_cast<const float4*>(x);
+        v.hi = *reinterpret_cast<const float4*>(x + 4);
     } else {
-        const uint2 u = *reinterpret_cast<const uint2*>(reinterpret_cast<const uint16_t*>(X) + off);
+        const uint4 u = *reinterpret_cast<const uint4*>(reinterpret_cast<const uint16_t*>(X) + off);
         if constexpr (std::is_same<TX, __half>::value) {
             const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&u.x));
             const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&u.y));
-            return make_float4(a.x, a.y, b.x, b.y);
+            const float2 c = __half22float2(*reinterpret_cast<const __half2*>(&u.z));
+            const float2 d = __half22float2(*reinterpret_cast<const __half2*>(&u.w));
+            v.lo = make_float4(a.x, a.y, b.x, b.y);
+            v.hi = make_float4(c.x, c.y, d.x, d.y);
         } else {
-            return make_float4(bf2f(u.x & 0xffff), bf2f(u.x >> 16), bf2f(u.y & 0xffff), bf2f(u.y >> 16));
+            v.lo = make_float4(bf2f(u.x & 0xffff), bf2f(u.x >> 16), bf2f(u.y & 0xffff), bf2f(u.y >> 16));
+            v.hi = make_float4(bf2f(u.z & 0xffff), bf2f(u.z >> 16), bf2f(u.w & 0xffff), bf2f(u.w >> 16));
         }
+    }
+    return v;
+}
+
+template <typename TX>
+__device__ __forceinline__ uint32_t pack_x2(float a, float b) {
+    if constexpr (std::is_same<TX, __half>::value) {
+        __half2 h = __floats2half2_rn(a, b);
+        return *reinterpret_cast<uint32_t*>(&h);
+    } else {
+        return pack_bf2(a, b);
     }
 }
 
 template <typename TX>
-__device__ __forceinline__ void store_x4(void* X, int64_t off, float4 v) {
+__device__ __forceinline__ void store_x8(void* X, int64_t off, const F8& v) {
     if constexpr (sizeof(TX) == 4) {
-        *reinterpret_cast<float4*>(reinterpret_cast<float*>(X) + off) = v;
-    } else if constexpr (std::is_same<TX, __half>::value) {
-        __half2 a = __floats2half2_rn(v.x, v.y), b = __floats2half2_rn(v.z, v.w);
-        *reinterpret_cast<uint2*>(reinterpret_cast<uint16_t*>(X) + off) =
-            make_uint2(*reinterpret_cast<uint32_t*>(&a), *reinterpret_cast<uint32_t*>(&b));
+        float* x = reinterpret_cast<float*>(X) + off;
+        *reinterpret_cast<float4*>(x) = v.lo;
+        *reinterpret_cast<float4*>(x + 4) = v.hi;
     } else {
-        __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
-        *reinterpret_cast<uint2*>(reinterpret_cast<uint16_t*>(X) + off) =
-            make_uint2(*reinterpret_cast<uint32_t*>(&a), *reinterpret_cast<uint32_t*>(&b));
+        *reinterpret_cast<uint4*>(reinterpret_cast<uint16_t*>(X) + off) =
+            make_uint4(pack_x2<TX>(v.lo.x, v.lo.y), pack_x2<TX>(v.lo.z, v.lo.w), pack_x2<TX>(v.hi.x, v.hi.y),
+                       pack_x2<TX>(v.hi.z, v.hi.w));
     }
+}
+
+__device__ __forceinline__ float dot8(const F8& a, const F8& b, float acc) {
+    acc = fmaf(a.lo.x, b.lo.x, acc);
+    acc = fmaf(a.lo.y, b.lo.y, acc);
+    acc = fmaf(a.lo.z, b.lo.z, acc);
+    acc = fmaf(a.lo.w, b.lo.w, acc);
+    acc = fmaf(a.hi.x, b.hi.x, acc);
+    acc = fmaf(a.hi.y, b.hi.y, acc);
+    acc = fmaf(a.hi.z, b.hi.z, acc);
+    acc = fmaf(a.hi.w, b.hi.w, acc);
+    return acc;
 }
 
 // ---- reductions ----------------------------------------------------------------
@@ -126,34 +174,6 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
     return s;  // valid in thread 0
 }
 
-// Deterministic sum of partials[base .. base+n) by warp 0, in double.
-__device__ __forceinline__ double sum_partials(const float* partials, int base, int n) {
-    double s = 0.0;
-    const int lane = threadIdx.x & 31;
-    for (int i = lane; i < n; i += 32) s += static_cast<double>(__ldcg(partials + base + i));
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    return s;
-}
-
-// Publishes this block's partial; true (in every thread) in the block that
-// completed the matrix.
-__device__ __forceinline__ bool finish_tile(const MemLaunch& p, int mat, int seq, float part,
-                                            int* flag_smem) {
-    if (threadIdx.x == 0) {
-        p.partials[p.tile_base[mat] + seq] = part;
-        __threadfence();
-        const uint32_t done = atomicAdd(p.counters + mat, 1u);
-        const bool last = done == static_cast<uint32_t>(p.tile_count[mat] - 1);
-        if (last) {
-            p.counters[mat] = 0u;  // leave the counter clean for the next call
-            __threadfence();
-        }
-        *flag_smem = last ? 1 : 0;
-    }
-    __syncthreads();
-    return *flag_smem != 0;
-}
-
 struct TileCoord {
     int r0, c;  // first row of this thread, its first column
 };
@@ -161,7 +181,7 @@ struct TileCoord {
 __device__ __forceinline__ TileCoord tile_coord(const MemItem& it) {
     TileCoord t;
     t.r0 = it.tile_r * kMemRows + int(threadIdx.x) / kVecPerRow;
-    t.c = it.tile_c * kMemCols + (int(threadIdx.x) % kVecPerRow) * 4;
+    t.c = it.tile_c * kMemCols + (int(threadIdx.x) % kVecPerRow) * kMemVec;
     return t;
 }
 
@@ -170,31 +190,19 @@ __device__ __forceinline__ TileCoord tile_coord(const MemItem& it) {
 template <typename TW>
 __global__ void __launch_bounds__(kThreads) sumsq_kernel(const MemLaunch p) {
     __shared__ float red[kThreads / 32];
-    __shared__ int flag;
     const MemItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
     const TW* W = reinterpret_cast<const TW*>(p.weights[it.mat]);
-    const bool vec = (md.n & 3) == 0;
+    const bool vec = (md.n & 7) == 0;
     const TileCoord tc = tile_coord(it);
-    float4 w[kPasses];
+    F8 w[kPasses];
 #pragma unroll
-    for (int k = 0; k < kPasses; ++k) w[k] = load_w4<TW>(W, md.m, md.n, tc.r0 + k * kRowsPerPass, tc.c, vec);
+    for (int k = 0; k < kPasses; ++k) w[k] = load_w8<TW>(W, md.m, md.n, tc.r0 + k * kRowsPerPass, tc.c, vec);
     float acc = 0.f;
 #pragma unroll
-    for (int k = 0; k < kPasses; ++k) {
-        acc = fmaf(w[k].x, w[k].x, acc);
-        acc = fmaf(w[k].y, w[k].y, acc);
-        acc = fmaf(w[k].z, w[k].z, acc);
-        acc = fmaf(w[k].w, w[k].w, acc);
-    }
+    for (int k = 0; k < kPasses; ++k) acc = dot8(w[k], w[k], acc);
     const float part = block_sum(acc, red);
-    if (finish_tile(p, it.mat, it.seq, part, &flag) && threadIdx.x < 32) {
-        const double s = sum_partials(p.partials, p.tile_base[it.mat], p.tile_count[it.mat]);
-        if (threadIdx.x == 0) {
-            p.scalars[it.mat].frob_sq = s;
-            if (!isfinite(s)) atomicOr(p.status, kStatusNonFinite);
-        }
-    }
+    if (threadIdx.x == 0) p.partials[p.tile_base[it.mat] + it.seq] = part;
 }
 
 // Items tile the padded buffer (rows x ld); zeros are written to the padding.
@@ -203,21 +211,22 @@ __global__ void __launch_bounds__(kThreads) cast_kernel(const MemLaunch p) {
     const MemItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
     const TW* W = reinterpret_cast<const TW*>(p.weights[it.mat]);
-    const double f = sqrt(p.scalars[it.mat].frob_sq);
-    const float scale = static_cast<float>(1.0 / (f + static_cast<double>(p.eps)));
     void* X = md.x[p.cur];
-    const bool vec = (md.n & 3) == 0;
+    const bool vec = (md.n & 7) == 0;
     const TileCoord tc = tile_coord(it);
     if (tc.c >= md.ld) return;
-    float4 w[kPasses];
+    F8 w[kPasses];
 #pragma unroll
-    for (int k = 0; k < kPasses; ++k) w[k] = load_w4<TW>(W, md.m, md.n, tc.r0 + k * kRowsPerPass, tc.c, vec);
+    for (int k = 0; k < kPasses; ++k) w[k] = load_w8<TW>(W, md.m, md.n, tc.r0 + k * kRowsPerPass, tc.c, vec);
+    const float scale = p.scalars[it.mat].scale;
 #pragma unroll
     for (int k = 0; k < kPasses; ++k) {
         const int r = tc.r0 + k * kRowsPerPass;
         if (r < md.rows) {
-            const float4 v = make_float4(w[k].x * scale, w[k].y * scale, w[k].z * scale, w[k].w * scale);
-            store_x4<TX>(X, int64_t(r) * md.ld + tc.c, v);
+            F8 v;
+            v.lo = make_float4(w[k].lo.x * scale, w[k].lo.y * scale, w[k].lo.z * scale, w[k].lo.w * scale);
+            v.hi = make_float4(w[k].hi.x * scale, w[k].hi.y * scale, w[k].hi.z * scale, w[k].hi.w * scale);
+            store_x8<TX>(X, int64_t(r) * md.ld + tc.c, v);
         }
     }
 }
@@ -225,106 +234,126 @@ __global__ void __launch_bounds__(kThreads) cast_kernel(const MemLaunch p) {
 template <typename TW, typename TX>
 __global__ void __launch_bounds__(kThreads) dot_kernel(const MemLaunch p) {
     __shared__ float red[kThreads / 32];
-    __shared__ int flag;
     const MemItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
     const TW* W = reinterpret_cast<const TW*>(p.weights[it.mat]);
     const void* X = md.x[p.cur];
-    const bool vec = (md.n & 3) == 0;
+    const bool vec = (md.n & 7) == 0;
     const TileCoord tc = tile_coord(it);
-    float4 w[kPasses], x[kPasses];
+    F8 w[kPasses], x[kPasses];
 #pragma unroll
     for (int k = 0; k < kPasses; ++k) {
         const int r = tc.r0 + k * kRowsPerPass;
-        w[k] = load_w4<TW>(W, md.m, md.n, r, tc.c, vec);
-        x[k] = (r < md.m && tc.c < md.n) ? load_x4<TX>(X, int64_t(r) * md.ld + tc.c)
-                                          : make_float4(0.f, 0.f, 0.f, 0.f);
+        w[k] = load_w8<TW>(W, md.m, md.n, r, tc.c, vec);
+        x[k] = (r < md.m && tc.c < md.n) ? load_x8<TX>(X, int64_t(r) * md.ld + tc.c) : zero8();
     }
     float acc = 0.f;
 #pragma unroll
-    for (int k = 0; k < kPasses; ++k) {
-        acc = fmaf(w[k].x, x[k].x, acc);
-        acc = fmaf(w[k].y, x[k].y, acc);
-        acc = fmaf(w[k].z, x[k].z, acc);
-        acc = fmaf(w[k].w, x[k].w, acc);
-    }
+    for (int k = 0; k < kPasses; ++k) acc = dot8(w[k], x[k], acc);
     const float part = block_sum(acc, red);
-    if (!finish_tile(p, it.mat, it.seq, part, &flag)) return;
-    if (threadIdx.x >= 32) return;
-    const double nh = sum_partials(p.partials, p.tile_base[it.mat], p.tile_count[it.mat]);
-    if (threadIdx.x == 0) {
-        p.scalars[it.mat].n_hat = nh;
-        if (!isfinite(nh)) atomicOr(p.status, kStatusNonFinite);
-        // The last matrix to finish writes the values and the loss in index order.
-        __threadfence();
-        const uint32_t done = atomicAdd(p.counters + p.count, 1u);
-        if (done == static_cast<uint32_t>(p.count - 1)) {
-            p.counters[p.count] = 0u;
-            __threadfence();
-            double loss = 0.0;
-            for (int i = 0; i < p.count; ++i) {
-                const double n_i = __ldcg(&p.scalars[i].n_hat);
-                double L;
-                if (p.variant == 0) {
-                    const double frob = sqrt(__ldcg(&p.scalars[i].frob_sq)) + static_cast<double>(p.eps);
-                    const double reg = n_i / frob;
-                    L = reg * reg;
-                } else {
-                    L = n_i;
-                }
-                if (p.per_matrix_out) p.per_matrix_out[i] = static_cast<float>(L);
-                loss += L;
-            }
-            *p.loss_out = static_cast<float>(static_cast<double>(p.lambda) * loss);
-        }
+    if (threadIdx.x == 0) p.partials[p.tile_base[it.mat] + it.seq] = part;
+}
+
+// One block per matrix: adds the matrix's tile partials in index order (double)
+// and derives the per-matrix coefficients the next pass needs.
+//   which = 0: ||W||_F^2 and the cast scale 1 / (||W||_F + eps);
+//   which = 1: n_hat and the gradient coefficients (Listing 1 backward times
+//              lambda * grad_scale): Hoyer alpha = 2 reg / frob,
+//              beta = 2 reg n_hat / frob^3 with reg = n_hat / frob; Nuc alpha = 1.
+//              The last block to finish also writes the values L_i and the loss
+//              lambda * sum_i L_i in index order.
+__global__ void __launch_bounds__(128) finalize_kernel(const MemLaunch p, int which) {
+    __shared__ double red[4];
+    const int mat = blockIdx.x;
+    const int base = p.tile_base[mat], n = p.tile_count[mat];
+    double s = 0.0;
+    for (int i = threadIdx.x; i < n; i += 128) s += static_cast<double>(__ldcg(p.partials + base + i));
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+    __syncthreads();
+    if (threadIdx.x != 0) return;
+    const double tot = (red[0] + red[1]) + (red[2] + red[3]);
+    MatScalars& sc = p.scalars[mat];
+    const double eps = static_cast<double>(p.eps);
+    if (which == 0) {
+        sc.frob_sq = tot;
+        sc.scale = static_cast<float>(1.0 / (sqrt(tot) + eps));
+        if (!isfinite(tot)) atomicOr(p.status, kStatusNonFinite);
+        return;
     }
+    sc.n_hat = tot;
+    const double frob = sqrt(sc.frob_sq) + eps;
+    const double lg = static_cast<double>(p.lambda) * static_cast<double>(p.grad_scale);
+    double alpha, beta;
+    if (p.variant == 0) {
+        const double reg = tot / frob;
+        alpha = lg * 2.0 * reg / frob;
+        beta = lg * 2.0 * reg * tot / (frob * frob * frob);
+    } else {
+        alpha = lg;
+        beta = 0.0;
+    }
+    const bool bad = !isfinite(tot) || !isfinite(alpha) || !isfinite(beta);
+    sc.alpha = static_cast<float>(alpha);
+    sc.beta = static_cast<float>(beta);
+    sc.skip = bad ? 1 : 0;
+    if (bad) atomicOr(p.status, kStatusNonFinite);
+    __threadfence();
+    const uint32_t done = atomicAdd(p.counters + p.count, 1u);
+    if (done != static_cast<uint32_t>(p.count - 1)) return;
+    p.counters[p.count] = 0u;  // leave the counter clean for the next call
+    __threadfence();
+    double loss = 0.0;
+    for (int i = 0; i < p.count; ++i) {
+        const double n_i = __ldcg(&p.scalars[i].n_hat);
+        double L;
+        if (p.variant == 0) {
+            const double fr = sqrt(__ldcg(&p.scalars[i].frob_sq)) + eps;
+            const double reg = n_i / fr;
+            L = reg * reg;
+        } else {
+            L = n_i;
+        }
+        if (p.per_matrix_out) p.per_matrix_out[i] = static_cast<float>(L);
+        loss += L;
+    }
+    *p.loss_out = static_cast<float>(static_cast<double>(p.lambda) * loss);
 }
 
 template <typename TW, typename TX>
 __global__ void __launch_bounds__(kThreads) combine_kernel(const MemLaunch p) {
     const MemItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
+    const TileCoord tc = tile_coord(it);
+    const MatScalars& sc = p.scalars[it.mat];
+    if (sc.skip || tc.c >= md.n) return;  // non-finite: leave the gradient untouched
     const TW* W = reinterpret_cast<const TW*>(p.weights[it.mat]);
     TW* G = reinterpret_cast<TW*>(p.grads[it.mat]);
     const void* X = md.x[p.cur];
-    const double nh = p.scalars[it.mat].n_hat;
-    const double frob = sqrt(p.scalars[it.mat].frob_sq) + static_cast<double>(p.eps);
-    const double lg = static_cast<double>(p.lambda) * static_cast<double>(p.grad_scale);
-    double alpha, beta;
-    if (p.variant == 0) {  // 2 reg (P_hat / frob - n_hat / frob^3 W)
-        const double reg = nh / frob;
-        alpha = lg * 2.0 * reg / frob;
-        beta = lg * 2.0 * reg * nh / (frob * frob * frob);
-    } else {               // P_hat
-        alpha = lg;
-        beta = 0.0;
-    }
-    if (!isfinite(alpha) || !isfinite(beta)) {
-        if (threadIdx.x == 0) atomicOr(p.status, kStatusNonFinite);
-        return;  // leave this matrix's gradient untouched
-    }
-    const float fa = static_cast<float>(alpha), fb = static_cast<float>(beta);
-    const bool vec = (md.n & 3) == 0;
-    const TileCoord tc = tile_coord(it);
-    if (tc.c >= md.n) return;
-    float4 w[kPasses], x[kPasses], g[kPasses];
+    const float fa = sc.alpha, fb = sc.beta;
+    const bool vec = (md.n & 7) == 0;
+    F8 w[kPasses], x[kPasses], g[kPasses];
 #pragma unroll
     for (int k = 0; k < kPasses; ++k) {
         const int r = tc.r0 + k * kRowsPerPass;
-        w[k] = load_w4<TW>(W, md.m, md.n, r, tc.c, vec);
-        g[k] = load_w4<TW>(G, md.m, md.n, r, tc.c, vec);
-        x[k] = r < md.m ? load_x4<TX>(X, int64_t(r) * md.ld + tc.c) : make_float4(0.f, 0.f, 0.f, 0.f);
+        w[k] = load_w8<TW>(W, md.m, md.n, r, tc.c, vec);
+        g[k] = load_w8<TW>(G, md.m, md.n, r, tc.c, vec);
+        x[k] = r < md.m ? load_x8<TX>(X, int64_t(r) * md.ld + tc.c) : zero8();
     }
 #pragma unroll
     for (int k = 0; k < kPasses; ++k) {
         const int r = tc.r0 + k * kRowsPerPass;
         if (r >= md.m) continue;
-        float4 o;
-        o.x = g[k].x + (fa * x[k].x - fb * w[k].x);
-        o.y = g[k].y + (fa * x[k].y - fb * w[k].y);
-        o.z = g[k].z + (fa * x[k].z - fb * w[k].z);
-        o.w = g[k].w + (fa * x[k].w - fb * w[k].w);
-        store_w4<TW>(G, md.n, r, tc.c, vec, o);
+        F8 o;
+        o.lo.x = g[k].lo.x + (fa * x[k].lo.x - fb * w[k].lo.x);
+        o.lo.y = g[k].lo.y + (fa * x[k].lo.y - fb * w[k].lo.y);
+        o.lo.z = g[k].lo.z + (fa * x[k].lo.z - fb * w[k].lo.z);
+        o.lo.w = g[k].lo.w + (fa * x[k].lo.w - fb * w[k].lo.w);
+        o.hi.x = g[k].hi.x + (fa * x[k].hi.x - fb * w[k].hi.x);
+        o.hi.y = g[k].hi.y + (fa * x[k].hi.y - fb * w[k].hi.y);
+        o.hi.z = g[k].hi.z + (fa * x[k].hi.z - fb * w[k].hi.z);
+        o.hi.w = g[k].hi.w + (fa * x[k].hi.w - fb * w[k].hi.w);
+        store_w8<TW>(G, md.n, r, tc.c, vec, o);
     }
 }
 
@@ -361,6 +390,11 @@ cudaError_t launch_cast(const MemLaunch& p, cudaStream_t s) {
 cudaError_t launch_dot(const MemLaunch& p, cudaStream_t s) {
     if (p.num_items == 0) return cudaSuccess;
     SLORR_DISPATCH_WX(dot_kernel);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_finalize(const MemLaunch& p, int which, cudaStream_t s) {
+    finalize_kernel<<<p.count, 128, 0, s>>>(p, which);
     return cudaGetLastError();
 }
 

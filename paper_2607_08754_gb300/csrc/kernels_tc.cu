@@ -129,6 +129,15 @@ __device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmI
     return pi;
 }
 
+// Symmetric products (Gram, Poly): only tiles holding some 128 x 128 block on
+// or above the diagonal are computed.  Tile (tm, tn) covers column blocks
+// 2 tn .. 2 tn + nblk - 1 (nblk = nsz / 128), so it is computed iff its last
+// column block reaches the diagonal: 2 tn + nblk - 1 >= tm.
+__device__ __forceinline__ bool sym_tile_computed(int tm, int tn, int Ppad) {
+    const int last_block = min(2 * tn + 1, Ppad / 128 - 1);
+    return last_block >= tm;
+}
+
 // Shared-memory descriptor of one K = 16 slice (kk) of a 64-wide K block:
 // K-major: rows of 128 bytes, slice kk starts 32 bytes further in the swizzle
 // atom; MN-major: 64-element MN chunks 8 KB apart (LBO), 8-row K groups 1 KB
@@ -169,6 +178,18 @@ __device__ void producer(const GemmLaunch& p, const Smem& s) {
                 const int mn = it.tn * kBNMax + j * 64, k = kb * kBK;
                 ptx::tma_load_2d(sb + j * kBoxBytes, pi.mapB, &s.full[stage], pi.b_mn ? mn : k,
                                  pi.b_mn ? k : mn);
+            }
+            if (p.prefetch > 0 && kb + p.prefetch < pi.nkb) {
+                // warm L2 with the k block `prefetch` steps ahead of this one
+                const int k = (kb + p.prefetch) * kBK;
+                for (int h = 0; h < 2; ++h) {
+                    const int mn = it.tm * kBM + h * 64;
+                    ptx::tma_prefetch_l2_2d(pi.mapA, pi.a_mn ? mn : k, pi.a_mn ? k : mn);
+                }
+                for (int j = 0; j < nboxes; ++j) {
+                    const int mn = it.tn * kBNMax + j * 64;
+                    ptx::tma_prefetch_l2_2d(pi.mapB, pi.b_mn ? mn : k, pi.b_mn ? k : mn);
+                }
             }
             issued_parity[stage] = int(phase);
             if (++stage == kStages) {
@@ -320,6 +341,15 @@ __device__ void epilogue(const GemmLaunch& p, const Smem& s, uint32_t tmem_base,
                 uint4* dst = reinterpret_cast<uint4*>(out + off);
 #pragma unroll
                 for (int q = 0; q < 4; ++q) dst[q] = o[q];
+                // The output is symmetric and strictly-lower tiles are skipped:
+                // write the transpose of this 128 x 128 block (I, J), J > I, when
+                // the tile that holds (J, I) is not computed.
+                const int I = it.tm, J = col0 / 128;
+                if (J > I && !sym_tile_computed(J, I / 2, md.Ppad)) {
+                    uint16_t* tdst = out + int64_t(col0) * ld + row;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) tdst[int64_t(j) * ld] = to16<BF16>(v[j]);
+                }
             }
         }
         ptx::tc_fence_before();

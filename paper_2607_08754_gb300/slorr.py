@@ -25,6 +25,7 @@ VARIANTS = {"hoyer": 0, "nuclear": 1}
 COMPUTES = {"fp16": 0, "bf16": 1, "fp32": 2}
 DTYPES = {"f32": 0, "bf16": 1}
 FLAG_SIMT_GEMM = 1
+FLAG_L2_PREFETCH = 2
 
 
 class SlorrError(RuntimeError):
