@@ -198,6 +198,23 @@ SLORR_API slorr_status slorr_partition(const slorr_shape* shapes, int32_t count,
 SLORR_API slorr_status slorr_set_timing(slorr_handle* h, int32_t enable);
 SLORR_API slorr_status slorr_read_timing(slorr_handle* h, double* ms, int64_t* launches, int32_t kinds);
 
+/* ||W||_F^2 of one matrix without any device allocation (the paper has no
+ * counterpart: this exists for callers that cannot provide a workspace, e.g.
+ * code running while a stream is captured, or under a framework that owns
+ * all device memory).
+ *   weight       device pointer, row-major m x n, of slorr_dtype `dtype`
+ *   out_frob_sq  device pointer to one double, written with sum_ij W_ij^2
+ * Enqueued on `stream`; deterministic (fixed-order partial sums).  Scratch is
+ * a fixed 256 KB array inside the library, present on every GPU that loads
+ * it until the process exits; m * n may not exceed 536870912 (INVALID_ARG
+ * otherwise).  All calls share that array: calls that overlap on the GPU
+ * (other streams or host threads) race and must be serialised by the caller.
+ * The first call on each device looks up the array's device address
+ * (cudaGetSymbolAddress); make that first call before any stream capture.
+ * Calls no cudaMalloc, cudaFree or other allocating routine. */
+SLORR_API slorr_status slorr_frob_sq_noalloc(const void* weight, int64_t m, int64_t n, int32_t dtype,
+                                             double* out_frob_sq, void* stream);
+
 SLORR_API void        slorr_destroy(slorr_handle* h);
 SLORR_API const char* slorr_status_string(slorr_status s);
 

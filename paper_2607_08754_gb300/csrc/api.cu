@@ -36,6 +36,12 @@ slorr_status cuda_fail(cudaError_t e, const char* what) {
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+}  // namespace
+
+void slorr::set_last_error(const std::string& msg) { g_last_error = msg; }
+
+namespace {
+
 struct Geom {
     int m, n, P, Q, Ppad, Qpad, transposed, rows, ld;
     size_t off_x[2], off_a, off_b;

@@ -15,6 +15,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <string>
 
 #include <cuda_runtime.h>
 
@@ -123,6 +124,9 @@ cudaError_t launch_combine(const MemLaunch& p, cudaStream_t s);
 cudaError_t launch_gemm_simt(const GemmLaunch& p, int elem, cudaStream_t s);
 cudaError_t launch_gemm_tc(const GemmLaunch& p, int elem, int grid, cudaStream_t s);
 int tc_smem_bytes();
+
+// Records the message slorr_last_error() returns on this thread (api.cu).
+void set_last_error(const std::string& msg);
 
 // Host Polar Express schedule (schedule.cpp).
 namespace host {

@@ -82,6 +82,7 @@ def load_library(path: str | None = None) -> ctypes.CDLL:
                                   ctypes.POINTER(i32)]),
         "slorr_set_timing": (i32, [vp, i32]),
         "slorr_read_timing": (i32, [vp, ctypes.POINTER(dbl), ctypes.POINTER(i64), i32]),
+        "slorr_frob_sq_noalloc": (i32, [vp, i64, i64, i32, vp, vp]),
         "slorr_destroy": (None, [vp]),
         "slorr_status_string": (ctypes.c_char_p, [i32]),
         "slorr_last_error": (ctypes.c_char_p, []),
@@ -212,6 +213,13 @@ def slorr_read_timing(handle) -> dict:
     cnt = (ctypes.c_int64 * n)()
     _check(load_library().slorr_read_timing(handle, ms, cnt, n))
     return {k: (float(ms[i]), int(cnt[i])) for i, k in enumerate(KERNEL_KINDS)}
+
+
+def slorr_frob_sq_noalloc(weight_ptr, m, n, dtype, out_ptr, stream) -> None:
+    """||W||_F^2 of one device matrix into a device double, with no device
+    allocation (fixed in-library scratch; see include/slorr.h)."""
+    _check(load_library().slorr_frob_sq_noalloc(ctypes.c_void_p(weight_ptr), int(m), int(n), int(dtype),
+                                                 ctypes.c_void_p(out_ptr), ctypes.c_void_p(stream or 0)))
 
 
 def slorr_destroy(handle) -> None:
