@@ -191,9 +191,10 @@ SLORR_API slorr_status slorr_partition(const slorr_shape* shapes, int32_t count,
  * launches is bracketed by a pair of CUDA events recorded on the caller's
  * stream (events are created on the host; no device memory is allocated).
  * slorr_read_timing() waits for the recorded events, adds the elapsed
- * milliseconds and launch counts per kernel kind into ms[k] / launches[k]
+ * milliseconds and kernel launch counts per kind into ms[k] / launches[k]
  * (k < kinds, kinds <= SLORR_NUM_KERNEL_KINDS; kinds are sumsq, cast, gram,
- * poly, update, dot, combine) and forgets them. */
+ * poly, update, dot, combine; sumsq and dot each include their finalize
+ * kernel) and forgets them. */
 #define SLORR_NUM_KERNEL_KINDS 7
 SLORR_API slorr_status slorr_set_timing(slorr_handle* h, int32_t enable);
 SLORR_API slorr_status slorr_read_timing(slorr_handle* h, double* ms, int64_t* launches, int32_t kinds);

@@ -74,7 +74,7 @@ struct slorr_handle {
     // tracing
     bool timing = false;
     std::vector<cudaEvent_t> ev_pool;
-    struct Mark { int kind; cudaEvent_t start, stop; };
+    struct Mark { int kind; int kernels; cudaEvent_t start, stop; };
     std::vector<Mark> marks;
     ~slorr_handle() {
         for (auto& m : marks) {
@@ -336,7 +336,7 @@ struct Traced {
     Traced(slorr_handle* h_, int kind_, cudaStream_t st_) : h(h_), st(st_), kind(kind_) {
         if (h->timing && (start = take_event(h)) != nullptr) cudaEventRecord(start, st);
     }
-    void done() {
+    void done(int kernels = 1) {
         if (!start) return;
         cudaEvent_t stop = take_event(h);
         if (!stop) {
@@ -344,7 +344,7 @@ struct Traced {
             return;
         }
         cudaEventRecord(stop, st);
-        h->marks.push_back({kind, start, stop});
+        h->marks.push_back({kind, kernels, start, stop});
         start = nullptr;
     }
 };
@@ -415,7 +415,7 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
         Traced tr(h, 0, st);
         if ((e = launch_sumsq(mp, st)) != cudaSuccess) return cuda_fail(e, "sumsq launch");
         if ((e = launch_finalize(mp, 0, st)) != cudaSuccess) return cuda_fail(e, "finalize launch");
-        tr.done();
+        tr.done(2);
     }
     MemLaunch cp = mp;
     cp.items = reinterpret_cast<const MemItem*>(ws + h->off_x_items);
@@ -462,7 +462,7 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
         Traced tr(h, 5, st);
         if ((e = launch_dot(dp, st)) != cudaSuccess) return cuda_fail(e, "dot launch");
         if ((e = launch_finalize(dp, 1, st)) != cudaSuccess) return cuda_fail(e, "finalize launch");
-        tr.done();
+        tr.done(2);
     }
     {
         Traced tr(h, 6, st);
@@ -657,7 +657,7 @@ slorr_status slorr_read_timing(slorr_handle* h, double* ms, int64_t* launches, i
         if (e != cudaSuccess && s == SLORR_OK) s = cuda_fail(e, "event timing");
         if (m.kind < kinds) {
             ms[m.kind] += double(t);
-            launches[m.kind] += 1;
+            launches[m.kind] += m.kernels;
         }
         h->ev_pool.push_back(m.start);
         h->ev_pool.push_back(m.stop);
