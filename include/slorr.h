@@ -97,6 +97,7 @@ typedef struct slorr_options {
 /* Flags. */
 #define SLORR_FLAG_SIMT_GEMM    1   /* run the 16-bit products on CUDA cores (debug)  */
 #define SLORR_FLAG_L2_PREFETCH  2   /* tensor-core producer also warms L2 ahead (tuning) */
+#define SLORR_FLAG_TC_BK32      4   /* 9 stages of K = 32 instead of 4 of K = 64 (tuning) */
 
 /* Fill *opt with the defaults listed beside each field above (App. C.1: T = 6,
  * ell = 1e-3, degree 5; eps, lambda and grad_scale as in Listing 1 / Alg. 2). */

@@ -178,7 +178,7 @@ void build_plan(slorr_handle* h) {
     h->off_mats = off;
     off = align_up(off + size_t(count) * sizeof(MatDev), 256);
     h->off_maps = off;
-    off = align_up(off + size_t(count) * 4 * 128, 256);
+    off = align_up(off + size_t(count) * kMapsPerMatrix * 128, 256);
     for (int ph = 0; ph < 3; ++ph) {
         h->off_tc_items[ph] = off;
         off = align_up(off + h->tc_items[ph].size() * sizeof(GemmItem), 256);
@@ -208,6 +208,9 @@ void build_plan(slorr_handle* h) {
     h->total_bytes = off;
 }
 
+// K depth of the tensor-core pipeline stages for this handle.
+int tc_bk(const slorr_handle* h) { return (h->opt.flags & SLORR_FLAG_TC_BK32) ? 32 : 64; }
+
 PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     if (!fn) {
@@ -221,16 +224,19 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
     return fn;
 }
 
-// Row-major rows x cols 16-bit matrix, 64 x 64 boxes, 128-byte swizzle.
-bool encode_map(CUtensorMap* map, void* base, int rows, int cols, bool bf16) {
+// Row-major rows x cols 16-bit matrix read in boxes of box_inner (contiguous)
+// x box_outer elements.  A 128-byte inner box uses the 128-byte swizzle, a
+// 64-byte one the 64-byte swizzle (the kernel's descriptors match).
+bool encode_map(CUtensorMap* map, void* base, int rows, int cols, bool bf16, int box_inner, int box_outer) {
     auto enc = get_encode();
     if (!enc) return false;
     cuuint64_t dims[2] = {cuuint64_t(cols), cuuint64_t(rows)};
     cuuint64_t strides[1] = {cuuint64_t(cols) * 2};
-    cuuint32_t box[2] = {64, 64};
+    cuuint32_t box[2] = {cuuint32_t(box_inner), cuuint32_t(box_outer)};
     cuuint32_t estr[2] = {1, 1};
+    const CUtensorMapSwizzle sw = box_inner * 2 == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
     CUresult r = enc(map, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, base,
-                     dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
@@ -253,7 +259,8 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
     const size_t base = h->off_tilebase;
     std::vector<int32_t> tb(count), tcnt(count);
     std::vector<MatDev> mats(count);
-    std::vector<uint8_t> maps(size_t(count) * 4 * 128, 0);
+    std::vector<uint8_t> maps(size_t(count) * kMapsPerMatrix * 128, 0);
+    const int bk = tc_bk(h);
     const bool tc = h->opt.compute != SLORR_COMPUTE_FP32;
     for (int i = 0; i < count; ++i) {
         const Geom& g = h->geom[i];
@@ -276,10 +283,16 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
         md.pad_ = 0;
         if (tc) {
             const bool bf = h->opt.compute == SLORR_COMPUTE_BF16;
-            CUtensorMap* mp = reinterpret_cast<CUtensorMap*>(maps.data() + size_t(i) * 4 * 128);
-            if (!encode_map(mp + 0, md.x[0], g.rows, g.ld, bf) || !encode_map(mp + 1, md.x[1], g.rows, g.ld, bf) ||
-                !encode_map(mp + 2, md.a, g.Ppad, g.Ppad, bf) || !encode_map(mp + 3, md.b, g.Ppad, g.Ppad, bf))
-                return fail(SLORR_ERR_CUDA, "cuTensorMapEncodeTiled failed");
+            CUtensorMap* mp = reinterpret_cast<CUtensorMap*>(maps.data() + size_t(i) * kMapsPerMatrix * 128);
+            // K-major boxes: bk (k) x 64 rows; MN-major boxes: 64 (mn) x bk rows
+            bool ok = true;
+            for (int b = 0; b < 2; ++b) {
+                ok = ok && encode_map(mp + b, md.x[b], g.rows, g.ld, bf, bk, 64);
+                ok = ok && encode_map(mp + 2 + b, md.x[b], g.rows, g.ld, bf, 64, bk);
+            }
+            ok = ok && encode_map(mp + 4, md.a, g.Ppad, g.Ppad, bf, bk, 64);
+            ok = ok && encode_map(mp + 5, md.b, g.Ppad, g.Ppad, bf, bk, 64);
+            if (!ok) return fail(SLORR_ERR_CUDA, "cuTensorMapEncodeTiled failed");
         }
     }
     put(plan, h->off_tilebase - base, tb.data(), tb.size());
@@ -433,6 +446,7 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
     g.status = reinterpret_cast<uint32_t*>(ws + h->off_status);
     g.timeout_ns = static_cast<unsigned long long>(h->opt.timeout_s * 1e9);
     g.prefetch = (h->opt.flags & SLORR_FLAG_L2_PREFETCH) ? 8 : 0;
+    g.bk = tc_bk(h);
     for (int t = 0; t < steps; ++t) {
         g.cur = t & 1;
         g.a = float(h->coeffs[3 * t + 0]);

@@ -87,11 +87,16 @@ struct GemmLaunch {
     int32_t cur;               // index of the current iterate buffer (0/1)
     float a, b, c;             // step coefficients (a_t, b_t, c_t)
     const MatDev* mats;
-    const void* maps;          // CUtensorMap array, 4 per matrix (X0, X1, A, B)
+    const void* maps;          // CUtensorMap array, kMapsPerMatrix per matrix
     uint32_t* status;
     unsigned long long timeout_ns;
     int32_t prefetch;          // k blocks of L2 prefetch lookahead (0 = off)
+    int32_t bk;                // K depth of a pipeline stage: 64 (4 stages) or 32 (9 stages)
 };
+
+// Tensor maps per matrix: X0 K-major, X1 K-major, X0 MN-major, X1 MN-major,
+// A K-major, M K-major.
+constexpr int kMapsPerMatrix = 6;
 
 struct MemLaunch {
     const MemItem* items;

@@ -254,32 +254,43 @@ __global__ void __launch_bounds__(kThreads) dot_kernel(const MemLaunch p) {
     if (threadIdx.x == 0) p.partials[p.tile_base[it.mat] + it.seq] = part;
 }
 
-// One block per matrix: adds the matrix's tile partials in index order (double)
-// and derives the per-matrix coefficients the next pass needs.
-//   which = 0: ||W||_F^2 and the cast scale 1 / (||W||_F + eps);
-//   which = 1: n_hat and the gradient coefficients (Listing 1 backward times
-//              lambda * grad_scale): Hoyer alpha = 2 reg / frob,
-//              beta = 2 reg n_hat / frob^3 with reg = n_hat / frob; Nuc alpha = 1.
-//              The last block to finish also writes the values L_i and the loss
-//              lambda * sum_i L_i in index order.
-__global__ void __launch_bounds__(128) finalize_kernel(const MemLaunch p, int which) {
+// Values L_i and the loss lambda * sum_i L_i, by one whole block: thread t
+// handles matrices t, t + 128, ...; the partial sums are combined in a fixed
+// tree, so the result does not depend on timing.
+__device__ void finalize_loss(const MemLaunch& p) {
     __shared__ double red[4];
-    const int mat = blockIdx.x;
-    const int base = p.tile_base[mat], n = p.tile_count[mat];
-    double s = 0.0;
-    for (int i = threadIdx.x; i < n; i += 128) s += static_cast<double>(__ldcg(p.partials + base + i));
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+    const double eps = static_cast<double>(p.eps);
+    double part = 0.0;
+    for (int i = threadIdx.x; i < p.count; i += 128) {
+        const double n_i = __ldcg(&p.scalars[i].n_hat);
+        double L;
+        if (p.variant == 0) {
+            const double fr = sqrt(__ldcg(&p.scalars[i].frob_sq)) + eps;
+            const double reg = n_i / fr;
+            L = reg * reg;
+        } else {
+            L = n_i;
+        }
+        if (p.per_matrix_out) p.per_matrix_out[i] = static_cast<float>(L);
+        part += L;
+    }
+    for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = part;
     __syncthreads();
-    if (threadIdx.x != 0) return;
-    const double tot = (red[0] + red[1]) + (red[2] + red[3]);
+    if (threadIdx.x == 0)
+        *p.loss_out = static_cast<float>(static_cast<double>(p.lambda) * ((red[0] + red[1]) + (red[2] + red[3])));
+}
+
+// Thread 0 of the block of matrix `mat`: stores the sum and the derived
+// coefficients; returns true in the last block to finish the n_hat pass.
+__device__ bool finalize_matrix(const MemLaunch& p, int which, int mat, double tot) {
     MatScalars& sc = p.scalars[mat];
     const double eps = static_cast<double>(p.eps);
     if (which == 0) {
         sc.frob_sq = tot;
         sc.scale = static_cast<float>(1.0 / (sqrt(tot) + eps));
         if (!isfinite(tot)) atomicOr(p.status, kStatusNonFinite);
-        return;
+        return false;
     }
     sc.n_hat = tot;
     const double frob = sqrt(sc.frob_sq) + eps;
@@ -299,25 +310,34 @@ __global__ void __launch_bounds__(128) finalize_kernel(const MemLaunch p, int wh
     sc.skip = bad ? 1 : 0;
     if (bad) atomicOr(p.status, kStatusNonFinite);
     __threadfence();
-    const uint32_t done = atomicAdd(p.counters + p.count, 1u);
-    if (done != static_cast<uint32_t>(p.count - 1)) return;
+    if (atomicAdd(p.counters + p.count, 1u) != static_cast<uint32_t>(p.count - 1)) return false;
     p.counters[p.count] = 0u;  // leave the counter clean for the next call
     __threadfence();
-    double loss = 0.0;
-    for (int i = 0; i < p.count; ++i) {
-        const double n_i = __ldcg(&p.scalars[i].n_hat);
-        double L;
-        if (p.variant == 0) {
-            const double fr = sqrt(__ldcg(&p.scalars[i].frob_sq)) + eps;
-            const double reg = n_i / fr;
-            L = reg * reg;
-        } else {
-            L = n_i;
-        }
-        if (p.per_matrix_out) p.per_matrix_out[i] = static_cast<float>(L);
-        loss += L;
-    }
-    *p.loss_out = static_cast<float>(static_cast<double>(p.lambda) * loss);
+    return true;
+}
+
+// One block per matrix: adds the matrix's tile partials in index order (double)
+// and derives the per-matrix coefficients the next pass needs.
+//   which = 0: ||W||_F^2 and the cast scale 1 / (||W||_F + eps);
+//   which = 1: n_hat and the gradient coefficients (Listing 1 backward times
+//              lambda * grad_scale): Hoyer alpha = 2 reg / frob,
+//              beta = 2 reg n_hat / frob^3 with reg = n_hat / frob; Nuc alpha = 1.
+//              The last block to finish also writes the values L_i and the loss
+//              lambda * sum_i L_i (finalize_loss).
+__global__ void __launch_bounds__(128) finalize_kernel(const MemLaunch p, int which) {
+    __shared__ double red[4];
+    __shared__ int is_last;
+    const int mat = blockIdx.x;
+    const int base = p.tile_base[mat], n = p.tile_count[mat];
+    double s = 0.0;
+    for (int i = threadIdx.x; i < n; i += 128) s += static_cast<double>(__ldcg(p.partials + base + i));
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+    __syncthreads();
+    const double tot = (red[0] + red[1]) + (red[2] + red[3]);
+    if (threadIdx.x == 0) is_last = finalize_matrix(p, which, mat, tot) ? 1 : 0;
+    __syncthreads();
+    if (is_last) finalize_loss(p);
 }
 
 template <typename TW, typename TX>

@@ -35,17 +35,36 @@ namespace {
 
 constexpr int kBM = 128;
 constexpr int kBNMax = 256;
-constexpr int kBK = 64;  // 64 x 16-bit = one 128-byte swizzle row
-constexpr int kStages = 4;
-constexpr int kABytes = kBM * kBK * 2;      // 16 KB
-constexpr int kBBytes = kBNMax * kBK * 2;   // 32 KB
-constexpr int kStageBytes = kABytes + kBBytes;
-constexpr int kBoxBytes = 64 * kBK * 2;     // one 64-row box, 8 KB
 constexpr int kTmemCols = 512;
 constexpr int kAccCols = 256;
 constexpr int kThreads = 192;
 constexpr int kEpiWarps = 4;
-constexpr size_t kSmemBytes = size_t(kStages) * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+constexpr int kMaxStages = 16;
+
+// Pipeline configuration: K depth of a stage and number of stages.
+//   BK = 64 (default): K-major boxes are 64 x 64 with the 128-byte swizzle,
+//                      48 KB stages, 4 stages;
+//   BK = 32 (option):  K-major boxes are 32 x 64 with the 64-byte swizzle,
+//                      24 KB stages, 9 stages.  Deeper, but its 64-byte rows
+//                      halve the bytes per L2 request; measured 1.5x slower.
+// MN-major boxes are always 64 (MN) x BK rows with the 128-byte swizzle.  Every
+// box holds 64 x BK elements.
+template <int BK_, int STAGES_>
+struct Cfg {
+    static constexpr int BK = BK_;
+    static constexpr int STAGES = STAGES_;
+    static constexpr int kBoxBytes = 64 * BK * 2;
+    static constexpr int kABytes = kBM * BK * 2;
+    static constexpr int kBBytes = kBNMax * BK * 2;
+    static constexpr int kStageBytes = kABytes + kBBytes;
+    static constexpr uint32_t kKLayout = BK == 64 ? 2u : 4u;  // SWIZZLE_128B / SWIZZLE_64B
+    static constexpr uint32_t kKSbo = 8 * BK * 2;              // 8 rows of BK 16-bit elements
+    static constexpr size_t kSmemBytes = size_t(STAGES) * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+    static_assert(STAGES <= kMaxStages, "too many stages");
+    static_assert(kSmemBytes <= 232448, "shared memory budget");
+};
+using Cfg64 = Cfg<64, 4>;
+using Cfg32 = Cfg<32, 9>;
 
 template <bool BF16>
 __device__ __forceinline__ uint32_t pack2(float lo, float hi) {
@@ -102,29 +121,36 @@ struct PhaseInfo {
     bool b_mn;   // B operand MN-major (else K-major)
 };
 
+// Tensor maps per matrix (kMapsPerMatrix of them, 128 bytes each):
+// X0 K-major, X1 K-major, X0 MN-major, X1 MN-major, A K-major, M K-major.
+__device__ __forceinline__ const void* xmap(const uint8_t* maps, int buf, bool mn) {
+    return maps + (mn ? 2 + buf : buf) * 128;
+}
+
+template <class C>
 __device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmItem& it) {
     const MatDev& md = p.mats[it.mat];
-    const uint8_t* maps = reinterpret_cast<const uint8_t*>(p.maps) + size_t(it.mat) * 4 * 128;
+    const uint8_t* maps = reinterpret_cast<const uint8_t*>(p.maps) + size_t(it.mat) * kMapsPerMatrix * 128;
     const bool tr = md.transposed != 0;
     PhaseInfo pi;
     if (p.phase == kGram) {
-        pi.mapA = maps + p.cur * 128;
-        pi.mapB = pi.mapA;
-        pi.nkb = md.Qpad / kBK;
         pi.a_mn = tr;
         pi.b_mn = tr;
-    } else if (p.phase == kPoly) {
-        pi.mapA = maps + 2 * 128;
+        pi.mapA = xmap(maps, p.cur, tr);
         pi.mapB = pi.mapA;
-        pi.nkb = md.Ppad / kBK;
+        pi.nkb = md.Qpad / C::BK;
+    } else if (p.phase == kPoly) {
         pi.a_mn = false;
         pi.b_mn = false;
+        pi.mapA = maps + 4 * 128;
+        pi.mapB = pi.mapA;
+        pi.nkb = md.Ppad / C::BK;
     } else {
-        pi.mapA = maps + 3 * 128;
-        pi.mapB = maps + p.cur * 128;
-        pi.nkb = md.Ppad / kBK;
         pi.a_mn = false;
         pi.b_mn = !tr;
+        pi.mapA = maps + 5 * 128;
+        pi.mapB = xmap(maps, p.cur, pi.b_mn);
+        pi.nkb = md.Ppad / C::BK;
     }
     return pi;
 }
@@ -138,26 +164,29 @@ __device__ __forceinline__ bool sym_tile_computed(int tm, int tn, int Ppad) {
     return last_block >= tm;
 }
 
-// Shared-memory descriptor of one K = 16 slice (kk) of a 64-wide K block:
-// K-major: rows of 128 bytes, slice kk starts 32 bytes further in the swizzle
-// atom; MN-major: 64-element MN chunks 8 KB apart (LBO), 8-row K groups 1 KB
-// apart (SBO), slice kk starts 16 rows = 2 KB further.
+// Shared-memory descriptor of one K = 16 slice (kk) of a BK-wide K block:
+// K-major: rows of 2 BK bytes (swizzle span), 8-row groups kKSbo apart, slice
+// kk starts 32 bytes further inside the swizzle atom; MN-major: 64-element MN
+// chunks one box apart (LBO), 8-row K groups 1 KB apart (SBO), slice kk starts
+// 16 rows = 2 KB further.
+template <class C>
 __device__ __forceinline__ uint64_t operand_desc(uint32_t base, int kk, bool mn) {
-    return mn ? ptx::sdesc_sw128(base + kk * 16 * 128, kBoxBytes, 1024)
-              : ptx::sdesc_sw128(base + kk * 32, 16, 1024);
+    return mn ? ptx::sdesc(base + kk * 16 * 128, C::kBoxBytes, 1024, 2u)
+              : ptx::sdesc(base + kk * 32, 16, C::kKSbo, C::kKLayout);
 }
 
+template <class C>
 __device__ void producer(const GemmLaunch& p, const Smem& s) {
     int stage = 0;
     uint32_t phase = 0;
-    int issued_parity[kStages];
+    int issued_parity[C::STAGES];
 #pragma unroll
-    for (int i = 0; i < kStages; ++i) issued_parity[i] = -1;
+    for (int i = 0; i < C::STAGES; ++i) issued_parity[i] = -1;
     bool ok = true;
     for (int idx = blockIdx.x; idx < p.num_items && ok; idx += gridDim.x) {
         const GemmItem it = p.items[idx];
-        const PhaseInfo pi = phase_info(p, it);
-        const uint32_t bytes = kABytes + uint32_t(it.nsz) * kBK * 2;
+        const PhaseInfo pi = phase_info<C>(p, it);
+        const uint32_t bytes = C::kABytes + uint32_t(it.nsz) * C::BK * 2;
         const int nboxes = it.nsz / 64;
         for (int kb = 0; kb < pi.nkb; ++kb) {
             if (!ptx::mbar_wait(&s.empty[stage], phase ^ 1u, s.abort, p.timeout_ns)) {
@@ -165,23 +194,23 @@ __device__ void producer(const GemmLaunch& p, const Smem& s) {
                 ok = false;
                 break;
             }
-            uint8_t* sa = s.stages + size_t(stage) * kStageBytes;
-            uint8_t* sb = sa + kABytes;
+            uint8_t* sa = s.stages + size_t(stage) * C::kStageBytes;
+            uint8_t* sb = sa + C::kABytes;
             ptx::mbar_arrive_expect_tx(&s.full[stage], bytes);
             // box coordinates are (inner, outer): (k, mn) for K-major, (mn, k) for MN-major
             for (int h = 0; h < 2; ++h) {
-                const int mn = it.tm * kBM + h * 64, k = kb * kBK;
-                ptx::tma_load_2d(sa + h * kBoxBytes, pi.mapA, &s.full[stage], pi.a_mn ? mn : k,
+                const int mn = it.tm * kBM + h * 64, k = kb * C::BK;
+                ptx::tma_load_2d(sa + h * C::kBoxBytes, pi.mapA, &s.full[stage], pi.a_mn ? mn : k,
                                  pi.a_mn ? k : mn);
             }
             for (int j = 0; j < nboxes; ++j) {
-                const int mn = it.tn * kBNMax + j * 64, k = kb * kBK;
-                ptx::tma_load_2d(sb + j * kBoxBytes, pi.mapB, &s.full[stage], pi.b_mn ? mn : k,
+                const int mn = it.tn * kBNMax + j * 64, k = kb * C::BK;
+                ptx::tma_load_2d(sb + j * C::kBoxBytes, pi.mapB, &s.full[stage], pi.b_mn ? mn : k,
                                  pi.b_mn ? k : mn);
             }
             if (p.prefetch > 0 && kb + p.prefetch < pi.nkb) {
                 // warm L2 with the k block `prefetch` steps ahead of this one
-                const int k = (kb + p.prefetch) * kBK;
+                const int k = (kb + p.prefetch) * C::BK;
                 for (int h = 0; h < 2; ++h) {
                     const int mn = it.tm * kBM + h * 64;
                     ptx::tma_prefetch_l2_2d(pi.mapA, pi.a_mn ? mn : k, pi.a_mn ? k : mn);
@@ -192,7 +221,7 @@ __device__ void producer(const GemmLaunch& p, const Smem& s) {
                 }
             }
             issued_parity[stage] = int(phase);
-            if (++stage == kStages) {
+            if (++stage == C::STAGES) {
                 stage = 0;
                 phase ^= 1u;
             }
@@ -200,13 +229,13 @@ __device__ void producer(const GemmLaunch& p, const Smem& s) {
     }
     if (!ok) {
         // Wait (bounded) for every copy this thread issued to land before exit.
-        for (int i = 0; i < kStages; ++i)
+        for (int i = 0; i < C::STAGES; ++i)
             if (issued_parity[i] >= 0)
                 ptx::mbar_wait(&s.full[i], uint32_t(issued_parity[i]), s.never, p.timeout_ns);
     }
 }
 
-template <bool BF16>
+template <bool BF16, class C>
 __device__ void mma_issuer(const GemmLaunch& p, const Smem& s, uint32_t tmem_base) {
     int stage = 0;
     uint32_t phase = 0;
@@ -215,7 +244,7 @@ __device__ void mma_issuer(const GemmLaunch& p, const Smem& s, uint32_t tmem_bas
     bool issued_any = false;
     for (int idx = blockIdx.x; idx < p.num_items && ok; idx += gridDim.x, ++local) {
         const GemmItem it = p.items[idx];
-        const PhaseInfo pi = phase_info(p, it);
+        const PhaseInfo pi = phase_info<C>(p, it);
         const uint32_t idesc = ptx::idesc_f16(kBM, it.nsz, BF16, pi.a_mn, pi.b_mn);
         const int buf = local & 1;
         const uint32_t tphase = (uint32_t(local) >> 1) & 1u;
@@ -233,16 +262,16 @@ __device__ void mma_issuer(const GemmLaunch& p, const Smem& s, uint32_t tmem_bas
                 break;
             }
             ptx::tc_fence_after();
-            const uint32_t a0 = ptx::smem_u32(s.stages + size_t(stage) * kStageBytes);
-            const uint32_t b0 = a0 + kABytes;
+            const uint32_t a0 = ptx::smem_u32(s.stages + size_t(stage) * C::kStageBytes);
+            const uint32_t b0 = a0 + C::kABytes;
 #pragma unroll
-            for (int kk = 0; kk < kBK / 16; ++kk) {
-                ptx::umma_f16(d_tmem, operand_desc(a0, kk, pi.a_mn), operand_desc(b0, kk, pi.b_mn), idesc,
+            for (int kk = 0; kk < C::BK / 16; ++kk) {
+                ptx::umma_f16(d_tmem, operand_desc<C>(a0, kk, pi.a_mn), operand_desc<C>(b0, kk, pi.b_mn), idesc,
                               (kb | kk) != 0 ? 1u : 0u);
             }
             issued_any = true;
             ptx::umma_commit(&s.empty[stage]);
-            if (++stage == kStages) {
+            if (++stage == C::STAGES) {
                 stage = 0;
                 phase ^= 1u;
             }
@@ -358,16 +387,16 @@ __device__ void epilogue(const GemmLaunch& p, const Smem& s, uint32_t tmem_base,
     }
 }
 
-template <bool BF16>
+template <bool BF16, class C>
 __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ GemmLaunch p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* base = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     Smem s;
     s.stages = base;
-    s.full = reinterpret_cast<uint64_t*>(base + size_t(kStages) * kStageBytes);
-    s.empty = s.full + kStages;
-    s.tfull = s.empty + kStages;
+    s.full = reinterpret_cast<uint64_t*>(base + size_t(C::STAGES) * C::kStageBytes);
+    s.empty = s.full + C::STAGES;
+    s.tfull = s.empty + C::STAGES;
     s.tempty = s.tfull + 2;
     s.drain = s.tempty + 2;
     s.tmem_slot = reinterpret_cast<uint32_t*>(s.drain + 1);
@@ -376,7 +405,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < kStages; ++i) {
+        for (int i = 0; i < C::STAGES; ++i) {
             ptx::mbar_init(&s.full[i], 1);
             ptx::mbar_init(&s.empty[i], 1);
         }
@@ -392,7 +421,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     if (warp == 0 && lane == 0) {
         // Warm the descriptors of the first item.
         if (blockIdx.x < p.num_items) {
-            const PhaseInfo pi = phase_info(p, p.items[blockIdx.x]);
+            const PhaseInfo pi = phase_info<C>(p, p.items[blockIdx.x]);
             ptx::prefetch_tmap(pi.mapA);
             ptx::prefetch_tmap(pi.mapB);
         }
@@ -407,10 +436,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     const uint32_t tmem_base = *s.tmem_slot;
 
     if (warp == 0) {
-        if (lane == 0) producer(p, s);
+        if (lane == 0) producer<C>(p, s);
         __syncwarp();
     } else if (warp == 1) {
-        if (lane == 0) mma_issuer<BF16>(p, s, tmem_base);
+        if (lane == 0) mma_issuer<BF16, C>(p, s, tmem_base);
         __syncwarp();
     } else {
         epilogue<BF16>(p, s, tmem_base, warp, lane);
@@ -423,27 +452,27 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     }
 }
 
-}  // namespace
+template <bool BF16, class C>
+cudaError_t launch_cfg(const GemmLaunch& p, int grid, cudaStream_t st) {
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<BF16, C>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             int(C::kSmemBytes));
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    tc_gemm_kernel<BF16, C><<<grid, kThreads, C::kSmemBytes, st>>>(p);
+    return cudaGetLastError();
+}
 
-int tc_smem_bytes() { return int(kSmemBytes); }
+}  // namespace
 
 cudaError_t launch_gemm_tc(const GemmLaunch& p, int elem, int grid, cudaStream_t st) {
     if (p.num_items == 0) return cudaSuccess;
-    static bool attr_set[2] = {false, false};
-    const int which = elem == kBF16 ? 1 : 0;
-    cudaError_t e;
-    if (!attr_set[which]) {
-        e = which ? cudaFuncSetAttribute(tc_gemm_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kSmemBytes))
-                  : cudaFuncSetAttribute(tc_gemm_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, int(kSmemBytes));
-        if (e != cudaSuccess) return e;
-        attr_set[which] = true;
-    }
     if (grid > p.num_items) grid = p.num_items;
-    if (which)
-        tc_gemm_kernel<true><<<grid, kThreads, kSmemBytes, st>>>(p);
-    else
-        tc_gemm_kernel<false><<<grid, kThreads, kSmemBytes, st>>>(p);
-    return cudaGetLastError();
+    const bool bf = elem == kBF16;
+    if (p.bk == 32) return bf ? launch_cfg<true, Cfg32>(p, grid, st) : launch_cfg<false, Cfg32>(p, grid, st);
+    return bf ? launch_cfg<true, Cfg64>(p, grid, st) : launch_cfg<false, Cfg64>(p, grid, st);
 }
 
 }  // namespace slorr

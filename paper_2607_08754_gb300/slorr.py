@@ -26,6 +26,7 @@ COMPUTES = {"fp16": 0, "bf16": 1, "fp32": 2}
 DTYPES = {"f32": 0, "bf16": 1}
 FLAG_SIMT_GEMM = 1
 FLAG_L2_PREFETCH = 2
+FLAG_TC_BK32 = 4
 
 
 class SlorrError(RuntimeError):

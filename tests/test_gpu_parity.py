@@ -147,13 +147,14 @@ def test_decoder_560m_layer_fp16():
 
 # ---- tensor cores vs CUDA cores on the same 16-bit arithmetic -------------------
 
-@pytest.mark.parametrize("compute", ["fp16", "bf16"])
-def test_tensor_core_iterates_match_simt(compute):
+@pytest.mark.parametrize("compute,flags", [("fp16", 0), ("bf16", 0), ("fp16", 4)])
+def test_tensor_core_iterates_match_simt(compute, flags):
+    """flags 4 = SLORR_FLAG_TC_BK32 (the 9-stage, 64-byte-swizzle pipeline)."""
     from paper_2607_08754_gb300.slorr import Regularizer, FLAG_SIMT_GEMM
     shapes = [(256, 768), (768, 256), (320, 1280), (384, 384)]
     Ws = [workloads.random_matrix(s, seed=70 + i, std=0.02) for i, s in enumerate(shapes)]
     w = [torch.from_numpy(W).cuda() for W in Ws]
-    tc = Regularizer(shapes, compute=compute)
+    tc = Regularizer(shapes, compute=compute, flags=flags)
     st = Regularizer(shapes, compute=compute, flags=FLAG_SIMT_GEMM)
     ulp = 2.0 ** -10 if compute == "fp16" else 2.0 ** -7
     for k in (1, 2, 6):
