@@ -98,6 +98,11 @@ typedef struct slorr_options {
 #define SLORR_FLAG_SIMT_GEMM    1   /* run the 16-bit products on CUDA cores (debug)  */
 #define SLORR_FLAG_L2_PREFETCH  2   /* tensor-core producer also warms L2 ahead (tuning) */
 #define SLORR_FLAG_TC_BK32      4   /* 9 stages of K = 32 instead of 4 of K = 64 (tuning) */
+#define SLORR_FLAG_TC_M128      8   /* 128 x 256 tensor-core tiles in every phase (tuning) */
+#define SLORR_FLAG_TEST_STALL  16   /* test only: every tensor-core CTA first waits on a
+                                       barrier nothing arrives on, so its bounded wait
+                                       runs out after timeout_s and the call reports
+                                       SLORR_ERR_TIMEOUT (failure-detection test)     */
 
 /* Fill *opt with the defaults listed beside each field above (App. C.1: T = 6,
  * ell = 1e-3, degree 5; eps, lambda and grad_scale as in Listing 1 / Alg. 2). */

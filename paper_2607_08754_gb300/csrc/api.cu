@@ -87,6 +87,19 @@ struct slorr_handle {
 
 namespace {
 
+// K depth of the tensor-core pipeline stages for this handle.
+int tc_bk(const slorr_handle* h) { return (h->opt.flags & SLORR_FLAG_TC_BK32) ? 32 : 64; }
+
+// 128-row M tiles per tensor-core CTA tile for one phase.  256 x 256 tiles
+// (mt = 2) move a third fewer operand rows per FLOP but cannot overlap a
+// tile's epilogue with the next main loop; they win for the long-K Gram and
+// the store-only Update, while the short-K Poly, whose epilogue also reads A,
+// keeps double-buffered 128 x 256 tiles.
+int tc_mt(const slorr_handle* h, int phase) {
+    if (h->opt.flags & (SLORR_FLAG_TC_M128 | SLORR_FLAG_TC_BK32)) return 1;
+    return phase == kPoly ? 1 : 2;
+}
+
 bool valid_options(const slorr_options& o, std::string* why) {
     if (o.variant != SLORR_HOYER && o.variant != SLORR_NUCLEAR) return *why = "variant", false;
     if (o.compute < SLORR_COMPUTE_FP16 || o.compute > SLORR_COMPUTE_FP32) return *why = "compute", false;
@@ -134,20 +147,25 @@ void build_plan(slorr_handle* h) {
         for (int r = 0; r < (g.rows + kMemRows - 1) / kMemRows; ++r)
             for (int c = 0; c < (g.ld + kMemCols - 1) / kMemCols; ++c)
                 h->x_items.push_back(MemItem{uint16_t(i), uint16_t(r), uint16_t(c), 0});
-        // tensor-core tiles: 128 x nsz, nsz <= 256.  The Gram and Poly outputs
-        // are symmetric: tiles lying strictly below the diagonal (in 128 x 128
-        // blocks) are skipped; the kernel mirrors the blocks they need.
+        // tensor-core tiles: msz x nsz with msz <= 128 mt, nsz <= 256.  The Gram
+        // and Poly outputs are symmetric: tiles lying strictly below the
+        // diagonal (in 128 x 128 blocks) are skipped; the kernel mirrors the
+        // blocks they need.
         for (int ph = 0; ph < 3; ++ph) {
+            const int mt = tc_mt(h, ph);
             const int N = ph == kUpdate ? g.Qpad : g.Ppad;
-            for (int tm = 0; tm < g.Ppad / 128; ++tm)
+            for (int tm = 0; tm * 128 * mt < g.Ppad; ++tm) {
+                const int msz = std::min(128 * mt, g.Ppad - tm * 128 * mt);
                 for (int tn = 0; tn * 256 < N; ++tn) {
                     const int nsz = std::min(256, N - tn * 256);
-                    if (ph != kUpdate && (2 * tn + nsz / 128 - 1) < tm) continue;
-                    h->tc_items[ph].push_back(GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), uint16_t(nsz)});
+                    if (ph != kUpdate && (2 * tn + nsz / 128 - 1) < tm * mt) continue;
+                    h->tc_items[ph].push_back(
+                        GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), uint16_t(nsz), uint16_t(msz), 0});
                 }
+            }
             for (int tm = 0; tm < g.Ppad / 64; ++tm)
                 for (int tn = 0; tn < N / 64; ++tn)
-                    h->simt_items[ph].push_back(GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), 64});
+                    h->simt_items[ph].push_back(GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), 64, 64, 0});
         }
     }
     h->total_w_tiles = tile_base;
@@ -207,9 +225,6 @@ void build_plan(slorr_handle* h) {
     }
     h->total_bytes = off;
 }
-
-// K depth of the tensor-core pipeline stages for this handle.
-int tc_bk(const slorr_handle* h) { return (h->opt.flags & SLORR_FLAG_TC_BK32) ? 32 : 64; }
 
 PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -447,6 +462,7 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
     g.timeout_ns = static_cast<unsigned long long>(h->opt.timeout_s * 1e9);
     g.prefetch = (h->opt.flags & SLORR_FLAG_L2_PREFETCH) ? 8 : 0;
     g.bk = tc_bk(h);
+    g.test_stall = (h->opt.flags & SLORR_FLAG_TEST_STALL) ? 1 : 0;
     for (int t = 0; t < steps; ++t) {
         g.cur = t & 1;
         g.a = float(h->coeffs[3 * t + 0]);
@@ -454,6 +470,7 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
         g.c = float(h->coeffs[3 * t + 2]);
         for (int ph = 0; ph < 3; ++ph) {
             g.phase = ph;
+            g.mt = tc_mt(h, ph);
             Traced tr(h, 2 + ph, st);
             if (use_tc) {
                 g.items = reinterpret_cast<const GemmItem*>(ws + h->off_tc_items[ph]);

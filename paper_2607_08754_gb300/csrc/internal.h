@@ -59,9 +59,11 @@ struct MatScalars {
 // One output tile of a grouped GEMM phase.
 struct GemmItem {
     uint16_t mat;
-    uint16_t tm;       // row tile index (tile rows = 128 for tcgen05, 64 for SIMT)
-    uint16_t tn;       // column tile index
+    uint16_t tm;       // row tile index (128 x mt rows per tcgen05 tile, 64 for SIMT)
+    uint16_t tn;       // column tile index (256 columns per tcgen05 tile, 64 for SIMT)
     uint16_t nsz;      // columns in this tile
+    uint16_t msz;      // rows in this tile
+    uint16_t pad_;
 };
 
 // One chunk of a memory-bound pass: a kMemRows x kMemCols tile of W (or of
@@ -92,6 +94,8 @@ struct GemmLaunch {
     unsigned long long timeout_ns;
     int32_t prefetch;          // k blocks of L2 prefetch lookahead (0 = off)
     int32_t bk;                // K depth of a pipeline stage: 64 (4 stages) or 32 (9 stages)
+    int32_t mt;                // 128-row M tiles per CTA tile: 1 or 2 (256 x 256 tiles)
+    int32_t test_stall;        // 1: the MMA thread first waits on a barrier nothing arrives on
 };
 
 // Tensor maps per matrix: X0 K-major, X1 K-major, X0 MN-major, X1 MN-major,

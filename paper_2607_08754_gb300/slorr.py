@@ -27,6 +27,8 @@ DTYPES = {"f32": 0, "bf16": 1}
 FLAG_SIMT_GEMM = 1
 FLAG_L2_PREFETCH = 2
 FLAG_TC_BK32 = 4
+FLAG_TC_M128 = 8
+FLAG_TEST_STALL = 16
 
 
 class SlorrError(RuntimeError):

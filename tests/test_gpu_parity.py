@@ -147,11 +147,13 @@ def test_decoder_560m_layer_fp16():
 
 # ---- tensor cores vs CUDA cores on the same 16-bit arithmetic -------------------
 
-@pytest.mark.parametrize("compute,flags", [("fp16", 0), ("bf16", 0), ("fp16", 4)])
+@pytest.mark.parametrize("compute,flags", [("fp16", 0), ("bf16", 0), ("fp16", 4), ("fp16", 8), ("bf16", 8)])
 def test_tensor_core_iterates_match_simt(compute, flags):
-    """flags 4 = SLORR_FLAG_TC_BK32 (the 9-stage, 64-byte-swizzle pipeline)."""
+    """Default tiles (256 x 256 for Gram/Update, 128 x 256 for Poly); flags 4 =
+    SLORR_FLAG_TC_BK32 (9-stage, 64-byte-swizzle pipeline); 8 =
+    SLORR_FLAG_TC_M128 (128 x 256 tiles everywhere)."""
     from paper_2607_08754_gb300.slorr import Regularizer, FLAG_SIMT_GEMM
-    shapes = [(256, 768), (768, 256), (320, 1280), (384, 384)]
+    shapes = [(256, 768), (768, 256), (320, 1280), (384, 384), (640, 1000)]
     Ws = [workloads.random_matrix(s, seed=70 + i, std=0.02) for i, s in enumerate(shapes)]
     w = [torch.from_numpy(W).cuda() for W in Ws]
     tc = Regularizer(shapes, compute=compute, flags=flags)
@@ -236,3 +238,21 @@ def test_vit_l16_full_size_sampled():
         L, G, _, _ = oracle.reg_single(W, "hoyer", co, EPS)
         assert abs(per[i] - L) <= 2e-2 * L
         assert rel(g[i].double().cpu().numpy(), G) <= 2e-2
+
+
+# ---- failure detection: a bounded device wait runs out -----------------------------
+
+def test_bounded_wait_timeout_reports_status_and_context_survives():
+    """SLORR_FLAG_TEST_STALL makes every tensor-core CTA wait on a barrier nothing
+    arrives on; with timeout_s = 0.05 each wait gives up, the kernel records
+    SLORR_ERR_TIMEOUT in the status word, drains and returns.  The same process
+    then runs a normal call that must still match the oracle."""
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_TEST_STALL
+    Ws = [workloads.random_matrix((256, 512), 21, 0.05), workloads.random_matrix((384, 128), 22, 0.05)]
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    stall = Regularizer([W.shape for W in Ws], flags=FLAG_TEST_STALL, timeout_s=0.05)
+    stall.run_steps(w, 1)
+    torch.cuda.synchronize()
+    assert stall.status() == 5          # SLORR_ERR_TIMEOUT
+    assert stall.status() == 0          # reading clears it
+    check(Ws, "hoyer", "fp16")          # the context is still usable
