@@ -103,6 +103,10 @@ typedef struct slorr_options {
                                        barrier nothing arrives on, so its bounded wait
                                        runs out after timeout_s and the call reports
                                        SLORR_ERR_TIMEOUT (failure-detection test)     */
+#define SLORR_FLAG_WRITE_GRAD  32   /* grads[i] = lambda * grad_scale * G_i instead of +=:
+                                       the pre-update gradient of the decoupled variant
+                                       (Alg. 1, App. C.2), applied by the caller as
+                                       W -= lr * grads[i] after its optimizer step      */
 
 /* Fill *opt with the defaults listed beside each field above (App. C.1: T = 6,
  * ell = 1e-3, degree 5; eps, lambda and grad_scale as in Listing 1 / Alg. 2). */

@@ -401,6 +401,7 @@ MemLaunch mem_params(slorr_handle* h, uint8_t* ws, float* loss, float* per, int 
     p.elem = h->elem;
     p.wdtype = h->opt.dtype == SLORR_BF16 ? 1 : 0;
     p.variant = h->opt.variant;
+    p.overwrite = (h->opt.flags & SLORR_FLAG_WRITE_GRAD) ? 1 : 0;
     p.eps = h->opt.eps;
     p.lambda = h->opt.lambda;
     p.grad_scale = h->opt.grad_scale;

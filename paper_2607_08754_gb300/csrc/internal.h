@@ -117,6 +117,7 @@ struct MemLaunch {
     int32_t elem;              // Elem of the iterate
     int32_t wdtype;            // 0 fp32, 1 bf16 weights/grads
     int32_t variant;           // 0 Hoyer, 1 Nuc
+    int32_t overwrite;         // 1: grad = lambda grad_scale G (Alg. 1 output), 0: grad +=
     float eps, lambda, grad_scale;
     float* loss_out;
     float* per_matrix_out;

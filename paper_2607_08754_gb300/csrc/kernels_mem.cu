@@ -4,6 +4,9 @@
 //   dot     n_hat_i = sum(W_i * P_hat_i), values L_i and the loss
 //                                                        (Sec. 3 "Computing the nuclear ...", Listing 1)
 //   combine W_i.grad += lambda * grad_scale * G_i       (Listing 1 backward, Alg. 2)
+//           or, in overwrite mode, out_i = lambda * grad_scale * G_i, the
+//           pre-update gradient Alg. 1 (decoupled SLORR) applies after the
+//           optimizer step
 // The iterates are stored in W's orientation (row-major, row length `ld`), so
 // every pass is elementwise.  A block handles one kMemRows x kMemCols tile:
 // each of its 256 threads owns 8 consecutive columns of 4 rows and issues all
@@ -357,7 +360,7 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const MemLaunch p) {
     for (int k = 0; k < kPasses; ++k) {
         const int r = tc.r0 + k * kRowsPerPass;
         w[k] = load_w8<TW>(W, md.m, md.n, r, tc.c, vec);
-        g[k] = load_w8<TW>(G, md.m, md.n, r, tc.c, vec);
+        g[k] = p.overwrite ? zero8() : load_w8<TW>(G, md.m, md.n, r, tc.c, vec);
         x[k] = r < md.m ? load_x8<TX>(X, int64_t(r) * md.ld + tc.c) : zero8();
     }
 #pragma unroll

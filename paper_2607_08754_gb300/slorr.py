@@ -29,6 +29,7 @@ FLAG_L2_PREFETCH = 2
 FLAG_TC_BK32 = 4
 FLAG_TC_M128 = 8
 FLAG_TEST_STALL = 16
+FLAG_WRITE_GRAD = 32
 
 
 class SlorrError(RuntimeError):

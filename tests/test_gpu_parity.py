@@ -256,3 +256,64 @@ def test_bounded_wait_timeout_reports_status_and_context_survives():
     assert stall.status() == 5          # SLORR_ERR_TIMEOUT
     assert stall.status() == 0          # reading clears it
     check(Ws, "hoyer", "fp16")          # the context is still usable
+
+
+# ---- decoupled variant (Alg. 1): write the pre-update gradient --------------------
+
+@pytest.mark.parametrize("variant", ["hoyer", "nuclear"])
+def test_write_grad_mode_matches_oracle_and_decoupled_step(variant):
+    """SLORR_FLAG_WRITE_GRAD overwrites the output with lambda * G_i (Alg. 1's
+    G_pre); the caller's decoupled step W <- W - lr * G_pre then matches the
+    oracle's."""
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_WRITE_GRAD
+    Ws = workloads.generate("vit_b16", range(4))
+    lam, lr = 0.002, 0.1
+    reg = Regularizer([W.shape for W in Ws], variant=variant, lam=lam, flags=FLAG_WRITE_GRAD)
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    out = [torch.full_like(x, 7.0) for x in w]         # garbage that must be overwritten
+    reg(w, out)
+    torch.cuda.synchronize()
+    assert reg.status() == 0
+    co = oracle.pe_coefficients(6)
+    _, _, ref = oracle.reg_forward_backward([W.astype(np.float64) for W in Ws], variant, co, lam)
+    for i, W in enumerate(Ws):
+        got = out[i].double().cpu().numpy()
+        assert grad_err(got, ref[i], W.astype(np.float64), variant, lam, 1.0) <= 2e-2
+        w_new = W.astype(np.float64) - lr * got
+        w_ref = W.astype(np.float64) - lr * ref[i]
+        assert np.linalg.norm(w_new - w_ref) <= 2e-2 * lr * np.linalg.norm(ref[i])
+
+
+# ---- T sweep and the ViT scaling ladder (next rows of the hot-path scope) --------
+
+@pytest.mark.parametrize("T", [1, 2, 4, 8, 10])
+def test_iteration_count_sweep(T):
+    Ws = [workloads.random_matrix(s, seed=300 + i, std=0.03) for i, s in enumerate([(256, 640), (640, 384)])]
+    check(Ws, "hoyer", "fp16", iters=T)
+    check(Ws, "hoyer", "fp32", iters=T)
+
+
+@pytest.mark.parametrize("name", ["vit_ladder_vit_ti", "vit_ladder_vit_256", "vit_ladder_vit_s"])
+def test_vit_ladder_small_sets(name):
+    check(workloads.generate(name), "hoyer", "fp16")
+
+
+def test_vit_ladder_vit_h_sampled():
+    from paper_2607_08754_gb300.slorr import Regularizer
+    name = "vit_ladder_vit_h"
+    shapes = workloads.shapes(name)
+    reg = Regularizer(shapes, compute="fp16")
+    w = [torch.from_numpy(workloads.generate_one(name, i)).cuda() for i in range(len(shapes))]
+    g = [torch.zeros_like(x) for x in w]
+    per = torch.empty(len(shapes), device="cuda")
+    loss = reg(w, g, per_matrix=per).item()
+    torch.cuda.synchronize()
+    assert reg.status() == 0
+    per = per.double().cpu().numpy()
+    assert loss == pytest.approx(per.sum(), rel=1e-6)
+    co = oracle.pe_coefficients(6)
+    for i in (0, 3, 125):
+        W = workloads.generate_one(name, i).astype(np.float64)
+        L, G, _, _ = oracle.reg_single(W, "hoyer", co, EPS)
+        assert abs(per[i] - L) <= 2e-2 * L
+        assert rel(g[i].double().cpu().numpy(), G) <= 2e-2

@@ -25,6 +25,12 @@ Shapes (conv kernels use the (C_out, C_in*k*k) view of App. D.1):
                     o 1280x1280, gate 3456x1280, up 3456x1280, down 1280x3456},
                     N(0, 0.02^2) (GQA, 20 query / 5 key-value heads of dim 64).
 * ``decoder_560m_mha``  the same with k, v 1280x1280 (multi-head attention).
+* ``vit_ladder_<name>``  the ViT scaling ladder of the paper's ViT configuration
+                    table (appendix "Scaling Up with Vision Transformers"):
+                    embed dim d and depth of vit_ti 192x12, vit_256 256x12,
+                    vit_s 384x12, vit_512 512x12, vit_b 768x12, vit_b24 768x24,
+                    vit_960_24 960x24, vit_l 1024x24, vit_1152_28 1152x28,
+                    vit_h 1280x32; MLP ratio 4; blocks as for ``vit_b16``.
 
 Matrix i of weight set number c (the order of ``WEIGHT_SETS``) is drawn in
 fp64 from ``numpy.random.default_rng(1000 * c + i)`` and rounded to fp32.
@@ -81,6 +87,13 @@ WEIGHT_SETS = {
     "decoder_560m": _decoder(24, 1280, 320, 3456),
     "decoder_560m_mha": _decoder(24, 1280, 1280, 3456),
 }
+
+# ViT scaling ladder (appended: the seeds of the sets above are unchanged).
+VIT_LADDER = [("vit_ti", 192, 12), ("vit_256", 256, 12), ("vit_s", 384, 12), ("vit_512", 512, 12),
+              ("vit_b", 768, 12), ("vit_b24", 768, 24), ("vit_960_24", 960, 24), ("vit_l", 1024, 24),
+              ("vit_1152_28", 1152, 28), ("vit_h", 1280, 32)]
+for _name, _d, _depth in VIT_LADDER:
+    WEIGHT_SETS["vit_ladder_" + _name] = _vit(_depth, _d, 4 * _d)
 
 SET_INDEX = {name: i for i, name in enumerate(WEIGHT_SETS)}
 
