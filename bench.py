@@ -3,6 +3,7 @@ over a whole weight set, Listing 1 / Alg. 2) on GB300.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload vit_l16]
                   [--variant hoyer|nuclear] [--compute fp16|bf16|fp32] [--impl ours|reference]
+                  [--iters T] [--op fwd_bwd|descent] [--eta ETA] [--flags F]
 
 A step is one slorr_reg_forward_backward call over the whole weight set
 (norm, cast, T = 6 Polar Express steps of three grouped GEMMs, dot, combine).
@@ -20,6 +21,8 @@ bounded sample of the same workload on this host's cores.
 With --gpus N > 1 (launched by torchrun) every rank regularizes its own full
 copy of the weight set (weak scaling, no collective on the data path); the
 time is the max over ranks.  --impl reference times the oracle instead.
+--op descent times slorr_reg_descent_step instead (the in-place regularizer-only
+step W -= eta lambda G of Alg. 1's last line; e2e then copies W in and out).
 """
 
 from __future__ import annotations
@@ -60,6 +63,10 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--flags", type=int, default=0, help="slorr_options.flags (tuning / debug)")
+    ap.add_argument("--op", default="fwd_bwd", choices=["fwd_bwd", "descent"],
+                    help="fwd_bwd: value + gradient accumulated into .grad (Alg. 2); descent: the in-place "
+                         "regularizer-only step W -= eta lambda G (Alg. 1, last line)")
+    ap.add_argument("--eta", type=float, default=1e-4, help="step size of --op descent")
     return ap.parse_args()
 
 
@@ -241,9 +248,17 @@ def main():
             dist.barrier()
         torch.cuda.synchronize(dev)
 
+    descent = args.op == "descent"
+
+    def step(w, g):
+        if descent:
+            reg.descent_step(w, args.eta, loss=loss)
+        else:
+            reg(w, g, loss=loss)
+
     # warm-up
     for _ in range(max(args.warmup, 3)):
-        reg(W, G, loss=loss)
+        step(W, G)
     barrier()
     assert reg.status() == 0, "device status word reports an error after warm-up"
 
@@ -257,7 +272,7 @@ def main():
     t1 = torch.cuda.Event(enable_timing=True)
     t0.record(stream)
     for _ in range(args.steps):
-        reg(W, G, loss=loss)
+        step(W, G)
     t1.record(stream)
     barrier()
     clk = clocks.stop()
@@ -277,16 +292,21 @@ def main():
     Lp = torch.zeros(1, dtype=torch.float32).pin_memory()
     Wd = [torch.empty_like(w) for w in W]
     Gd = [torch.empty_like(w) for w in W]
-    h2d = sum(w.numel() * w.element_size() for w in Wp) + sum(g.numel() * g.element_size() for g in Gp)
-    d2h = sum(g.numel() * g.element_size() for g in Gp) + 4
+    wbytes = sum(w.numel() * w.element_size() for w in Wp)
+    gbytes = 0 if descent else sum(g.numel() * g.element_size() for g in Gp)
+    h2d = wbytes + gbytes
+    d2h = (wbytes if descent else gbytes) + 4
 
     def e2e_step():
+        # inputs in (W, and .grad unless descending), the result out (the updated
+        # W or .grad) and the loss
         for d, h in zip(Wd, Wp):
             d.copy_(h, non_blocking=True)
-        for d, h in zip(Gd, Gp):
-            d.copy_(h, non_blocking=True)
-        reg(Wd, Gd, loss=loss)
-        for d, h in zip(Gp, Gd):
+        if not descent:
+            for d, h in zip(Gd, Gp):
+                d.copy_(h, non_blocking=True)
+        step(Wd, Gd)
+        for d, h in zip(Wp if descent else Gp, Wd if descent else Gd):
             d.copy_(h, non_blocking=True)
         Lp.copy_(loss, non_blocking=True)
 
@@ -322,9 +342,10 @@ def main():
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f16" if args.compute == "fp16" else args.compute,
             "data": "synthetic",
-            "config": {"workload": f"{name} {args.variant}: {len(shapes)} matrices, T={args.iters}, "
+            "config": {"workload": f"{name} {args.variant}{' descent step' if descent else ''}: "
+                                   f"{len(shapes)} matrices, T={args.iters}, "
                                    f"{args.compute} operands / fp32 accumulate, fp32 weights and grads",
-                       "matrices": len(shapes), "iters": args.iters, "variant": args.variant,
+                       "matrices": len(shapes), "iters": args.iters, "variant": args.variant, "op": args.op,
                        "gflop_per_step": flops_step / 1e9,
                        "l2": "inputs larger than L2 (fp32 weights %.2f GB)" %
                              (sum(w.numel() for w in W) * 4 / 1e9)},

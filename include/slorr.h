@@ -142,6 +142,26 @@ SLORR_API slorr_status slorr_reg_forward_backward(slorr_handle* h, const void* c
                                         float* per_matrix_out, void* workspace,
                                         size_t workspace_bytes, void* stream);
 
+/* One regularizer-only gradient descent step, in place, over the whole weight
+ * set:  W_i <- W_i - eta * lambda * grad_scale * G_i(W_i),  with G_i the same
+ * Polar Express gradient slorr_reg_forward_backward produces (Eq. 1).  It is the
+ * last line of Alg. 1 (App. C.2, decoupled SLORR: W -= eta lambda G_pre) with
+ * no task update in between, i.e. the "regularizer-only gradient step" of
+ * Props. 2 and 3 (Sec. 3.1).  The gradient pass reads each W_i once and writes
+ * it back; no grad buffer is involved, and SLORR_FLAG_WRITE_GRAD is ignored.
+ *   weights[i]      device pointer to W_i, row-major m_i x n_i, 16-byte
+ *                   aligned; READ AND OVERWRITTEN
+ *   eta             step size (finite; eta * lambda * grad_scale must be finite)
+ *   loss_out        device pointer to 1 float: lambda * sum_i L_i at the
+ *                   weights BEFORE the step
+ *   per_matrix_out, workspace, workspace_bytes, stream: as for
+ *                   slorr_reg_forward_backward
+ * A matrix whose norm or estimate is non-finite is left unchanged and the
+ * status word records SLORR_ERR_NONFINITE.  Asynchronous. */
+SLORR_API slorr_status slorr_reg_descent_step(slorr_handle* h, void* const* weights, float eta,
+                                    float* loss_out, float* per_matrix_out, void* workspace,
+                                    size_t workspace_bytes, void* stream);
+
 /* Forget which workspace holds the plan; the next call re-writes it. */
 SLORR_API slorr_status slorr_reset_workspace(slorr_handle* h);
 

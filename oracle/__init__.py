@@ -10,6 +10,9 @@ computes, written from the paper (SLORR, arXiv 2607.08754):
   SLORR-Hoyer and SLORR-Nuc (Sec. 3 problem statement and Eq. 1, Listing 1,
   Alg. 2), the exact SVD-based quantities, and the FLOP model of Sec. 3
   "Computational cost".
+* ``descent``        -- the regularizer-only descent step (last line of Alg. 1
+  with no task update; the setting of Props. 2 and 3) and the retained-energy
+  metric E(P) and rank P* of App. D.4.
 * ``svd_jacobi``     -- an independent one-sided Jacobi SVD used only as a
   brute-force second opinion on tiny inputs.
 
@@ -44,4 +47,12 @@ from .slorr import (  # noqa: F401
     exact_grad,
     pe_flops,
     weight_set_flops,
+)
+from .descent import (  # noqa: F401
+    descent_step,
+    descent_trajectory,
+    singular_values,
+    hoyer_tau,
+    energy,
+    energy_rank,
 )

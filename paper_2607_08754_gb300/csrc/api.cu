@@ -401,7 +401,7 @@ MemLaunch mem_params(slorr_handle* h, uint8_t* ws, float* loss, float* per, int 
     p.elem = h->elem;
     p.wdtype = h->opt.dtype == SLORR_BF16 ? 1 : 0;
     p.variant = h->opt.variant;
-    p.overwrite = (h->opt.flags & SLORR_FLAG_WRITE_GRAD) ? 1 : 0;
+    p.out_mode = (h->opt.flags & SLORR_FLAG_WRITE_GRAD) ? kOutOverwrite : kOutAccumulate;
     p.eps = h->opt.eps;
     p.lambda = h->opt.lambda;
     p.grad_scale = h->opt.grad_scale;
@@ -412,17 +412,29 @@ MemLaunch mem_params(slorr_handle* h, uint8_t* ws, float* loss, float* per, int 
     return p;
 }
 
+// descent: grads is NULL and the combine pass applies W -= eta * lambda *
+// grad_scale * G in place (the weights are then written, through a non-const
+// pointer the caller gave slorr_reg_descent_step).
 slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads, float* loss, float* per,
-                 void* workspace, size_t ws_bytes, int steps, bool finish, cudaStream_t st) {
+                 void* workspace, size_t ws_bytes, int steps, bool finish, cudaStream_t st,
+                 bool descent = false, float eta = 0.f) {
     if (!h) return fail(SLORR_ERR_INVALID_ARG, "handle is NULL");
     slorr_status s = check_matrix_ptrs(h, weights, "weight");
     if (s != SLORR_OK) return s;
+    if (descent) {
+        if (!std::isfinite(eta)) return fail(SLORR_ERR_INVALID_ARG, "eta must be finite");
+        if (!std::isfinite(eta * h->opt.lambda * h->opt.grad_scale))
+            return fail(SLORR_ERR_INVALID_ARG, "eta * lambda * grad_scale overflows");
+        grads = const_cast<void* const*>(weights);
+    }
     if (finish) {
-        s = check_matrix_ptrs(h, grads, "grad");
-        if (s != SLORR_OK) return s;
         if (!loss) return fail(SLORR_ERR_INVALID_ARG, "loss_out is NULL");
-        for (size_t i = 0; i < h->shapes.size(); ++i)
-            if (grads[i] == weights[i]) return fail(SLORR_ERR_INVALID_ARG, "a grad aliases its weight");
+        if (!descent) {
+            s = check_matrix_ptrs(h, grads, "grad");
+            if (s != SLORR_OK) return s;
+            for (size_t i = 0; i < h->shapes.size(); ++i)
+                if (grads[i] == weights[i]) return fail(SLORR_ERR_INVALID_ARG, "a grad aliases its weight");
+        }
     }
     if (!workspace) return fail(SLORR_ERR_WORKSPACE, "workspace is NULL");
     if (reinterpret_cast<uintptr_t>(workspace) % 256 != 0)
@@ -488,6 +500,10 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
     }
     if (!finish) return SLORR_OK;
     MemLaunch dp = mem_params(h, ws, loss, per, steps & 1);
+    if (descent) {
+        dp.out_mode = kOutDescent;
+        dp.grad_scale = -eta * h->opt.grad_scale;  // alpha, beta then carry -eta * lambda * grad_scale
+    }
     dp.items = reinterpret_cast<const MemItem*>(ws + h->off_w_items);
     dp.num_items = int(h->w_items.size());
     {
@@ -572,6 +588,14 @@ slorr_status slorr_reg_forward_backward(slorr_handle* h, const void* const* weig
     if (!h) return fail(SLORR_ERR_INVALID_ARG, "handle is NULL");
     return run(h, weights, grads, loss_out, per_matrix_out, workspace, workspace_bytes, h->opt.iters, true,
                static_cast<cudaStream_t>(stream));
+}
+
+slorr_status slorr_reg_descent_step(slorr_handle* h, void* const* weights, float eta, float* loss_out,
+                                    float* per_matrix_out, void* workspace, size_t workspace_bytes,
+                                    void* stream) {
+    if (!h) return fail(SLORR_ERR_INVALID_ARG, "handle is NULL");
+    return run(h, const_cast<const void* const*>(weights), nullptr, loss_out, per_matrix_out, workspace,
+               workspace_bytes, h->opt.iters, true, static_cast<cudaStream_t>(stream), true, eta);
 }
 
 slorr_status slorr_reset_workspace(slorr_handle* h) {

@@ -102,6 +102,13 @@ struct GemmLaunch {
 // A K-major, M K-major.
 constexpr int kMapsPerMatrix = 6;
 
+// Where the combine pass puts lambda * grad_scale * G_i.
+enum OutMode : int32_t {
+    kOutAccumulate = 0,  // grads[i] += (Listing 1 backward, Alg. 2)
+    kOutOverwrite = 1,   // grads[i] =  (the pre-update gradient of Alg. 1)
+    kOutDescent = 2,     // weights[i] += (grad_scale already holds -eta * grad_scale), in place
+};
+
 struct MemLaunch {
     const MemItem* items;
     int32_t num_items;
@@ -117,7 +124,7 @@ struct MemLaunch {
     int32_t elem;              // Elem of the iterate
     int32_t wdtype;            // 0 fp32, 1 bf16 weights/grads
     int32_t variant;           // 0 Hoyer, 1 Nuc
-    int32_t overwrite;         // 1: grad = lambda grad_scale G (Alg. 1 output), 0: grad +=
+    int32_t out_mode;          // kOutAccumulate, kOutOverwrite or kOutDescent
     float eps, lambda, grad_scale;
     float* loss_out;
     float* per_matrix_out;

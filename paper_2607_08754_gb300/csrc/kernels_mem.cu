@@ -6,7 +6,9 @@
 //   combine W_i.grad += lambda * grad_scale * G_i       (Listing 1 backward, Alg. 2)
 //           or, in overwrite mode, out_i = lambda * grad_scale * G_i, the
 //           pre-update gradient Alg. 1 (decoupled SLORR) applies after the
-//           optimizer step
+//           optimizer step, or, in descent mode, W_i -= eta * lambda *
+//           grad_scale * G_i in place (the last line of Alg. 1 with no task
+//           update in between: the regularizer-only step of Props. 2 and 3)
 // The iterates are stored in W's orientation (row-major, row length `ld`), so
 // every pass is elementwise.  A block handles one kMemRows x kMemCols tile:
 // each of its 256 threads owns 8 consecutive columns of 4 rows and issues all
@@ -360,7 +362,12 @@ __global__ void __launch_bounds__(kThreads) combine_kernel(const MemLaunch p) {
     for (int k = 0; k < kPasses; ++k) {
         const int r = tc.r0 + k * kRowsPerPass;
         w[k] = load_w8<TW>(W, md.m, md.n, r, tc.c, vec);
-        g[k] = p.overwrite ? zero8() : load_w8<TW>(G, md.m, md.n, r, tc.c, vec);
+        if (p.out_mode == kOutAccumulate)
+            g[k] = load_w8<TW>(G, md.m, md.n, r, tc.c, vec);
+        else if (p.out_mode == kOutDescent)
+            g[k] = w[k];  // G points at W itself: the step is applied in place
+        else
+            g[k] = zero8();
         x[k] = r < md.m ? load_x8<TX>(X, int64_t(r) * md.ld + tc.c) : zero8();
     }
 #pragma unroll

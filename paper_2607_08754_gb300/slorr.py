@@ -74,6 +74,8 @@ def load_library(path: str | None = None) -> ctypes.CDLL:
         "slorr_workspace_size": (i32, [vp, ctypes.POINTER(ctypes.c_size_t)]),
         "slorr_reg_forward_backward": (i32, [vp, ctypes.POINTER(vp), ctypes.POINTER(vp), vp, vp, vp,
                                              ctypes.c_size_t, vp]),
+        "slorr_reg_descent_step": (i32, [vp, ctypes.POINTER(vp), ctypes.c_float, vp, vp, vp, ctypes.c_size_t,
+                                         vp]),
         "slorr_reset_workspace": (i32, [vp]),
         "slorr_get_status": (i32, [vp, vp, vp]),
         "slorr_run_steps": (i32, [vp, ctypes.POINTER(vp), vp, ctypes.c_size_t, i32, vp]),
@@ -149,6 +151,13 @@ def slorr_reg_forward_backward(handle, weight_ptrs, grad_ptrs, loss_ptr, per_mat
         handle, _ptr_array(weight_ptrs), _ptr_array(grad_ptrs), ctypes.c_void_p(loss_ptr),
         ctypes.c_void_p(per_matrix_ptr or 0), ctypes.c_void_p(workspace_ptr), workspace_bytes,
         ctypes.c_void_p(stream or 0)))
+
+
+def slorr_reg_descent_step(handle, weight_ptrs, eta, loss_ptr, per_matrix_ptr, workspace_ptr, workspace_bytes,
+                           stream) -> None:
+    _check(load_library().slorr_reg_descent_step(
+        handle, _ptr_array(weight_ptrs), float(eta), ctypes.c_void_p(loss_ptr), ctypes.c_void_p(per_matrix_ptr or 0),
+        ctypes.c_void_p(workspace_ptr), workspace_bytes, ctypes.c_void_p(stream or 0)))
 
 
 def slorr_reset_workspace(handle) -> None:
@@ -293,6 +302,18 @@ class Regularizer:
         slorr_reg_forward_backward(self.handle, [w.data_ptr() for w in weights], [g.data_ptr() for g in grads],
                                    loss.data_ptr(), per_matrix.data_ptr() if per_matrix is not None else 0,
                                    ws, self.workspace_bytes, s)
+        return loss
+
+    def descent_step(self, weights, eta: float, loss=None, per_matrix=None, stream=None):
+        """W_i -= eta * lambda * grad_scale * G_i(W_i) in place; returns the loss at the old weights."""
+        import torch
+        dev = weights[0].device
+        ws = self.workspace(dev)
+        if loss is None:
+            loss = torch.empty(1, dtype=torch.float32, device=dev)
+        s = stream if stream is not None else torch.cuda.current_stream(dev).cuda_stream
+        slorr_reg_descent_step(self.handle, [w.data_ptr() for w in weights], eta, loss.data_ptr(),
+                               per_matrix.data_ptr() if per_matrix is not None else 0, ws, self.workspace_bytes, s)
         return loss
 
     def run_steps(self, weights, steps: int, stream=None):

@@ -89,6 +89,24 @@ def test_validation_rejects_bad_requests(lib):
     with pytest.raises(slorr.SlorrError) as e:
         slorr.slorr_reg_forward_backward(h, [256], [512], 768, 0, 1030, ws, 0)
     assert e.value.status == 4       # misaligned workspace
+    # the in-place descent step: a non-finite step, a NULL loss, a short workspace
+    for eta in [float("nan"), float("inf"), -float("inf")]:
+        with pytest.raises(slorr.SlorrError) as e:
+            slorr.slorr_reg_descent_step(h, [256], eta, 768, 0, 1024, ws, 0)
+        assert e.value.status == 1 and "eta" in str(e.value)
+    with pytest.raises(slorr.SlorrError) as e:
+        slorr.slorr_reg_descent_step(h, [256], 0.1, 0, 0, 1024, ws, 0)
+    assert e.value.status == 1
+    with pytest.raises(slorr.SlorrError) as e:
+        slorr.slorr_reg_descent_step(h, [256], 0.1, 768, 0, 1024, ws - 1, 0)
+    assert e.value.status == 4
+    slorr.slorr_destroy(h)
+    o = slorr.slorr_default_options()
+    o.lambda_ = 1e30
+    h = slorr.slorr_create([(4, 4)], o)
+    with pytest.raises(slorr.SlorrError) as e:
+        slorr.slorr_reg_descent_step(h, [256], 1e30, 768, 0, 1024, slorr.slorr_workspace_size(h), 0)
+    assert e.value.status == 1 and "overflows" in str(e.value)
     slorr.slorr_destroy(h)
 
 
