@@ -12,8 +12,10 @@ The default workload is the ViT-L/16-shaped set (96 matrices, 302 M weights,
 
 Printed: one JSON line.  value = algorithmic TFLOP/s of the whole job, using
 the paper's count T * sum_i (4 P_i^2 Q_i + 2 P_i^3) (Sec. 3 "Computational
-cost"); e2e = the same through the C ABI with the weights and grads copied from
-pinned host memory and the grads and loss copied back inside the timed region;
+cost"); e2e = the same through the C ABI's host-buffer call (slorr_pipeline_forward_backward):
+the weights and grads copied from page-locked host memory and the grads and
+loss copied back inside the timed region, group by group, overlapped with the
+kernels of the other groups;
 roofline = the tensor-core GEMM kernel measured live with CUDA events around
 each of its launches on the call's stream; cpu_baseline = the fp64 oracle on a
 bounded sample of the same workload on this host's cores.
@@ -45,8 +47,10 @@ import workloads  # noqa: E402
 
 METRIC = "regularizer fwd+bwd ms/step & TFLOP/s (% GB300 dense peak) per weight set"
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
-PROFILE_FILE = os.path.join(ROOT, "profiles", "tc_gemm_vit_l16.txt")
-TC_SOURCE = os.path.join(ROOT, "paper_2607_08754_gb300", "csrc", "kernels_tc.cu")
+PROFILE_FILE = os.path.join(ROOT, "profiles", "tc_pair_vit_l16.txt")
+# the default tensor-core GEMM (the CTA-pair kernel) and the headers it is built from
+TC_SOURCES = [os.path.join(ROOT, "paper_2607_08754_gb300", "csrc", f)
+              for f in ("kernels_tc_pair.cu", "tc_common.cuh", "ptx.cuh")]
 
 
 def parse():
@@ -67,6 +71,8 @@ def parse():
                     help="fwd_bwd: value + gradient accumulated into .grad (Alg. 2); descent: the in-place "
                          "regularizer-only step W -= eta lambda G (Alg. 1, last line)")
     ap.add_argument("--eta", type=float, default=1e-4, help="step size of --op descent")
+    ap.add_argument("--e2e-groups", type=int, default=8,
+                    help="groups of the host-buffer pipeline timed as e2e (slorr_pipeline_forward_backward)")
     return ap.parse_args()
 
 
@@ -164,11 +170,19 @@ class ClockSampler:
                 "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons), "samples": len(rows)}
 
 
+def tc_source_hash() -> str:
+    """sha256 over the default tensor-core kernel's source files, in order."""
+    h = hashlib.sha256()
+    for f in TC_SOURCES:
+        h.update(open(f, "rb").read())
+    return h.hexdigest()
+
+
 def tc_traffic():
     """dram bytes per launch of the tensor-core GEMM from the committed ncu
     summary, or None when the kernel source changed since it was taken."""
     try:
-        src = hashlib.sha256(open(TC_SOURCE, "rb").read()).hexdigest()
+        src = tc_source_hash()
         vals = {}
         with open(PROFILE_FILE) as f:
             for line in f:
@@ -297,16 +311,21 @@ def main():
     h2d = wbytes + gbytes
     d2h = (wbytes if descent else gbytes) + 4
 
+    pipe = None if descent else slorr.Pipeline(shapes, groups=args.e2e_groups, variant=args.variant,
+                                               compute=args.compute, iters=args.iters, lam=1.0, flags=args.flags)
+
     def e2e_step():
-        # inputs in (W, and .grad unless descending), the result out (the updated
-        # W or .grad) and the loss
+        if pipe is not None:
+            # the public host-buffer call: W and .grad copied in from page-locked
+            # host memory, .grad and the loss copied back, per group of matrices,
+            # overlapped with the kernels of the other groups
+            pipe(Wp, Gp, Wd, Gd, Lp)
+            return
+        # descent: W in, the updated W and the loss out
         for d, h in zip(Wd, Wp):
             d.copy_(h, non_blocking=True)
-        if not descent:
-            for d, h in zip(Gd, Gp):
-                d.copy_(h, non_blocking=True)
         step(Wd, Gd)
-        for d, h in zip(Wp if descent else Gp, Wd if descent else Gd):
+        for d, h in zip(Wp, Wd):
             d.copy_(h, non_blocking=True)
         Lp.copy_(loss, non_blocking=True)
 
@@ -323,10 +342,13 @@ def main():
     if world > 1:
         dist.all_reduce(ems, op=dist.ReduceOp.MAX)
     e2e_ms = ems.item() / args.e2e_steps
+    if pipe is not None:
+        assert pipe.status() == 0, "device status word reports an error in the e2e region"
     e2e_val = world * flops_step / (e2e_ms * 1e-3) / 1e12
 
     if rank == 0:
         pk = peaks()
+        single_cta = bool(args.flags & (slorr.FLAG_TC_SINGLE_CTA | slorr.FLAG_TC_BK32 | slorr.FLAG_TC_M128))
         gemm_ms = sum(kt[k][0] for k in ("gram", "poly", "update"))
         gemm_launches = sum(kt[k][1] for k in ("gram", "poly", "update"))
         launches = sum(v[1] for v in kt.values())
@@ -351,14 +373,17 @@ def main():
                              (sum(w.numel() for w in W) * 4 / 1e9)},
             "pct_of_dense_peak": value / world / pk["bf16"],
             "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                         "frac": achieved / peak, "traffic": tc_traffic(),
-                         "kernel": "tc_gemm_kernel (Gram/Poly/Update launches)",
+                         "frac": achieved / peak, "traffic": None if single_cta else tc_traffic(),
+                         "kernel": ("tc_gemm_kernel" if single_cta else "tc_pair_kernel")
+                                   + " (Gram/Poly/Update launches)",
                          "peak_source": pk["source"] + " bf16 burst (fp16 dense rate equal)"},
             "memory_phases_ms_per_step": mem_ms,
             "kernels": kernel_breakdown,
             "gpu_launches": launches,
             "e2e": {"value": e2e_val, "unit": "TFLOP/s", "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d,
-                    "d2h_bytes_per_step": d2h},
+                    "d2h_bytes_per_step": d2h,
+                    "call": "slorr_reg_descent_step with torch copies" if descent else
+                            f"slorr_pipeline_forward_backward, {args.e2e_groups} groups"},
             "clocks": clk,
         }
         if not args.no_cpu_baseline:

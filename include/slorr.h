@@ -107,6 +107,12 @@ typedef struct slorr_options {
                                        the pre-update gradient of the decoupled variant
                                        (Alg. 1, App. C.2), applied by the caller as
                                        W -= lr * grads[i] after its optimizer step      */
+#define SLORR_FLAG_TC_SINGLE_CTA 64 /* one-CTA tensor-core kernels (256 x 256 Gram/Update
+                                       tiles, 128 x 256 Poly tiles) instead of the
+                                       default CTA-pair kernel (tcgen05 cta_group::2);
+                                       implied by TC_BK32 and TC_M128 (tuning)           */
+#define SLORR_FLAG_PAIR_ONE_SLOT 128 /* CTA-pair kernel with one accumulator per SM (no
+                                       epilogue overlap; tuning)                         */
 
 /* Fill *opt with the defaults listed beside each field above (App. C.1: T = 6,
  * ell = 1e-3, degree 5; eps, lambda and grad_scale as in Listing 1 / Alg. 2). */
@@ -248,6 +254,54 @@ SLORR_API slorr_status slorr_frob_sq_noalloc(const void* weight, int64_t m, int6
 
 SLORR_API void        slorr_destroy(slorr_handle* h);
 SLORR_API const char* slorr_status_string(slorr_status s);
+
+/* ---- Host-resident weights and grads: a copy/compute pipeline ---------------
+ * The same forward + backward as slorr_reg_forward_backward (Listing 1,
+ * Alg. 2) for a weight set whose weights and grads live in host memory.  The
+ * set is split into `groups` runs of consecutive matrices of about equal size
+ * (the regularizer is a sum of independent per-matrix terms, Sec. 3), each
+ * with its own plan; while group g is regularized on the caller's stream, the
+ * weights and grads of the next groups are copied in on a second stream and
+ * the updated grads of the previous ones are copied out on a third, so that
+ * the host<->device copies in both directions overlap each other and the
+ * kernels.  The results equal those of slorr_reg_forward_backward on the same
+ * data (per-matrix values and grads bit for bit; the loss adds the groups'
+ * partial losses in group order).
+ *
+ * slorr_pipeline_create: shapes / opt as for slorr_create; groups >= 1 (more
+ * than `count` is clamped).  Host-only: no CUDA call until the first run,
+ * which creates the two copy streams and the events on the current device;
+ * every later run must use that device. */
+typedef struct slorr_pipeline slorr_pipeline;
+SLORR_API slorr_status slorr_pipeline_create(slorr_pipeline** out, const slorr_shape* shapes, int32_t count,
+                                   const slorr_options* opt, int32_t groups);
+
+/* Device workspace bytes a run needs (the groups' workspaces, the partial
+ * losses and the per-matrix values); host-only. */
+SLORR_API slorr_status slorr_pipeline_workspace_size(const slorr_pipeline* p, size_t* bytes);
+
+/* One pipelined forward + backward, enqueued on `stream`:
+ *   host_weights[i]  W_i in host memory, row-major m_i x n_i (page-locked,
+ *                    e.g. cudaHostAlloc, for the copies to overlap)
+ *   host_grads[i]    W_i.grad in host memory, same layout; ACCUMULATED (+=):
+ *                    copied in, accumulated on the device, copied back
+ *   host_loss        page-locked host float, written with lambda * sum_i L_i
+ *   host_per_matrix  page-locked host array of `count` floats, or NULL
+ *   dev_weights[i], dev_grads[i]
+ *                    device staging buffers of W_i's size (16-byte aligned),
+ *                    owned by the caller; overwritten
+ *   workspace        >= slorr_pipeline_workspace_size() bytes, 256-byte aligned
+ * When `stream` reaches the end of the call's work, every copy back to the
+ * host has completed.  Host buffers must not be touched until then. */
+SLORR_API slorr_status slorr_pipeline_forward_backward(slorr_pipeline* p, const void* const* host_weights,
+                                             void* const* host_grads, float* host_loss, float* host_per_matrix,
+                                             void* const* dev_weights, void* const* dev_grads, void* workspace,
+                                             size_t workspace_bytes, void* stream);
+
+/* As slorr_get_status, over every group of the pipeline. */
+SLORR_API slorr_status slorr_pipeline_get_status(slorr_pipeline* p, const void* workspace, void* stream);
+
+SLORR_API void slorr_pipeline_destroy(slorr_pipeline* p);
 
 /* Human-readable reason for the last non-OK status returned on this thread. */
 SLORR_API const char* slorr_last_error(void);

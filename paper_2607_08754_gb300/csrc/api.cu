@@ -87,15 +87,26 @@ struct slorr_handle {
 
 namespace {
 
-// K depth of the tensor-core pipeline stages for this handle.
-int tc_bk(const slorr_handle* h) { return (h->opt.flags & SLORR_FLAG_TC_BK32) ? 32 : 64; }
+// The CTA-pair kernel (256 x 256 tiles over two SMs, two accumulators per SM)
+// runs every phase unless a one-CTA kernel is asked for.
+bool tc_pair(const slorr_handle* h) {
+    return (h->opt.flags & (SLORR_FLAG_TC_SINGLE_CTA | SLORR_FLAG_TC_BK32 | SLORR_FLAG_TC_M128)) == 0;
+}
 
-// 128-row M tiles per tensor-core CTA tile for one phase.  256 x 256 tiles
-// (mt = 2) move a third fewer operand rows per FLOP but cannot overlap a
-// tile's epilogue with the next main loop; they win for the long-K Gram and
-// the store-only Update, while the short-K Poly, whose epilogue also reads A,
-// keeps double-buffered 128 x 256 tiles.
+// K depth of the tensor-core pipeline stages for this handle.
+int tc_bk(const slorr_handle* h) {
+    if (tc_pair(h)) return 64;  // the pair kernel's stages are K = 64
+    return (h->opt.flags & SLORR_FLAG_TC_BK32) ? 32 : 64;
+}
+
+// 128-row M tiles per tensor-core tile for one phase.  The pair kernel always
+// takes 256 x 256 tiles.  Of the one-CTA kernels, 256 x 256 tiles (mt = 2) move
+// a third fewer operand rows per FLOP but cannot overlap a tile's epilogue
+// with the next main loop; they win for the long-K Gram and the store-only
+// Update, while the short-K Poly, whose epilogue also reads A, keeps
+// double-buffered 128 x 256 tiles.
 int tc_mt(const slorr_handle* h, int phase) {
+    if (tc_pair(h)) return 2;
     if (h->opt.flags & (SLORR_FLAG_TC_M128 | SLORR_FLAG_TC_BK32)) return 1;
     return phase == kPoly ? 1 : 2;
 }
@@ -476,6 +487,8 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
     g.prefetch = (h->opt.flags & SLORR_FLAG_L2_PREFETCH) ? 8 : 0;
     g.bk = tc_bk(h);
     g.test_stall = (h->opt.flags & SLORR_FLAG_TEST_STALL) ? 1 : 0;
+    const bool pair = tc_pair(h);
+    g.pair_slots = (h->opt.flags & SLORR_FLAG_PAIR_ONE_SLOT) ? 1 : 2;
     for (int t = 0; t < steps; ++t) {
         g.cur = t & 1;
         g.a = float(h->coeffs[3 * t + 0]);
@@ -488,7 +501,8 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
             if (use_tc) {
                 g.items = reinterpret_cast<const GemmItem*>(ws + h->off_tc_items[ph]);
                 g.num_items = int(h->tc_items[ph].size());
-                e = launch_gemm_tc(g, h->elem, h->num_sms, st);
+                e = pair ? launch_gemm_tc_pair(g, h->elem, h->num_sms, st)
+                         : launch_gemm_tc(g, h->elem, h->num_sms, st);
             } else {
                 g.items = reinterpret_cast<const GemmItem*>(ws + h->off_simt_items[ph]);
                 g.num_items = int(h->simt_items[ph].size());
@@ -517,6 +531,24 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
         if ((e = launch_combine(dp, st)) != cudaSuccess) return cuda_fail(e, "combine launch");
         tr.done();
     }
+    return SLORR_OK;
+}
+
+// Reads and clears the device status word of a workspace (after the caller
+// synchronised the stream that used it).
+slorr_status take_status_word(const slorr_handle* h, const void* workspace, uint32_t* word) {
+    uint8_t* ws = static_cast<uint8_t*>(const_cast<void*>(workspace));
+    cudaError_t e = cudaMemcpy(word, ws + h->off_status, 4, cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess) e = cudaMemset(ws + h->off_status, 0, 4);
+    if (e != cudaSuccess) return cuda_fail(e, "status read");
+    return SLORR_OK;
+}
+
+slorr_status status_from_word(uint32_t word) {
+    if (word & kStatusTimeout) return fail(SLORR_ERR_TIMEOUT, "a device-side wait timed out");
+    if (word & kStatusNonFinite) return fail(SLORR_ERR_NONFINITE, "non-finite norm or estimate");
+    if (word & kStatusInternal)
+        return fail(SLORR_ERR_UNSUPPORTED, "the two CTAs of a tensor-core pair received different TMEM addresses");
     return SLORR_OK;
 }
 
@@ -611,13 +643,9 @@ slorr_status slorr_get_status(slorr_handle* h, const void* workspace, void* stre
     cudaError_t e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
     uint32_t word = 0;
-    uint8_t* ws = static_cast<uint8_t*>(const_cast<void*>(workspace));
-    e = cudaMemcpy(&word, ws + h->off_status, 4, cudaMemcpyDeviceToHost);
-    if (e == cudaSuccess) e = cudaMemset(ws + h->off_status, 0, 4);
-    if (e != cudaSuccess) return cuda_fail(e, "status read");
-    if (word & kStatusTimeout) return fail(SLORR_ERR_TIMEOUT, "a device-side wait timed out");
-    if (word & kStatusNonFinite) return fail(SLORR_ERR_NONFINITE, "non-finite norm or estimate");
-    return SLORR_OK;
+    slorr_status s = take_status_word(h, workspace, &word);
+    if (s != SLORR_OK) return s;
+    return status_from_word(word);
 }
 
 slorr_status slorr_run_steps(slorr_handle* h, const void* const* weights, void* workspace, size_t workspace_bytes,
@@ -738,5 +766,203 @@ const char* slorr_status_string(slorr_status s) {
 }
 
 const char* slorr_last_error(void) { return g_last_error.c_str(); }
+
+}  // extern "C"
+
+// ---- host-resident weight sets: the copy / compute pipeline ----------------------
+
+struct slorr_pipeline {
+    std::vector<slorr_handle*> groups;  // one plan per run of consecutive matrices
+    std::vector<int> first;             // first matrix of each group; first[G] = count
+    std::vector<size_t> ws_off;         // offset of each group's workspace slice
+    std::vector<size_t> bytes;          // bytes of W_i (and of its grad)
+    size_t off_loss = 0;                // G partial losses, the total, `count` per-matrix values
+    size_t total_bytes = 0;
+    int count = 0;
+    int device = -1;                    // streams and events live on this device
+    cudaStream_t s_in = nullptr, s_out = nullptr;
+    cudaEvent_t ev_start = nullptr, ev_out = nullptr;
+    std::vector<cudaEvent_t> ev_in, ev_done;
+    ~slorr_pipeline() {
+        for (auto* g : groups) delete g;
+        for (auto e : ev_in) cudaEventDestroy(e);
+        for (auto e : ev_done) cudaEventDestroy(e);
+        if (ev_start) cudaEventDestroy(ev_start);
+        if (ev_out) cudaEventDestroy(ev_out);
+        if (s_in) cudaStreamDestroy(s_in);
+        if (s_out) cudaStreamDestroy(s_out);
+    }
+};
+
+namespace {
+
+// Streams and events, created on the current device at the first run.
+slorr_status pipeline_init(slorr_pipeline* p) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (p->device >= 0) {
+        if (dev != p->device) return fail(SLORR_ERR_INVALID_ARG, "pipeline used on another device than its first run");
+        return SLORR_OK;
+    }
+    const int G = int(p->groups.size());
+    e = cudaStreamCreateWithFlags(&p->s_in, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&p->s_out, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p->ev_start, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p->ev_out, cudaEventDisableTiming);
+    for (int g = 0; g < G && e == cudaSuccess; ++g) {
+        cudaEvent_t a = nullptr, b = nullptr;
+        e = cudaEventCreateWithFlags(&a, cudaEventDisableTiming);
+        if (e == cudaSuccess) {
+            p->ev_in.push_back(a);
+            e = cudaEventCreateWithFlags(&b, cudaEventDisableTiming);
+            if (e == cudaSuccess) p->ev_done.push_back(b);
+        }
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "pipeline stream / event creation");
+    p->device = dev;
+    return SLORR_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+slorr_status slorr_pipeline_create(slorr_pipeline** out, const slorr_shape* shapes, int32_t count,
+                                   const slorr_options* opt, int32_t groups) {
+    if (!out) return fail(SLORR_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    if (groups < 1) return fail(SLORR_ERR_INVALID_ARG, "groups must be >= 1");
+    // validates shapes, count and options
+    slorr_handle* probe = nullptr;
+    slorr_status s = slorr_create(&probe, shapes, count, opt);
+    if (s != SLORR_OK) return s;
+    const int esz = probe->opt.dtype == SLORR_BF16 ? 2 : 4;
+    delete probe;
+    auto* p = new slorr_pipeline();
+    p->count = count;
+    size_t total = 0;
+    for (int i = 0; i < count; ++i) {
+        p->bytes.push_back(size_t(shapes[i].m) * size_t(shapes[i].n) * size_t(esz));
+        total += p->bytes.back();
+    }
+    // Consecutive runs of about total / G bytes each, none empty.
+    const int G = std::min<int>(groups, count);
+    p->first.push_back(0);
+    size_t acc = 0;
+    for (int i = 0; i < count; ++i) {
+        acc += p->bytes[i];
+        const int g = int(p->first.size());  // group being filled is g - 1
+        const int left = count - (i + 1);     // matrices not yet assigned
+        const int needed = G - g;             // groups still to start after this one
+        if (g < G && (acc * size_t(G) >= total * size_t(g) || left == needed) && left >= needed)
+            p->first.push_back(i + 1);
+    }
+    p->first.push_back(count);
+    size_t off = 0;
+    for (size_t g = 0; g + 1 < p->first.size(); ++g) {
+        slorr_handle* h = nullptr;
+        s = slorr_create(&h, shapes + p->first[g], p->first[g + 1] - p->first[g], opt);
+        if (s != SLORR_OK) {
+            delete p;
+            return s;
+        }
+        p->groups.push_back(h);
+        p->ws_off.push_back(off);
+        off = align_up(off + h->total_bytes, 1024);
+    }
+    p->off_loss = off;
+    off = align_up(off + (p->groups.size() + 1 + size_t(count)) * sizeof(float), 256);
+    p->total_bytes = off;
+    *out = p;
+    return SLORR_OK;
+}
+
+slorr_status slorr_pipeline_workspace_size(const slorr_pipeline* p, size_t* bytes) {
+    if (!p || !bytes) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
+    *bytes = p->total_bytes;
+    return SLORR_OK;
+}
+
+slorr_status slorr_pipeline_forward_backward(slorr_pipeline* p, const void* const* host_weights,
+                                             void* const* host_grads, float* host_loss, float* host_per_matrix,
+                                             void* const* dev_weights, void* const* dev_grads, void* workspace,
+                                             size_t workspace_bytes, void* stream) {
+    if (!p) return fail(SLORR_ERR_INVALID_ARG, "pipeline is NULL");
+    if (!host_weights || !host_grads || !host_loss || !dev_weights || !dev_grads)
+        return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
+    for (int i = 0; i < p->count; ++i)
+        if (!host_weights[i] || !host_grads[i]) return fail(SLORR_ERR_INVALID_ARG, "host pointer is NULL");
+    if (!workspace) return fail(SLORR_ERR_WORKSPACE, "workspace is NULL");
+    if (reinterpret_cast<uintptr_t>(workspace) % 256 != 0)
+        return fail(SLORR_ERR_WORKSPACE, "workspace is not 256-byte aligned");
+    if (workspace_bytes < p->total_bytes) return fail(SLORR_ERR_WORKSPACE, "workspace too small");
+    slorr_status s = pipeline_init(p);
+    if (s != SLORR_OK) return s;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    float* parts = reinterpret_cast<float*>(ws + p->off_loss);
+    const int G = int(p->groups.size());
+    float* total = parts + G;
+    float* per = total + 1;
+    // Copies start after the caller's earlier work on `stream`.
+    cudaError_t e = cudaEventRecord(p->ev_start, st);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(p->s_in, p->ev_start, 0);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(p->s_out, p->ev_start, 0);
+    // in: every group's weights and grads, in group order
+    for (int g = 0; g < G && e == cudaSuccess; ++g) {
+        for (int i = p->first[g]; i < p->first[g + 1] && e == cudaSuccess; ++i) {
+            e = cudaMemcpyAsync(dev_weights[i], host_weights[i], p->bytes[i], cudaMemcpyHostToDevice, p->s_in);
+            if (e == cudaSuccess)
+                e = cudaMemcpyAsync(dev_grads[i], host_grads[i], p->bytes[i], cudaMemcpyHostToDevice, p->s_in);
+        }
+        if (e == cudaSuccess) e = cudaEventRecord(p->ev_in[g], p->s_in);
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "pipeline copy-in");
+    // compute: group g once its copies have landed
+    for (int g = 0; g < G; ++g) {
+        e = cudaStreamWaitEvent(st, p->ev_in[g], 0);
+        if (e != cudaSuccess) return cuda_fail(e, "pipeline wait");
+        slorr_handle* h = p->groups[g];
+        const int f = p->first[g];
+        s = run(h, reinterpret_cast<const void* const*>(dev_weights + f), dev_grads + f, parts + g, per + f,
+                ws + p->ws_off[g], h->total_bytes, h->opt.iters, true, st);
+        if (s != SLORR_OK) return s;
+        e = cudaEventRecord(p->ev_done[g], st);
+        if (e != cudaSuccess) return cuda_fail(e, "pipeline record");
+    }
+    // out: each group's grads once its kernels are done
+    for (int g = 0; g < G && e == cudaSuccess; ++g) {
+        e = cudaStreamWaitEvent(p->s_out, p->ev_done[g], 0);
+        for (int i = p->first[g]; i < p->first[g + 1] && e == cudaSuccess; ++i)
+            e = cudaMemcpyAsync(host_grads[i], dev_grads[i], p->bytes[i], cudaMemcpyDeviceToHost, p->s_out);
+    }
+    if (e == cudaSuccess) e = cudaEventRecord(p->ev_out, p->s_out);
+    if (e != cudaSuccess) return cuda_fail(e, "pipeline copy-out");
+    // the loss (partial losses added in group order) and the per-matrix values
+    e = launch_sum_parts(parts, G, total, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(host_loss, total, sizeof(float), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess && host_per_matrix)
+        e = cudaMemcpyAsync(host_per_matrix, per, size_t(p->count) * sizeof(float), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(st, p->ev_out, 0);
+    if (e != cudaSuccess) return cuda_fail(e, "pipeline finish");
+    return SLORR_OK;
+}
+
+slorr_status slorr_pipeline_get_status(slorr_pipeline* p, const void* workspace, void* stream) {
+    if (!p || !workspace) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
+    cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+    uint32_t all = 0;
+    for (size_t g = 0; g < p->groups.size(); ++g) {
+        uint32_t word = 0;
+        slorr_status s = take_status_word(p->groups[g], static_cast<const uint8_t*>(workspace) + p->ws_off[g], &word);
+        if (s != SLORR_OK) return s;
+        all |= word;
+    }
+    return status_from_word(all);
+}
+
+void slorr_pipeline_destroy(slorr_pipeline* p) { delete p; }
 
 }  // extern "C"

@@ -24,13 +24,15 @@ namespace slorr {
 constexpr int kMaxMatrices = 4096;
 constexpr int kMaxIters = 16;
 constexpr int kPadRows = 128;   // Ppad granularity (tcgen05 tile M)
-constexpr int kPadCols = 64;    // Qpad granularity (one 128-byte swizzle row of 16-bit)
+constexpr int kPadCols = 128;   // Qpad granularity (a CTA pair splits a tile's 2 x 64 columns)
 
 // Element type of the iterate buffers X, A, B.
 enum Elem : int32_t { kF32 = 0, kF16 = 1, kBF16 = 2 };
 
 // Status bits written by kernels into the workspace status word.
-enum StatusBits : uint32_t { kStatusTimeout = 1u, kStatusNonFinite = 2u };
+// kStatusInternal: the two CTAs of a pair received different TMEM addresses
+// (the pair kernel then does no work).
+enum StatusBits : uint32_t { kStatusTimeout = 1u, kStatusNonFinite = 2u, kStatusInternal = 4u };
 
 // Per-matrix device descriptor (lives in the workspace).
 struct MatDev {
@@ -96,6 +98,7 @@ struct GemmLaunch {
     int32_t bk;                // K depth of a pipeline stage: 64 (4 stages) or 32 (9 stages)
     int32_t mt;                // 128-row M tiles per CTA tile: 1 or 2 (256 x 256 tiles)
     int32_t test_stall;        // 1: the MMA thread first waits on a barrier nothing arrives on
+    int32_t pair_slots;        // CTA-pair kernel: accumulators per CTA (1 or 2)
 };
 
 // Tensor maps per matrix: X0 K-major, X1 K-major, X0 MN-major, X1 MN-major,
@@ -138,8 +141,10 @@ cudaError_t launch_cast(const MemLaunch& p, cudaStream_t s);
 cudaError_t launch_dot(const MemLaunch& p, cudaStream_t s);
 cudaError_t launch_finalize(const MemLaunch& p, int which, cudaStream_t s);
 cudaError_t launch_combine(const MemLaunch& p, cudaStream_t s);
+cudaError_t launch_sum_parts(const float* parts, int n, float* out, cudaStream_t s);
 cudaError_t launch_gemm_simt(const GemmLaunch& p, int elem, cudaStream_t s);
 cudaError_t launch_gemm_tc(const GemmLaunch& p, int elem, int grid, cudaStream_t s);
+cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t s);
 int tc_smem_bytes();
 
 // Records the message slorr_last_error() returns on this thread (api.cu).

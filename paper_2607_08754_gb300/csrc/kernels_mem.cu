@@ -428,6 +428,20 @@ cudaError_t launch_finalize(const MemLaunch& p, int which, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+// One thread: out = sum of the n partial losses in index order (double).
+__global__ void sum_parts_kernel(const float* __restrict__ parts, int n, float* __restrict__ out) {
+    if (threadIdx.x == 0 && blockIdx.x == 0) {
+        double t = 0.0;
+        for (int i = 0; i < n; ++i) t += static_cast<double>(parts[i]);
+        *out = static_cast<float>(t);
+    }
+}
+
+cudaError_t launch_sum_parts(const float* parts, int n, float* out, cudaStream_t s) {
+    sum_parts_kernel<<<1, 32, 0, s>>>(parts, n, out);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_combine(const MemLaunch& p, cudaStream_t s) {
     if (p.num_items == 0) return cudaSuccess;
     SLORR_DISPATCH_WX(combine_kernel);

@@ -30,16 +30,14 @@
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
-#include "internal.h"
-#include "ptx.cuh"
+#include "tc_common.cuh"
 
 namespace slorr {
 namespace {
 
-constexpr int kBM = 128;       // rows of one UMMA
-constexpr int kBNMax = 256;
+using namespace tc;
+
 constexpr int kTmemCols = 512;
-constexpr int kAccCols = 256;  // fp32 columns of one 128 x 256 accumulator
 constexpr int kMaxStages = 16;
 
 // Pipeline configuration: K depth BK of a stage, stages, M tiles per CTA.
@@ -72,36 +70,6 @@ using Cfg64 = Cfg<64, 4, 1>;
 using Cfg32 = Cfg<32, 9, 1>;
 using Cfg256 = Cfg<64, 3, 2>;
 
-template <bool BF16>
-__device__ __forceinline__ uint32_t pack2(float lo, float hi) {
-    if constexpr (BF16) {
-        __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-        return *reinterpret_cast<uint32_t*>(&v);
-    } else {
-        __half2 v = __floats2half2_rn(lo, hi);
-        return *reinterpret_cast<uint32_t*>(&v);
-    }
-}
-
-template <bool BF16>
-__device__ __forceinline__ uint16_t to16(float x) {
-    if constexpr (BF16)
-        return __bfloat16_as_ushort(__float2bfloat16_rn(x));
-    else
-        return __half_as_ushort(__float2half_rn(x));
-}
-
-template <bool BF16>
-__device__ __forceinline__ float2 unpack2(uint32_t u) {
-    if constexpr (BF16) {
-        __nv_bfloat162 v = *reinterpret_cast<__nv_bfloat162*>(&u);
-        return __bfloat1622float2(v);
-    } else {
-        __half2 v = *reinterpret_cast<__half2*>(&u);
-        return __half22float2(v);
-    }
-}
-
 struct Smem {
     uint8_t* stages;
     uint64_t* full;
@@ -117,68 +85,6 @@ struct Smem {
 __device__ __forceinline__ void record_timeout(const GemmLaunch& p, const Smem& s) {
     *s.abort = 1;
     atomicOr(p.status, kStatusTimeout);
-}
-
-struct PhaseInfo {
-    const void* mapA;
-    const void* mapB;
-    int nkb;
-    bool a_mn;   // A operand MN-major (else K-major)
-    bool b_mn;   // B operand MN-major (else K-major)
-};
-
-// Tensor maps per matrix (kMapsPerMatrix of them, 128 bytes each):
-// X0 K-major, X1 K-major, X0 MN-major, X1 MN-major, A K-major, M K-major.
-__device__ __forceinline__ const void* xmap(const uint8_t* maps, int buf, bool mn) {
-    return maps + (mn ? 2 + buf : buf) * 128;
-}
-
-template <class C>
-__device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmItem& it) {
-    const MatDev& md = p.mats[it.mat];
-    const uint8_t* maps = reinterpret_cast<const uint8_t*>(p.maps) + size_t(it.mat) * kMapsPerMatrix * 128;
-    const bool tr = md.transposed != 0;
-    PhaseInfo pi;
-    if (p.phase == kGram) {
-        pi.a_mn = tr;
-        pi.b_mn = tr;
-        pi.mapA = xmap(maps, p.cur, tr);
-        pi.mapB = pi.mapA;
-        pi.nkb = md.Qpad / C::BK;
-    } else if (p.phase == kPoly) {
-        pi.a_mn = false;
-        pi.b_mn = false;
-        pi.mapA = maps + 4 * 128;
-        pi.mapB = pi.mapA;
-        pi.nkb = md.Ppad / C::BK;
-    } else {
-        pi.a_mn = false;
-        pi.b_mn = !tr;
-        pi.mapA = maps + 5 * 128;
-        pi.mapB = xmap(maps, p.cur, pi.b_mn);
-        pi.nkb = md.Ppad / C::BK;
-    }
-    return pi;
-}
-
-// Symmetric products (Gram, Poly): only tiles holding some 128 x 128 block on
-// or above the diagonal are computed.  Tile (tm, tn) covers row blocks from
-// tm MT on and column blocks 2 tn .. min(2 tn + 1, nb - 1) (nb = Ppad / 128), so
-// it is computed iff its last column block reaches its first row block.
-__device__ __forceinline__ bool sym_tile_computed(int tm, int tn, int Ppad, int mt) {
-    const int last_col_block = min(2 * tn + 1, Ppad / 128 - 1);
-    return last_col_block >= tm * mt;
-}
-
-// Shared-memory descriptor of one K = 16 slice (kk) of a BK-wide K block:
-// K-major: rows of 2 BK bytes (swizzle span), 8-row groups kKSbo apart, slice
-// kk starts 32 bytes further inside the swizzle atom; MN-major: 64-element MN
-// chunks one box apart (LBO), 8-row K groups 1 KB apart (SBO), slice kk starts
-// 16 rows = 2 KB further.
-template <class C>
-__device__ __forceinline__ uint64_t operand_desc(uint32_t base, int kk, bool mn) {
-    return mn ? ptx::sdesc(base + kk * 16 * 128, C::kBoxBytes, 1024, 2u)
-              : ptx::sdesc(base + kk * 32, 16, C::kKSbo, C::kKLayout);
 }
 
 template <class C>
@@ -333,99 +239,9 @@ __device__ void epilogue(const GemmLaunch& p, const Smem& s, uint32_t tmem_base,
         ptx::tc_fence_after();
         if (half < it.msz / kBM) {
             const int row0 = it.tm * (kBM * C::MT) + half * kBM;  // first row of this 128-row tile
-            const int row = row0 + quad * 32 + lane;
             const uint32_t t_row =
                 tmem_base + (uint32_t(quad * 32) << 16) + uint32_t((slot + half) * kAccCols);
-            const int nch = it.nsz / 32;
-            if (p.phase == kUpdate) {
-                uint16_t* out = reinterpret_cast<uint16_t*>(md.x[p.cur ^ 1]);
-                const int64_t ld = md.ld;
-                for (int ch = 0; ch < nch; ++ch) {
-                    uint32_t r[32];
-                    ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
-                    ptx::tmem_ld_wait();
-                    const int col0 = it.tn * kBNMax + ch * 32;
-                    if (md.transposed) {
-                        // X^T[q][p]: for each column the warp's 32 rows are contiguous
-                        uint16_t* dst = out + int64_t(col0) * ld + row;
-#pragma unroll
-                        for (int j = 0; j < 32; ++j) dst[int64_t(j) * ld] = to16<BF16>(__uint_as_float(r[j]));
-                    } else {
-                        uint4 o[4];
-                        uint32_t* ow = reinterpret_cast<uint32_t*>(o);
-#pragma unroll
-                        for (int j = 0; j < 16; ++j)
-                            ow[j] = pack2<BF16>(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
-                        uint4* dst = reinterpret_cast<uint4*>(out + int64_t(row) * ld + col0);
-#pragma unroll
-                        for (int v = 0; v < 4; ++v) dst[v] = o[v];
-                    }
-                }
-            } else {
-                uint16_t* out = reinterpret_cast<uint16_t*>(p.phase == kGram ? md.a : md.b);
-                const uint16_t* amat = reinterpret_cast<const uint16_t*>(md.a);
-                const int64_t ld = md.Ppad;
-                const bool poly = p.phase == kPoly;
-                const float cacc = poly ? p.c : 1.f;
-                // Poly reads b A at the output position: loads for the next chunk are
-                // issued before the current chunk is processed.
-                uint4 e_next[4];
-                if (poly) {
-                    const uint4* src = reinterpret_cast<const uint4*>(amat + int64_t(row) * ld + it.tn * kBNMax);
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) e_next[q] = src[q];
-                }
-                for (int ch = 0; ch < nch; ++ch) {
-                    const int col0 = it.tn * kBNMax + ch * 32;
-                    const int64_t off = int64_t(row) * ld + col0;
-                    uint4 e[4];
-                    if (poly) {
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) e[q] = e_next[q];
-                        if (ch + 1 < nch) {
-                            const uint4* src = reinterpret_cast<const uint4*>(amat + off + 32);
-#pragma unroll
-                            for (int q = 0; q < 4; ++q) e_next[q] = src[q];
-                        }
-                    }
-                    uint32_t r[32];
-                    ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
-                    ptx::tmem_ld_wait();
-                    uint4 o[4];
-                    uint32_t* ow = reinterpret_cast<uint32_t*>(o);
-                    const int d = row - col0;  // diagonal element of this row, if in the chunk
-                    const uint32_t* ew = reinterpret_cast<const uint32_t*>(e);
-#pragma unroll
-                    for (int j = 0; j < 16; ++j) {
-                        float lo = cacc * __uint_as_float(r[2 * j]);
-                        float hi = cacc * __uint_as_float(r[2 * j + 1]);
-                        if (poly) {
-                            // M = c A^2 + b A + a I
-                            const float2 x = unpack2<BF16>(ew[j]);
-                            lo = fmaf(p.b, x.x, lo) + (2 * j == d ? p.a : 0.f);
-                            hi = fmaf(p.b, x.y, hi) + (2 * j + 1 == d ? p.a : 0.f);
-                        }
-                        ow[j] = pack2<BF16>(lo, hi);
-                    }
-                    uint4* dst = reinterpret_cast<uint4*>(out + off);
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) dst[q] = o[q];
-                    // The output is symmetric and strictly-lower tiles are skipped:
-                    // write the transpose of this 128 x 128 block (I, J), J > I, when
-                    // the tile that holds (J, I) is not computed.  The mirrored copy
-                    // uses the same rounded 16-bit values, so the stored matrix is
-                    // exactly symmetric.
-                    const int I = row0 / kBM, J = col0 / kBM;
-                    if (J > I && !sym_tile_computed(J / C::MT, I / 2, md.Ppad, C::MT)) {
-                        uint16_t* tdst = out + int64_t(col0) * ld + row;
-#pragma unroll
-                        for (int j = 0; j < 16; ++j) {
-                            tdst[int64_t(2 * j) * ld] = uint16_t(ow[j] & 0xffffu);
-                            tdst[int64_t(2 * j + 1) * ld] = uint16_t(ow[j] >> 16);
-                        }
-                    }
-                }
-            }
+            store_rows<BF16, C::MT>(p, it, md, row0, t_row, quad, lane, 0, it.nsz / 32);
         }
         ptx::tc_fence_before();
         __syncwarp();

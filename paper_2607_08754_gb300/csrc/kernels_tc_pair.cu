@@ -1,0 +1,395 @@
+// Grouped persistent tensor-core GEMM on CTA pairs (tcgen05 cta_group::2), for
+// the same three phases of a Polar Express step as kernels_tc.cu (Sec. 3
+// "Computing the polar factor"): Gram A = X X^T, Poly M = a I + b A + c A A,
+// Update X' = M X, over every matrix of the weight set in one launch.
+//
+// A cluster of two CTAs on two SMs computes one 256 x 256 tile.  CTA r of the
+// pair holds rows [128 r, 128 r + 128) of the tile's A operand and columns
+// [nsz/2 r, nsz/2 (r + 1)) of its B operand in shared memory, and rows
+// [128 r, 128 r + 128) of the fp32 accumulator in its own tensor memory; one
+// thread of the even CTA issues M = 256 UMMAs that read both CTAs' operands and
+// write both CTAs' accumulators.  Each SM therefore moves the same bytes per
+// FLOP as a single-CTA 256 x 256 tile, while a tile's accumulator takes only
+// 256 TMEM columns per SM: two of them fit, so a tile's epilogue overlaps the
+// next tile's main loop.
+//
+// Roles (192 threads per CTA; 320 for Poly):
+//   warp 0 lane 0   TMA producer (both CTAs): waits for a stage to be free and
+//                   loads its CTA's A rows and B half into its own shared
+//                   memory, counting the bytes on the even CTA's stage barrier
+//                   (the cta_group::2 form of the tensor copy);
+//   warp 1          allocates the pair's TMEM (with the peer); lane 0 of the
+//                   even CTA "arms" each stage barrier with the bytes of both
+//                   CTAs' copies one ring ahead (as soon as the stage's current
+//                   data has landed), issues the pair UMMAs, and multicasts
+//                   each stage release and each tile completion to both CTAs;
+//   warps 2..       epilogue (both CTAs): 128 rows of the tile from TMEM, one
+//                   warp (two for Poly, each taking half of the columns) per
+//                   32-row TMEM lane quadrant; then release the accumulator
+//                   slot on the even CTA's barrier.
+// A stage is released only by a commit the MMA thread issues after arming the
+// stage's next phase, so every copy of either CTA is counted on a phase the
+// MMA thread armed; on a timeout that thread waits (bounded) for the last
+// armed phase of every stage, and the exit cluster barrier keeps the odd CTA
+// alive until then.  Every wait is bounded; a CTA that gives up sets the
+// abort flag of both CTAs.  The only unbounded waits are the two cluster
+// barriers at entry and exit, which every thread reaches after finitely many
+// bounded waits.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include "tc_common.cuh"
+
+namespace slorr {
+namespace {
+
+using namespace tc;
+
+template <int STAGES_, int SLOTS_, int EPIW_>
+struct PairCfg {
+    static constexpr int BK = 64;
+    static constexpr int STAGES = STAGES_;
+    static constexpr int kSlots = SLOTS_;                 // accumulators per CTA in TMEM
+    static constexpr int kBoxBytes = 64 * BK * 2;         // one 64 x 64 box
+    static constexpr int kABytes = kBM * BK * 2;          // this CTA's 128 rows of A
+    static constexpr int kBBytes = (kBNMax / 2) * BK * 2; // this CTA's half of B (<= 128 rows)
+    static constexpr int kStageBytes = kABytes + kBBytes;
+    static constexpr int kEpiWarps = EPIW_;               // 4, or 8: two per TMEM lane quadrant
+    static_assert(EPIW_ == 4 || EPIW_ == 8, "epilogue warps");
+    static constexpr int kThreads = 64 + 32 * kEpiWarps;
+    static constexpr uint32_t kKLayout = 2u;              // SWIZZLE_128B
+    static constexpr uint32_t kKSbo = 8 * BK * 2;
+    static constexpr uint32_t kTmemCols = uint32_t(kSlots) * kAccCols;
+    static constexpr size_t kBarrierBytes = 512;
+    static constexpr size_t kSmemBytes = size_t(STAGES) * kStageBytes + 1024 /*align*/ + kBarrierBytes;
+    static_assert((2 * STAGES + 2 * kSlots + 1) * 8 + 16 <= kBarrierBytes, "barrier area");
+    static_assert(kSmemBytes <= 232448, "shared memory budget");
+    static_assert(kTmemCols <= 512, "tensor memory budget");
+};
+// Ring depth (a build-time tuning knob): 6 stages of 32 KB; 7 still fit.
+#ifndef SLORR_PAIR_STAGES
+#define SLORR_PAIR_STAGES 6
+#endif
+// Two accumulators per CTA (the tile epilogue overlaps the next main loop);
+// the Poly epilogue, which also reads b A, takes 8 warps, the others 4 (more
+// polling warps slow the producer and MMA threads of the long-K phases).
+using PairCfg1 = PairCfg<SLORR_PAIR_STAGES, 1, 4>;   // one accumulator per CTA: no overlap
+using PairCfg2 = PairCfg<SLORR_PAIR_STAGES, 2, 4>;
+using PairCfg2Wide = PairCfg<SLORR_PAIR_STAGES, 2, 8>;
+
+struct PairSmem {
+    uint8_t* stages;
+    uint64_t* full;    // even CTA: both CTAs' copies of the stage landed
+    uint64_t* empty;   // stage consumed by the pair UMMAs (multicast commit)
+    uint64_t* tfull;   // accumulator slot complete (multicast commit)
+    uint64_t* tempty;  // even CTA: both CTAs' epilogues released the slot
+    uint64_t* drain;
+    uint32_t* tmem_slot;
+    volatile int* abort;
+    volatile int* never;  // stays 0: drain waits ignore the abort flag
+    uint32_t peer;        // cluster rank of the other CTA
+};
+
+__device__ __forceinline__ void record_timeout(const GemmLaunch& p, const PairSmem& s) {
+    *s.abort = 1;
+    ptx::st_cluster_u32(ptx::mapa(ptx::smem_u32(const_cast<int*>(s.abort)), s.peer), 1u);
+    atomicOr(p.status, kStatusTimeout);
+}
+
+// Bytes one CTA of the pair copies per stage of a tile: its A rows, unless they
+// lie beyond the matrix (the UMMA rows they would feed are never stored), and
+// its half of the B columns.
+template <class C>
+__device__ __forceinline__ uint32_t pair_stage_bytes(const GemmItem& it, int rank) {
+    return (rank * kBM < it.msz ? uint32_t(C::kABytes) : 0u) + uint32_t(it.nsz / 2) * C::BK * 2;
+}
+
+template <class C>
+__device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, int pair, int npairs) {
+    int stage = 0;
+    uint32_t phase = 0;
+    const uint32_t even_full = ptx::mapa(ptx::smem_u32(s.full), 0);
+    for (int idx = pair; idx < p.num_items; idx += npairs) {
+        const GemmItem it = p.items[idx];
+        const PhaseInfo pi = phase_info<C>(p, it);
+        const bool load_a = rank * kBM < it.msz;
+        const int bhalf = it.nsz / 2;  // 64 or 128 rows of B per CTA
+        for (int kb = 0; kb < pi.nkb; ++kb) {
+            if (!ptx::mbar_wait(&s.empty[stage], phase ^ 1u, s.abort, p.timeout_ns)) {
+                record_timeout(p, s);
+                return;
+            }
+            uint8_t* sa = s.stages + size_t(stage) * C::kStageBytes;
+            uint8_t* sb = sa + C::kABytes;
+            const int k = kb * C::BK;
+            const uint32_t bar = even_full + uint32_t(stage * 8);
+            // box coordinates are (inner, outer): (k, mn) for K-major, (mn, k) for MN-major
+            if (load_a)
+                for (int b = 0; b < 2; ++b) {
+                    const int mn = it.tm * (2 * kBM) + rank * kBM + b * 64;
+                    ptx::tma_load_2d_pair(sa + b * C::kBoxBytes, pi.mapA, bar, pi.a_mn ? mn : k, pi.a_mn ? k : mn);
+                }
+            for (int j = 0; j < bhalf / 64; ++j) {
+                const int mn = it.tn * kBNMax + rank * bhalf + j * 64;
+                ptx::tma_load_2d_pair(sb + j * C::kBoxBytes, pi.mapB, bar, pi.b_mn ? mn : k, pi.b_mn ? k : mn);
+            }
+            if (++stage == C::STAGES) {
+                stage = 0;
+                phase ^= 1u;
+            }
+        }
+    }
+}
+
+// Walks this pair's (tile, K block) sequence; the MMA thread keeps one cursor
+// STAGES K blocks ahead of the one it consumes, to arm stage barriers.
+template <class C>
+struct KCursor {
+    const GemmLaunch* p;
+    int idx, kb, nkb, step;
+    uint32_t bytes;  // bytes both CTAs copy for the current K block
+    __device__ void load() {
+        if (idx < p->num_items) {
+            const GemmItem it = p->items[idx];
+            nkb = phase_info<C>(*p, it).nkb;
+            bytes = pair_stage_bytes<C>(it, 0) + pair_stage_bytes<C>(it, 1);
+        }
+    }
+    __device__ KCursor(const GemmLaunch& gp, int first, int stride) : p(&gp), idx(first), kb(0), nkb(0), step(stride),
+                                                                      bytes(0) {
+        load();
+    }
+    __device__ bool valid() const { return idx < p->num_items; }
+    __device__ void next() {
+        if (++kb == nkb) {
+            kb = 0;
+            idx += step;
+            load();
+        }
+    }
+};
+
+template <bool BF16, class C>
+__device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_base, int pair, int npairs) {
+    int armed_parity[C::STAGES];
+#pragma unroll
+    for (int i = 0; i < C::STAGES; ++i) armed_parity[i] = -1;
+    // Arm the first ring: phase 0 of every stage the sequence reaches.
+    KCursor<C> arm(p, pair, npairs);
+    for (int i = 0; i < C::STAGES && arm.valid(); ++i, arm.next()) {
+        ptx::mbar_arrive_expect_tx(&s.full[i], arm.bytes);
+        armed_parity[i] = 0;
+    }
+    int stage = 0;
+    uint32_t phase = 0;
+    int local = 0;
+    bool ok = true;
+    bool issued_any = false;
+    if (p.test_stall) {
+        // Failure-detection test: wait on the drain barrier, which nothing
+        // arrives on before the end, so the bounded wait runs out.
+        if (!ptx::mbar_wait(s.drain, 0u, s.abort, p.timeout_ns)) {
+            record_timeout(p, s);
+            ok = false;
+        }
+    }
+    for (int idx = pair; idx < p.num_items && ok; idx += npairs, ++local) {
+        const GemmItem it = p.items[idx];
+        const PhaseInfo pi = phase_info<C>(p, it);
+        const uint32_t idesc = ptx::idesc_f16(2 * kBM, it.nsz, BF16, pi.a_mn, pi.b_mn);
+        const int slot = local % C::kSlots;
+        const uint32_t tphase = uint32_t(local / C::kSlots) & 1u;
+        if (!ptx::mbar_wait<true>(&s.tempty[slot], tphase ^ 1u, s.abort, p.timeout_ns)) {
+            record_timeout(p, s);
+            ok = false;
+            break;
+        }
+        ptx::tc_fence_after();
+        const uint32_t d_tmem = tmem_base + uint32_t(slot * kAccCols);
+        for (int kb = 0; kb < pi.nkb; ++kb) {
+            if (!ptx::mbar_wait(&s.full[stage], phase, s.abort, p.timeout_ns)) {
+                record_timeout(p, s);
+                ok = false;
+                break;
+            }
+            // This stage's data has landed, so its barrier is in its next phase:
+            // arm it now for the K block one ring ahead.
+            if (arm.valid()) {
+                ptx::mbar_arrive_expect_tx(&s.full[stage], arm.bytes);
+                armed_parity[stage] = int(phase ^ 1u);
+                arm.next();
+            }
+            ptx::tc_fence_after();
+            const uint32_t a0 = ptx::smem_u32(s.stages + size_t(stage) * C::kStageBytes);
+            const uint32_t b0 = a0 + C::kABytes;
+#pragma unroll
+            for (int kk = 0; kk < C::BK / 16; ++kk)
+                ptx::umma_f16_pair(d_tmem, operand_desc<C>(a0, kk, pi.a_mn), operand_desc<C>(b0, kk, pi.b_mn), idesc,
+                                   (kb | kk) != 0 ? 1u : 0u);
+            issued_any = true;
+            ptx::umma_commit_pair_mc(&s.empty[stage], 0x3);
+            if (++stage == C::STAGES) {
+                stage = 0;
+                phase ^= 1u;
+            }
+        }
+        if (!ok) break;
+        ptx::umma_commit_pair_mc(&s.tfull[slot], 0x3);
+    }
+    if (!ok) {
+        if (issued_any) {
+            // No UMMA may still be writing either CTA's TMEM when it is released.
+            ptx::umma_commit_pair_mc(s.drain, 0x1);
+            ptx::mbar_wait(s.drain, 0u, s.never, p.timeout_ns);
+        }
+        // Every copy either CTA issued was counted on an armed phase: wait
+        // (bounded) for the last armed phase of each stage before exit.
+        for (int i = 0; i < C::STAGES; ++i)
+            if (armed_parity[i] >= 0) ptx::mbar_wait(&s.full[i], uint32_t(armed_parity[i]), s.never, p.timeout_ns);
+    }
+}
+
+template <bool BF16, class C>
+__device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_base, int rank, int pair,
+                              int npairs, int warp, int lane) {
+    const int quad = warp & 3;             // TMEM lanes [32 quad, 32 quad + 32) (hardware rule)
+    const int ngroups = C::kEpiWarps / 4;  // warps per lane quadrant, splitting the columns
+    const int group = (warp - 2) / 4;
+    int local = 0;
+    const uint32_t even_tempty = ptx::mapa(ptx::smem_u32(s.tempty), 0);
+    for (int idx = pair; idx < p.num_items; idx += npairs, ++local) {
+        const GemmItem it = p.items[idx];
+        const MatDev& md = p.mats[it.mat];
+        const int slot = local % C::kSlots;
+        const uint32_t tphase = uint32_t(local / C::kSlots) & 1u;
+        int ok = 1;
+        if (lane == 0) ok = ptx::mbar_wait(&s.tfull[slot], tphase, s.abort, p.timeout_ns) ? 1 : 0;
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok) {
+            if (lane == 0) record_timeout(p, s);
+            break;
+        }
+        ptx::tc_fence_after();
+        if (rank * kBM < it.msz) {
+            const int row0 = it.tm * (2 * kBM) + rank * kBM;
+            const uint32_t t_row = tmem_base + (uint32_t(quad * 32) << 16) + uint32_t(slot * kAccCols);
+            const int per = it.nsz / 32 / ngroups;  // 32-column chunks per warp
+            store_rows<BF16, 2>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per);
+        }
+        // The slot may be overwritten once this warp's TMEM loads are done
+        // (tcgen05.wait::ld above); the stores need no ordering with the
+        // next UMMAs, so the arrive is relaxed.
+        ptx::tc_fence_before();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive_cluster_relaxed(even_tempty + uint32_t(slot * 8));
+    }
+}
+
+template <bool BF16, class C>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(C::kThreads, 1)
+    tc_pair_kernel(const __grid_constant__ GemmLaunch p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* base = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    PairSmem s;
+    s.stages = base;
+    s.full = reinterpret_cast<uint64_t*>(base + size_t(C::STAGES) * C::kStageBytes);
+    s.empty = s.full + C::STAGES;
+    s.tfull = s.empty + C::STAGES;
+    s.tempty = s.tfull + C::kSlots;
+    s.drain = s.tempty + C::kSlots;
+    s.tmem_slot = reinterpret_cast<uint32_t*>(s.drain + 1);
+    s.abort = reinterpret_cast<volatile int*>(s.tmem_slot + 1);
+    s.never = s.abort + 1;
+    const int rank = int(ptx::cluster_ctarank());
+    s.peer = uint32_t(rank ^ 1);
+    const int pair = blockIdx.x / 2, npairs = gridDim.x / 2;
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < C::STAGES; ++i) {
+            ptx::mbar_init(&s.full[i], 1);
+            ptx::mbar_init(&s.empty[i], 1);
+        }
+        for (int i = 0; i < C::kSlots; ++i) {
+            ptx::mbar_init(&s.tfull[i], 1);
+            ptx::mbar_init(&s.tempty[i], 2 * C::kEpiWarps);
+        }
+        ptx::mbar_init(s.drain, 1);
+        *s.abort = 0;
+        *s.never = 0;
+        ptx::fence_mbar_init();
+    }
+    if (warp == 0 && lane == 0 && pair < p.num_items) {
+        const PhaseInfo pi = phase_info<C>(p, p.items[pair]);
+        ptx::prefetch_tmap(pi.mapA);
+        ptx::prefetch_tmap(pi.mapB);
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc_pair(s.tmem_slot, C::kTmemCols);
+        ptx::tmem_relinquish_pair();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::cluster_sync();  // barriers initialised and TMEM allocated in both CTAs
+    ptx::tc_fence_after();
+    const uint32_t tmem_base = *s.tmem_slot;
+    // The UMMAs address both CTAs' accumulators with the even CTA's TMEM
+    // address: the two allocations must agree, else no work is done.
+    const uint32_t peer_base = ptx::ld_cluster_u32(ptx::mapa(ptx::smem_u32(s.tmem_slot), s.peer));
+    if (peer_base != tmem_base) {
+        if (threadIdx.x == 0) atomicOr(p.status, kStatusInternal);
+    } else if (warp == 0) {
+        if (lane == 0) pair_producer<C>(p, s, rank, pair, npairs);
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0 && rank == 0) pair_mma<BF16, C>(p, s, tmem_base, pair, npairs);
+        __syncwarp();
+    } else {
+        pair_epilogue<BF16, C>(p, s, tmem_base, rank, pair, npairs, warp, lane);
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::cluster_sync();  // no remote arrive, UMMA or copy of either CTA is outstanding
+    if (warp == 1) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc_pair(tmem_base, C::kTmemCols);
+    }
+}
+
+template <bool BF16, class C>
+cudaError_t launch_pair_cfg(const GemmLaunch& p, int num_sms, cudaStream_t st) {
+    static int max_pairs = 0;
+    if (max_pairs == 0) {
+        cudaError_t e = cudaFuncSetAttribute(tc_pair_kernel<BF16, C>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             int(C::kSmemBytes));
+        if (e != cudaSuccess) return e;
+        cudaLaunchConfig_t probe = {};
+        probe.gridDim = dim3(unsigned(2 * (num_sms / 2)));
+        probe.blockDim = dim3(C::kThreads);
+        probe.dynamicSmemBytes = C::kSmemBytes;
+        int clusters = 0;
+        e = cudaOccupancyMaxActiveClusters(&clusters, tc_pair_kernel<BF16, C>, &probe);
+        if (e != cudaSuccess) return e;
+        if (clusters < 1) return cudaErrorInvalidConfiguration;
+        max_pairs = clusters < num_sms / 2 ? clusters : num_sms / 2;
+    }
+    const int npairs = p.num_items < max_pairs ? p.num_items : max_pairs;
+    tc_pair_kernel<BF16, C><<<2 * npairs, C::kThreads, C::kSmemBytes, st>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t st) {
+    if (p.num_items == 0) return cudaSuccess;
+    const bool bf = elem == kBF16;
+    if (p.pair_slots == 2 && p.phase == kPoly)
+        return bf ? launch_pair_cfg<true, PairCfg2Wide>(p, num_sms, st)
+                  : launch_pair_cfg<false, PairCfg2Wide>(p, num_sms, st);
+    if (p.pair_slots == 2)
+        return bf ? launch_pair_cfg<true, PairCfg2>(p, num_sms, st) : launch_pair_cfg<false, PairCfg2>(p, num_sms, st);
+    return bf ? launch_pair_cfg<true, PairCfg1>(p, num_sms, st) : launch_pair_cfg<false, PairCfg1>(p, num_sms, st);
+}
+
+}  // namespace slorr

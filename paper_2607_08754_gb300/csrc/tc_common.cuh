@@ -1,0 +1,218 @@
+// Pieces shared by the tensor-core GEMM kernels (kernels_tc.cu: one CTA per
+// tile; kernels_tc_pair.cu: a CTA pair per tile): 16-bit packing, the operand
+// maps and orientation of each phase, the symmetric-tile rule, shared-memory
+// operand descriptors and the epilogue of one 128-row block.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace slorr {
+namespace tc {
+
+constexpr int kBM = 128;       // rows of one UMMA M tile (per CTA)
+constexpr int kBNMax = 256;    // columns of a tile
+constexpr int kAccCols = 256;  // fp32 TMEM columns of one 128 x 256 accumulator
+
+template <bool BF16>
+__device__ __forceinline__ uint32_t pack2(float lo, float hi) {
+    if constexpr (BF16) {
+        __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+        return *reinterpret_cast<uint32_t*>(&v);
+    } else {
+        __half2 v = __floats2half2_rn(lo, hi);
+        return *reinterpret_cast<uint32_t*>(&v);
+    }
+}
+
+template <bool BF16>
+__device__ __forceinline__ uint16_t to16(float x) {
+    if constexpr (BF16)
+        return __bfloat16_as_ushort(__float2bfloat16_rn(x));
+    else
+        return __half_as_ushort(__float2half_rn(x));
+}
+
+template <bool BF16>
+__device__ __forceinline__ float2 unpack2(uint32_t u) {
+    if constexpr (BF16) {
+        __nv_bfloat162 v = *reinterpret_cast<__nv_bfloat162*>(&u);
+        return __bfloat1622float2(v);
+    } else {
+        __half2 v = *reinterpret_cast<__half2*>(&u);
+        return __half22float2(v);
+    }
+}
+
+struct PhaseInfo {
+    const void* mapA;
+    const void* mapB;
+    int nkb;
+    bool a_mn;   // A operand MN-major (else K-major)
+    bool b_mn;   // B operand MN-major (else K-major)
+};
+
+// Tensor maps per matrix (kMapsPerMatrix of them, 128 bytes each):
+// X0 K-major, X1 K-major, X0 MN-major, X1 MN-major, A K-major, M K-major.
+__device__ __forceinline__ const void* xmap(const uint8_t* maps, int buf, bool mn) {
+    return maps + (mn ? 2 + buf : buf) * 128;
+}
+
+template <class C>
+__device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmItem& it) {
+    const MatDev& md = p.mats[it.mat];
+    const uint8_t* maps = reinterpret_cast<const uint8_t*>(p.maps) + size_t(it.mat) * kMapsPerMatrix * 128;
+    const bool tr = md.transposed != 0;
+    PhaseInfo pi;
+    if (p.phase == kGram) {
+        pi.a_mn = tr;
+        pi.b_mn = tr;
+        pi.mapA = xmap(maps, p.cur, tr);
+        pi.mapB = pi.mapA;
+        pi.nkb = md.Qpad / C::BK;
+    } else if (p.phase == kPoly) {
+        pi.a_mn = false;
+        pi.b_mn = false;
+        pi.mapA = maps + 4 * 128;
+        pi.mapB = pi.mapA;
+        pi.nkb = md.Ppad / C::BK;
+    } else {
+        pi.a_mn = false;
+        pi.b_mn = !tr;
+        pi.mapA = maps + 5 * 128;
+        pi.mapB = xmap(maps, p.cur, pi.b_mn);
+        pi.nkb = md.Ppad / C::BK;
+    }
+    return pi;
+}
+
+// Symmetric products (Gram, Poly): only tiles holding some 128 x 128 block on
+// or above the diagonal are computed.  Tile (tm, tn) covers row blocks from
+// tm MT on and column blocks 2 tn .. min(2 tn + 1, nb - 1) (nb = Ppad / 128), so
+// it is computed iff its last column block reaches its first row block.
+__device__ __forceinline__ bool sym_tile_computed(int tm, int tn, int Ppad, int mt) {
+    const int last_col_block = min(2 * tn + 1, Ppad / 128 - 1);
+    return last_col_block >= tm * mt;
+}
+
+// Shared-memory descriptor of one K = 16 slice (kk) of a BK-wide K block:
+// K-major: rows of 2 BK bytes (swizzle span), 8-row groups kKSbo apart, slice
+// kk starts 32 bytes further inside the swizzle atom; MN-major: 64-element MN
+// chunks one box apart (LBO), 8-row K groups 1 KB apart (SBO), slice kk starts
+// 16 rows = 2 KB further.
+template <class C>
+__device__ __forceinline__ uint64_t operand_desc(uint32_t base, int kk, bool mn) {
+    return mn ? ptx::sdesc(base + kk * 16 * 128, C::kBoxBytes, 1024, 2u)
+              : ptx::sdesc(base + kk * 32, 16, C::kKSbo, C::kKLayout);
+}
+
+// Epilogue of one 128-row block of a finished tile: this warp's 32 TMEM lanes
+// (rows row0 + 32 quad + [0, 32)) and the tile's 32-column chunks
+// [ch_begin, ch_end) (chunk c: columns tn * 256 + 32 c, TMEM columns t_row + 32 c).
+//   Update: X' rows, stored in W's orientation (transposed iterates take one
+//           coalesced 64-byte segment per column);
+//   Gram / Poly: c * acc (+ b A + a I for Poly) into the Ppad x Ppad output,
+//           plus the transpose of every 128 x 128 block (I, J), J > I, whose
+//           mirror tile is skipped (tiles are MT x 128 rows by 256 columns).
+template <bool BF16, int MT>
+__device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& it, const MatDev& md, int row0,
+                                           uint32_t t_row, int quad, int lane, int ch_begin, int ch_end) {
+    const int row = row0 + quad * 32 + lane;
+    const int nch = ch_end;
+    if (p.phase == kUpdate) {
+        uint16_t* out = reinterpret_cast<uint16_t*>(md.x[p.cur ^ 1]);
+        const int64_t ld = md.ld;
+        for (int ch = ch_begin; ch < nch; ++ch) {
+            uint32_t r[32];
+            ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
+            ptx::tmem_ld_wait();
+            const int col0 = it.tn * kBNMax + ch * 32;
+            if (md.transposed) {
+                // X^T[q][p]: for each column the warp's 32 rows are contiguous
+                uint16_t* dst = out + int64_t(col0) * ld + row;
+#pragma unroll
+                for (int j = 0; j < 32; ++j) dst[int64_t(j) * ld] = to16<BF16>(__uint_as_float(r[j]));
+            } else {
+                uint4 o[4];
+                uint32_t* ow = reinterpret_cast<uint32_t*>(o);
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                    ow[j] = pack2<BF16>(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
+                uint4* dst = reinterpret_cast<uint4*>(out + int64_t(row) * ld + col0);
+#pragma unroll
+                for (int v = 0; v < 4; ++v) dst[v] = o[v];
+            }
+        }
+    } else {
+        uint16_t* out = reinterpret_cast<uint16_t*>(p.phase == kGram ? md.a : md.b);
+        const uint16_t* amat = reinterpret_cast<const uint16_t*>(md.a);
+        const int64_t ld = md.Ppad;
+        const bool poly = p.phase == kPoly;
+        const float cacc = poly ? p.c : 1.f;
+        // Poly reads b A at the output position: loads for the next chunk are
+        // issued before the current chunk is processed.
+        uint4 e_next[4];
+        if (poly) {
+            const uint4* src =
+                reinterpret_cast<const uint4*>(amat + int64_t(row) * ld + it.tn * kBNMax + ch_begin * 32);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) e_next[q] = src[q];
+        }
+        for (int ch = ch_begin; ch < nch; ++ch) {
+            const int col0 = it.tn * kBNMax + ch * 32;
+            const int64_t off = int64_t(row) * ld + col0;
+            uint4 e[4];
+            if (poly) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) e[q] = e_next[q];
+                if (ch + 1 < nch) {
+                    const uint4* src = reinterpret_cast<const uint4*>(amat + off + 32);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) e_next[q] = src[q];
+                }
+            }
+            uint32_t r[32];
+            ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
+            ptx::tmem_ld_wait();
+            uint4 o[4];
+            uint32_t* ow = reinterpret_cast<uint32_t*>(o);
+            const int d = row - col0;  // diagonal element of this row, if in the chunk
+            const uint32_t* ew = reinterpret_cast<const uint32_t*>(e);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                float lo = cacc * __uint_as_float(r[2 * j]);
+                float hi = cacc * __uint_as_float(r[2 * j + 1]);
+                if (poly) {
+                    // M = c A^2 + b A + a I
+                    const float2 x = unpack2<BF16>(ew[j]);
+                    lo = fmaf(p.b, x.x, lo) + (2 * j == d ? p.a : 0.f);
+                    hi = fmaf(p.b, x.y, hi) + (2 * j + 1 == d ? p.a : 0.f);
+                }
+                ow[j] = pack2<BF16>(lo, hi);
+            }
+            uint4* dst = reinterpret_cast<uint4*>(out + off);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) dst[q] = o[q];
+            // The output is symmetric and strictly-lower tiles are skipped:
+            // write the transpose of this 128 x 128 block (I, J), J > I, when
+            // the tile that holds (J, I) is not computed.  The mirrored copy
+            // uses the same rounded 16-bit values, so the stored matrix is
+            // exactly symmetric.
+            const int I = row0 / kBM, J = col0 / kBM;
+            if (J > I && !sym_tile_computed(J / MT, I / 2, md.Ppad, MT)) {
+                uint16_t* tdst = out + int64_t(col0) * ld + row;
+#pragma unroll
+                for (int j = 0; j < 16; ++j) {
+                    tdst[int64_t(2 * j) * ld] = uint16_t(ow[j] & 0xffffu);
+                    tdst[int64_t(2 * j + 1) * ld] = uint16_t(ow[j] >> 16);
+                }
+            }
+        }
+    }
+}
+
+}  // namespace tc
+}  // namespace slorr

@@ -30,6 +30,8 @@ FLAG_TC_BK32 = 4
 FLAG_TC_M128 = 8
 FLAG_TEST_STALL = 16
 FLAG_WRITE_GRAD = 32
+FLAG_TC_SINGLE_CTA = 64
+FLAG_PAIR_ONE_SLOT = 128
 
 
 class SlorrError(RuntimeError):
@@ -89,6 +91,13 @@ def load_library(path: str | None = None) -> ctypes.CDLL:
         "slorr_set_timing": (i32, [vp, i32]),
         "slorr_read_timing": (i32, [vp, ctypes.POINTER(dbl), ctypes.POINTER(i64), i32]),
         "slorr_frob_sq_noalloc": (i32, [vp, i64, i64, i32, vp, vp]),
+        "slorr_pipeline_create": (i32, [ctypes.POINTER(vp), ctypes.POINTER(Shape), i32, ctypes.POINTER(Options),
+                                        i32]),
+        "slorr_pipeline_workspace_size": (i32, [vp, ctypes.POINTER(ctypes.c_size_t)]),
+        "slorr_pipeline_forward_backward": (i32, [vp, ctypes.POINTER(vp), ctypes.POINTER(vp), vp, vp,
+                                                  ctypes.POINTER(vp), ctypes.POINTER(vp), vp, ctypes.c_size_t, vp]),
+        "slorr_pipeline_get_status": (i32, [vp, vp, vp]),
+        "slorr_pipeline_destroy": (None, [vp]),
         "slorr_destroy": (None, [vp]),
         "slorr_status_string": (ctypes.c_char_p, [i32]),
         "slorr_last_error": (ctypes.c_char_p, []),
@@ -243,7 +252,58 @@ def slorr_status_string(status: int) -> str:
     return load_library().slorr_status_string(int(status)).decode()
 
 
+def slorr_pipeline_create(shapes, options: Options | None = None, groups: int = 8) -> ctypes.c_void_p:
+    arr, n = _shapes(shapes)
+    p = ctypes.c_void_p()
+    _check(load_library().slorr_pipeline_create(ctypes.byref(p), arr, n,
+                                                ctypes.byref(options) if options is not None else None, int(groups)))
+    return p
+
+
+def slorr_pipeline_workspace_size(pipe) -> int:
+    out = ctypes.c_size_t()
+    _check(load_library().slorr_pipeline_workspace_size(pipe, ctypes.byref(out)))
+    return out.value
+
+
+def slorr_pipeline_forward_backward(pipe, host_weight_ptrs, host_grad_ptrs, host_loss_ptr, host_per_matrix_ptr,
+                                    dev_weight_ptrs, dev_grad_ptrs, workspace_ptr, workspace_bytes, stream) -> None:
+    _check(load_library().slorr_pipeline_forward_backward(
+        pipe, _ptr_array(host_weight_ptrs), _ptr_array(host_grad_ptrs), ctypes.c_void_p(host_loss_ptr),
+        ctypes.c_void_p(host_per_matrix_ptr or 0), _ptr_array(dev_weight_ptrs), _ptr_array(dev_grad_ptrs),
+        ctypes.c_void_p(workspace_ptr), workspace_bytes, ctypes.c_void_p(stream or 0)))
+
+
+def slorr_pipeline_get_status(pipe, workspace_ptr, stream) -> int:
+    return int(load_library().slorr_pipeline_get_status(pipe, ctypes.c_void_p(workspace_ptr),
+                                                        ctypes.c_void_p(stream or 0)))
+
+
+def slorr_pipeline_destroy(pipe) -> None:
+    load_library().slorr_pipeline_destroy(pipe)
+
+
 # ---- torch-facing convenience ----------------------------------------------------
+
+def make_options(variant: str = "hoyer", compute: str = "fp16", dtype: str = "f32", iters: int = 6,
+                 lam: float = 1.0, eps: float = 1e-7, grad_scale: float = 1.0, ell: float = 1e-3,
+                 cushion: float = -1.0, safety: float = 1.01, flags: int = 0, timeout_s: float = 2.0) -> Options:
+    """slorr_options from keyword arguments (defaults as slorr_default_options)."""
+    o = slorr_default_options()
+    o.variant = VARIANTS[variant]
+    o.compute = COMPUTES[compute]
+    o.dtype = DTYPES[dtype]
+    o.iters = int(iters)
+    o.lambda_ = float(lam)
+    o.eps = float(eps)
+    o.grad_scale = float(grad_scale)
+    o.ell = float(ell)
+    o.cushion = float(cushion)
+    o.safety = float(safety)
+    o.flags = int(flags)
+    o.timeout_s = float(timeout_s)
+    return o
+
 
 class Regularizer:
     """One planned weight set.  Holds the handle and a torch-allocated workspace.
@@ -256,19 +316,8 @@ class Regularizer:
                  iters: int = 6, lam: float = 1.0, eps: float = 1e-7, grad_scale: float = 1.0,
                  ell: float = 1e-3, cushion: float = -1.0, safety: float = 1.01, flags: int = 0,
                  timeout_s: float = 2.0):
-        o = slorr_default_options()
-        o.variant = VARIANTS[variant]
-        o.compute = COMPUTES[compute]
-        o.dtype = DTYPES[dtype]
-        o.iters = int(iters)
-        o.lambda_ = float(lam)
-        o.eps = float(eps)
-        o.grad_scale = float(grad_scale)
-        o.ell = float(ell)
-        o.cushion = float(cushion)
-        o.safety = float(safety)
-        o.flags = int(flags)
-        o.timeout_s = float(timeout_s)
+        o = make_options(variant, compute, dtype, iters, lam, eps, grad_scale, ell, cushion, safety, flags,
+                         timeout_s)
         self.shapes = [(int(m), int(n)) for m, n in shapes]
         self.iters = int(iters)
         self.options = o
@@ -347,6 +396,53 @@ class Regularizer:
         dev = self._ws.device
         s = stream if stream is not None else torch.cuda.current_stream(dev).cuda_stream
         return slorr_get_status(self.handle, self.workspace(dev), s)
+
+
+class Pipeline:
+    """A weight set whose weights and grads live in (page-locked) host memory.
+
+    ``pipe(host_w, host_g, dev_w, dev_g, host_loss)`` enqueues the pipelined
+    forward + backward on the current CUDA stream: copies in, kernels and
+    copies out of consecutive groups of matrices overlap.  ``host_g`` is
+    accumulated into (+=); ``host_loss`` (a page-locked 1-element float tensor)
+    receives lambda * sum_i L_i.  Keyword options as for ``Regularizer``."""
+
+    def __init__(self, shapes, groups: int = 8, **kw):
+        self.shapes = [(int(m), int(n)) for m, n in shapes]
+        self.options = make_options(**kw)
+        self.handle = slorr_pipeline_create(self.shapes, self.options, groups)
+        self.workspace_bytes = slorr_pipeline_workspace_size(self.handle)
+        self._ws = None
+
+    def __del__(self):
+        h = getattr(self, "handle", None)
+        if h is not None and _lib is not None:
+            slorr_pipeline_destroy(h)
+            self.handle = None
+
+    def workspace(self, device):
+        import torch
+        if self._ws is None or self._ws.device != torch.device(device):
+            self._ws = torch.empty(self.workspace_bytes + 256, dtype=torch.uint8, device=device)
+        base = self._ws.data_ptr()
+        return base + (-base) % 256
+
+    def __call__(self, host_weights, host_grads, dev_weights, dev_grads, host_loss, host_per_matrix=None,
+                 stream=None):
+        import torch
+        dev = dev_weights[0].device
+        ws = self.workspace(dev)
+        s = stream if stream is not None else torch.cuda.current_stream(dev).cuda_stream
+        slorr_pipeline_forward_backward(
+            self.handle, [w.data_ptr() for w in host_weights], [g.data_ptr() for g in host_grads],
+            host_loss.data_ptr(), host_per_matrix.data_ptr() if host_per_matrix is not None else 0,
+            [w.data_ptr() for w in dev_weights], [g.data_ptr() for g in dev_grads], ws, self.workspace_bytes, s)
+
+    def status(self, stream=None) -> int:
+        import torch
+        dev = self._ws.device
+        s = stream if stream is not None else torch.cuda.current_stream(dev).cuda_stream
+        return slorr_pipeline_get_status(self.handle, self.workspace(dev), s)
 
 
 class _DeviceArray:

@@ -1,0 +1,131 @@
+"""The CTA-pair tensor-core kernel (the default: tcgen05 cta_group::2, 256 x 256
+tiles over two SMs) against the CUDA-core path, the one-CTA kernels and the
+oracle.
+
+Shapes are chosen to reach every tile case of the pair kernel: a last row tile
+with only 128 rows (the odd CTA's half idle), last column tiles of 128 columns
+(64 B rows per CTA), K-major and MN-major operands (m <= n and m > n), a
+matrix smaller than one tile, and more tiles than pairs.  Test ids carry
+"one_slot" (one accumulator per SM) or "two_slot" (two, the overlapped
+epilogue).
+
+Tolerances are those of the tensor-core-vs-CUDA-core test: 4 ulp of the
+operand type per step (at most 6 steps' worth), and the oracle parity bounds
+(2e-2 for fp16 operands)."""
+
+import numpy as np
+import pytest
+
+import oracle
+import workloads
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+EPS = 1e-7
+MODES = {"one_slot": 128, "two_slot": 0}   # SLORR_FLAG_PAIR_ONE_SLOT, default
+SHAPES = [(256, 768), (768, 256), (320, 1280), (384, 384), (640, 1000), (64, 64), (130, 700), (1000, 130)]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _need_gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2607_08754_gb300 import slorr
+    slorr.load_library()
+
+
+def rel(a, b):
+    return np.linalg.norm(a - b) / np.linalg.norm(b)
+
+
+@pytest.mark.parametrize("mode", list(MODES))
+@pytest.mark.parametrize("compute", ["fp16", "bf16"])
+def test_pair_iterates_match_simt(mode, compute):
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_SIMT_GEMM
+    Ws = [workloads.random_matrix(s, seed=90 + i, std=0.02) for i, s in enumerate(SHAPES)]
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    tc = Regularizer(SHAPES, compute=compute, flags=MODES[mode])
+    st = Regularizer(SHAPES, compute=compute, flags=FLAG_SIMT_GEMM)
+    ulp = 2.0 ** -10 if compute == "fp16" else 2.0 ** -7
+    for k in (1, 2, 6):
+        tc.run_steps(w, k)
+        st.run_steps(w, k)
+        torch.cuda.synchronize()
+        assert tc.status() == 0 and st.status() == 0
+        for i in range(len(SHAPES)):
+            a = tc.iterate(i, k).double().cpu().numpy()
+            b = st.iterate(i, k).double().cpu().numpy()
+            assert rel(a, b) <= 4 * ulp * (k if k < 6 else 6), (k, i, SHAPES[i], rel(a, b))
+
+
+@pytest.mark.parametrize("mode", list(MODES))
+@pytest.mark.parametrize("variant", ["hoyer", "nuclear"])
+def test_pair_forward_backward_matches_oracle(mode, variant):
+    from paper_2607_08754_gb300.slorr import Regularizer
+    Ws = [workloads.random_matrix(s, seed=120 + i, std=0.05) for i, s in enumerate(SHAPES)]
+    Ws += workloads.generate("resnet18", [0, 5, 12, 20])
+    shapes = [W.shape for W in Ws]
+    reg = Regularizer(shapes, variant=variant, compute="fp16", lam=0.5, flags=MODES[mode])
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    g = [torch.zeros_like(x) for x in w]
+    per = torch.empty(len(Ws), device="cuda")
+    loss = reg(w, g, per_matrix=per).item()
+    torch.cuda.synchronize()
+    assert reg.status() == 0
+    co = oracle.pe_coefficients(6)
+    ref_loss, ref_per, ref_inc = oracle.reg_forward_backward([W.astype(np.float64) for W in Ws], variant, co,
+                                                             0.5, EPS)
+    assert abs(loss - ref_loss) <= 2e-2 * abs(ref_loss)
+    per = per.double().cpu().numpy()
+    for i in range(len(Ws)):
+        assert abs(per[i] - ref_per[i]) <= 2e-2 * abs(ref_per[i]), (i, shapes[i])
+        assert rel(g[i].double().cpu().numpy(), ref_inc[i]) <= 2e-2, (i, shapes[i])
+
+
+@pytest.mark.parametrize("mode", ["two_slot"])
+def test_pair_vit_l16_layers_match_single_cta_kernel(mode):
+    """Paper-sized matrices (one ViT-L/16 block): the pair kernel and the one-CTA
+    kernels give the same iterates up to 16-bit rounding."""
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_TC_SINGLE_CTA
+    Ws = workloads.generate("vit_l16", [0, 1, 2, 3])
+    shapes = [W.shape for W in Ws]
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    a_reg = Regularizer(shapes, flags=MODES[mode])
+    b_reg = Regularizer(shapes, flags=FLAG_TC_SINGLE_CTA)
+    a_reg.run_steps(w, 6)
+    b_reg.run_steps(w, 6)
+    torch.cuda.synchronize()
+    assert a_reg.status() == 0 and b_reg.status() == 0
+    for i in range(len(shapes)):
+        a = a_reg.iterate(i, 6).double().cpu().numpy()
+        b = b_reg.iterate(i, 6).double().cpu().numpy()
+        assert rel(a, b) <= 24 * 2.0 ** -10, (i, rel(a, b))
+
+
+@pytest.mark.parametrize("mode", ["two_slot"])
+def test_pair_bounded_wait_timeout_and_recovery(mode):
+    """SLORR_FLAG_TEST_STALL in the pair kernel: the even CTA's MMA thread waits on
+    a barrier nothing arrives on, gives up after timeout_s, and sets both CTAs'
+    abort flags; every role unwinds, the even CTA drains the pair's copies, and
+    the call reports SLORR_ERR_TIMEOUT.  A normal pair call afterwards matches
+    the CUDA-core path."""
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_TEST_STALL, FLAG_SIMT_GEMM
+    shapes = [(256, 512), (384, 128), (640, 1000)]
+    Ws = [workloads.random_matrix(s, 31 + i, 0.05) for i, s in enumerate(shapes)]
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    stall = Regularizer(shapes, flags=MODES[mode] | FLAG_TEST_STALL, timeout_s=0.05)
+    stall.run_steps(w, 1)
+    torch.cuda.synchronize()
+    assert stall.status() == 5          # SLORR_ERR_TIMEOUT
+    assert stall.status() == 0
+    tc = Regularizer(shapes, flags=MODES[mode])
+    st = Regularizer(shapes, flags=FLAG_SIMT_GEMM)
+    tc.run_steps(w, 2)
+    st.run_steps(w, 2)
+    torch.cuda.synchronize()
+    assert tc.status() == 0 and st.status() == 0
+    for i in range(len(shapes)):
+        a = tc.iterate(i, 2).double().cpu().numpy()
+        b = st.iterate(i, 2).double().cpu().numpy()
+        assert rel(a, b) <= 8 * 2.0 ** -10, (i, rel(a, b))

@@ -147,9 +147,11 @@ def test_decoder_560m_layer_fp16():
 
 # ---- tensor cores vs CUDA cores on the same 16-bit arithmetic -------------------
 
-@pytest.mark.parametrize("compute,flags", [("fp16", 0), ("bf16", 0), ("fp16", 4), ("fp16", 8), ("bf16", 8)])
+@pytest.mark.parametrize("compute,flags", [("fp16", 0), ("bf16", 0), ("fp16", 64), ("bf16", 64), ("fp16", 4),
+                                           ("fp16", 8), ("bf16", 8)])
 def test_tensor_core_iterates_match_simt(compute, flags):
-    """Default tiles (256 x 256 for Gram/Update, 128 x 256 for Poly); flags 4 =
+    """Default: the CTA-pair kernel (256 x 256 tiles); 64 = SLORR_FLAG_TC_SINGLE_CTA
+    (one-CTA kernels: 256 x 256 Gram/Update, 128 x 256 Poly); 4 =
     SLORR_FLAG_TC_BK32 (9-stage, 64-byte-swizzle pipeline); 8 =
     SLORR_FLAG_TC_M128 (128 x 256 tiles everywhere)."""
     from paper_2607_08754_gb300.slorr import Regularizer, FLAG_SIMT_GEMM
@@ -247,10 +249,11 @@ def test_bounded_wait_timeout_reports_status_and_context_survives():
     arrives on; with timeout_s = 0.05 each wait gives up, the kernel records
     SLORR_ERR_TIMEOUT in the status word, drains and returns.  The same process
     then runs a normal call that must still match the oracle."""
-    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_TEST_STALL
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_TEST_STALL, FLAG_TC_SINGLE_CTA
     Ws = [workloads.random_matrix((256, 512), 21, 0.05), workloads.random_matrix((384, 128), 22, 0.05)]
     w = [torch.from_numpy(W).cuda() for W in Ws]
-    stall = Regularizer([W.shape for W in Ws], flags=FLAG_TEST_STALL, timeout_s=0.05)
+    # the one-CTA kernel here; tests/test_gpu_pair.py stalls the pair kernel
+    stall = Regularizer([W.shape for W in Ws], flags=FLAG_TEST_STALL | FLAG_TC_SINGLE_CTA, timeout_s=0.05)
     stall.run_steps(w, 1)
     torch.cuda.synchronize()
     assert stall.status() == 5          # SLORR_ERR_TIMEOUT

@@ -185,3 +185,28 @@ def test_layer_partition_two_ranks_gloo(lib):
     assert loss == pytest.approx(ref_loss, rel=1e-12)
     for g, r in zip(grads, ref):
         assert np.allclose(g, r, rtol=1e-12, atol=1e-15)
+
+
+def test_pipeline_validation_and_workspace(lib):
+    """The host-buffer pipeline rejects bad requests before any CUDA call, and
+    its workspace holds every group's plan."""
+    shapes = [(64, 576), (128, 1152), (256, 2304), (512, 4608), (1000, 512)]
+    with pytest.raises(slorr.SlorrError) as e:
+        slorr.slorr_pipeline_create(shapes, None, 0)
+    assert e.value.status == 1
+    with pytest.raises(slorr.SlorrError):
+        slorr.slorr_pipeline_create([(0, 4)], None, 2)
+    single = slorr.slorr_workspace_size(slorr.slorr_create(shapes))
+    for groups in (1, 2, 5, 50):
+        p = slorr.slorr_pipeline_create(shapes, None, groups)
+        ws = slorr.slorr_pipeline_workspace_size(p)
+        assert ws >= single - 1024 * groups   # each group carries its own plan
+        with pytest.raises(slorr.SlorrError) as e:   # NULL host pointer
+            slorr.slorr_pipeline_forward_backward(p, [256] * 4 + [0], [512] * 5, 768, 0, [1024] * 5, [2048] * 5,
+                                                  4096, ws, 0)
+        assert e.value.status == 1
+        with pytest.raises(slorr.SlorrError) as e:   # short workspace
+            slorr.slorr_pipeline_forward_backward(p, [256] * 5, [512] * 5, 768, 0, [1024] * 5, [2048] * 5,
+                                                  4096, ws - 1, 0)
+        assert e.value.status == 4
+        slorr.slorr_pipeline_destroy(p)
