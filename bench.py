@@ -71,7 +71,7 @@ def parse():
                     help="fwd_bwd: value + gradient accumulated into .grad (Alg. 2); descent: the in-place "
                          "regularizer-only step W -= eta lambda G (Alg. 1, last line)")
     ap.add_argument("--eta", type=float, default=1e-4, help="step size of --op descent")
-    ap.add_argument("--e2e-groups", type=int, default=8,
+    ap.add_argument("--e2e-groups", type=int, default=16,
                     help="groups of the host-buffer pipeline timed as e2e (slorr_pipeline_forward_backward)")
     return ap.parse_args()
 
