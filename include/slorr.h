@@ -113,6 +113,9 @@ typedef struct slorr_options {
                                        implied by TC_BK32 and TC_M128 (tuning)           */
 #define SLORR_FLAG_PAIR_ONE_SLOT 128 /* CTA-pair kernel with one accumulator per SM (no
                                        epilogue overlap; tuning)                         */
+#define SLORR_FLAG_TC_QUAD     256  /* clusters of two CTA pairs computing two tiles that
+                                       share an operand, loaded once by TMA multicast
+                                       (tuning)                                          */
 
 /* Fill *opt with the defaults listed beside each field above (App. C.1: T = 6,
  * ell = 1e-3, degree 5; eps, lambda and grad_scale as in Listing 1 / Alg. 2). */

@@ -59,13 +59,15 @@ struct slorr_handle {
     int esize;
     // item lists (host)
     std::vector<GemmItem> tc_items[3];
+    std::vector<GemmItem> quad_items[3];  // super-tiles: 2 items each (the second may be empty)
     std::vector<GemmItem> simt_items[3];
     std::vector<MemItem> w_items;  // tiles of W (sumsq, dot, combine)
     std::vector<MemItem> x_items;  // tiles of the padded iterate (cast)
     int total_w_tiles = 0;
     // workspace layout
     size_t off_status = 0, off_counters = 0, off_scalars = 0, off_partials = 0, off_tilebase = 0,
-           off_tilecount = 0, off_mats = 0, off_maps = 0, off_tc_items[3] = {}, off_simt_items[3] = {},
+           off_tilecount = 0, off_mats = 0, off_maps = 0, off_tc_items[3] = {}, off_quad_items[3] = {},
+           off_simt_items[3] = {},
            off_w_items = 0, off_x_items = 0, off_ptrs = 0, off_plan_end = 0, total_bytes = 0;
     // device state
     const void* prepared_ws = nullptr;
@@ -125,11 +127,50 @@ bool valid_options(const slorr_options& o, std::string* why) {
     return true;
 }
 
+// Super-tiles of the 4-CTA kernel for one matrix and phase: two 256 x 256
+// tiles that share an operand, one per CTA pair of the cluster.  The tiles of
+// each row (the same A rows) are paired left to right; a row's odd last tile
+// waits, and the leftovers of each column (the same B columns) are paired top
+// to bottom; a final odd leftover runs alone (second item empty, msz = 0).
+// Gram and Poly keep only the tiles on or above the diagonal, as the pair
+// kernel does.
+void add_quad_items(std::vector<GemmItem>& out, int mat, int ph, int Ppad, int N) {
+    const GemmItem none{uint16_t(mat), 0, 0, 0, 0, 0};
+    std::vector<std::vector<GemmItem>> by_col((N + 255) / 256);
+    for (int tm = 0; tm * 256 < Ppad; ++tm) {
+        const int msz = std::min(256, Ppad - tm * 256);
+        std::vector<GemmItem> row;
+        for (int tn = 0; tn * 256 < N; ++tn) {
+            const int nsz = std::min(256, N - tn * 256);
+            if (ph != kUpdate && (2 * tn + nsz / 128 - 1) < tm * 2) continue;
+            row.push_back(GemmItem{uint16_t(mat), uint16_t(tm), uint16_t(tn), uint16_t(nsz), uint16_t(msz), 0});
+        }
+        size_t j = 0;
+        for (; j + 1 < row.size(); j += 2) {
+            out.push_back(row[j]);
+            out.push_back(row[j + 1]);
+        }
+        if (j < row.size()) by_col[row[j].tn].push_back(row[j]);
+    }
+    for (auto& col : by_col) {
+        size_t j = 0;
+        for (; j + 1 < col.size(); j += 2) {
+            out.push_back(col[j]);
+            out.push_back(col[j + 1]);
+        }
+        if (j < col.size()) {
+            out.push_back(col[j]);
+            out.push_back(none);
+        }
+    }
+}
+
 void build_plan(slorr_handle* h) {
     const int count = int(h->shapes.size());
     h->geom.resize(count);
     for (int i = 0; i < 3; ++i) {
         h->tc_items[i].clear();
+        h->quad_items[i].clear();
         h->simt_items[i].clear();
     }
     h->w_items.clear();
@@ -174,6 +215,7 @@ void build_plan(slorr_handle* h) {
                         GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), uint16_t(nsz), uint16_t(msz), 0});
                 }
             }
+            add_quad_items(h->quad_items[ph], i, ph, g.Ppad, N);
             for (int tm = 0; tm < g.Ppad / 64; ++tm)
                 for (int tn = 0; tn < N / 64; ++tn)
                     h->simt_items[ph].push_back(GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), 64, 64, 0});
@@ -188,6 +230,19 @@ void build_plan(slorr_handle* h) {
         };
         std::stable_sort(h->tc_items[ph].begin(), h->tc_items[ph].end(),
                          [&](const GemmItem& a, const GemmItem& b) { return kdim(a) > kdim(b); });
+        // super-tiles move as units of two items
+        std::vector<std::pair<GemmItem, GemmItem>> sup;
+        for (size_t j = 0; j + 1 < h->quad_items[ph].size(); j += 2)
+            sup.push_back({h->quad_items[ph][j], h->quad_items[ph][j + 1]});
+        std::stable_sort(sup.begin(), sup.end(), [&](const std::pair<GemmItem, GemmItem>& a,
+                                                     const std::pair<GemmItem, GemmItem>& b) {
+            return kdim(a.first) > kdim(b.first);
+        });
+        h->quad_items[ph].clear();
+        for (auto& pr : sup) {
+            h->quad_items[ph].push_back(pr.first);
+            h->quad_items[ph].push_back(pr.second);
+        }
     }
 
     // Workspace layout.
@@ -211,6 +266,8 @@ void build_plan(slorr_handle* h) {
     for (int ph = 0; ph < 3; ++ph) {
         h->off_tc_items[ph] = off;
         off = align_up(off + h->tc_items[ph].size() * sizeof(GemmItem), 256);
+        h->off_quad_items[ph] = off;
+        off = align_up(off + h->quad_items[ph].size() * sizeof(GemmItem), 256);
         h->off_simt_items[ph] = off;
         off = align_up(off + h->simt_items[ph].size() * sizeof(GemmItem), 256);
     }
@@ -327,6 +384,7 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
     put(plan, h->off_maps - base, maps.data(), maps.size());
     for (int ph = 0; ph < 3; ++ph) {
         put(plan, h->off_tc_items[ph] - base, h->tc_items[ph].data(), h->tc_items[ph].size());
+        put(plan, h->off_quad_items[ph] - base, h->quad_items[ph].data(), h->quad_items[ph].size());
         put(plan, h->off_simt_items[ph] - base, h->simt_items[ph].data(), h->simt_items[ph].size());
     }
     put(plan, h->off_w_items - base, h->w_items.data(), h->w_items.size());
@@ -488,6 +546,7 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
     g.bk = tc_bk(h);
     g.test_stall = (h->opt.flags & SLORR_FLAG_TEST_STALL) ? 1 : 0;
     const bool pair = tc_pair(h);
+    const bool quad = pair && (h->opt.flags & SLORR_FLAG_TC_QUAD) != 0;
     g.pair_slots = (h->opt.flags & SLORR_FLAG_PAIR_ONE_SLOT) ? 1 : 2;
     for (int t = 0; t < steps; ++t) {
         g.cur = t & 1;
@@ -498,7 +557,11 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
             g.phase = ph;
             g.mt = tc_mt(h, ph);
             Traced tr(h, 2 + ph, st);
-            if (use_tc) {
+            if (use_tc && quad) {
+                g.items = reinterpret_cast<const GemmItem*>(ws + h->off_quad_items[ph]);
+                g.num_items = int(h->quad_items[ph].size() / 2);
+                e = launch_gemm_tc_quad(g, h->elem, h->num_sms, st);
+            } else if (use_tc) {
                 g.items = reinterpret_cast<const GemmItem*>(ws + h->off_tc_items[ph]);
                 g.num_items = int(h->tc_items[ph].size());
                 e = pair ? launch_gemm_tc_pair(g, h->elem, h->num_sms, st)

@@ -145,6 +145,8 @@ cudaError_t launch_sum_parts(const float* parts, int n, float* out, cudaStream_t
 cudaError_t launch_gemm_simt(const GemmLaunch& p, int elem, cudaStream_t s);
 cudaError_t launch_gemm_tc(const GemmLaunch& p, int elem, int grid, cudaStream_t s);
 cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t s);
+// items: 2 per super-tile (num_items super-tiles); see kernels_tc_quad.cu
+cudaError_t launch_gemm_tc_quad(const GemmLaunch& p, int elem, int num_sms, cudaStream_t s);
 int tc_smem_bytes();
 
 // Records the message slorr_last_error() returns on this thread (api.cu).

@@ -156,6 +156,19 @@ __device__ __forceinline__ void tma_load_2d_pair(void* dst, const void* map, uin
         : "memory");
 }
 
+// As tma_load_2d_pair, multicast: the box lands at the same shared-memory
+// offset in every CTA of `cta_mask`, and its bytes are counted, for each
+// destination, on the barrier at bar_cluster's offset in that destination's
+// pair leader (the even CTA of its pair).
+__device__ __forceinline__ void tma_load_2d_pair_mc(void* dst, const void* map, uint32_t bar_cluster, int32_t x,
+                                                    int32_t y, uint16_t cta_mask) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+        ".multicast::cluster [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
+        "l"(map), "r"(bar_cluster), "r"(x), "r"(y), "h"(cta_mask)
+        : "memory");
+}
+
 // Hint: bring one box of a tensor into L2 (no shared memory, no completion).
 __device__ __forceinline__ void tma_prefetch_l2_2d(const void* map, int32_t x, int32_t y) {
     asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(map), "r"(x),

@@ -32,6 +32,7 @@ FLAG_TEST_STALL = 16
 FLAG_WRITE_GRAD = 32
 FLAG_TC_SINGLE_CTA = 64
 FLAG_PAIR_ONE_SLOT = 128
+FLAG_TC_QUAD = 256
 
 
 class SlorrError(RuntimeError):
