@@ -96,12 +96,21 @@ __device__ __forceinline__ void record_timeout(const GemmLaunch& p, const PairSm
     atomicOr(p.status, kStatusTimeout);
 }
 
+// Diagonal tiles of the symmetric products (Gram A = X X^T, Poly A A): with
+// tm == tn and a full 256 x 256 tile, each CTA's A rows and B columns are the
+// same 128 rows of the same matrix, so they are copied once and both UMMA
+// operands read them (the B descriptor points at the A half).
+__device__ __forceinline__ bool shared_operand(const GemmLaunch& p, const GemmItem& it) {
+    return p.phase != kUpdate && it.tm == it.tn && it.msz == 2 * kBM && it.nsz == kBNMax;
+}
+
 // Bytes one CTA of the pair copies per stage of a tile: its A rows, unless they
 // lie beyond the matrix (the UMMA rows they would feed are never stored), and
-// its half of the B columns.
+// its half of the B columns, unless they are its A rows (shared_operand).
 template <class C>
-__device__ __forceinline__ uint32_t pair_stage_bytes(const GemmItem& it, int rank) {
-    return (rank * kBM < it.msz ? uint32_t(C::kABytes) : 0u) + uint32_t(it.nsz / 2) * C::BK * 2;
+__device__ __forceinline__ uint32_t pair_stage_bytes(const GemmLaunch& p, const GemmItem& it, int rank) {
+    const uint32_t a = rank * kBM < it.msz ? uint32_t(C::kABytes) : 0u;
+    return shared_operand(p, it) ? a : a + uint32_t(it.nsz / 2) * C::BK * 2;
 }
 
 template <class C>
@@ -113,6 +122,7 @@ __device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, 
         const GemmItem it = p.items[idx];
         const PhaseInfo pi = phase_info<C>(p, it);
         const bool load_a = rank * kBM < it.msz;
+        const bool load_b = !shared_operand(p, it);
         const int bhalf = it.nsz / 2;  // 64 or 128 rows of B per CTA
         for (int kb = 0; kb < pi.nkb; ++kb) {
             if (!ptx::mbar_wait(&s.empty[stage], phase ^ 1u, s.abort, p.timeout_ns)) {
@@ -129,7 +139,7 @@ __device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, 
                     const int mn = it.tm * (2 * kBM) + rank * kBM + b * 64;
                     ptx::tma_load_2d_pair(sa + b * C::kBoxBytes, pi.mapA, bar, pi.a_mn ? mn : k, pi.a_mn ? k : mn);
                 }
-            for (int j = 0; j < bhalf / 64; ++j) {
+            for (int j = 0; load_b && j < bhalf / 64; ++j) {
                 const int mn = it.tn * kBNMax + rank * bhalf + j * 64;
                 ptx::tma_load_2d_pair(sb + j * C::kBoxBytes, pi.mapB, bar, pi.b_mn ? mn : k, pi.b_mn ? k : mn);
             }
@@ -152,7 +162,7 @@ struct KCursor {
         if (idx < p->num_items) {
             const GemmItem it = p->items[idx];
             nkb = phase_info<C>(*p, it).nkb;
-            bytes = pair_stage_bytes<C>(it, 0) + pair_stage_bytes<C>(it, 1);
+            bytes = pair_stage_bytes<C>(*p, it, 0) + pair_stage_bytes<C>(*p, it, 1);
         }
     }
     __device__ KCursor(const GemmLaunch& gp, int first, int stride) : p(&gp), idx(first), kb(0), nkb(0), step(stride),
@@ -221,7 +231,7 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
             }
             ptx::tc_fence_after();
             const uint32_t a0 = ptx::smem_u32(s.stages + size_t(stage) * C::kStageBytes);
-            const uint32_t b0 = a0 + C::kABytes;
+            const uint32_t b0 = shared_operand(p, it) ? a0 : a0 + C::kABytes;
 #pragma unroll
             for (int kk = 0; kk < C::BK / 16; ++kk)
                 ptx::umma_f16_pair(d_tmem, operand_desc<C>(a0, kk, pi.a_mn), operand_desc<C>(b0, kk, pi.b_mn), idesc,
