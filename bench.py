@@ -71,8 +71,9 @@ def parse():
                     help="fwd_bwd: value + gradient accumulated into .grad (Alg. 2); descent: the in-place "
                          "regularizer-only step W -= eta lambda G (Alg. 1, last line)")
     ap.add_argument("--eta", type=float, default=1e-4, help="step size of --op descent")
-    ap.add_argument("--e2e-groups", type=int, default=16,
-                    help="groups of the host-buffer pipeline timed as e2e (slorr_pipeline_forward_backward)")
+    ap.add_argument("--e2e-groups", type=int, default=0,
+                    help="groups of the host-buffer pipeline timed as e2e (slorr_pipeline_forward_backward); "
+                         "0: about 64 MiB of weights per group, at most 16")
     return ap.parse_args()
 
 
@@ -311,7 +312,7 @@ def main():
     h2d = wbytes + gbytes
     d2h = (wbytes if descent else gbytes) + 4
 
-    pipe = None if descent else slorr.Pipeline(shapes, groups=args.e2e_groups, variant=args.variant,
+    pipe = None if descent else slorr.Pipeline(shapes, groups=args.e2e_groups or None, variant=args.variant,
                                                compute=args.compute, iters=args.iters, lam=1.0, flags=args.flags)
 
     def e2e_step():
@@ -383,7 +384,7 @@ def main():
             "e2e": {"value": e2e_val, "unit": "TFLOP/s", "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h,
                     "call": "slorr_reg_descent_step with torch copies" if descent else
-                            f"slorr_pipeline_forward_backward, {args.e2e_groups} groups"},
+                            f"slorr_pipeline_forward_backward, {pipe.groups} groups"},
             "clocks": clk,
         }
         if not args.no_cpu_baseline:

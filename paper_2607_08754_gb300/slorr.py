@@ -408,8 +408,20 @@ class Pipeline:
     accumulated into (+=); ``host_loss`` (a page-locked 1-element float tensor)
     receives lambda * sum_i L_i.  Keyword options as for ``Regularizer``."""
 
-    def __init__(self, shapes, groups: int = 8, **kw):
+    @staticmethod
+    def auto_groups(shapes, dtype: str = "f32") -> int:
+        """About 64 MiB of weights per group, 1 to 16 groups: enough groups for the
+        copies to overlap the kernels, few enough that a group's launches stay
+        cheap next to its copies."""
+        esz = 4 if dtype == "f32" else 2
+        total = sum(int(m) * int(n) for m, n in shapes) * esz
+        return max(1, min(16, total // (64 << 20)))
+
+    def __init__(self, shapes, groups: int | None = None, **kw):
         self.shapes = [(int(m), int(n)) for m, n in shapes]
+        if groups is None:
+            groups = self.auto_groups(self.shapes, kw.get("dtype", "f32"))
+        self.groups = int(groups)
         self.options = make_options(**kw)
         self.handle = slorr_pipeline_create(self.shapes, self.options, groups)
         self.workspace_bytes = slorr_pipeline_workspace_size(self.handle)
