@@ -116,6 +116,11 @@ typedef struct slorr_options {
 #define SLORR_FLAG_TC_QUAD     256  /* clusters of two CTA pairs computing two tiles that
                                        share an operand, loaded once by TMA multicast
                                        (tuning)                                          */
+#define SLORR_FLAG_NO_PDL      512  /* launch every kernel after the previous one completes.
+                                       By default the memory passes and the CTA-pair
+                                       kernel are programmatic dependents of the kernel
+                                       before them, so each one's launch and prologue
+                                       overlap the previous one's tail (tuning)          */
 
 /* Fill *opt with the defaults listed beside each field above (App. C.1: T = 6,
  * ell = 1e-3, degree 5; eps, lambda and grad_scale as in Listing 1 / Alg. 2). */

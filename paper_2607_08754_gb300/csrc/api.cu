@@ -95,6 +95,9 @@ bool tc_pair(const slorr_handle* h) {
     return (h->opt.flags & (SLORR_FLAG_TC_SINGLE_CTA | SLORR_FLAG_TC_BK32 | SLORR_FLAG_TC_M128)) == 0;
 }
 
+// Programmatic dependent launch of the memory passes and the pair kernel.
+bool use_pdl(const slorr_handle* h) { return (h->opt.flags & SLORR_FLAG_NO_PDL) == 0; }
+
 // K depth of the tensor-core pipeline stages for this handle.
 int tc_bk(const slorr_handle* h) {
     if (tc_pair(h)) return 64;  // the pair kernel's stages are K = 64
@@ -471,6 +474,7 @@ MemLaunch mem_params(slorr_handle* h, uint8_t* ws, float* loss, float* per, int 
     p.wdtype = h->opt.dtype == SLORR_BF16 ? 1 : 0;
     p.variant = h->opt.variant;
     p.out_mode = (h->opt.flags & SLORR_FLAG_WRITE_GRAD) ? kOutOverwrite : kOutAccumulate;
+    p.pdl = use_pdl(h) ? 1 : 0;
     p.eps = h->opt.eps;
     p.lambda = h->opt.lambda;
     p.grad_scale = h->opt.grad_scale;
@@ -548,6 +552,7 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
     const bool pair = tc_pair(h);
     const bool quad = pair && (h->opt.flags & SLORR_FLAG_TC_QUAD) != 0;
     g.pair_slots = (h->opt.flags & SLORR_FLAG_PAIR_ONE_SLOT) ? 1 : 2;
+    g.pdl = (use_pdl(h) && pair && !quad) ? 1 : 0;
     for (int t = 0; t < steps; ++t) {
         g.cur = t & 1;
         g.a = float(h->coeffs[3 * t + 0]);

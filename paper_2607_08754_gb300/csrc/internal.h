@@ -16,6 +16,7 @@
 #include <cstddef>
 #include <cstdint>
 #include <string>
+#include <utility>
 
 #include <cuda_runtime.h>
 
@@ -99,6 +100,7 @@ struct GemmLaunch {
     int32_t mt;                // 128-row M tiles per CTA tile: 1 or 2 (256 x 256 tiles)
     int32_t test_stall;        // 1: the MMA thread first waits on a barrier nothing arrives on
     int32_t pair_slots;        // CTA-pair kernel: accumulators per CTA (1 or 2)
+    int32_t pdl;               // launch with programmatic dependent launch
 };
 
 // Tensor maps per matrix: X0 K-major, X1 K-major, X0 MN-major, X1 MN-major,
@@ -128,6 +130,7 @@ struct MemLaunch {
     int32_t wdtype;            // 0 fp32, 1 bf16 weights/grads
     int32_t variant;           // 0 Hoyer, 1 Nuc
     int32_t out_mode;          // kOutAccumulate, kOutOverwrite or kOutDescent
+    int32_t pdl;               // launch with programmatic dependent launch
     float eps, lambda, grad_scale;
     float* loss_out;
     float* per_matrix_out;
@@ -148,6 +151,27 @@ cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cuda
 // items: 2 per super-tile (num_items super-tiles); see kernels_tc_quad.cu
 cudaError_t launch_gemm_tc_quad(const GemmLaunch& p, int elem, int num_sms, cudaStream_t s);
 int tc_smem_bytes();
+
+#if defined(__CUDACC__)
+// Launches `kernel` on `st`; with pdl, as a programmatic dependent of the
+// stream's previous kernel (the kernel must call griddep_wait() before it
+// reads anything an earlier kernel wrote).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_kernel(void (*kernel)(KArgs...), unsigned grid, unsigned block, size_t smem, cudaStream_t st,
+                          bool pdl, Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(block);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = pdl ? attr : nullptr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+#endif
 
 // Records the message slorr_last_error() returns on this thread (api.cu).
 void set_last_error(const std::string& msg);

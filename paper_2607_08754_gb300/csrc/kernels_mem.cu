@@ -23,6 +23,7 @@
 #include <cuda_fp16.h>
 
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace slorr {
 namespace {
@@ -195,6 +196,8 @@ __device__ __forceinline__ TileCoord tile_coord(const MemItem& it) {
 template <typename TW>
 // Six blocks per SM (at most 40 registers a thread).
 __global__ void __launch_bounds__(kThreads, 6) sumsq_kernel(const MemLaunch p) {
+    ptx::griddep_wait();  // inputs come from the previous kernel (programmatic launch)
+    ptx::griddep_launch_dependents();
     __shared__ float red[kThreads / 32];
     const MemItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
@@ -214,6 +217,8 @@ __global__ void __launch_bounds__(kThreads, 6) sumsq_kernel(const MemLaunch p) {
 // Items tile the padded buffer (rows x ld); zeros are written to the padding.
 template <typename TW, typename TX>
 __global__ void __launch_bounds__(kThreads) cast_kernel(const MemLaunch p) {
+    ptx::griddep_wait();  // inputs come from the previous kernel (programmatic launch)
+    ptx::griddep_launch_dependents();
     const MemItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
     const TW* W = reinterpret_cast<const TW*>(p.weights[it.mat]);
@@ -242,6 +247,8 @@ template <typename TW, typename TX>
 // (68 registers) the pass reached 0.69 of the measured HBM bandwidth on the
 // ViT-L/16 set, with four it is 11% faster.
 __global__ void __launch_bounds__(kThreads, 4) dot_kernel(const MemLaunch p) {
+    ptx::griddep_wait();  // inputs come from the previous kernel (programmatic launch)
+    ptx::griddep_launch_dependents();
     __shared__ float red[kThreads / 32];
     const MemItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
@@ -334,6 +341,8 @@ __device__ bool finalize_matrix(const MemLaunch& p, int which, int mat, double t
 //              The last block to finish also writes the values L_i and the loss
 //              lambda * sum_i L_i (finalize_loss).
 __global__ void __launch_bounds__(128) finalize_kernel(const MemLaunch p, int which) {
+    ptx::griddep_wait();  // inputs come from the previous kernel (programmatic launch)
+    ptx::griddep_launch_dependents();
     __shared__ double red[4];
     __shared__ int is_last;
     const int mat = blockIdx.x;
@@ -354,6 +363,8 @@ template <typename TW, typename TX>
 // thread needs 128 registers (two blocks per SM); in halves it fits four
 // blocks per SM, 20% faster on the ViT-L/16 set.
 __global__ void __launch_bounds__(kThreads, 4) combine_kernel(const MemLaunch p) {
+    ptx::griddep_wait();  // inputs come from the previous kernel (programmatic launch)
+    ptx::griddep_launch_dependents();
     const MemItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
     const TileCoord tc = tile_coord(it);
@@ -398,45 +409,41 @@ __global__ void __launch_bounds__(kThreads, 4) combine_kernel(const MemLaunch p)
 
 cudaError_t launch_sumsq(const MemLaunch& p, cudaStream_t s) {
     if (p.num_items == 0) return cudaSuccess;
-    if (p.wdtype == 0)
-        sumsq_kernel<float><<<p.num_items, kThreads, 0, s>>>(p);
-    else
-        sumsq_kernel<__nv_bfloat16><<<p.num_items, kThreads, 0, s>>>(p);
-    return cudaGetLastError();
+    if (p.wdtype == 0) return launch_kernel(sumsq_kernel<float>, p.num_items, kThreads, 0, s, p.pdl != 0, p);
+    return launch_kernel(sumsq_kernel<__nv_bfloat16>, p.num_items, kThreads, 0, s, p.pdl != 0, p);
 }
 
+#define SLORR_LAUNCH_WX(KERNEL, TW, TX) launch_kernel(KERNEL<TW, TX>, p.num_items, kThreads, 0, s, p.pdl != 0, p)
 #define SLORR_DISPATCH_WX(KERNEL)                                                                  \
     do {                                                                                           \
         if (p.wdtype == 0) {                                                                       \
-            if (p.elem == kF32) KERNEL<float, float><<<p.num_items, kThreads, 0, s>>>(p);          \
-            else if (p.elem == kF16) KERNEL<float, __half><<<p.num_items, kThreads, 0, s>>>(p);    \
-            else KERNEL<float, __nv_bfloat16><<<p.num_items, kThreads, 0, s>>>(p);                \
-        } else {                                                                                   \
-            if (p.elem == kF32) KERNEL<__nv_bfloat16, float><<<p.num_items, kThreads, 0, s>>>(p);  \
-            else if (p.elem == kF16) KERNEL<__nv_bfloat16, __half><<<p.num_items, kThreads, 0, s>>>(p); \
-            else KERNEL<__nv_bfloat16, __nv_bfloat16><<<p.num_items, kThreads, 0, s>>>(p);        \
+            if (p.elem == kF32) return SLORR_LAUNCH_WX(KERNEL, float, float);                      \
+            if (p.elem == kF16) return SLORR_LAUNCH_WX(KERNEL, float, __half);                     \
+            return SLORR_LAUNCH_WX(KERNEL, float, __nv_bfloat16);                                  \
         }                                                                                          \
+        if (p.elem == kF32) return SLORR_LAUNCH_WX(KERNEL, __nv_bfloat16, float);                  \
+        if (p.elem == kF16) return SLORR_LAUNCH_WX(KERNEL, __nv_bfloat16, __half);                 \
+        return SLORR_LAUNCH_WX(KERNEL, __nv_bfloat16, __nv_bfloat16);                              \
     } while (0)
 
 cudaError_t launch_cast(const MemLaunch& p, cudaStream_t s) {
     if (p.num_items == 0) return cudaSuccess;
     SLORR_DISPATCH_WX(cast_kernel);
-    return cudaGetLastError();
 }
 
 cudaError_t launch_dot(const MemLaunch& p, cudaStream_t s) {
     if (p.num_items == 0) return cudaSuccess;
     SLORR_DISPATCH_WX(dot_kernel);
-    return cudaGetLastError();
 }
 
 cudaError_t launch_finalize(const MemLaunch& p, int which, cudaStream_t s) {
-    finalize_kernel<<<p.count, 128, 0, s>>>(p, which);
-    return cudaGetLastError();
+    return launch_kernel(finalize_kernel, p.count, 128, 0, s, p.pdl != 0, p, which);
 }
 
 // One thread: out = sum of the n partial losses in index order (double).
 __global__ void sum_parts_kernel(const float* __restrict__ parts, int n, float* __restrict__ out) {
+    ptx::griddep_wait();
+    ptx::griddep_launch_dependents();
     if (threadIdx.x == 0 && blockIdx.x == 0) {
         double t = 0.0;
         for (int i = 0; i < n; ++i) t += static_cast<double>(parts[i]);
@@ -445,14 +452,12 @@ __global__ void sum_parts_kernel(const float* __restrict__ parts, int n, float* 
 }
 
 cudaError_t launch_sum_parts(const float* parts, int n, float* out, cudaStream_t s) {
-    sum_parts_kernel<<<1, 32, 0, s>>>(parts, n, out);
-    return cudaGetLastError();
+    return launch_kernel(sum_parts_kernel, 1, 32, 0, s, false, parts, n, out);
 }
 
 cudaError_t launch_combine(const MemLaunch& p, cudaStream_t s) {
     if (p.num_items == 0) return cudaSuccess;
     SLORR_DISPATCH_WX(combine_kernel);
-    return cudaGetLastError();
 }
 
 }  // namespace slorr

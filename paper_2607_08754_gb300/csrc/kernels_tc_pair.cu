@@ -347,6 +347,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(C::kThreads, 1)
     // The UMMAs address both CTAs' accumulators with the even CTA's TMEM
     // address: the two allocations must agree, else no work is done.
     const uint32_t peer_base = ptx::ld_cluster_u32(ptx::mapa(ptx::smem_u32(s.tmem_slot), s.peer));
+    // Under programmatic dependent launch everything above overlapped the
+    // previous kernel's tail; wait for its results before any role starts.
+    ptx::griddep_wait();
+    ptx::griddep_launch_dependents();
     if (peer_base != tmem_base) {
         if (threadIdx.x == 0) atomicOr(p.status, kStatusInternal);
     } else if (warp == 0) {
@@ -385,8 +389,7 @@ cudaError_t launch_pair_cfg(const GemmLaunch& p, int num_sms, cudaStream_t st) {
         max_pairs = clusters < num_sms / 2 ? clusters : num_sms / 2;
     }
     const int npairs = p.num_items < max_pairs ? p.num_items : max_pairs;
-    tc_pair_kernel<BF16, C><<<2 * npairs, C::kThreads, C::kSmemBytes, st>>>(p);
-    return cudaGetLastError();
+    return launch_kernel(tc_pair_kernel<BF16, C>, unsigned(2 * npairs), C::kThreads, C::kSmemBytes, st, p.pdl != 0, p);
 }
 
 }  // namespace

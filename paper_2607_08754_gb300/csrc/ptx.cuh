@@ -84,6 +84,20 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
     }
 }
 
+// ---- programmatic dependent launch -------------------------------------------------
+
+// Blocks until every grid this one depends on programmatically has completed
+// and its memory is visible (a no-op when the kernel was launched without the
+// programmatic-serialisation attribute).
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Lets the next grid in the stream be scheduled once every block of this grid
+// has issued this (or exited); that grid still waits in griddep_wait() for
+// this one to complete before it reads anything.
+__device__ __forceinline__ void griddep_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ---- thread-block clusters ------------------------------------------------------
 
 __device__ __forceinline__ uint32_t cluster_ctarank() {

@@ -33,6 +33,7 @@ FLAG_WRITE_GRAD = 32
 FLAG_TC_SINGLE_CTA = 64
 FLAG_PAIR_ONE_SLOT = 128
 FLAG_TC_QUAD = 256
+FLAG_NO_PDL = 512
 
 
 class SlorrError(RuntimeError):

@@ -129,3 +129,24 @@ def test_pair_bounded_wait_timeout_and_recovery(mode):
         a = tc.iterate(i, 2).double().cpu().numpy()
         b = st.iterate(i, 2).double().cpu().numpy()
         assert rel(a, b) <= 8 * 2.0 ** -10, (i, rel(a, b))
+
+
+def test_programmatic_dependent_launch_is_bit_identical():
+    """Programmatic dependent launch (the default; SLORR_FLAG_NO_PDL turns it
+    off) only changes when kernels launch, not what they compute: three
+    consecutive calls (accumulating into .grad) and the loss equal the
+    serialised launches bit for bit."""
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_NO_PDL
+    Ws = [workloads.random_matrix(s, seed=900 + i, std=0.05) for i, s in enumerate(SHAPES)]
+    out = []
+    for flags in (0, FLAG_NO_PDL):
+        reg = Regularizer(SHAPES, flags=flags)
+        w = [torch.from_numpy(W).cuda() for W in Ws]
+        g = [torch.zeros_like(x) for x in w]
+        losses = [reg(w, g).clone() for _ in range(3)]
+        torch.cuda.synchronize()
+        assert reg.status() == 0
+        out.append(([x.cpu() for x in g], torch.cat(losses).cpu()))
+    for a, b in zip(out[0][0], out[1][0]):
+        assert torch.equal(a, b)
+    assert torch.equal(out[0][1], out[1][1])

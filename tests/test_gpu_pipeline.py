@@ -90,3 +90,37 @@ def test_pipeline_vit_b16_matches_oracle_sampled():
         assert abs(hp[i].item() - L) <= 2e-2 * L
         got = hg[i].double().numpy()
         assert np.linalg.norm(got - G) <= 2e-2 * np.linalg.norm(G), i
+
+
+@pytest.mark.parametrize("dtype,variant,flags", [("bf16", "hoyer", 0), ("f32", "nuclear", 0), ("f32", "hoyer", 32),
+                                                 ("bf16", "nuclear", 32)])
+def test_pipeline_options_equal_device_call(dtype, variant, flags):
+    """bf16 weight storage, the nuclear variant and SLORR_FLAG_WRITE_GRAD (32) go
+    through the pipeline unchanged: grads and per-matrix values equal the
+    device-resident call bit for bit."""
+    from paper_2607_08754_gb300.slorr import Regularizer, Pipeline
+    tdt = torch.float32 if dtype == "f32" else torch.bfloat16
+    Ws = [torch.from_numpy(workloads.random_matrix(s, seed=700 + i, std=0.05)).to(tdt) for i, s in enumerate(SHAPES)]
+    G0 = [torch.from_numpy(workloads.random_matrix(s, seed=800 + i, std=0.01)).to(tdt) for i, s in enumerate(SHAPES)]
+    kw = dict(variant=variant, dtype=dtype, flags=flags, lam=0.7)
+    reg = Regularizer(SHAPES, **kw)
+    w = [x.cuda() for x in Ws]
+    g = [x.cuda() for x in G0]
+    per = torch.empty(len(SHAPES), device="cuda")
+    loss = reg(w, g, per_matrix=per).item()
+    torch.cuda.synchronize()
+    assert reg.status() == 0
+    pipe = Pipeline(SHAPES, groups=3, **kw)
+    hw = [x.pin_memory() for x in Ws]
+    hg = [x.clone().pin_memory() for x in G0]
+    dw = [torch.empty_like(x) for x in w]
+    dg = [torch.empty_like(x) for x in w]
+    hl = torch.zeros(1).pin_memory()
+    hp = torch.zeros(len(SHAPES)).pin_memory()
+    pipe(hw, hg, dw, dg, hl, hp)
+    torch.cuda.synchronize()
+    assert pipe.status() == 0
+    assert hl.item() == pytest.approx(loss, rel=1e-6)
+    assert torch.equal(hp, per.cpu())
+    for a, b in zip(hg, g):
+        assert torch.equal(a, b.cpu())
