@@ -63,6 +63,7 @@ def parse():
     ap.add_argument("--workload", default="vit_l16", choices=list(workloads.WEIGHT_SETS))
     ap.add_argument("--variant", default="hoyer", choices=["hoyer", "nuclear"])
     ap.add_argument("--compute", default="fp16", choices=["fp16", "bf16", "fp32"])
+    ap.add_argument("--dtype", default="f32", choices=["f32", "bf16"], help="storage of the weights and grads")
     ap.add_argument("--iters", type=int, default=6)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=10)
@@ -94,6 +95,23 @@ def cpu_cores() -> int:
         return len(os.sched_getaffinity(0))
     except AttributeError:  # pragma: no cover
         return os.cpu_count() or 1
+
+
+def blas_info() -> dict:
+    """numpy's BLAS library and its thread limit, as threadpoolctl or numpy reports them."""
+    try:
+        from threadpoolctl import threadpool_info
+        libs = [d for d in threadpool_info() if d.get("user_api") == "blas"]
+        if libs:
+            return {"library": libs[0].get("internal_api"), "threads": libs[0].get("num_threads")}
+    except Exception:
+        pass
+    try:
+        cfg = np.show_config(mode="dicts")
+        blas = cfg.get("Build Dependencies", {}).get("blas", {})
+        return {"library": blas.get("name"), "threads": None}
+    except Exception:
+        return {"library": None, "threads": None}
 
 
 def oracle_sample(name: str, variant: str, iters: int, budget_s: float, max_steps: int = 1):
@@ -223,7 +241,8 @@ def run_reference(args, rank, world):
             "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
             "config": {"workload": f"{args.workload} {args.variant}, T={args.iters}", "matrices": len(shapes)},
             "cpu_baseline": {"value": tflops, "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
-                             "sample": f"each step: {desc}; ms_per_step extrapolated to the whole set by FLOPs"},
+                             "sample": f"each step: {desc}; ms_per_step extrapolated to the whole set by FLOPs",
+                             "blas": blas_info()},
             "e2e": {"value": tflops, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -251,14 +270,16 @@ def main():
     dev = torch.device("cuda", local)
     name = args.workload
     shapes = workloads.shapes(name)
-    reg = slorr.Regularizer(shapes, variant=args.variant, compute=args.compute, iters=args.iters, lam=1.0,
-                            flags=args.flags)
-    W_host = [torch.from_numpy(workloads.generate_one(name, i)) for i in range(len(shapes))]
+    reg = slorr.Regularizer(shapes, variant=args.variant, compute=args.compute, dtype=args.dtype, iters=args.iters,
+                            lam=1.0, flags=args.flags)
+    tdt = torch.float32 if args.dtype == "f32" else torch.bfloat16
+    W_host = [torch.from_numpy(workloads.generate_one(name, i)).to(tdt) for i in range(len(shapes))]
     W = [w.to(dev) for w in W_host]
     G = [torch.zeros_like(w) for w in W]
     loss = torch.zeros(1, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
     flops_step = slorr.slorr_flops(shapes, args.iters)
+    flops_exec = slorr.slorr_executed_flops(reg.handle)  # incl. padding, minus skipped symmetric tiles
 
     def barrier():
         if world > 1:
@@ -286,15 +307,17 @@ def main():
     clocks = ClockSampler(local)
     clocks.start()
     barrier()
-    t0 = torch.cuda.Event(enable_timing=True)
-    t1 = torch.cuda.Event(enable_timing=True)
-    t0.record(stream)
-    for _ in range(args.steps):
+    # one event between calls (a call starts with a memset, so this costs no
+    # overlap): per-call times for the percentiles
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    evs[0].record(stream)
+    for k in range(args.steps):
         step(W, G)
-    t1.record(stream)
+        evs[k + 1].record(stream)
     barrier()
     clk = clocks.stop()
-    ms_total = t0.elapsed_time(t1)
+    ms_total = evs[0].elapsed_time(evs[-1])
+    per_call = sorted(evs[k].elapsed_time(evs[k + 1]) for k in range(args.steps))
     assert reg.status() == 0, "device status word reports an error in the timed region"
     # per-kernel CUDA events on the call's stream (roofline of the GEMM kernel)
     slorr.slorr_set_timing(reg.handle, True)
@@ -324,7 +347,8 @@ def main():
     d2h = (wbytes if descent else gbytes) + 4
 
     pipe = None if descent else slorr.Pipeline(shapes, groups=args.e2e_groups or None, variant=args.variant,
-                                               compute=args.compute, iters=args.iters, lam=1.0, flags=args.flags)
+                                               compute=args.compute, dtype=args.dtype, iters=args.iters, lam=1.0,
+                                               flags=args.flags)
 
     def e2e_step():
         if pipe is not None:
@@ -368,7 +392,27 @@ def main():
         flops_per_launch = flops_step / (3 * args.iters)
         achieved = flops_per_launch / (per_launch_ms * 1e-3) / 1e12
         peak = pk["bf16"]  # fp16 and bf16 share the dense tensor rate (nominal ratio 1)
+        wbytes_dev = sum(w.numel() * w.element_size() for w in W)
+        l2_note = ("inputs larger than L2: %s weights %.3f GB (129 MB L2), no flush" % (args.dtype, wbytes_dev / 1e9)
+                   if wbytes_dev > 129e6 else
+                   "inputs smaller than L2: %s weights %.1f MB, L2-warm timing" % (args.dtype, wbytes_dev / 1e6))
         mem_ms = sum(kt[k][0] for k in ("sumsq", "cast", "dot", "combine")) / args.steps
+        # memory passes against the measured HBM copy bandwidth: algorithmic bytes per call
+        # (sumsq: W; cast: W + the padded iterate; dot: W + X_T; combine: W + X_T + grad
+        # read and written, or W read and written in place for --op descent)
+        wsz = 4 if args.dtype == "f32" else 2
+        xsz = 4 if args.compute == "fp32" else 2
+        elems = sum(m * n for m, n in shapes)
+        xelems = sum(((max(m, n) + 127) // 128 * 128) * ((min(m, n) + 127) // 128 * 128) for m, n in shapes)
+        comb = (2 * wsz + xsz) if descent else (3 * wsz + xsz)
+        mem_bytes = {"sumsq": wsz * elems, "cast": wsz * elems + xsz * xelems, "dot": (wsz + xsz) * elems,
+                     "combine": comb * elems}
+        memory_roofline = {}
+        for k, b in mem_bytes.items():
+            t = kt[k][0] / args.steps * 1e-3
+            gbs = b / t / 1e9
+            memory_roofline[k] = {"bytes": b, "ms": kt[k][0] / args.steps, "achieved_gbs": gbs,
+                                  "frac": gbs / pk["hbm"]}
         kernel_breakdown = {k: {"ms_per_step": v[0] / args.steps, "launches_per_step": v[1] / args.steps}
                             for k, v in kt.items()}
         line = {
@@ -378,18 +422,25 @@ def main():
             "data": "synthetic",
             "config": {"workload": f"{name} {args.variant}{' descent step' if descent else ''}: "
                                    f"{len(shapes)} matrices, T={args.iters}, "
-                                   f"{args.compute} operands / fp32 accumulate, fp32 weights and grads",
+                                   f"{args.compute} operands / fp32 accumulate, {args.dtype} weights and grads",
                        "matrices": len(shapes), "iters": args.iters, "variant": args.variant, "op": args.op,
                        "gflop_per_step": flops_step / 1e9,
-                       "l2": "inputs larger than L2 (fp32 weights %.2f GB)" %
-                             (sum(w.numel() for w in W) * 4 / 1e9)},
+                       "l2": l2_note},
             "pct_of_dense_peak": value / world / pk["bf16"],
+            "step_ms": {"mean": ms_step, "p10": per_call[len(per_call) // 10],
+                        "p50": per_call[len(per_call) // 2], "p90": per_call[(9 * len(per_call)) // 10]},
+            "executed": {"gflop_per_step": flops_exec / 1e9,
+                         "tflops": world * flops_exec / (ms_step * 1e-3) / 1e12,
+                         "note": "MMA FLOPs the kernels execute: padding included, strictly-lower "
+                                 "symmetric tiles skipped"},
             "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                          "frac": achieved / peak, "traffic": None if single_cta else tc_traffic(),
+                         "frac_of_sustained": achieved / pk["bf16_sustained"],
                          "kernel": ("tc_gemm_kernel" if single_cta else "tc_pair_kernel")
                                    + " (Gram/Poly/Update launches)",
                          "peak_source": pk["source"] + " bf16 burst (fp16 dense rate equal)"},
             "memory_phases_ms_per_step": mem_ms,
+            "memory_roofline": memory_roofline,
             "kernels": kernel_breakdown,
             "gpu_launches": launches,
             "e2e": {"value": e2e_val, "unit": "TFLOP/s", "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d,
@@ -401,7 +452,8 @@ def main():
         if not args.no_cpu_baseline:
             f, t, desc = oracle_sample(name, args.variant, args.iters, args.cpu_seconds)
             line["cpu_baseline"] = {"value": f / t / 1e12, "unit": "TFLOP/s", "cores": cpu_cores(),
-                                    "kind": "oracle", "sample": desc}
+                                    "kind": "oracle", "sample": desc, "blas": blas_info(),
+                                    "ms_per_step_est": flops_step / (f / t) * 1e3}
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.barrier()

@@ -231,6 +231,14 @@ SLORR_API int64_t slorr_flops(const slorr_shape* shapes, int32_t count, int32_t 
 SLORR_API slorr_status slorr_partition(const slorr_shape* shapes, int32_t count, int32_t world,
                              int32_t rank, int32_t* out_indices, int32_t* out_count);
 
+/* FLOPs the matrix products of one call execute on the path the handle's
+ * options select (host-only): 2 x rows x columns x K over every tile of every
+ * Gram, Poly and Update launch, counting the zero padding (P to a multiple of
+ * 128, Q to a multiple of 128) and the 256-row CTA-pair MMAs, and skipping
+ * the strictly-lower tiles of the symmetric products.  slorr_flops gives the
+ * paper's algorithmic count (Sec. 3 "Computational cost") instead. */
+SLORR_API slorr_status slorr_executed_flops(const slorr_handle* h, double* out);
+
 /* Per-kernel timing (tracing).  While enabled, every kernel this handle
  * launches is bracketed by a pair of CUDA events recorded on the caller's
  * stream (events are created on the host; no device memory is allocated).

@@ -676,6 +676,27 @@ slorr_status slorr_create(slorr_handle** out, const slorr_shape* shapes, int32_t
     return SLORR_OK;
 }
 
+slorr_status slorr_executed_flops(const slorr_handle* h, double* out) {
+    if (!h || !out) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
+    const bool simt = h->opt.compute == SLORR_COMPUTE_FP32 || (h->opt.flags & SLORR_FLAG_SIMT_GEMM);
+    const bool pair = !simt && tc_pair(h);
+    const bool quad = pair && (h->opt.flags & SLORR_FLAG_TC_QUAD);
+    double total = 0.0;
+    for (int ph = 0; ph < 3; ++ph) {
+        const std::vector<GemmItem>& items =
+            simt ? h->simt_items[ph] : (quad ? h->quad_items[ph] : h->tc_items[ph]);
+        for (const GemmItem& it : items) {
+            if (it.msz == 0) continue;  // empty half of a super-tile
+            const Geom& g = h->geom[it.mat];
+            const double K = ph == kGram ? g.Qpad : g.Ppad;
+            const double rows = pair ? 256.0 : double(it.msz);  // pair UMMAs are always M = 256
+            total += 2.0 * rows * double(it.nsz) * K;
+        }
+    }
+    *out = total * double(h->opt.iters);
+    return SLORR_OK;
+}
+
 slorr_status slorr_workspace_size(const slorr_handle* h, size_t* bytes) {
     if (!h || !bytes) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
     *bytes = h->total_bytes;

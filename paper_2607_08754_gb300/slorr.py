@@ -90,6 +90,7 @@ def load_library(path: str | None = None) -> ctypes.CDLL:
         "slorr_flops": (i64, [ctypes.POINTER(Shape), i32, i32]),
         "slorr_partition": (i32, [ctypes.POINTER(Shape), i32, i32, i32, ctypes.POINTER(i32),
                                   ctypes.POINTER(i32)]),
+        "slorr_executed_flops": (i32, [vp, ctypes.POINTER(dbl)]),
         "slorr_set_timing": (i32, [vp, i32]),
         "slorr_read_timing": (i32, [vp, ctypes.POINTER(dbl), ctypes.POINTER(i64), i32]),
         "slorr_frob_sq_noalloc": (i32, [vp, i64, i64, i32, vp, vp]),
@@ -213,6 +214,12 @@ def slorr_cushion_ratio() -> float:
 def slorr_flops(shapes, iters: int = 6) -> int:
     arr, n = _shapes(shapes)
     return int(load_library().slorr_flops(arr, n, int(iters)))
+
+
+def slorr_executed_flops(handle) -> float:
+    out = ctypes.c_double()
+    _check(load_library().slorr_executed_flops(handle, ctypes.byref(out)))
+    return out.value
 
 
 def slorr_partition(shapes, world: int, rank: int) -> list[int]:

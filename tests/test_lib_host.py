@@ -210,3 +210,28 @@ def test_pipeline_validation_and_workspace(lib):
                                                   4096, ws - 1, 0)
         assert e.value.status == 4
         slorr.slorr_pipeline_destroy(p)
+
+
+def test_executed_flops_counts_pair_tiles(lib):
+    """slorr_executed_flops: 2 x 256 x nsz x K over the CTA-pair tiles of every
+    phase (P and Q padded to multiples of 128, strictly-lower 256 x 256 tiles of
+    the symmetric Gram and Poly products skipped), times T.  A square 256 x 256
+    matrix executes exactly the paper's count."""
+    def expected(shapes, T):
+        tot = 0
+        for m, n in shapes:
+            P, Q = min(m, n), max(m, n)
+            Pp, Qp = -(-P // 128) * 128, -(-Q // 128) * 128
+            for ph, (N, K) in enumerate([(Pp, Qp), (Pp, Pp), (Qp, Pp)]):
+                for tm in range(-(-Pp // 256)):
+                    for tn in range(-(-N // 256)):
+                        nsz = min(256, N - tn * 256)
+                        if ph < 2 and tn < tm:
+                            continue
+                        tot += 2 * 256 * nsz * K
+        return tot * T
+    for shapes in ([(256, 256)], [(1000, 512)], [(64, 147), (3072, 1024), (1024, 4096), (130, 700)]):
+        r = slorr.Regularizer(shapes, iters=4)
+        assert slorr.slorr_executed_flops(r.handle) == expected(shapes, 4)
+    assert slorr.slorr_executed_flops(slorr.Regularizer([(256, 256)]).handle) == \
+        slorr.slorr_flops([(256, 256)], 6)
