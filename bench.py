@@ -396,19 +396,23 @@ def main():
         l2_note = ("inputs larger than L2: %s weights %.3f GB (129 MB L2), no flush" % (args.dtype, wbytes_dev / 1e9)
                    if wbytes_dev > 129e6 else
                    "inputs smaller than L2: %s weights %.1f MB, L2-warm timing" % (args.dtype, wbytes_dev / 1e6))
-        mem_ms = sum(kt[k][0] for k in ("sumsq", "cast", "dot", "combine")) / args.steps
+        mem_ms = sum(kt[k][0] for k in ("sumsq", "cast", "normcast", "dot", "combine")) / args.steps
         # memory passes against the measured HBM copy bandwidth: algorithmic bytes per call
-        # (sumsq: W; cast: W + the padded iterate; dot: W + X_T; combine: W + X_T + grad
-        # read and written, or W read and written in place for --op descent)
+        # (sumsq: W; cast: W + the padded iterate; normcast, both in one pass: W + the
+        # padded iterate; dot: W + X_T; combine: W + X_T + grad read and written, or W
+        # read and written in place for --op descent); passes that did not run are left out
         wsz = 4 if args.dtype == "f32" else 2
         xsz = 4 if args.compute == "fp32" else 2
         elems = sum(m * n for m, n in shapes)
         xelems = sum(((max(m, n) + 127) // 128 * 128) * ((min(m, n) + 127) // 128 * 128) for m, n in shapes)
         comb = (2 * wsz + xsz) if descent else (3 * wsz + xsz)
-        mem_bytes = {"sumsq": wsz * elems, "cast": wsz * elems + xsz * xelems, "dot": (wsz + xsz) * elems,
+        mem_bytes = {"sumsq": wsz * elems, "cast": wsz * elems + xsz * xelems,
+                     "normcast": wsz * elems + xsz * xelems, "dot": (wsz + xsz) * elems,
                      "combine": comb * elems}
         memory_roofline = {}
         for k, b in mem_bytes.items():
+            if kt[k][1] == 0:
+                continue
             t = kt[k][0] / args.steps * 1e-3
             gbs = b / t / 1e9
             memory_roofline[k] = {"bytes": b, "ms": kt[k][0] / args.steps, "achieved_gbs": gbs,

@@ -121,6 +121,12 @@ typedef struct slorr_options {
                                        kernel are programmatic dependents of the kernel
                                        before them, so each one's launch and prologue
                                        overlap the previous one's tail (tuning)          */
+#define SLORR_FLAG_SEPARATE_NORM 1024 /* 16-bit iterates: take ||W||_F and write X_0 in two
+                                       passes over W.  By default one pass does both:
+                                       it stores W rounded to 16 bits and the first
+                                       Gram and Update epilogues apply 1/(||W||_F+eps)
+                                       (a matrix with max |w| > 2^15, or ||W||_F < 1 in
+                                       fp16, is re-cast with the scale); tuning          */
 
 /* Fill *opt with the defaults listed beside each field above (App. C.1: T = 6,
  * ell = 1e-3, degree 5; eps, lambda and grad_scale as in Listing 1 / Alg. 2). */
@@ -202,6 +208,8 @@ typedef struct slorr_matrix_view {
     int32_t       transposed;
     const double* frob_sq;
     const double* n_hat;
+    const float*  x0_scale;  /* X_0 = *x0_scale times the array at after_steps = 0
+                                (16-bit iterates store W unscaled; else 1)    */
 } slorr_matrix_view;
 SLORR_API slorr_status slorr_iterate_view(const slorr_handle* h, const void* workspace, int32_t i,
                                 int32_t after_steps, slorr_matrix_view* out);
@@ -245,9 +253,10 @@ SLORR_API slorr_status slorr_executed_flops(const slorr_handle* h, double* out);
  * slorr_read_timing() waits for the recorded events, adds the elapsed
  * milliseconds and kernel launch counts per kind into ms[k] / launches[k]
  * (k < kinds, kinds <= SLORR_NUM_KERNEL_KINDS; kinds are sumsq, cast, gram,
- * poly, update, dot, combine; sumsq and dot each include their finalize
- * kernel) and forgets them. */
-#define SLORR_NUM_KERNEL_KINDS 7
+ * poly, update, dot, combine, normcast: the 16-bit iterates' single pass
+ * for the norm and X_0, which replaces sumsq and cast; sumsq, normcast and
+ * dot each include their finalize kernel) and forgets them. */
+#define SLORR_NUM_KERNEL_KINDS 8
 SLORR_API slorr_status slorr_set_timing(slorr_handle* h, int32_t enable);
 SLORR_API slorr_status slorr_read_timing(slorr_handle* h, double* ms, int64_t* launches, int32_t kinds);
 

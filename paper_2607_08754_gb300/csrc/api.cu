@@ -45,7 +45,8 @@ namespace {
 struct Geom {
     int m, n, P, Q, Ppad, Qpad, transposed, rows, ld;
     size_t off_x[2], off_a, off_b;
-    int tile_base, tile_count;
+    int tile_base, tile_count;      // tiles of W (sumsq, dot, combine)
+    int xtile_base, xtile_count;    // tiles of the padded iterate (cast, normcast)
 };
 
 }  // namespace
@@ -64,9 +65,10 @@ struct slorr_handle {
     std::vector<MemItem> w_items;  // tiles of W (sumsq, dot, combine)
     std::vector<MemItem> x_items;  // tiles of the padded iterate (cast)
     int total_w_tiles = 0;
+    int total_x_tiles = 0;
     // workspace layout
-    size_t off_status = 0, off_counters = 0, off_scalars = 0, off_partials = 0, off_tilebase = 0,
-           off_tilecount = 0, off_mats = 0, off_maps = 0, off_tc_items[3] = {}, off_quad_items[3] = {},
+    size_t off_status = 0, off_counters = 0, off_scalars = 0, off_partials = 0, off_partials_max = 0,
+           off_tilebase = 0, off_tilecount = 0, off_xtilebase = 0, off_xtilecount = 0, off_mats = 0, off_maps = 0, off_tc_items[3] = {}, off_quad_items[3] = {},
            off_simt_items[3] = {},
            off_w_items = 0, off_x_items = 0, off_ptrs = 0, off_plan_end = 0, total_bytes = 0;
     // device state
@@ -97,6 +99,13 @@ bool tc_pair(const slorr_handle* h) {
 
 // Programmatic dependent launch of the memory passes and the pair kernel.
 bool use_pdl(const slorr_handle* h) { return (h->opt.flags & SLORR_FLAG_NO_PDL) == 0; }
+
+// 16-bit iterates on the tensor cores: the norm and the cast share one read of
+// W (normcast), and the first Gram and Update epilogues apply the scale.
+bool fused_norm(const slorr_handle* h) {
+    return h->opt.compute != SLORR_COMPUTE_FP32 &&
+           (h->opt.flags & (SLORR_FLAG_SIMT_GEMM | SLORR_FLAG_SEPARATE_NORM)) == 0;
+}
 
 // K depth of the tensor-core pipeline stages for this handle.
 int tc_bk(const slorr_handle* h) {
@@ -178,7 +187,7 @@ void build_plan(slorr_handle* h) {
     }
     h->w_items.clear();
     h->x_items.clear();
-    int tile_base = 0;
+    int tile_base = 0, xtile_base = 0;
     for (int i = 0; i < count; ++i) {
         Geom& g = h->geom[i];
         g.m = int(h->shapes[i].m);
@@ -199,9 +208,13 @@ void build_plan(slorr_handle* h) {
             for (int c = 0; c < tc; ++c)
                 h->w_items.push_back(MemItem{uint16_t(i), uint16_t(r), uint16_t(c), uint16_t(seq++)});
         tile_base += g.tile_count;
+        g.xtile_base = xtile_base;
+        int xseq = 0;
         for (int r = 0; r < (g.rows + kMemRows - 1) / kMemRows; ++r)
             for (int c = 0; c < (g.ld + kMemCols - 1) / kMemCols; ++c)
-                h->x_items.push_back(MemItem{uint16_t(i), uint16_t(r), uint16_t(c), 0});
+                h->x_items.push_back(MemItem{uint16_t(i), uint16_t(r), uint16_t(c), uint16_t(xseq++)});
+        g.xtile_count = xseq;
+        xtile_base += xseq;
         // tensor-core tiles: msz x nsz with msz <= 128 mt, nsz <= 256.  The Gram
         // and Poly outputs are symmetric: tiles lying strictly below the
         // diagonal (in 128 x 128 blocks) are skipped; the kernel mirrors the
@@ -225,6 +238,7 @@ void build_plan(slorr_handle* h) {
         }
     }
     h->total_w_tiles = tile_base;
+    h->total_x_tiles = xtile_base;
     // Longest K first (stable: keeps a matrix's tiles together).
     for (int ph = 0; ph < 3; ++ph) {
         auto kdim = [&](const GemmItem& it) {
@@ -257,10 +271,16 @@ void build_plan(slorr_handle* h) {
     h->off_scalars = off;
     off = align_up(off + size_t(count) * sizeof(MatScalars), 256);
     h->off_partials = off;
-    off = align_up(off + size_t(h->total_w_tiles) * 4, 256);
+    off = align_up(off + size_t(std::max(h->total_w_tiles, h->total_x_tiles)) * 4, 256);
+    h->off_partials_max = off;
+    off = align_up(off + size_t(h->total_x_tiles) * 4, 256);
     h->off_tilebase = off;
     off = align_up(off + size_t(count) * 4, 256);
     h->off_tilecount = off;
+    off = align_up(off + size_t(count) * 4, 256);
+    h->off_xtilebase = off;
+    off = align_up(off + size_t(count) * 4, 256);
+    h->off_xtilecount = off;
     off = align_up(off + size_t(count) * 4, 256);
     h->off_mats = off;
     off = align_up(off + size_t(count) * sizeof(MatDev), 256);
@@ -343,7 +363,7 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
     }
     std::vector<uint8_t> plan(h->off_plan_end - h->off_tilebase, 0);
     const size_t base = h->off_tilebase;
-    std::vector<int32_t> tb(count), tcnt(count);
+    std::vector<int32_t> tb(count), tcnt(count), xtb(count), xtcnt(count);
     std::vector<MatDev> mats(count);
     std::vector<uint8_t> maps(size_t(count) * kMapsPerMatrix * 128, 0);
     const int bk = tc_bk(h);
@@ -352,6 +372,8 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
         const Geom& g = h->geom[i];
         tb[i] = g.tile_base;
         tcnt[i] = g.tile_count;
+        xtb[i] = g.xtile_base;
+        xtcnt[i] = g.xtile_count;
         MatDev& md = mats[i];
         md.x[0] = ws + g.off_x[0];
         md.x[1] = ws + g.off_x[1];
@@ -383,6 +405,8 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
     }
     put(plan, h->off_tilebase - base, tb.data(), tb.size());
     put(plan, h->off_tilecount - base, tcnt.data(), tcnt.size());
+    put(plan, h->off_xtilebase - base, xtb.data(), xtb.size());
+    put(plan, h->off_xtilecount - base, xtcnt.data(), xtcnt.size());
     put(plan, h->off_mats - base, mats.data(), mats.size());
     put(plan, h->off_maps - base, maps.data(), maps.size());
     for (int ph = 0; ph < 3; ++ph) {
@@ -464,6 +488,7 @@ MemLaunch mem_params(slorr_handle* h, uint8_t* ws, float* loss, float* per, int 
     p.mats = reinterpret_cast<const MatDev*>(ws + h->off_mats);
     p.scalars = reinterpret_cast<MatScalars*>(ws + h->off_scalars);
     p.partials = reinterpret_cast<float*>(ws + h->off_partials);
+    p.partials_max = reinterpret_cast<float*>(ws + h->off_partials_max);
     p.tile_base = reinterpret_cast<const int32_t*>(ws + h->off_tilebase);
     p.tile_count = reinterpret_cast<const int32_t*>(ws + h->off_tilecount);
     p.counters = reinterpret_cast<uint32_t*>(ws + h->off_counters);
@@ -522,25 +547,33 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
     cudaError_t e = cudaMemsetAsync(ws + h->off_counters, 0, (h->shapes.size() + 1) * 4, st);
     if (e != cudaSuccess) return cuda_fail(e, "counter reset");
 
+    const bool use_tc = h->opt.compute != SLORR_COMPUTE_FP32 && !(h->opt.flags & SLORR_FLAG_SIMT_GEMM);
+    const bool fuse_norm = use_tc && fused_norm(h);
     MemLaunch mp = mem_params(h, ws, loss, per, 0);
-    mp.items = reinterpret_cast<const MemItem*>(ws + h->off_w_items);
-    mp.num_items = int(h->w_items.size());
-    {
-        Traced tr(h, 0, st);
-        if ((e = launch_sumsq(mp, st)) != cudaSuccess) return cuda_fail(e, "sumsq launch");
-        if ((e = launch_finalize(mp, 0, st)) != cudaSuccess) return cuda_fail(e, "finalize launch");
-        tr.done(2);
-    }
-    MemLaunch cp = mp;
+    MemLaunch cp = mp;  // tiles of the padded iterate
     cp.items = reinterpret_cast<const MemItem*>(ws + h->off_x_items);
     cp.num_items = int(h->x_items.size());
-    {
+    if (fuse_norm) {
+        cp.tile_base = reinterpret_cast<const int32_t*>(ws + h->off_xtilebase);
+        cp.tile_count = reinterpret_cast<const int32_t*>(ws + h->off_xtilecount);
+        Traced tr(h, 7, st);
+        if ((e = launch_normcast(cp, st)) != cudaSuccess) return cuda_fail(e, "normcast launch");
+        if ((e = launch_finalize(cp, 2, st)) != cudaSuccess) return cuda_fail(e, "finalize launch");
+        tr.done(2);
+    } else {
+        mp.items = reinterpret_cast<const MemItem*>(ws + h->off_w_items);
+        mp.num_items = int(h->w_items.size());
+        {
+            Traced tr(h, 0, st);
+            if ((e = launch_sumsq(mp, st)) != cudaSuccess) return cuda_fail(e, "sumsq launch");
+            if ((e = launch_finalize(mp, 0, st)) != cudaSuccess) return cuda_fail(e, "finalize launch");
+            tr.done(2);
+        }
         Traced tr(h, 1, st);
         if ((e = launch_cast(cp, st)) != cudaSuccess) return cuda_fail(e, "cast launch");
         tr.done();
     }
 
-    const bool use_tc = h->opt.compute != SLORR_COMPUTE_FP32 && !(h->opt.flags & SLORR_FLAG_SIMT_GEMM);
     GemmLaunch g{};
     g.mats = reinterpret_cast<const MatDev*>(ws + h->off_mats);
     g.maps = ws + h->off_maps;
@@ -553,6 +586,7 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
     const bool quad = pair && (h->opt.flags & SLORR_FLAG_TC_QUAD) != 0;
     g.pair_slots = (h->opt.flags & SLORR_FLAG_PAIR_ONE_SLOT) ? 1 : 2;
     g.pdl = (use_pdl(h) && pair && !quad) ? 1 : 0;
+    g.scalars = reinterpret_cast<const MatScalars*>(ws + h->off_scalars);
     for (int t = 0; t < steps; ++t) {
         g.cur = t & 1;
         g.a = float(h->coeffs[3 * t + 0]);
@@ -561,6 +595,7 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
         for (int ph = 0; ph < 3; ++ph) {
             g.phase = ph;
             g.mt = tc_mt(h, ph);
+            g.x0_scaled = (fuse_norm && t == 0 && ph != kPoly) ? 1 : 0;
             Traced tr(h, 2 + ph, st);
             if (use_tc && quad) {
                 g.items = reinterpret_cast<const GemmItem*>(ws + h->off_quad_items[ph]);
@@ -672,6 +707,11 @@ slorr_status slorr_create(slorr_handle** out, const slorr_shape* shapes, int32_t
         h->esize = 2;
     }
     build_plan(h);
+    for (const Geom& g : h->geom)
+        if (g.tile_count > 65535 || g.xtile_count > 65535) {
+            delete h;
+            return fail(SLORR_ERR_UNSUPPORTED, "matrix too large: more than 65535 tiles of 16 x 512 elements");
+        }
     *out = h;
     return SLORR_OK;
 }
@@ -759,6 +799,7 @@ slorr_status slorr_iterate_view(const slorr_handle* h, const void* workspace, in
     const MatScalars* sc = reinterpret_cast<const MatScalars*>(ws + h->off_scalars) + i;
     out->frob_sq = &sc->frob_sq;
     out->n_hat = &sc->n_hat;
+    out->x0_scale = &sc->x0_scale;
     return SLORR_OK;
 }
 

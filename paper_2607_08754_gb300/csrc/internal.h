@@ -54,9 +54,12 @@ struct MatScalars {
     double frob_sq;    // ||W||_F^2
     double n_hat;      // sum(W * P_hat)
     float scale;       // 1 / (||W||_F + eps): the normalisation of X_0
+    float x0_scale;    // X_0 = x0_scale * (the stored X_0 buffer): scale when the
+                       // fused norm pass stored W unscaled, else 1
     float alpha;       // gradient = alpha * P_hat - beta * W (lambda, grad_scale included)
     float beta;
     int32_t skip;      // non-finite norm or estimate: leave the gradient untouched
+    int32_t pad_;
 };
 
 // One output tile of a grouped GEMM phase.
@@ -101,6 +104,11 @@ struct GemmLaunch {
     int32_t test_stall;        // 1: the MMA thread first waits on a barrier nothing arrives on
     int32_t pair_slots;        // CTA-pair kernel: accumulators per CTA (1 or 2)
     int32_t pdl;               // launch with programmatic dependent launch
+    // x0_scaled = 1 (first step after the fused norm pass, which stores X_0
+    // as W rounded to 16 bits): the Gram epilogue multiplies by
+    // scalars[i].x0_scale^2 and the Update epilogue by scalars[i].x0_scale.
+    int32_t x0_scaled;
+    const MatScalars* scalars;
 };
 
 // Tensor maps per matrix: X0 K-major, X1 K-major, X0 MN-major, X1 MN-major,
@@ -120,6 +128,7 @@ struct MemLaunch {
     const MatDev* mats;
     MatScalars* scalars;
     float* partials;           // one float per (matrix, tile)
+    float* partials_max;       // fused norm pass: max |w| per tile
     const int32_t* tile_base;  // first partial index of each matrix
     const int32_t* tile_count; // tiles per matrix
     uint32_t* counters;        // per-matrix completion counters
@@ -141,7 +150,9 @@ struct MemLaunch {
 // Launchers (return cudaGetLastError() of the launch).
 cudaError_t launch_sumsq(const MemLaunch& p, cudaStream_t s);
 cudaError_t launch_cast(const MemLaunch& p, cudaStream_t s);
+cudaError_t launch_normcast(const MemLaunch& p, cudaStream_t s);
 cudaError_t launch_dot(const MemLaunch& p, cudaStream_t s);
+// which: 0 after sumsq, 1 after dot (and the loss), 2 after normcast
 cudaError_t launch_finalize(const MemLaunch& p, int which, cudaStream_t s);
 cudaError_t launch_combine(const MemLaunch& p, cudaStream_t s);
 cudaError_t launch_sum_parts(const float* parts, int n, float* out, cudaStream_t s);

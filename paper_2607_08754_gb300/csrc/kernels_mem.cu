@@ -1,6 +1,11 @@
 // Memory-bound passes of the SLORR hot path, grouped over all weight matrices:
 //   sumsq   ||W_i||_F^2                                  (Listing 1, frob)
 //   cast    X_0 = W_i / (||W_i||_F + eps), zero padded    (Sec. 3 "Computing the polar factor")
+//   normcast  sumsq and cast in one read of W, for 16-bit iterates: the
+//           buffer receives W itself rounded to 16 bits, and the first Gram
+//           and Update epilogues apply the scale (x0_scale); the finalize
+//           kernel re-casts, with the scale, a matrix whose values would lose
+//           precision in an unscaled fp16 copy
 //   dot     n_hat_i = sum(W_i * P_hat_i), values L_i and the loss
 //                                                        (Sec. 3 "Computing the nuclear ...", Listing 1)
 //   combine W_i.grad += lambda * grad_scale * G_i       (Listing 1 backward, Alg. 2)
@@ -180,6 +185,44 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
     return s;  // valid in thread 0
 }
 
+// Block-wide sum and max of one value per thread: valid in thread 0.
+__device__ __forceinline__ float2 block_sum_max(float v, float m) {
+    __shared__ float rs[kThreads / 32], rm[kThreads / 32];
+    for (int o = 16; o > 0; o >>= 1) {
+        v += __shfl_xor_sync(0xffffffffu, v, o);
+        m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    }
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) {
+        rs[warp] = v;
+        rm[warp] = m;
+    }
+    __syncthreads();
+    float2 r = make_float2(0.f, 0.f);
+    if (warp == 0) {
+        r.x = lane < (kThreads / 32) ? rs[lane] : 0.f;
+        r.y = lane < (kThreads / 32) ? rm[lane] : 0.f;
+        for (int o = 16; o > 0; o >>= 1) {
+            r.x += __shfl_xor_sync(0xffffffffu, r.x, o);
+            r.y = fmaxf(r.y, __shfl_xor_sync(0xffffffffu, r.y, o));
+        }
+    }
+    return r;
+}
+
+__device__ __forceinline__ float absmax8(const F8& a, float m) {
+    m = fmaxf(m, fmaxf(fmaxf(fabsf(a.lo.x), fabsf(a.lo.y)), fmaxf(fabsf(a.lo.z), fabsf(a.lo.w))));
+    return fmaxf(m, fmaxf(fmaxf(fabsf(a.hi.x), fabsf(a.hi.y)), fmaxf(fabsf(a.hi.z), fabsf(a.hi.w))));
+}
+
+// An unscaled fp16 copy keeps every value of W at full relative precision
+// and below overflow when max |w| <= 2^15, and its subnormal spacing (2^-24)
+// costs no more than in the scaled X_0 when ||W||_F >= 1; bf16 has fp32's
+// exponent range.
+__device__ __forceinline__ bool unscaled_cast_ok(int elem, float maxabs, double frob) {
+    return elem == kBF16 || maxabs == 0.f || (maxabs <= 32768.f && frob >= 1.0);
+}
+
 struct TileCoord {
     int r0, c;  // first row of this thread, its first column
 };
@@ -212,6 +255,42 @@ __global__ void __launch_bounds__(kThreads, 6) sumsq_kernel(const MemLaunch p) {
     for (int k = 0; k < kPasses; ++k) acc = dot8(w[k], w[k], acc);
     const float part = block_sum(acc, red);
     if (threadIdx.x == 0) p.partials[p.tile_base[it.mat] + it.seq] = part;
+}
+
+// sumsq and cast in one read of W (16-bit iterates).  Items tile the padded
+// buffer (rows x ld); the buffer receives W rounded to 16 bits, unscaled, and
+// zeros in the padding; one partial of ||W||^2 and one of max |w| per item.
+template <typename TW, typename TX>
+__global__ void __launch_bounds__(kThreads, 4) normcast_kernel(const MemLaunch p) {
+    ptx::griddep_wait();  // inputs come from the previous kernel (programmatic launch)
+    ptx::griddep_launch_dependents();
+    const MemItem it = p.items[blockIdx.x];
+    const MatDev md = p.mats[it.mat];
+    const TW* W = reinterpret_cast<const TW*>(p.weights[it.mat]);
+    void* X = md.x[p.cur];
+    const bool vec = (md.n & 7) == 0;
+    const TileCoord tc = tile_coord(it);
+    F8 w[kPasses];
+#pragma unroll
+    for (int k = 0; k < kPasses; ++k) w[k] = load_w8<TW>(W, md.m, md.n, tc.r0 + k * kRowsPerPass, tc.c, vec);
+    if (tc.c < md.ld) {
+#pragma unroll
+        for (int k = 0; k < kPasses; ++k) {
+            const int r = tc.r0 + k * kRowsPerPass;
+            if (r < md.rows) store_x8<TX>(X, int64_t(r) * md.ld + tc.c, w[k]);
+        }
+    }
+    float acc = 0.f, mx = 0.f;
+#pragma unroll
+    for (int k = 0; k < kPasses; ++k) {
+        acc = dot8(w[k], w[k], acc);
+        mx = absmax8(w[k], mx);
+    }
+    const float2 sm = block_sum_max(acc, mx);
+    if (threadIdx.x == 0) {
+        p.partials[p.tile_base[it.mat] + it.seq] = sm.x;
+        p.partials_max[p.tile_base[it.mat] + it.seq] = sm.y;
+    }
 }
 
 // Items tile the padded buffer (rows x ld); zeros are written to the padding.
@@ -305,6 +384,7 @@ __device__ bool finalize_matrix(const MemLaunch& p, int which, int mat, double t
     if (which == 0) {
         sc.frob_sq = tot;
         sc.scale = static_cast<float>(1.0 / (sqrt(tot) + eps));
+        sc.x0_scale = 1.f;
         if (!isfinite(tot)) atomicOr(p.status, kStatusNonFinite);
         return false;
     }
@@ -335,6 +415,9 @@ __device__ bool finalize_matrix(const MemLaunch& p, int which, int mat, double t
 // One block per matrix: adds the matrix's tile partials in index order (double)
 // and derives the per-matrix coefficients the next pass needs.
 //   which = 0: ||W||_F^2 and the cast scale 1 / (||W||_F + eps);
+//   which = 2: the same after normcast, and x0_scale: the scale when the
+//              unscaled copy is kept, else 1 after this block re-casts
+//              X_0 = scale * W;
 //   which = 1: n_hat and the gradient coefficients (Listing 1 backward times
 //              lambda * grad_scale): Hoyer alpha = 2 reg / frob,
 //              beta = 2 reg n_hat / frob^3 with reg = n_hat / frob; Nuc alpha = 1.
@@ -344,18 +427,60 @@ __global__ void __launch_bounds__(128) finalize_kernel(const MemLaunch p, int wh
     ptx::griddep_wait();  // inputs come from the previous kernel (programmatic launch)
     ptx::griddep_launch_dependents();
     __shared__ double red[4];
+    __shared__ float redm[4];
     __shared__ int is_last;
     const int mat = blockIdx.x;
     const int base = p.tile_base[mat], n = p.tile_count[mat];
+    const bool fused = which == 2;
     double s = 0.0;
-    for (int i = threadIdx.x; i < n; i += 128) s += static_cast<double>(__ldcg(p.partials + base + i));
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+    float m = 0.f;
+    for (int i = threadIdx.x; i < n; i += 128) {
+        s += static_cast<double>(__ldcg(p.partials + base + i));
+        if (fused) m = fmaxf(m, __ldcg(p.partials_max + base + i));
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+        s += __shfl_xor_sync(0xffffffffu, s, o);
+        m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    }
+    if ((threadIdx.x & 31) == 0) {
+        red[threadIdx.x >> 5] = s;
+        redm[threadIdx.x >> 5] = m;
+    }
     __syncthreads();
     const double tot = (red[0] + red[1]) + (red[2] + red[3]);
-    if (threadIdx.x == 0) is_last = finalize_matrix(p, which, mat, tot) ? 1 : 0;
-    __syncthreads();
-    if (is_last) finalize_loss(p);
+    if (!fused) {
+        if (threadIdx.x == 0) is_last = finalize_matrix(p, which, mat, tot) ? 1 : 0;
+        __syncthreads();
+        if (is_last) finalize_loss(p);
+        return;
+    }
+    // after normcast: keep the unscaled copy (x0_scale = scale) or re-cast it
+    const float mx = fmaxf(fmaxf(redm[0], redm[1]), fmaxf(redm[2], redm[3]));
+    const double fr = sqrt(tot);
+    const float scale = static_cast<float>(1.0 / (fr + static_cast<double>(p.eps)));
+    const bool ok = unscaled_cast_ok(p.elem, mx, fr);
+    if (threadIdx.x == 0) {
+        MatScalars& sc = p.scalars[mat];
+        sc.frob_sq = tot;
+        sc.scale = scale;
+        sc.x0_scale = ok ? scale : 1.f;
+        if (!isfinite(tot)) atomicOr(p.status, kStatusNonFinite);
+    }
+    if (ok) return;
+    // X_0 = scale * W over W's region (the padding already holds zeros)
+    const MatDev md = p.mats[mat];
+    const void* W = p.weights[mat];
+    const int64_t total = int64_t(md.m) * md.n;
+    for (int64_t i = threadIdx.x; i < total; i += 128) {
+        const int64_t r = i / md.n, c = i - r * md.n;
+        const float w = p.wdtype == 0 ? reinterpret_cast<const float*>(W)[i]
+                                      : bf2f(reinterpret_cast<const uint16_t*>(W)[i]);
+        const int64_t o = r * md.ld + c;
+        if (p.elem == kF16)
+            reinterpret_cast<__half*>(md.x[p.cur])[o] = __float2half_rn(w * scale);
+        else
+            reinterpret_cast<__nv_bfloat16*>(md.x[p.cur])[o] = __float2bfloat16_rn(w * scale);
+    }
 }
 
 template <typename TW, typename TX>
@@ -434,6 +559,12 @@ cudaError_t launch_cast(const MemLaunch& p, cudaStream_t s) {
 cudaError_t launch_dot(const MemLaunch& p, cudaStream_t s) {
     if (p.num_items == 0) return cudaSuccess;
     SLORR_DISPATCH_WX(dot_kernel);
+}
+
+cudaError_t launch_normcast(const MemLaunch& p, cudaStream_t s) {
+    if (p.num_items == 0) return cudaSuccess;
+    if (p.elem == kF32) return cudaErrorInvalidValue;  // 16-bit iterates only
+    SLORR_DISPATCH_WX(normcast_kernel);
 }
 
 cudaError_t launch_finalize(const MemLaunch& p, int which, cudaStream_t s) {

@@ -117,11 +117,14 @@ __device__ __forceinline__ uint64_t operand_desc(uint32_t base, int kk, bool mn)
 //   Gram / Poly: c * acc (+ b A + a I for Poly) into the Ppad x Ppad output,
 //           plus the transpose of every 128 x 128 block (I, J), J > I, whose
 //           mirror tile is skipped (tiles are MT x 128 rows by 256 columns).
+// In the first step after the fused norm pass (p.x0_scaled) the stored X_0
+// is W itself: the Gram scales acc by x0_scale^2 and the Update by x0_scale.
 template <bool BF16, int MT>
 __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& it, const MatDev& md, int row0,
                                            uint32_t t_row, int quad, int lane, int ch_begin, int ch_end) {
     const int row = row0 + quad * 32 + lane;
     const int nch = ch_end;
+    const float xs = p.x0_scaled ? p.scalars[it.mat].x0_scale : 1.f;
     if (p.phase == kUpdate) {
         uint16_t* out = reinterpret_cast<uint16_t*>(md.x[p.cur ^ 1]);
         const int64_t ld = md.ld;
@@ -134,13 +137,13 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
                 // X^T[q][p]: for each column the warp's 32 rows are contiguous
                 uint16_t* dst = out + int64_t(col0) * ld + row;
 #pragma unroll
-                for (int j = 0; j < 32; ++j) dst[int64_t(j) * ld] = to16<BF16>(__uint_as_float(r[j]));
+                for (int j = 0; j < 32; ++j) dst[int64_t(j) * ld] = to16<BF16>(xs * __uint_as_float(r[j]));
             } else {
                 uint4 o[4];
                 uint32_t* ow = reinterpret_cast<uint32_t*>(o);
 #pragma unroll
                 for (int j = 0; j < 16; ++j)
-                    ow[j] = pack2<BF16>(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
+                    ow[j] = pack2<BF16>(xs * __uint_as_float(r[2 * j]), xs * __uint_as_float(r[2 * j + 1]));
                 uint4* dst = reinterpret_cast<uint4*>(out + int64_t(row) * ld + col0);
 #pragma unroll
                 for (int v = 0; v < 4; ++v) dst[v] = o[v];
@@ -151,7 +154,7 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
         const uint16_t* amat = reinterpret_cast<const uint16_t*>(md.a);
         const int64_t ld = md.Ppad;
         const bool poly = p.phase == kPoly;
-        const float cacc = poly ? p.c : 1.f;
+        const float cacc = poly ? p.c : xs * xs;
         // Poly reads b A at the output position: loads for the next chunk are
         // issued before the current chunk is processed.
         uint4 e_next[4];

@@ -34,6 +34,7 @@ FLAG_TC_SINGLE_CTA = 64
 FLAG_PAIR_ONE_SLOT = 128
 FLAG_TC_QUAD = 256
 FLAG_NO_PDL = 512
+FLAG_SEPARATE_NORM = 1024
 
 
 class SlorrError(RuntimeError):
@@ -56,7 +57,7 @@ class Options(ctypes.Structure):
 class MatrixView(ctypes.Structure):
     _fields_ = [("x", ctypes.c_void_p), ("rows", ctypes.c_int64), ("cols", ctypes.c_int64),
                 ("ld", ctypes.c_int64), ("elem", ctypes.c_int32), ("transposed", ctypes.c_int32),
-                ("frob_sq", ctypes.c_void_p), ("n_hat", ctypes.c_void_p)]
+                ("frob_sq", ctypes.c_void_p), ("n_hat", ctypes.c_void_p), ("x0_scale", ctypes.c_void_p)]
 
 
 _lib = None
@@ -230,7 +231,7 @@ def slorr_partition(shapes, world: int, rank: int) -> list[int]:
     return [int(out[i]) for i in range(cnt.value)]
 
 
-KERNEL_KINDS = ("sumsq", "cast", "gram", "poly", "update", "dot", "combine")
+KERNEL_KINDS = ("sumsq", "cast", "gram", "poly", "update", "dot", "combine", "normcast")
 
 
 def slorr_set_timing(handle, enable: bool) -> None:
@@ -391,6 +392,8 @@ class Regularizer:
         if v.elem == 2:
             raw = raw.view(torch.bfloat16)
         x = raw[:, : v.cols].float()
+        if after_steps == 0:  # 16-bit iterates hold W unscaled: X_0 = x0_scale * buffer
+            x = x * device_view(v.x0_scale, (1,), "<f4", dev).clone()
         return x.t().contiguous() if v.transposed else x
 
     def scalars(self, i: int):

@@ -1,0 +1,135 @@
+"""The fused norm pass of the 16-bit iterates.
+
+One read of W gives two things:
+- the norm ||W||_F (Listing 1);
+- the stored X_0, which is W itself rounded to 16 bits.
+
+The scale 1 / (||W||_F + eps) (Sec. 3 "Computing the polar factor") is applied in the first Gram
+and Update epilogues. The tests compare this against the two-pass path
+(SLORR_FLAG_SEPARATE_NORM) and the oracle.
+
+Matrices whose values would lose precision in an unscaled fp16 copy are re-cast with the scale by
+the kernel that finalizes their norm:
+- ||W||_F < 1;
+- max |w| > 2^15.
+
+bf16 keeps fp32's exponent range and never needs the re-cast. The Hoyer value is scale invariant
+(L(a W) = L(W), Sec. 3), so scaled copies of one set must give the same values; the oracle decides.
+"""
+
+import numpy as np
+import pytest
+
+import oracle
+import workloads
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+EPS = 1e-7
+TOL = {"fp16": (2e-2, 2e-2), "bf16": (2e-2, 5e-2)}
+SHAPES = [(256, 768), (768, 256), (130, 700), (64, 147), (1000, 130), (384, 384)]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _need_gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2607_08754_gb300 import slorr
+    slorr.load_library()
+
+
+def rel(a, b):
+    return np.linalg.norm(a - b) / np.linalg.norm(b)
+
+
+def run(Ws, compute, flags=0, variant="hoyer"):
+    from paper_2607_08754_gb300.slorr import Regularizer
+    reg = Regularizer([W.shape for W in Ws], variant=variant, compute=compute, flags=flags)
+    w = [torch.from_numpy(np.ascontiguousarray(W, dtype=np.float32)).cuda() for W in Ws]
+    g = [torch.zeros_like(x) for x in w]
+    per = torch.empty(len(Ws), device="cuda")
+    loss = reg(w, g, per_matrix=per).item()
+    torch.cuda.synchronize()
+    assert reg.status() == 0
+    return loss, per.double().cpu().numpy(), [x.double().cpu().numpy() for x in g], reg, w
+
+
+def check_oracle(Ws, out, compute, variant="hoyer"):
+    loss, per, grads = out[:3]
+    tl, tg = TOL[compute]
+    W64 = [W.astype(np.float32).astype(np.float64) for W in Ws]
+    ref_loss, ref_per, ref_inc = oracle.reg_forward_backward(W64, variant, oracle.pe_coefficients(6), 1.0, EPS)
+    assert abs(loss - ref_loss) <= tl * abs(ref_loss)
+    for i in range(len(Ws)):
+        assert abs(per[i] - ref_per[i]) <= tl * abs(ref_per[i]), (i, per[i], ref_per[i])
+        assert rel(grads[i], ref_inc[i]) <= tg, (i, rel(grads[i], ref_inc[i]))
+
+
+def x0_scale(reg, i):
+    from paper_2607_08754_gb300.slorr import slorr_iterate_view, device_view
+    dev = reg._ws.device
+    v = slorr_iterate_view(reg.handle, reg.workspace(dev), i, 0)
+    return float(device_view(v.x0_scale, (1,), "<f4", dev).cpu()[0])
+
+
+@pytest.mark.parametrize("variant", ["hoyer", "nuclear"])
+@pytest.mark.parametrize("compute", ["fp16", "bf16"])
+def test_fused_norm_matches_two_pass_path_and_oracle(compute, variant):
+    from paper_2607_08754_gb300.slorr import FLAG_SEPARATE_NORM
+    Ws = [workloads.random_matrix(s, seed=300 + i, std=0.05) for i, s in enumerate(SHAPES)]
+    fused = run(Ws, compute, 0, variant)
+    split = run(Ws, compute, FLAG_SEPARATE_NORM, variant)
+    check_oracle(Ws, fused, compute, variant)
+    check_oracle(Ws, split, compute, variant)
+    # ||W||_F^2 is the same sum of the same squares in both passes
+    for i in range(len(Ws)):
+        f_a, _ = fused[3].scalars(i)
+        f_b, _ = split[3].scalars(i)
+        assert f_a == pytest.approx(float(np.sum(Ws[i].astype(np.float64) ** 2)), rel=1e-6)
+        assert f_a == pytest.approx(f_b, rel=1e-6)
+        assert x0_scale(split[3], i) == 1.0
+        assert x0_scale(fused[3], i) == pytest.approx(1.0 / (np.sqrt(f_a) + EPS), rel=1e-6)
+
+
+@pytest.mark.parametrize("compute", ["fp16", "bf16"])
+def test_x0_is_the_normalised_weight(compute):
+    """After 0 steps the iterate view (stored buffer times x0_scale) is
+    W / (||W||_F + eps) up to one 16-bit rounding of W."""
+    from paper_2607_08754_gb300.slorr import Regularizer
+    Ws = [workloads.random_matrix(s, seed=320 + i, std=0.05) for i, s in enumerate(SHAPES)]
+    reg = Regularizer(SHAPES, compute=compute)
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    reg.run_steps(w, 0)
+    torch.cuda.synchronize()
+    assert reg.status() == 0
+    ulp = 2.0 ** -11 if compute == "fp16" else 2.0 ** -8
+    for i, W in enumerate(Ws):
+        W64 = W.astype(np.float64)
+        ref = W64 / (np.linalg.norm(W64) + EPS)
+        ref = ref.T if W.shape[0] > W.shape[1] else ref
+        assert rel(reg.iterate(i, 0).double().cpu().numpy(), ref) <= ulp
+
+
+@pytest.mark.parametrize("compute", ["fp16", "bf16"])
+def test_values_outside_the_unscaled_range_are_recast(compute):
+    """One set mixing matrices that suit the unscaled copy (std 0.05) with
+    ones that do not in fp16: ||W||_F < 1 (times 1e-4) and max |w| > 2^15
+    (times 1e6).  Each matrix is decided on its own.  In fp16 the re-cast
+    matrices have x0_scale = 1; in bf16 every matrix keeps the unscaled copy.
+    The values and gradients match the oracle, and the Hoyer values equal
+    those of the unscaled set (scale invariance)."""
+    base = [workloads.random_matrix(s, seed=340 + i, std=0.05) for i, s in enumerate(SHAPES)]
+    factors = [1.0, 1e-4, 1e6, 1.0, 1e-4, 1e6]
+    Ws = [W * np.float32(f) for W, f in zip(base, factors)]
+    out = run(Ws, compute)
+    check_oracle(Ws, out, compute)
+    ref = run(base, compute)
+    np.testing.assert_allclose(out[1], ref[1], rtol=2e-2)
+    for i, f in enumerate(factors):
+        fsq, _ = out[3].scalars(i)
+        expect = 1.0 / (np.sqrt(fsq) + EPS)
+        if compute == "fp16" and f != 1.0:
+            assert x0_scale(out[3], i) == 1.0, i
+        else:
+            assert x0_scale(out[3], i) == pytest.approx(expect, rel=1e-6), i
