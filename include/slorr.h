@@ -121,6 +121,12 @@ typedef struct slorr_options {
                                        kernel are programmatic dependents of the kernel
                                        before them, so each one's launch and prologue
                                        overlap the previous one's tail (tuning)          */
+#define SLORR_FLAG_NO_SPLIT_K  2048  /* never split the K range of a Gram tile across CTA
+                                       pairs.  By default a set whose few Gram tiles have
+                                       a long K (Q >> P, e.g. ResNet-18's 512 x 4608
+                                       layers) splits each such tile into up to 2 parts
+                                       whose fp32 partials are added, in part order, by
+                                       the last part's epilogue (tuning)                */
 #define SLORR_FLAG_SEPARATE_NORM 1024 /* 16-bit iterates: take ||W||_F and write X_0 in two
                                        passes over W.  By default one pass does both:
                                        it stores W rounded to 16 bits and the first
@@ -246,6 +252,12 @@ SLORR_API slorr_status slorr_partition(const slorr_shape* shapes, int32_t count,
  * the strictly-lower tiles of the symmetric products.  slorr_flops gives the
  * paper's algorithmic count (Sec. 3 "Computational cost") instead. */
 SLORR_API slorr_status slorr_executed_flops(const slorr_handle* h, double* out);
+
+/* Work items of one GEMM launch of the plan (host-only): phase 0 Gram, 1 Poly,
+ * 2 Update.  For the tensor-core kernels an item is a 256 x 256 output tile,
+ * or one K part of a split Gram tile (SLORR_FLAG_NO_SPLIT_K); for the 4-CTA
+ * kernel a pair of tiles; for the CUDA-core kernel a 64 x 64 tile. */
+SLORR_API slorr_status slorr_gemm_items(const slorr_handle* h, int32_t phase, int32_t* items);
 
 /* Per-kernel timing (tracing).  While enabled, every kernel this handle
  * launches is bracketed by a pair of CUDA events recorded on the caller's

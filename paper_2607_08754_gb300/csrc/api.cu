@@ -66,9 +66,11 @@ struct slorr_handle {
     std::vector<MemItem> x_items;  // tiles of the padded iterate (cast)
     int total_w_tiles = 0;
     int total_x_tiles = 0;
+    int total_split_parts = 0;  // 256 x 256 fp32 partial slots of split-K Gram tiles
     // workspace layout
     size_t off_status = 0, off_counters = 0, off_scalars = 0, off_partials = 0, off_partials_max = 0,
-           off_tilebase = 0, off_tilecount = 0, off_xtilebase = 0, off_xtilecount = 0, off_mats = 0, off_maps = 0, off_tc_items[3] = {}, off_quad_items[3] = {},
+           off_tilebase = 0, off_tilecount = 0, off_xtilebase = 0, off_xtilecount = 0, off_split_cnt = 0,
+           off_split_part = 0, off_mats = 0, off_maps = 0, off_tc_items[3] = {}, off_quad_items[3] = {},
            off_simt_items[3] = {},
            off_w_items = 0, off_x_items = 0, off_ptrs = 0, off_plan_end = 0, total_bytes = 0;
     // device state
@@ -177,6 +179,49 @@ void add_quad_items(std::vector<GemmItem>& out, int mat, int ph, int Ppad, int N
     }
 }
 
+// Split K of the CTA-pair kernel's Gram tiles (A = X X^T with K = Qpad).  A
+// Gram launch lasts at least as long as its longest tile, and a set with few
+// tiles of long K (ResNet-18's 512 x 4608 layers: 3 tiles of K = 4608) leaves
+// most pairs idle meanwhile.  The plan assumes 76 pairs (152 SMs): a tile's K
+// is split into parts of about max(1024, the launch's K per pair), at most
+// kMaxSplit (2) parts.  Each part accumulates its K range; the epilogue warp that
+// finishes last adds the parts' fp32 partials in part order.  That warp
+// reads every part's 256 x 256 partial, so more parts shorten the main loop
+// but lengthen the last epilogue.
+constexpr int kPlanPairs = 76;
+#ifndef SLORR_SPLIT_MIN_K
+#define SLORR_SPLIT_MIN_K 1024
+#endif
+
+void split_gram_items(slorr_handle* h) {
+    h->total_split_parts = 0;
+    if (h->opt.compute == SLORR_COMPUTE_FP32 || !tc_pair(h) ||
+        (h->opt.flags & (SLORR_FLAG_SIMT_GEMM | SLORR_FLAG_TC_QUAD | SLORR_FLAG_NO_SPLIT_K)))
+        return;
+    std::vector<GemmItem>& items = h->tc_items[kGram];
+    double work = 0.0;
+    for (const GemmItem& it : items) work += h->geom[it.mat].Qpad;
+    const double target = std::max(double(SLORR_SPLIT_MIN_K), work / kPlanPairs);
+    std::vector<GemmItem> out;
+    for (const GemmItem& it : items) {
+        const int K = h->geom[it.mat].Qpad;
+        int parts = int(std::ceil(K / target));
+        parts = std::min(std::min(parts, kMaxSplit), K / 64);
+        if (parts <= 1) {
+            out.push_back(it);
+            continue;
+        }
+        for (int q = 0; q < parts; ++q) {
+            GemmItem part = it;
+            part.ksplit = uint16_t(q | (parts << 8));
+            part.sid = uint32_t(h->total_split_parts);
+            out.push_back(part);
+        }
+        h->total_split_parts += parts;
+    }
+    items.swap(out);
+}
+
 void build_plan(slorr_handle* h) {
     const int count = int(h->shapes.size());
     h->geom.resize(count);
@@ -239,11 +284,15 @@ void build_plan(slorr_handle* h) {
     }
     h->total_w_tiles = tile_base;
     h->total_x_tiles = xtile_base;
+    split_gram_items(h);
     // Longest K first (stable: keeps a matrix's tiles together).
     for (int ph = 0; ph < 3; ++ph) {
         auto kdim = [&](const GemmItem& it) {
             const Geom& g = h->geom[it.mat];
-            return ph == kGram ? g.Qpad : g.Ppad;
+            const int K = ph == kGram ? g.Qpad : g.Ppad;
+            int b, e;
+            split_range(it, K / 64, &b, &e);
+            return it.ksplit ? (e - b) * 64 : K;
         };
         std::stable_sort(h->tc_items[ph].begin(), h->tc_items[ph].end(),
                          [&](const GemmItem& a, const GemmItem& b) { return kdim(a) > kdim(b); });
@@ -274,6 +323,8 @@ void build_plan(slorr_handle* h) {
     off = align_up(off + size_t(std::max(h->total_w_tiles, h->total_x_tiles)) * 4, 256);
     h->off_partials_max = off;
     off = align_up(off + size_t(h->total_x_tiles) * 4, 256);
+    h->off_split_cnt = off;
+    off = align_up(off + size_t(h->total_split_parts) * 8 * 4, 256);
     h->off_tilebase = off;
     off = align_up(off + size_t(count) * 4, 256);
     h->off_tilecount = off;
@@ -301,6 +352,8 @@ void build_plan(slorr_handle* h) {
     h->off_ptrs = off;
     off = align_up(off + size_t(2 * count) * sizeof(void*), 1024);
     h->off_plan_end = off;
+    h->off_split_part = off;
+    off = align_up(off + size_t(h->total_split_parts) * 65536 * 4, 1024);
     for (int i = 0; i < count; ++i) {
         Geom& g = h->geom[i];
         const size_t xbytes = size_t(g.rows) * g.ld * h->esize;
@@ -545,6 +598,10 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
     s = upload_ptrs(h, ws, weights, finish ? grads : nullptr, st);
     if (s != SLORR_OK) return s;
     cudaError_t e = cudaMemsetAsync(ws + h->off_counters, 0, (h->shapes.size() + 1) * 4, st);
+    // split-K part counts: each Gram's last parts leave them at zero, but a
+    // call that timed out may not have
+    if (e == cudaSuccess && h->total_split_parts > 0)
+        e = cudaMemsetAsync(ws + h->off_split_cnt, 0, size_t(h->total_split_parts) * 8 * 4, st);
     if (e != cudaSuccess) return cuda_fail(e, "counter reset");
 
     const bool use_tc = h->opt.compute != SLORR_COMPUTE_FP32 && !(h->opt.flags & SLORR_FLAG_SIMT_GEMM);
@@ -587,6 +644,8 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
     g.pair_slots = (h->opt.flags & SLORR_FLAG_PAIR_ONE_SLOT) ? 1 : 2;
     g.pdl = (use_pdl(h) && pair && !quad) ? 1 : 0;
     g.scalars = reinterpret_cast<const MatScalars*>(ws + h->off_scalars);
+    g.split_part = reinterpret_cast<float*>(ws + h->off_split_part);
+    g.split_cnt = reinterpret_cast<uint32_t*>(ws + h->off_split_cnt);
     for (int t = 0; t < steps; ++t) {
         g.cur = t & 1;
         g.a = float(h->coeffs[3 * t + 0]);
@@ -728,12 +787,25 @@ slorr_status slorr_executed_flops(const slorr_handle* h, double* out) {
         for (const GemmItem& it : items) {
             if (it.msz == 0) continue;  // empty half of a super-tile
             const Geom& g = h->geom[it.mat];
-            const double K = ph == kGram ? g.Qpad : g.Ppad;
+            const int Kfull = ph == kGram ? g.Qpad : g.Ppad;
+            int kb0, kb1;
+            split_range(it, Kfull / 64, &kb0, &kb1);
+            const double K = it.ksplit ? double(kb1 - kb0) * 64 : double(Kfull);
             const double rows = pair ? 256.0 : double(it.msz);  // pair UMMAs are always M = 256
             total += 2.0 * rows * double(it.nsz) * K;
         }
     }
     *out = total * double(h->opt.iters);
+    return SLORR_OK;
+}
+
+slorr_status slorr_gemm_items(const slorr_handle* h, int32_t phase, int32_t* items) {
+    if (!h || !items) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
+    if (phase < 0 || phase > 2) return fail(SLORR_ERR_INVALID_ARG, "phase must be 0 (Gram), 1 (Poly) or 2 (Update)");
+    const bool simt = h->opt.compute == SLORR_COMPUTE_FP32 || (h->opt.flags & SLORR_FLAG_SIMT_GEMM);
+    const bool quad = !simt && tc_pair(h) && (h->opt.flags & SLORR_FLAG_TC_QUAD);
+    *items = int32_t(simt ? h->simt_items[phase].size()
+                          : quad ? h->quad_items[phase].size() / 2 : h->tc_items[phase].size());
     return SLORR_OK;
 }
 

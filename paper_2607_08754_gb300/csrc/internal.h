@@ -69,8 +69,27 @@ struct GemmItem {
     uint16_t tn;       // column tile index (256 columns per tcgen05 tile, 64 for SIMT)
     uint16_t nsz;      // columns in this tile
     uint16_t msz;      // rows in this tile
-    uint16_t pad_;
+    uint16_t ksplit;   // split K (CTA-pair Gram): part s | (parts S << 8); 0 = whole K
+    uint32_t sid;      // split K: the tile's first 256 x 256 partial slot (parts sid .. sid + S - 1)
 };
+
+// K blocks [begin, end) of an item's nkb: part s of S takes an equal share.
+__host__ __device__ inline void split_range(const GemmItem& it, int nkb, int* begin, int* end) {
+    const int parts = it.ksplit >> 8;
+    if (parts <= 1) {
+        *begin = 0;
+        *end = nkb;
+        return;
+    }
+    const int s = it.ksplit & 0xff;
+    *begin = s * nkb / parts;
+    *end = (s + 1) * nkb / parts;
+}
+
+#ifndef SLORR_MAX_SPLIT
+#define SLORR_MAX_SPLIT 2
+#endif
+constexpr int kMaxSplit = SLORR_MAX_SPLIT;  // K parts of a split Gram tile (a build-time tuning knob)
 
 // One chunk of a memory-bound pass: a kMemRows x kMemCols tile of W (or of
 // the padded iterate buffer for the cast).
@@ -109,6 +128,12 @@ struct GemmLaunch {
     // scalars[i].x0_scale^2 and the Update epilogue by scalars[i].x0_scale.
     int32_t x0_scaled;
     const MatScalars* scalars;
+    // split K (CTA-pair Gram): part s of a split tile leaves its fp32 partial
+    // at split_part + ((sid + s) * 256 + column) * 256 + row (tile
+    // coordinates), and counts it in split_cnt[sid * 8 + rank * 4 + quad];
+    // the epilogue warp that counts last adds the parts and stores the tile.
+    float* split_part;
+    uint32_t* split_cnt;
 };
 
 // Tensor maps per matrix: X0 K-major, X1 K-major, X0 MN-major, X1 MN-major,

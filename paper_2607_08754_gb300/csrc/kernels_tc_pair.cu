@@ -124,7 +124,9 @@ __device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, 
         const bool load_a = rank * kBM < it.msz;
         const bool load_b = !shared_operand(p, it);
         const int bhalf = it.nsz / 2;  // 64 or 128 rows of B per CTA
-        for (int kb = 0; kb < pi.nkb; ++kb) {
+        int kb_begin, kb_end;
+        split_range(it, pi.nkb, &kb_begin, &kb_end);
+        for (int kb = kb_begin; kb < kb_end; ++kb) {
             if (!ptx::mbar_wait(&s.empty[stage], phase ^ 1u, s.abort, p.timeout_ns)) {
                 record_timeout(p, s);
                 return;
@@ -161,7 +163,9 @@ struct KCursor {
     __device__ void load() {
         if (idx < p->num_items) {
             const GemmItem it = p->items[idx];
-            nkb = phase_info<C>(*p, it).nkb;
+            int b, e;
+            split_range(it, phase_info<C>(*p, it).nkb, &b, &e);
+            nkb = e - b;
             bytes = pair_stage_bytes<C>(*p, it, 0) + pair_stage_bytes<C>(*p, it, 1);
         }
     }
@@ -216,7 +220,9 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
         }
         ptx::tc_fence_after();
         const uint32_t d_tmem = tmem_base + uint32_t(slot * kAccCols);
-        for (int kb = 0; kb < pi.nkb; ++kb) {
+        int kb_begin, kb_end;
+        split_range(it, pi.nkb, &kb_begin, &kb_end);
+        for (int kb = kb_begin; kb < kb_end; ++kb) {
             if (!ptx::mbar_wait(&s.full[stage], phase, s.abort, p.timeout_ns)) {
                 record_timeout(p, s);
                 ok = false;
@@ -235,7 +241,7 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
 #pragma unroll
             for (int kk = 0; kk < C::BK / 16; ++kk)
                 ptx::umma_f16_pair(d_tmem, operand_desc<C>(a0, kk, pi.a_mn), operand_desc<C>(b0, kk, pi.b_mn), idesc,
-                                   (kb | kk) != 0 ? 1u : 0u);
+                                   (kb != kb_begin || kk != 0) ? 1u : 0u);
             issued_any = true;
             ptx::umma_commit_pair_mc(&s.empty[stage], 0x3);
             if (++stage == C::STAGES) {
@@ -284,7 +290,14 @@ __device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t t
             const int row0 = it.tm * (2 * kBM) + rank * kBM;
             const uint32_t t_row = tmem_base + (uint32_t(quad * 32) << 16) + uint32_t(slot * kAccCols);
             const int per = it.nsz / 32 / ngroups;  // 32-column chunks per warp
-            store_rows<BF16, 2>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per);
+            const int parts = it.ksplit >> 8;
+            if (parts <= 1) {
+                store_rows<BF16, 2>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per);
+            } else if constexpr (C::kEpiWarps == 4) {  // split K: Gram only, one warp per lane quadrant
+                if (split_partial_is_last(p, it, rank, quad, lane, t_row, 0, per))
+                    store_rows<BF16, 2>(p, it, md, row0, t_row, quad, lane, 0, per,
+                                        p.split_part + size_t(it.sid) * 65536, parts, rank * kBM + quad * 32 + lane);
+            }
         }
         // The slot may be overwritten once this warp's TMEM loads are done
         // (tcgen05.wait::ld above); the stores need no ordering with the

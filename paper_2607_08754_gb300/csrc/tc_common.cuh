@@ -109,6 +109,38 @@ __device__ __forceinline__ uint64_t operand_desc(uint32_t base, int kk, bool mn)
               : ptx::sdesc(base + kk * 32, 16, C::kKSbo, C::kKLayout);
 }
 
+// Split K, one part of a tile: this warp stores its 32 rows of the part's
+// fp32 accumulator (columns [32 ch_begin, 32 ch_end) of the tile) in the
+// part's 256 x 256 slot, split_part + (sid + s) * 65536, column-major so that
+// each column's 32 rows are one coalesced segment, and counts them in
+// split_cnt[sid * 8 + rank * 4 + quad].  Returns true in the warp that
+// counts last for its rows (the other parts' rows are then visible to it);
+// that warp resets the count for the next launch.
+__device__ __forceinline__ bool split_partial_is_last(const GemmLaunch& p, const GemmItem& it, int rank, int quad,
+                                                      int lane, uint32_t t_row, int ch_begin, int ch_end) {
+    const int parts = it.ksplit >> 8, own = it.ksplit & 0xff;
+    const int row_t = rank * kBM + quad * 32 + lane;
+    float* dst = p.split_part + (size_t(it.sid) + own) * 65536 + row_t;
+    for (int ch = ch_begin; ch < ch_end; ++ch) {
+        uint32_t r[32];
+        ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
+        ptx::tmem_ld_wait();
+#pragma unroll
+        for (int j = 0; j < 32; ++j) dst[size_t(ch * 32 + j) * 256] = __uint_as_float(r[j]);
+    }
+    __threadfence();
+    __syncwarp();
+    uint32_t* cnt = p.split_cnt + size_t(it.sid) * 8 + rank * 4 + quad;
+    int last = 0;
+    if (lane == 0) {
+        last = atomicAdd(cnt, 1u) == uint32_t(parts - 1) ? 1 : 0;
+        if (last) *cnt = 0u;
+    }
+    last = __shfl_sync(0xffffffffu, last, 0);
+    if (last) __threadfence();
+    return last != 0;
+}
+
 // Epilogue of one 128-row block of a finished tile: this warp's 32 TMEM lanes
 // (rows row0 + 32 quad + [0, 32)) and the tile's 32-column chunks
 // [ch_begin, ch_end) (chunk c: columns tn * 256 + 32 c, TMEM columns t_row + 32 c).
@@ -119,9 +151,13 @@ __device__ __forceinline__ uint64_t operand_desc(uint32_t base, int kk, bool mn)
 //           mirror tile is skipped (tiles are MT x 128 rows by 256 columns).
 // In the first step after the fused norm pass (p.x0_scaled) the stored X_0
 // is W itself: the Gram scales acc by x0_scale^2 and the Update by x0_scale.
+// With split K (Gram), the accumulator is replaced by the sum, in part
+// order, of the `parts` fp32 partials at split_tile (row row_t of the tile;
+// this warp's own part among them).
 template <bool BF16, int MT>
 __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& it, const MatDev& md, int row0,
-                                           uint32_t t_row, int quad, int lane, int ch_begin, int ch_end) {
+                                           uint32_t t_row, int quad, int lane, int ch_begin, int ch_end,
+                                           const float* split_tile = nullptr, int parts = 1, int row_t = 0) {
     const int row = row0 + quad * 32 + lane;
     const int nch = ch_end;
     const float xs = p.x0_scaled ? p.scalars[it.mat].x0_scale : 1.f;
@@ -178,8 +214,33 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
                 }
             }
             uint32_t r[32];
-            ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
-            ptx::tmem_ld_wait();
+            if (split_tile == nullptr) {
+                ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
+                ptx::tmem_ld_wait();
+            } else {
+                // every part from memory, in part order, two parts' loads in
+                // flight at a time: the sum does not depend on which part
+                // finished last
+                const float* src = split_tile + size_t(ch * 32) * 256 + row_t;
+#pragma unroll
+                for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(__ldcg(src + size_t(j) * 256));
+                for (int q = 1; q < parts; q += 2) {
+                    const float* s1 = src + size_t(q) * 65536;
+                    float a[32], b[32];
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) a[j] = __ldcg(s1 + size_t(j) * 256);
+                    if (q + 1 < parts) {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) b[j] = __ldcg(s1 + 65536 + size_t(j) * 256);
+                    }
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        float v = __uint_as_float(r[j]) + a[j];
+                        if (q + 1 < parts) v += b[j];
+                        r[j] = __float_as_uint(v);
+                    }
+                }
+            }
             uint4 o[4];
             uint32_t* ow = reinterpret_cast<uint32_t*>(o);
             const int d = row - col0;  // diagonal element of this row, if in the chunk

@@ -35,6 +35,7 @@ FLAG_PAIR_ONE_SLOT = 128
 FLAG_TC_QUAD = 256
 FLAG_NO_PDL = 512
 FLAG_SEPARATE_NORM = 1024
+FLAG_NO_SPLIT_K = 2048
 
 
 class SlorrError(RuntimeError):
@@ -92,6 +93,7 @@ def load_library(path: str | None = None) -> ctypes.CDLL:
         "slorr_partition": (i32, [ctypes.POINTER(Shape), i32, i32, i32, ctypes.POINTER(i32),
                                   ctypes.POINTER(i32)]),
         "slorr_executed_flops": (i32, [vp, ctypes.POINTER(dbl)]),
+        "slorr_gemm_items": (i32, [vp, i32, ctypes.POINTER(i32)]),
         "slorr_set_timing": (i32, [vp, i32]),
         "slorr_read_timing": (i32, [vp, ctypes.POINTER(dbl), ctypes.POINTER(i64), i32]),
         "slorr_frob_sq_noalloc": (i32, [vp, i64, i64, i32, vp, vp]),
@@ -221,6 +223,13 @@ def slorr_executed_flops(handle) -> float:
     out = ctypes.c_double()
     _check(load_library().slorr_executed_flops(handle, ctypes.byref(out)))
     return out.value
+
+
+def slorr_gemm_items(handle, phase: int) -> int:
+    """Work items of one GEMM launch of the plan: phase 0 Gram, 1 Poly, 2 Update."""
+    out = ctypes.c_int32(0)
+    _check(load_library().slorr_gemm_items(handle, int(phase), ctypes.byref(out)))
+    return int(out.value)
 
 
 def slorr_partition(shapes, world: int, rank: int) -> list[int]:

@@ -150,3 +150,61 @@ def test_programmatic_dependent_launch_is_bit_identical():
     for a, b in zip(out[0][0], out[1][0]):
         assert torch.equal(a, b)
     assert torch.equal(out[0][1], out[1][1])
+
+
+def test_split_k_gram_matches_whole_k_and_oracle():
+    """Split K of long Gram tiles (the default for sets whose few Gram tiles
+    have a long K): the parts' fp32 partials, added in part order by the last
+    part's epilogue, give the same iterates as whole-K tiles
+    (SLORR_FLAG_NO_SPLIT_K) up to fp32 summation order, and the values and
+    gradients match the oracle.  Shapes: K = Q up to 4608, a transposed
+    matrix (m > n: MN-major Gram operands), a tile of 128 rows and a set
+    small enough that its tiles are split."""
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_NO_SPLIT_K, slorr_gemm_items
+    shapes = [(512, 4608), (4608, 384), (256, 2304), (130, 1152), (512, 1000)]
+    Ws = [workloads.random_matrix(s, seed=510 + i, std=0.02) for i, s in enumerate(shapes)]
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    split = Regularizer(shapes)
+    whole = Regularizer(shapes, flags=FLAG_NO_SPLIT_K)
+    assert slorr_gemm_items(split.handle, 0) > slorr_gemm_items(whole.handle, 0)
+    for k in (1, 2, 6):
+        split.run_steps(w, k)
+        whole.run_steps(w, k)
+        torch.cuda.synchronize()
+        assert split.status() == 0 and whole.status() == 0
+        for i in range(len(shapes)):
+            a = split.iterate(i, k).double().cpu().numpy()
+            b = whole.iterate(i, k).double().cpu().numpy()
+            assert rel(a, b) <= 4 * 2.0 ** -10 * k, (k, i, shapes[i], rel(a, b))
+    g = [torch.zeros_like(x) for x in w]
+    per = torch.empty(len(shapes), device="cuda")
+    loss = split(w, g, per_matrix=per).item()
+    torch.cuda.synchronize()
+    assert split.status() == 0
+    co = oracle.pe_coefficients(6)
+    ref_loss, ref_per, ref_inc = oracle.reg_forward_backward([W.astype(np.float64) for W in Ws], "hoyer", co,
+                                                             1.0, EPS)
+    assert abs(loss - ref_loss) <= 2e-2 * abs(ref_loss)
+    per = per.double().cpu().numpy()
+    for i in range(len(shapes)):
+        assert abs(per[i] - ref_per[i]) <= 2e-2 * abs(ref_per[i]), (i, shapes[i])
+        assert rel(g[i].double().cpu().numpy(), ref_inc[i]) <= 2e-2, (i, shapes[i])
+
+
+def test_split_k_is_deterministic():
+    """The last part adds every part's partial in part order, so repeated
+    calls give bit-identical iterates whichever part finishes last."""
+    from paper_2607_08754_gb300.slorr import Regularizer
+    shapes = [(512, 4608), (256, 2304), (512, 1000)]
+    Ws = [workloads.random_matrix(s, seed=530 + i, std=0.02) for i, s in enumerate(shapes)]
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    reg = Regularizer(shapes)
+    outs = []
+    for _ in range(3):
+        reg.run_steps(w, 6)
+        torch.cuda.synchronize()
+        assert reg.status() == 0
+        outs.append([reg.iterate(i, 6).cpu() for i in range(len(shapes))])
+    for o in outs[1:]:
+        for a, b in zip(outs[0], o):
+            assert torch.equal(a, b)

@@ -36,11 +36,11 @@ def rel(a, b):
 
 @pytest.mark.parametrize("compute", ["fp16", "bf16"])
 def test_quad_iterates_match_simt_and_pair(compute):
-    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_SIMT_GEMM
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_SIMT_GEMM, FLAG_NO_SPLIT_K
     Ws = [workloads.random_matrix(s, seed=500 + i, std=0.02) for i, s in enumerate(SHAPES)]
     w = [torch.from_numpy(W).cuda() for W in Ws]
     qd = Regularizer(SHAPES, compute=compute, flags=QUAD)
-    pr = Regularizer(SHAPES, compute=compute)
+    pr = Regularizer(SHAPES, compute=compute, flags=FLAG_NO_SPLIT_K)  # the quad kernel takes whole-K tiles
     st = Regularizer(SHAPES, compute=compute, flags=FLAG_SIMT_GEMM)
     ulp = 2.0 ** -10 if compute == "fp16" else 2.0 ** -7
     for k in (1, 2, 6):
@@ -85,7 +85,7 @@ def test_quad_bounded_wait_timeout_and_recovery():
     nothing arrives on and give up after timeout_s; all four CTAs unwind, each
     leader drains its pair's copies, and the call reports SLORR_ERR_TIMEOUT.  A
     normal call afterwards matches the pair kernel."""
-    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_TEST_STALL
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_TEST_STALL, FLAG_NO_SPLIT_K
     shapes = [(256, 512), (384, 128), (640, 1000)]
     Ws = [workloads.random_matrix(s, 41 + i, 0.05) for i, s in enumerate(shapes)]
     w = [torch.from_numpy(W).cuda() for W in Ws]
@@ -95,7 +95,7 @@ def test_quad_bounded_wait_timeout_and_recovery():
     assert stall.status() == 5          # SLORR_ERR_TIMEOUT
     assert stall.status() == 0
     qd = Regularizer(shapes, flags=QUAD)
-    pr = Regularizer(shapes)
+    pr = Regularizer(shapes, flags=FLAG_NO_SPLIT_K)
     qd.run_steps(w, 2)
     pr.run_steps(w, 2)
     torch.cuda.synchronize()

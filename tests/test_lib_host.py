@@ -235,3 +235,33 @@ def test_executed_flops_counts_pair_tiles(lib):
         assert slorr.slorr_executed_flops(r.handle) == expected(shapes, 4)
     assert slorr.slorr_executed_flops(slorr.Regularizer([(256, 256)]).handle) == \
         slorr.slorr_flops([(256, 256)], 6)
+
+
+def test_split_k_plan(lib):
+    """The Gram tiles of a set with few long-K tiles are split into K parts
+    (at most 2, about max(1024, the launch's K per pair) each); sets
+    whose Gram tiles already fill the pairs, Poly and Update, the
+    CUDA-core path and SLORR_FLAG_NO_SPLIT_K are not.  Splitting changes
+    neither the tiles' total K nor the executed FLOPs."""
+    import workloads
+    rn = workloads.shapes("resnet18")
+    split = slorr.Regularizer(rn)
+    whole = slorr.Regularizer(rn, flags=slorr.FLAG_NO_SPLIT_K)
+    g_split = slorr.slorr_gemm_items(split.handle, 0)
+    g_whole = slorr.slorr_gemm_items(whole.handle, 0)
+    assert g_whole < g_split <= 2 * g_whole
+    for ph in (1, 2):
+        assert slorr.slorr_gemm_items(split.handle, ph) == slorr.slorr_gemm_items(whole.handle, ph)
+    assert slorr.slorr_executed_flops(split.handle) == slorr.slorr_executed_flops(whole.handle)
+    assert split.workspace_bytes > whole.workspace_bytes      # the parts' fp32 partial slots
+    # one 512 x 4608 matrix alone: its 3 Gram tiles (K = 4608, 72 K blocks) become 3 x 2 parts
+    one = slorr.Regularizer([(512, 4608)])
+    assert slorr.slorr_gemm_items(one.handle, 0) == 6
+    # the ViT-L/16 set's 960 Gram tiles fill the 76 pairs many times over
+    vl = workloads.shapes("vit_l16")
+    assert slorr.slorr_gemm_items(slorr.Regularizer(vl).handle, 0) == \
+        slorr.slorr_gemm_items(slorr.Regularizer(vl, flags=slorr.FLAG_NO_SPLIT_K).handle, 0) == 960
+    assert slorr.slorr_gemm_items(slorr.Regularizer(rn, compute="fp32").handle, 0) == \
+        slorr.slorr_gemm_items(slorr.Regularizer(rn, compute="fp32", flags=slorr.FLAG_NO_SPLIT_K).handle, 0)
+    with pytest.raises(slorr.SlorrError):
+        slorr.slorr_gemm_items(split.handle, 3)
