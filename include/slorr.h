@@ -127,6 +127,14 @@ typedef struct slorr_options {
                                        layers) splits each such tile into up to 2 parts
                                        whose fp32 partials are added, in part order, by
                                        the last part's epilogue (tuning)                */
+#define SLORR_FLAG_GRAPH       4096  /* capture the launches of a forward/backward or
+                                       descent call into a CUDA graph once and replay it
+                                       while the workspace, loss_out, per_matrix_out, T
+                                       and eta are unchanged (the weight and grad
+                                       pointers may change: they are read from the
+                                       workspace).  Ignored while timing is on; a stream
+                                       that is being captured gets the launches.  Saves
+                                       the launch gaps of small sets                    */
 #define SLORR_FLAG_SEPARATE_NORM 1024 /* 16-bit iterates: take ||W||_F and write X_0 in two
                                        passes over W.  By default one pass does both:
                                        it stores W rounded to 16 bits and the first

@@ -82,7 +82,13 @@ struct slorr_handle {
     std::vector<cudaEvent_t> ev_pool;
     struct Mark { int kind; int kernels; cudaEvent_t start, stop; };
     std::vector<Mark> marks;
+    // SLORR_FLAG_GRAPH
+    cudaGraphExec_t graph_exec = nullptr;
+    std::vector<uintptr_t> graph_key;
+    cudaStream_t capture_stream = nullptr;
     ~slorr_handle() {
+        if (graph_exec) cudaGraphExecDestroy(graph_exec);
+        if (capture_stream) cudaStreamDestroy(capture_stream);
         for (auto& m : marks) {
             cudaEventDestroy(m.start);
             cudaEventDestroy(m.stop);
@@ -566,6 +572,65 @@ MemLaunch mem_params(slorr_handle* h, uint8_t* ws, float* loss, float* per, int 
 // descent: grads is NULL and the combine pass applies W -= eta * lambda *
 // grad_scale * G in place (the weights are then written, through a non-const
 // pointer the caller gave slorr_reg_descent_step).
+slorr_status launch_all(slorr_handle* h, uint8_t* ws, float* loss, float* per, int steps, bool finish,
+                        cudaStream_t st, bool descent, float eta);
+
+// SLORR_FLAG_GRAPH: the call's launches are captured once into a CUDA graph
+// and replayed while the workspace, the loss and value outputs, T and eta
+// stay the same (the weight and gradient pointers live in the workspace, so
+// new tensors need no new graph).  A stream that is already being captured
+// gets the launches themselves.
+slorr_status launch_graph(slorr_handle* h, uint8_t* ws, float* loss, float* per, int steps, cudaStream_t st,
+                          bool descent, float eta) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    cudaError_t e = cudaStreamIsCapturing(st, &cs);
+    if (e != cudaSuccess) return cuda_fail(e, "stream query");
+    if (cs != cudaStreamCaptureStatusNone) return launch_all(h, ws, loss, per, steps, true, st, descent, eta);
+    uint32_t eta_bits = 0;
+    std::memcpy(&eta_bits, &eta, 4);
+    const std::vector<uintptr_t> key = {reinterpret_cast<uintptr_t>(ws), reinterpret_cast<uintptr_t>(loss),
+                                        reinterpret_cast<uintptr_t>(per), uintptr_t(steps), uintptr_t(descent),
+                                        uintptr_t(eta_bits)};
+    if (h->graph_exec == nullptr || key != h->graph_key) {
+        if (h->graph_exec != nullptr) {
+            cudaGraphExecDestroy(h->graph_exec);
+            h->graph_exec = nullptr;
+        }
+        // relaxed: the first launch of each kernel configuration queries its
+        // occupancy, which the stricter capture modes forbid
+        // captured on a stream of the handle's own (the caller's may be the
+        // legacy default stream, which cannot be captured); launched on st
+        if (h->capture_stream == nullptr) {
+            e = cudaStreamCreateWithFlags(&h->capture_stream, cudaStreamNonBlocking);
+            if (e != cudaSuccess) {
+                h->capture_stream = nullptr;
+                return cuda_fail(e, "capture stream");
+            }
+        }
+        cudaStream_t cap = h->capture_stream;
+        e = cudaStreamBeginCapture(cap, cudaStreamCaptureModeRelaxed);
+        if (e != cudaSuccess) return cuda_fail(e, "graph capture");
+        const slorr_status s = launch_all(h, ws, loss, per, steps, true, cap, descent, eta);
+        cudaGraph_t graph = nullptr;
+        e = cudaStreamEndCapture(cap, &graph);
+        if (s != SLORR_OK) {
+            if (graph) cudaGraphDestroy(graph);
+            return s;
+        }
+        if (e != cudaSuccess) return cuda_fail(e, "graph capture");
+        e = cudaGraphInstantiate(&h->graph_exec, graph, 0);
+        cudaGraphDestroy(graph);
+        if (e != cudaSuccess) {
+            h->graph_exec = nullptr;
+            return cuda_fail(e, "graph instantiation");
+        }
+        h->graph_key = key;
+    }
+    e = cudaGraphLaunch(h->graph_exec, st);
+    if (e != cudaSuccess) return cuda_fail(e, "graph launch");
+    return SLORR_OK;
+}
+
 slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads, float* loss, float* per,
                  void* workspace, size_t ws_bytes, int steps, bool finish, cudaStream_t st,
                  bool descent = false, float eta = 0.f) {
@@ -597,6 +662,15 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
     if (s != SLORR_OK) return s;
     s = upload_ptrs(h, ws, weights, finish ? grads : nullptr, st);
     if (s != SLORR_OK) return s;
+    if ((h->opt.flags & SLORR_FLAG_GRAPH) && finish && !h->timing)
+        return launch_graph(h, ws, loss, per, steps, st, descent, eta);
+    return launch_all(h, ws, loss, per, steps, finish, st, descent, eta);
+}
+
+// Every launch of one call, on `st` (after run() checked the arguments, the
+// plan is in the workspace and the pointer arrays are uploaded).
+slorr_status launch_all(slorr_handle* h, uint8_t* ws, float* loss, float* per, int steps, bool finish,
+                        cudaStream_t st, bool descent, float eta) {
     cudaError_t e = cudaMemsetAsync(ws + h->off_counters, 0, (h->shapes.size() + 1) * 4, st);
     // split-K part counts: each Gram's last parts leave them at zero, but a
     // call that timed out may not have

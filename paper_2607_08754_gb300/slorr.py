@@ -36,6 +36,7 @@ FLAG_TC_QUAD = 256
 FLAG_NO_PDL = 512
 FLAG_SEPARATE_NORM = 1024
 FLAG_NO_SPLIT_K = 2048
+FLAG_GRAPH = 4096
 
 
 class SlorrError(RuntimeError):
@@ -360,12 +361,22 @@ class Regularizer:
     def coefficients(self) -> np.ndarray:
         return slorr_get_coefficients(self.handle, self.iters)
 
+    def _loss_buffer(self, dev):
+        """A fresh loss tensor per call, or with FLAG_GRAPH one reused by every
+        call (the graph replays while the output pointer stays the same)."""
+        import torch
+        if not (self.options.flags & FLAG_GRAPH):
+            return torch.empty(1, dtype=torch.float32, device=dev)
+        if getattr(self, "_loss", None) is None or self._loss.device != dev:
+            self._loss = torch.empty(1, dtype=torch.float32, device=dev)
+        return self._loss
+
     def __call__(self, weights, grads, loss=None, per_matrix=None, stream=None):
         import torch
         dev = weights[0].device
         ws = self.workspace(dev)
         if loss is None:
-            loss = torch.empty(1, dtype=torch.float32, device=dev)
+            loss = self._loss_buffer(dev)
         s = stream if stream is not None else torch.cuda.current_stream(dev).cuda_stream
         slorr_reg_forward_backward(self.handle, [w.data_ptr() for w in weights], [g.data_ptr() for g in grads],
                                    loss.data_ptr(), per_matrix.data_ptr() if per_matrix is not None else 0,
@@ -378,7 +389,7 @@ class Regularizer:
         dev = weights[0].device
         ws = self.workspace(dev)
         if loss is None:
-            loss = torch.empty(1, dtype=torch.float32, device=dev)
+            loss = self._loss_buffer(dev)
         s = stream if stream is not None else torch.cuda.current_stream(dev).cuda_stream
         slorr_reg_descent_step(self.handle, [w.data_ptr() for w in weights], eta, loss.data_ptr(),
                                per_matrix.data_ptr() if per_matrix is not None else 0, ws, self.workspace_bytes, s)
