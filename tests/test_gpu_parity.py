@@ -242,6 +242,44 @@ def test_vit_l16_full_size_sampled():
         assert rel(g[i].double().cpu().numpy(), G) <= 2e-2
 
 
+def full_set_sampled(name, samples, variant="hoyer", compute="fp16"):
+    """The whole weight set in one call, as bench.py times it; the sampled
+    matrices' values and gradients against the oracle, and the loss against
+    the sum of the values."""
+    from paper_2607_08754_gb300.slorr import Regularizer
+    shapes = workloads.shapes(name)
+    reg = Regularizer(shapes, variant=variant, compute=compute, lam=1.0)
+    w = [torch.from_numpy(workloads.generate_one(name, i)).cuda() for i in range(len(shapes))]
+    g = [torch.zeros_like(x) for x in w]
+    per = torch.empty(len(shapes), device="cuda")
+    loss = reg(w, g, per_matrix=per).item()
+    torch.cuda.synchronize()
+    assert reg.status() == 0
+    per = per.double().cpu().numpy()
+    assert loss == pytest.approx(per.sum(), rel=1e-6)
+    co = oracle.pe_coefficients(6)
+    tl, tg = TOL[compute]
+    for i in samples:
+        W = workloads.generate_one(name, i).astype(np.float64)
+        L, G, _, _ = oracle.reg_single(W, variant, co, EPS)
+        assert abs(per[i] - L) <= tl * abs(L), (name, i)
+        assert grad_err(g[i].double().cpu().numpy(), G, W, variant, 1.0, 1.0) <= tg, (name, i)
+
+
+def test_decoder_560m_full_size_sampled():
+    """The 560M decoder set (168 matrices, 417 M weights): q, k, o, gate and
+    down projections of the first and last blocks."""
+    full_set_sampled("decoder_560m", (0, 1, 3, 4, 6, 167))
+
+
+def test_decoder_560m_mha_full_size_sampled_nuclear():
+    full_set_sampled("decoder_560m_mha", (1, 5, 160), variant="nuclear")
+
+
+def test_vit_b16_full_size_sampled_bf16():
+    full_set_sampled("vit_b16", (0, 1, 2, 3, 47), compute="bf16")
+
+
 # ---- failure detection: a bounded device wait runs out -----------------------------
 
 def test_bounded_wait_timeout_reports_status_and_context_survives():
