@@ -137,6 +137,30 @@ def oracle_sample(name: str, variant: str, iters: int, budget_s: float, max_step
     return flops, t_total, desc
 
 
+def gpu_local_cpus(gpu_index: int):
+    """The host CPUs next to the GPU (its PCI device's local_cpulist in sysfs),
+    or None.  Page-locked buffers allocated from a thread on them land in the
+    GPU's own NUMA node, so host<->device copies do not cross the CPU-CPU link."""
+    try:
+        out = subprocess.run(["nvidia-smi", f"--id={gpu_index}", "--query-gpu=pci.bus_id",
+                              "--format=csv,noheader"], capture_output=True, text=True, timeout=20).stdout.strip()
+        dom, rest = out.split(":", 1)
+        bus = f"{int(dom, 16):04x}:{rest.lower()}"
+        with open(f"/sys/bus/pci/devices/{bus}/local_cpulist") as f:
+            text = f.read().strip()
+        cpus = set()
+        for part in text.split(","):
+            if "-" in part:
+                a, b = part.split("-")
+                cpus.update(range(int(a), int(b) + 1))
+            elif part:
+                cpus.add(int(part))
+        cpus &= os.sched_getaffinity(0)
+        return cpus or None
+    except Exception:
+        return None
+
+
 class ClockSampler:
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -335,7 +359,12 @@ def main():
     value = world * flops_step / (ms_step * 1e-3) / 1e12
     assert reg.status() == 0, "device status word reports an error in the timed region"
 
-    # e2e: pinned host buffers, copies inside the timed region
+    # e2e: pinned host buffers, copies inside the timed region.  The buffers
+    # are allocated, and the copies issued, from the GPU's local CPUs.
+    all_cpus = os.sched_getaffinity(0)
+    local_cpus = gpu_local_cpus(local)
+    if local_cpus:
+        os.sched_setaffinity(0, local_cpus)
     Wp = [w.pin_memory() for w in W_host]
     Gp = [torch.zeros_like(w).pin_memory() for w in W_host]
     Lp = torch.zeros(1, dtype=torch.float32).pin_memory()
@@ -378,6 +407,7 @@ def main():
     if world > 1:
         dist.all_reduce(ems, op=dist.ReduceOp.MAX)
     e2e_ms = ems.item() / args.e2e_steps
+    os.sched_setaffinity(0, all_cpus)
     if pipe is not None:
         assert pipe.status() == 0, "device status word reports an error in the e2e region"
     e2e_val = world * flops_step / (e2e_ms * 1e-3) / 1e12
@@ -450,7 +480,9 @@ def main():
             "e2e": {"value": e2e_val, "unit": "TFLOP/s", "ms_per_step": e2e_ms, "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h,
                     "call": "slorr_reg_descent_step with torch copies" if descent else
-                            f"slorr_pipeline_forward_backward, {pipe.groups} groups"},
+                            f"slorr_pipeline_forward_backward, {pipe.groups} groups",
+                    "host_buffers": ("page-locked, allocated on the GPU's %d local CPUs" % len(local_cpus))
+                                    if local_cpus else "page-locked (GPU-local CPUs unknown)"},
             "clocks": clk,
         }
         if not args.no_cpu_baseline:
