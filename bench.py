@@ -422,6 +422,17 @@ def main():
         flops_per_launch = flops_step / (3 * args.iters)
         achieved = flops_per_launch / (per_launch_ms * 1e-3) / 1e12
         peak = pk["bf16"]  # fp16 and bf16 share the dense tensor rate (nominal ratio 1)
+        # CUDA-core GEMM (fp32 mode, or the 16-bit check path): bound by FP32
+        # instruction issue.  128 FP32 lanes per SM at the maximum SM clock; the
+        # compensated (Dot2) multiply-add of fp32 mode takes 10 FP32 operations
+        # (product, its FMA error, two-sum, two error adds), the plain one 1.
+        simt = args.compute == "fp32" or bool(args.flags & slorr.FLAG_SIMT_GEMM)
+        ops_per_mac = 10 if args.compute == "fp32" else 1
+        sm_max = (clk or {}).get("sm_max_mhz") or 2070.0
+        nsm = torch.cuda.get_device_properties(dev).multi_processor_count
+        alu_peak = nsm * 128 * sm_max * 1e6 * 2 / ops_per_mac / 1e12
+        alu_source = ("derived: %d SMs x 128 FP32 lanes x %.0f MHz x 2 FLOP per multiply-add / %d FP32 "
+                      "operations per multiply-add" % (nsm, sm_max, ops_per_mac))
         wbytes_dev = sum(w.numel() * w.element_size() for w in W)
         l2_note = ("inputs larger than L2: %s weights %.3f GB (129 MB L2), no flush" % (args.dtype, wbytes_dev / 1e9)
                    if wbytes_dev > 129e6 else
@@ -467,12 +478,18 @@ def main():
                          "tflops": world * flops_exec / (ms_step * 1e-3) / 1e12,
                          "note": "MMA FLOPs the kernels execute: padding included, strictly-lower "
                                  "symmetric tiles skipped"},
-            "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                         "frac": achieved / peak, "traffic": None if single_cta else tc_traffic(),
-                         "frac_of_sustained": achieved / pk["bf16_sustained"],
-                         "kernel": ("tc_gemm_kernel" if single_cta else "tc_pair_kernel")
-                                   + " (Gram/Poly/Update launches)",
-                         "peak_source": pk["source"] + " bf16 burst (fp16 dense rate equal)"},
+            "roofline": ({"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                          "frac": achieved / peak, "traffic": None if single_cta else tc_traffic(),
+                          "frac_of_sustained": achieved / pk["bf16_sustained"],
+                          "kernel": ("tc_gemm_kernel" if single_cta else "tc_pair_kernel")
+                                    + " (Gram/Poly/Update launches)",
+                          "peak_source": pk["source"] + " bf16 burst (fp16 dense rate equal)"}
+                         if not simt else
+                         {"bound": "alu", "achieved": achieved, "peak": alu_peak, "unit": "TFLOP/s",
+                          "frac": achieved / alu_peak, "traffic": None,
+                          "kernel": "simt_gemm_kernel (Gram/Poly/Update launches, compensated fp32 sums)"
+                                    if args.compute == "fp32" else "simt_gemm_kernel (Gram/Poly/Update launches)",
+                          "peak_source": alu_source}),
             "memory_phases_ms_per_step": mem_ms,
             "memory_roofline": memory_roofline,
             "kernels": kernel_breakdown,

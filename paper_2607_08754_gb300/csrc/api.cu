@@ -283,9 +283,11 @@ void build_plan(slorr_handle* h) {
                 }
             }
             add_quad_items(h->quad_items[ph], i, ph, g.Ppad, N);
-            for (int tm = 0; tm < g.Ppad / 64; ++tm)
-                for (int tn = 0; tn < N / 64; ++tn)
-                    h->simt_items[ph].push_back(GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), 64, 64, 0});
+            // CUDA-core tiles; the symmetric Gram and Poly keep those on or above the diagonal
+            for (int tm = 0; tm < g.Ppad / kSimtTile; ++tm)
+                for (int tn = (ph == kUpdate ? 0 : tm); tn < N / kSimtTile; ++tn)
+                    h->simt_items[ph].push_back(
+                        GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), kSimtTile, kSimtTile, 0});
         }
     }
     h->total_w_tiles = tile_base;

@@ -89,7 +89,8 @@ __host__ __device__ inline void split_range(const GemmItem& it, int nkb, int* be
 #ifndef SLORR_MAX_SPLIT
 #define SLORR_MAX_SPLIT 2
 #endif
-constexpr int kMaxSplit = SLORR_MAX_SPLIT;  // K parts of a split Gram tile (a build-time tuning knob)
+constexpr int kMaxSplit = SLORR_MAX_SPLIT;
+constexpr int kSimtTile = 32;  // output tile of the CUDA-core GEMM (32 x 32)  // K parts of a split Gram tile (a build-time tuning knob)
 
 // One chunk of a memory-bound pass: a kMemRows x kMemCols tile of W (or of
 // the padded iterate buffer for the cast).

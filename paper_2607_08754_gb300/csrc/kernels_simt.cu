@@ -1,9 +1,13 @@
 // Grouped SIMT (CUDA-core) GEMM for the three phases of a Polar Express step
 // (Sec. 3 "Computational cost": A = X X^T, M = a I + b A + c A^2, X <- M X on
-// the P x Q Gram side; M X is the step's a X + (b A + c A^2) X).  Used for the fp32 compute mode and, with 16-bit
-// storage, as a CUDA-core check of the tensor-core kernel.  64 x 64 output
-// tile per block, 256 threads, 4 x 4 per thread, K staged 16 at a time through
-// shared memory.
+// the P x Q Gram side; M X is the step's a X + (b A + c A^2) X).  Used for the
+// fp32 compute mode and, with 16-bit storage, as a CUDA-core check of the
+// tensor-core kernel.  32 x 32 output tile per block (small sets still fill
+// the GPU), 256 threads, 2 x 2 outputs per thread, K staged 32 at a time
+// through two shared-memory buffers: the next stage's global loads are in
+// flight while the current one is used.  Gram and Poly are symmetric: only
+// tiles on or above the diagonal are computed, and each writes its
+// transposed block as well.
 //
 // In fp32 mode the dot products are compensated (Ogita-Rump-Oishi "Dot2":
 // each product is split exactly with an FMA, each addition with Knuth's
@@ -21,7 +25,7 @@
 namespace slorr {
 namespace {
 
-constexpr int kBM = 64, kBN = 64, kBK = 16;
+constexpr int kT = kSimtTile, kBK = 32;
 
 template <typename T>
 __device__ __forceinline__ float ld_f(const T* p);
@@ -43,8 +47,8 @@ __device__ __forceinline__ void st_f<__nv_bfloat16>(__nv_bfloat16* p, float v) {
 
 template <typename T>
 __global__ void __launch_bounds__(256) simt_gemm_kernel(const GemmLaunch p) {
-    __shared__ float As[kBK][kBM + 4];
-    __shared__ float Bs[kBK][kBN + 4];
+    __shared__ float As[2][kBK][kT + 1];  // [buffer][k][i]
+    __shared__ float Bs[2][kBK][kT + 1];  // [buffer][k][j]
     const GemmItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
     const T* X = reinterpret_cast<const T*>(md.x[p.cur]);
@@ -64,35 +68,49 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const GemmLaunch p) {
     } else {                         // M X
         opA = Bm; sa_i = md.Ppad; sa_k = 1; opB = X; sb_j = sq; sb_k = sp; K = md.Ppad;
     }
-    const int m0 = it.tm * kBM, n0 = it.tn * kBN;
+    const int m0 = it.tm * kT, n0 = it.tn * kT;
     const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
     constexpr bool kDot2 = sizeof(T) == 4;
-    float acc[4][4] = {};
-    float cmp[4][4] = {};
+    // Each stage: 32 x 32 values of each operand, 4 per thread, consecutive
+    // threads along the operand's contiguous dimension.
+    float ra[4], rb[4];
+    auto gload = [&](int k0) {
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            const int e = int(threadIdx.x) + 256 * r;
+            const int ia = sa_k == 1 ? e / kBK : e % kT, ka = sa_k == 1 ? e % kBK : e / kT;
+            const int jb = sb_k == 1 ? e / kBK : e % kT, kb = sb_k == 1 ? e % kBK : e / kT;
+            ra[r] = ld_f<T>(opA + int64_t(m0 + ia) * sa_i + int64_t(k0 + ka) * sa_k);
+            rb[r] = ld_f<T>(opB + int64_t(n0 + jb) * sb_j + int64_t(k0 + kb) * sb_k);
+        }
+    };
+    auto sstore = [&](int buf) {
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            const int e = int(threadIdx.x) + 256 * r;
+            const int ia = sa_k == 1 ? e / kBK : e % kT, ka = sa_k == 1 ? e % kBK : e / kT;
+            const int jb = sb_k == 1 ? e / kBK : e % kT, kb = sb_k == 1 ? e % kBK : e / kT;
+            As[buf][ka][ia] = ra[r];
+            Bs[buf][kb][jb] = rb[r];
+        }
+    };
+    float acc[2][2] = {};
+    float cmp[2][2] = {};
+    gload(0);
+    sstore(0);
+    __syncthreads();
+    int buf = 0;
     for (int k0 = 0; k0 < K; k0 += kBK) {
-        // 64 x 16 of each operand: 1024 values, 4 per thread.
-        for (int e = threadIdx.x; e < kBM * kBK; e += 256) {
-            int i, k;
-            if (sa_k == 1) { i = e / kBK; k = e % kBK; } else { k = e / kBM; i = e % kBM; }
-            As[k][i] = ld_f<T>(opA + static_cast<int64_t>(m0 + i) * sa_i + static_cast<int64_t>(k0 + k) * sa_k);
-        }
-        for (int e = threadIdx.x; e < kBN * kBK; e += 256) {
-            int j, k;
-            if (sb_k == 1) { j = e / kBK; k = e % kBK; } else { k = e / kBN; j = e % kBN; }
-            Bs[k][j] = ld_f<T>(opB + static_cast<int64_t>(n0 + j) * sb_j + static_cast<int64_t>(k0 + k) * sb_k);
-        }
-        __syncthreads();
-#pragma unroll
+        const bool more = k0 + kBK < K;
+        if (more) gload(k0 + kBK);  // in flight while this stage is used
+#pragma unroll 8
         for (int k = 0; k < kBK; ++k) {
-            float a[4], b[4];
+            const float a[2] = {As[buf][k][ty * 2], As[buf][k][ty * 2 + 1]};
+            const float b[2] = {Bs[buf][k][tx * 2], Bs[buf][k][tx * 2 + 1]};
 #pragma unroll
-            for (int u = 0; u < 4; ++u) a[u] = As[k][ty * 4 + u];
+            for (int u = 0; u < 2; ++u)
 #pragma unroll
-            for (int v = 0; v < 4; ++v) b[v] = Bs[k][tx * 4 + v];
-#pragma unroll
-            for (int u = 0; u < 4; ++u)
-#pragma unroll
-                for (int v = 0; v < 4; ++v) {
+                for (int v = 0; v < 2; ++v) {
                     if constexpr (kDot2) {
                         const float pr = a[u] * b[v];
                         const float pe = fmaf(a[u], b[v], -pr);   // a b = pr + pe exactly
@@ -106,21 +124,28 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const GemmLaunch p) {
                     }
                 }
         }
+        if (more) sstore(buf ^ 1);  // the other buffer: last read before the previous barrier
         __syncthreads();
+        buf ^= 1;
     }
+    const bool mirror = p.phase != kUpdate && it.tn > it.tm;
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < 2; ++u) {
 #pragma unroll
-        for (int v = 0; v < 4; ++v) {
-            const int i = m0 + ty * 4 + u, j = n0 + tx * 4 + v;
+        for (int v = 0; v < 2; ++v) {
+            const int i = m0 + ty * 2 + u, j = n0 + tx * 2 + v;
             const float acc_uv = acc[u][v] + cmp[u][v];
             if (p.phase == kGram) {
-                st_f<T>(reinterpret_cast<T*>(md.a) + static_cast<int64_t>(i) * md.Ppad + j, acc_uv);
-            } else if (p.phase == kPoly) {      // M = c A^2 + b A + a I
+                T* a = reinterpret_cast<T*>(md.a);
+                st_f<T>(a + static_cast<int64_t>(i) * md.Ppad + j, acc_uv);
+                if (mirror) st_f<T>(a + static_cast<int64_t>(j) * md.Ppad + i, acc_uv);
+            } else if (p.phase == kPoly) {      // M = c A^2 + b A + a I (A is stored symmetric)
                 const int64_t idx = static_cast<int64_t>(i) * md.Ppad + j;
                 float val = fmaf(p.b, ld_f<T>(Am + idx), p.c * acc_uv);
                 if (i == j) val += p.a;
-                st_f<T>(reinterpret_cast<T*>(md.b) + idx, val);
+                T* m = reinterpret_cast<T*>(md.b);
+                st_f<T>(m + idx, val);
+                if (mirror) st_f<T>(m + static_cast<int64_t>(j) * md.Ppad + i, val);
             } else {                            // X' = M X
                 st_f<T>(reinterpret_cast<T*>(md.x[p.cur ^ 1]) + static_cast<int64_t>(i) * sp +
                             static_cast<int64_t>(j) * sq, acc_uv);
