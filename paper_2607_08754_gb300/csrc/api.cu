@@ -251,20 +251,34 @@ void build_plan(slorr_handle* h) {
         // iterate buffer in W's orientation
         g.rows = g.transposed ? g.Qpad : g.Ppad;
         g.ld = g.transposed ? g.Ppad : g.Qpad;
-        const int tr = (g.m + kMemRows - 1) / kMemRows, tc = (g.n + kMemCols - 1) / kMemCols;
+        // memory-pass tiles: kMemRows x kMemCols of the matrix (of the padded
+        // iterate buffer for the cast), or, when the rows are a multiple of 128
+        // elements (then ld == n), runs of that many consecutive elements
+        const bool flat = g.ld == g.n;
+        constexpr int64_t kTileElems = int64_t(kMemRows) * kMemCols;
         g.tile_base = tile_base;
-        g.tile_count = tr * tc;
-        int seq = 0;
-        for (int r = 0; r < tr; ++r)
-            for (int c = 0; c < tc; ++c)
-                h->w_items.push_back(MemItem{uint16_t(i), uint16_t(r), uint16_t(c), uint16_t(seq++)});
-        tile_base += g.tile_count;
         g.xtile_base = xtile_base;
-        int xseq = 0;
-        for (int r = 0; r < (g.rows + kMemRows - 1) / kMemRows; ++r)
-            for (int c = 0; c < (g.ld + kMemCols - 1) / kMemCols; ++c)
-                h->x_items.push_back(MemItem{uint16_t(i), uint16_t(r), uint16_t(c), uint16_t(xseq++)});
+        int seq = 0, xseq = 0;
+        if (flat) {
+            const int64_t wt = (int64_t(g.m) * g.n + kTileElems - 1) / kTileElems;
+            const int64_t xt = (int64_t(g.rows) * g.ld + kTileElems - 1) / kTileElems;
+            for (int64_t t = 0; t < wt && t <= 65535; ++t)
+                h->w_items.push_back(MemItem{uint16_t(i), kFlatTile, 0, uint16_t(seq++)});
+            for (int64_t t = 0; t < xt && t <= 65535; ++t)
+                h->x_items.push_back(MemItem{uint16_t(i), kFlatTile, 0, uint16_t(xseq++)});
+            if (wt > 65535 || xt > 65535) seq = xseq = 65536;  // rejected by slorr_create
+        } else {
+            const int tr = (g.m + kMemRows - 1) / kMemRows, tc = (g.n + kMemCols - 1) / kMemCols;
+            for (int r = 0; r < tr; ++r)
+                for (int c = 0; c < tc; ++c)
+                    h->w_items.push_back(MemItem{uint16_t(i), uint16_t(r), uint16_t(c), uint16_t(seq++)});
+            for (int r = 0; r < (g.rows + kMemRows - 1) / kMemRows; ++r)
+                for (int c = 0; c < (g.ld + kMemCols - 1) / kMemCols; ++c)
+                    h->x_items.push_back(MemItem{uint16_t(i), uint16_t(r), uint16_t(c), uint16_t(xseq++)});
+        }
+        g.tile_count = seq;
         g.xtile_count = xseq;
+        tile_base += seq;
         xtile_base += xseq;
         // tensor-core tiles: msz x nsz with msz <= 128 mt, nsz <= 256.  The Gram
         // and Poly outputs are symmetric: tiles lying strictly below the

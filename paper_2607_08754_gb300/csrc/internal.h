@@ -99,10 +99,14 @@ constexpr int kMemCols = 512;
 constexpr int kMemVec = 8;      // consecutive columns per thread
 struct MemItem {
     uint16_t mat;
-    uint16_t tile_r;   // tile row index (kMemRows rows)
+    uint16_t tile_r;   // tile row index (kMemRows rows), or kFlatTile
     uint16_t tile_c;   // tile column index (kMemCols cols)
     uint16_t seq;      // index of this tile within its matrix
 };
+// tile_r of a flat tile: elements [8192 seq, 8192 seq + 8192) of a matrix
+// whose rows are a multiple of 128 elements (ld == n), W and the iterate
+// buffer at the same offset.
+constexpr uint16_t kFlatTile = 0xffff;
 
 // Phases of one Polar Express step (the step's polynomial is applied as
 // X <- M X with M = a I + b A + c A^2, the same product as a X + (b A + c A^2) X).

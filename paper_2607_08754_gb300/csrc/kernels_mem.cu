@@ -18,7 +18,10 @@
 // every pass is elementwise.  A block handles one kMemRows x kMemCols tile:
 // each of its 256 threads owns 8 consecutive columns of 4 rows and issues all
 // its 128-bit loads before using them.  Rows whose length is not a multiple
-// of 8 take a scalar path.  Per-matrix coefficients (the cast scale, the
+// of 8 take a scalar path.  A matrix whose rows are a multiple of 128
+// elements has an iterate buffer without column padding (ld == n); its tiles
+// are runs of 8192 consecutive elements instead ("flat"), so rows that are
+// not a multiple of 512 long leave no thread idle.  Per-matrix coefficients (the cast scale, the
 // gradient's alpha and beta) are computed once by the finalize kernels, in
 // double precision, and read as floats by the streaming passes.  Cross-tile sums are
 // deterministic: each streaming block writes one partial per tile and exits;
@@ -83,22 +86,43 @@ __device__ __forceinline__ F8 load_w8(const TW* W, int m, int n, int r, int c, b
     return v;
 }
 
+// Eight W elements at a 16-byte aligned offset (the flat tiles).
+template <typename TW>
+__device__ __forceinline__ F8 load_w8_at(const TW* W, int64_t idx) {
+    F8 v;
+    if constexpr (sizeof(TW) == 4) {
+        v.lo = *reinterpret_cast<const float4*>(W + idx);
+        v.hi = *reinterpret_cast<const float4*>(W + idx + 4);
+    } else {
+        const uint4 u = *reinterpret_cast<const uint4*>(W + idx);
+        v.lo = make_float4(bf2f(u.x & 0xffff), bf2f(u.x >> 16), bf2f(u.y & 0xffff), bf2f(u.y >> 16));
+        v.hi = make_float4(bf2f(u.z & 0xffff), bf2f(u.z >> 16), bf2f(u.w & 0xffff), bf2f(u.w >> 16));
+    }
+    return v;
+}
+
 __device__ __forceinline__ uint32_t pack_bf2(float a, float b) {
     return uint32_t(__bfloat16_as_ushort(__float2bfloat16_rn(a))) |
            (uint32_t(__bfloat16_as_ushort(__float2bfloat16_rn(b))) << 16);
+}
+
+// Eight elements at a 16-byte aligned offset.
+template <typename TW>
+__device__ __forceinline__ void store_w8_at(TW* W, int64_t idx, const F8& v) {
+    if constexpr (sizeof(TW) == 4) {
+        *reinterpret_cast<float4*>(W + idx) = v.lo;
+        *reinterpret_cast<float4*>(W + idx + 4) = v.hi;
+    } else {
+        *reinterpret_cast<uint4*>(W + idx) = make_uint4(pack_bf2(v.lo.x, v.lo.y), pack_bf2(v.lo.z, v.lo.w),
+                                                        pack_bf2(v.hi.x, v.hi.y), pack_bf2(v.hi.z, v.hi.w));
+    }
 }
 
 template <typename TW>
 __device__ __forceinline__ void store_w8(TW* W, int n, int r, int c, bool vec, const F8& v) {
     const int64_t idx = int64_t(r) * n + c;
     if (vec) {
-        if constexpr (sizeof(TW) == 4) {
-            *reinterpret_cast<float4*>(W + idx) = v.lo;
-            *reinterpret_cast<float4*>(W + idx + 4) = v.hi;
-        } else {
-            *reinterpret_cast<uint4*>(W + idx) = make_uint4(pack_bf2(v.lo.x, v.lo.y), pack_bf2(v.lo.z, v.lo.w),
-                                                            pack_bf2(v.hi.x, v.hi.y), pack_bf2(v.hi.z, v.hi.w));
-        }
+        store_w8_at<TW>(W, idx, v);
     } else {
         const float t[8] = {v.lo.x, v.lo.y, v.lo.z, v.lo.w, v.hi.x, v.hi.y, v.hi.z, v.hi.w};
         for (int e = 0; e < 8 && c + e < n; ++e) {
@@ -223,15 +247,57 @@ __device__ __forceinline__ bool unscaled_cast_ok(int elem, float maxabs, double 
     return elem == kBF16 || maxabs == 0.f || (maxabs <= 32768.f && frob >= 1.0);
 }
 
-struct TileCoord {
-    int r0, c;  // first row of this thread, its first column
+// Where this thread's 8-element group of row pass k lies: in a 2-D tile
+// (row r0 + 4 k, columns c .. c + 7), or in a flat tile (elements e0 + 2048 k
+// .. + 7 of W and, at the same offset, of the iterate buffer).
+constexpr int kPassElems = kThreads * kMemVec;
+struct Span {
+    bool flat;
+    int r0, c;   // 2-D: the thread's first row, its first column
+    int64_t e0;  // flat: the thread's first element
 };
 
-__device__ __forceinline__ TileCoord tile_coord(const MemItem& it) {
-    TileCoord t;
+__device__ __forceinline__ Span span_of(const MemItem& it) {
+    Span t;
+    t.flat = it.tile_r == kFlatTile;
     t.r0 = it.tile_r * kMemRows + int(threadIdx.x) / kVecPerRow;
     t.c = it.tile_c * kMemCols + (int(threadIdx.x) % kVecPerRow) * kMemVec;
+    t.e0 = int64_t(it.seq) * (kMemRows * kMemCols) + int64_t(threadIdx.x) * kMemVec;
     return t;
+}
+
+// Pass k's group lies in W (all 8 elements in a flat tile, where n % 8 == 0;
+// in a 2-D tile the row does, and the first column: the scalar paths mask
+// the rest).
+__device__ __forceinline__ bool in_w(const Span& t, const MatDev& md, int k) {
+    if (t.flat) return t.e0 + int64_t(k) * kPassElems < int64_t(md.m) * md.n;
+    return t.r0 + k * kRowsPerPass < md.m && t.c < md.n;
+}
+
+// Pass k's group lies in the (padded) iterate buffer.
+__device__ __forceinline__ bool in_x(const Span& t, const MatDev& md, int k) {
+    if (t.flat) return t.e0 + int64_t(k) * kPassElems < int64_t(md.rows) * md.ld;
+    return t.r0 + k * kRowsPerPass < md.rows && t.c < md.ld;
+}
+
+__device__ __forceinline__ int64_t x_off(const Span& t, const MatDev& md, int k) {
+    if (t.flat) return t.e0 + int64_t(k) * kPassElems;
+    return int64_t(t.r0 + k * kRowsPerPass) * md.ld + t.c;
+}
+
+// W's (or a same-shaped gradient's) 8 elements of pass k, zero outside.
+template <typename TW>
+__device__ __forceinline__ F8 load_w(const TW* W, const MatDev& md, const Span& t, int k, bool vec) {
+    if (t.flat) return in_w(t, md, k) ? load_w8_at<TW>(W, t.e0 + int64_t(k) * kPassElems) : zero8();
+    return load_w8<TW>(W, md.m, md.n, t.r0 + k * kRowsPerPass, t.c, vec);
+}
+
+template <typename TW>
+__device__ __forceinline__ void store_w(TW* W, const MatDev& md, const Span& t, int k, bool vec, const F8& v) {
+    if (t.flat)
+        store_w8_at<TW>(W, t.e0 + int64_t(k) * kPassElems, v);
+    else
+        store_w8<TW>(W, md.n, t.r0 + k * kRowsPerPass, t.c, vec, v);
 }
 
 // ---- kernels ---------------------------------------------------------------------
@@ -246,10 +312,10 @@ __global__ void __launch_bounds__(kThreads, 6) sumsq_kernel(const MemLaunch p) {
     const MatDev md = p.mats[it.mat];
     const TW* W = reinterpret_cast<const TW*>(p.weights[it.mat]);
     const bool vec = (md.n & 7) == 0;
-    const TileCoord tc = tile_coord(it);
+    const Span tc = span_of(it);
     F8 w[kPasses];
 #pragma unroll
-    for (int k = 0; k < kPasses; ++k) w[k] = load_w8<TW>(W, md.m, md.n, tc.r0 + k * kRowsPerPass, tc.c, vec);
+    for (int k = 0; k < kPasses; ++k) w[k] = load_w<TW>(W, md, tc, k, vec);
     float acc = 0.f;
 #pragma unroll
     for (int k = 0; k < kPasses; ++k) acc = dot8(w[k], w[k], acc);
@@ -269,17 +335,13 @@ __global__ void __launch_bounds__(kThreads, 4) normcast_kernel(const MemLaunch p
     const TW* W = reinterpret_cast<const TW*>(p.weights[it.mat]);
     void* X = md.x[p.cur];
     const bool vec = (md.n & 7) == 0;
-    const TileCoord tc = tile_coord(it);
+    const Span tc = span_of(it);
     F8 w[kPasses];
 #pragma unroll
-    for (int k = 0; k < kPasses; ++k) w[k] = load_w8<TW>(W, md.m, md.n, tc.r0 + k * kRowsPerPass, tc.c, vec);
-    if (tc.c < md.ld) {
+    for (int k = 0; k < kPasses; ++k) w[k] = load_w<TW>(W, md, tc, k, vec);
 #pragma unroll
-        for (int k = 0; k < kPasses; ++k) {
-            const int r = tc.r0 + k * kRowsPerPass;
-            if (r < md.rows) store_x8<TX>(X, int64_t(r) * md.ld + tc.c, w[k]);
-        }
-    }
+    for (int k = 0; k < kPasses; ++k)
+        if (in_x(tc, md, k)) store_x8<TX>(X, x_off(tc, md, k), w[k]);
     float acc = 0.f, mx = 0.f;
 #pragma unroll
     for (int k = 0; k < kPasses; ++k) {
@@ -303,20 +365,19 @@ __global__ void __launch_bounds__(kThreads) cast_kernel(const MemLaunch p) {
     const TW* W = reinterpret_cast<const TW*>(p.weights[it.mat]);
     void* X = md.x[p.cur];
     const bool vec = (md.n & 7) == 0;
-    const TileCoord tc = tile_coord(it);
-    if (tc.c >= md.ld) return;
+    const Span tc = span_of(it);
+    if (!tc.flat && tc.c >= md.ld) return;
     F8 w[kPasses];
 #pragma unroll
-    for (int k = 0; k < kPasses; ++k) w[k] = load_w8<TW>(W, md.m, md.n, tc.r0 + k * kRowsPerPass, tc.c, vec);
+    for (int k = 0; k < kPasses; ++k) w[k] = load_w<TW>(W, md, tc, k, vec);
     const float scale = p.scalars[it.mat].scale;
 #pragma unroll
     for (int k = 0; k < kPasses; ++k) {
-        const int r = tc.r0 + k * kRowsPerPass;
-        if (r < md.rows) {
+        if (in_x(tc, md, k)) {
             F8 v;
             v.lo = make_float4(w[k].lo.x * scale, w[k].lo.y * scale, w[k].lo.z * scale, w[k].lo.w * scale);
             v.hi = make_float4(w[k].hi.x * scale, w[k].hi.y * scale, w[k].hi.z * scale, w[k].hi.w * scale);
-            store_x8<TX>(X, int64_t(r) * md.ld + tc.c, v);
+            store_x8<TX>(X, x_off(tc, md, k), v);
         }
     }
 }
@@ -333,18 +394,32 @@ __global__ void __launch_bounds__(kThreads, 4) dot_kernel(const MemLaunch p) {
     const MatDev md = p.mats[it.mat];
     const TW* W = reinterpret_cast<const TW*>(p.weights[it.mat]);
     const void* X = md.x[p.cur];
-    const bool vec = (md.n & 7) == 0;
-    const TileCoord tc = tile_coord(it);
-    F8 w[kPasses], x[kPasses];
-#pragma unroll
-    for (int k = 0; k < kPasses; ++k) {
-        const int r = tc.r0 + k * kRowsPerPass;
-        w[k] = load_w8<TW>(W, md.m, md.n, r, tc.c, vec);
-        x[k] = (r < md.m && tc.c < md.n) ? load_x8<TX>(X, int64_t(r) * md.ld + tc.c) : zero8();
-    }
     float acc = 0.f;
+    if (it.tile_r == kFlatTile) {
+        // flat tile: W and X_T at the same offsets
+        const int64_t e0 = int64_t(it.seq) * (kMemRows * kMemCols) + int64_t(threadIdx.x) * kMemVec;
+        const int64_t total = int64_t(md.m) * md.n;
+        F8 w[kPasses], x[kPasses];
 #pragma unroll
-    for (int k = 0; k < kPasses; ++k) acc = dot8(w[k], x[k], acc);
+        for (int k = 0; k < kPasses; ++k) {
+            const int64_t e = e0 + int64_t(k) * kPassElems;
+            w[k] = e < total ? load_w8_at<TW>(W, e) : zero8();
+            x[k] = e < total ? load_x8<TX>(X, e) : zero8();
+        }
+#pragma unroll
+        for (int k = 0; k < kPasses; ++k) acc = dot8(w[k], x[k], acc);
+    } else {
+        const bool vec = (md.n & 7) == 0;
+        const Span tc = span_of(it);
+        F8 w[kPasses], x[kPasses];
+#pragma unroll
+        for (int k = 0; k < kPasses; ++k) {
+            w[k] = load_w<TW>(W, md, tc, k, vec);
+            x[k] = in_w(tc, md, k) ? load_x8<TX>(X, x_off(tc, md, k)) : zero8();
+        }
+#pragma unroll
+        for (int k = 0; k < kPasses; ++k) acc = dot8(w[k], x[k], acc);
+    }
     const float part = block_sum(acc, red);
     if (threadIdx.x == 0) p.partials[p.tile_base[it.mat] + it.seq] = part;
 }
@@ -492,9 +567,9 @@ __global__ void __launch_bounds__(kThreads, 4) combine_kernel(const MemLaunch p)
     ptx::griddep_launch_dependents();
     const MemItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
-    const TileCoord tc = tile_coord(it);
+    const Span tc = span_of(it);
     const MatScalars& sc = p.scalars[it.mat];
-    if (sc.skip || tc.c >= md.n) return;  // non-finite: leave the gradient untouched
+    if (sc.skip || (!tc.flat && tc.c >= md.n)) return;  // non-finite: leave the gradient untouched
     const TW* W = reinterpret_cast<const TW*>(p.weights[it.mat]);
     TW* G = reinterpret_cast<TW*>(p.grads[it.mat]);
     const void* X = md.x[p.cur];
@@ -505,17 +580,15 @@ __global__ void __launch_bounds__(kThreads, 4) combine_kernel(const MemLaunch p)
         F8 w[2], x[2], g[2];
 #pragma unroll
         for (int q = 0; q < 2; ++q) {
-            const int r = tc.r0 + (h + q) * kRowsPerPass;
-            w[q] = load_w8<TW>(W, md.m, md.n, r, tc.c, vec);
-            if (p.out_mode == kOutAccumulate) g[q] = load_w8<TW>(G, md.m, md.n, r, tc.c, vec);
+            w[q] = load_w<TW>(W, md, tc, h + q, vec);
+            if (p.out_mode == kOutAccumulate) g[q] = load_w<TW>(G, md, tc, h + q, vec);
             else if (p.out_mode == kOutDescent) g[q] = w[q];  // G points at W: applied in place
             else g[q] = zero8();
-            x[q] = r < md.m ? load_x8<TX>(X, int64_t(r) * md.ld + tc.c) : zero8();
+            x[q] = in_w(tc, md, h + q) ? load_x8<TX>(X, x_off(tc, md, h + q)) : zero8();
         }
 #pragma unroll
         for (int q = 0; q < 2; ++q) {
-            const int r = tc.r0 + (h + q) * kRowsPerPass;
-            if (r >= md.m) continue;
+            if (!in_w(tc, md, h + q)) continue;
             F8 o;
             o.lo.x = g[q].lo.x + (fa * x[q].lo.x - fb * w[q].lo.x);
             o.lo.y = g[q].lo.y + (fa * x[q].lo.y - fb * w[q].lo.y);
@@ -525,7 +598,7 @@ __global__ void __launch_bounds__(kThreads, 4) combine_kernel(const MemLaunch p)
             o.hi.y = g[q].hi.y + (fa * x[q].hi.y - fb * w[q].hi.y);
             o.hi.z = g[q].hi.z + (fa * x[q].hi.z - fb * w[q].hi.z);
             o.hi.w = g[q].hi.w + (fa * x[q].hi.w - fb * w[q].hi.w);
-            store_w8<TW>(G, md.n, r, tc.c, vec, o);
+            store_w<TW>(G, md, tc, h + q, vec, o);
         }
     }
 }
