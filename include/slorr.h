@@ -121,6 +121,12 @@ typedef struct slorr_options {
                                        kernel are programmatic dependents of the kernel
                                        before them, so each one's launch and prologue
                                        overlap the previous one's tail (tuning)          */
+#define SLORR_FLAG_SEPARATE_NORM 1024 /* 16-bit iterates: take ||W||_F and write X_0 in two
+                                       passes over W.  By default one pass does both:
+                                       it stores W rounded to 16 bits and the first
+                                       Gram and Update epilogues apply 1/(||W||_F+eps)
+                                       (a matrix with max |w| > 2^15, or ||W||_F < 1 in
+                                       fp16, is re-cast with the scale); tuning          */
 #define SLORR_FLAG_NO_SPLIT_K  2048  /* never split the K range of a Gram tile across CTA
                                        pairs.  By default a set whose few Gram tiles have
                                        a long K (Q >> P, e.g. ResNet-18's 512 x 4608
@@ -135,12 +141,6 @@ typedef struct slorr_options {
                                        workspace).  Ignored while timing is on; a stream
                                        that is being captured gets the launches.  Saves
                                        the launch gaps of small sets                    */
-#define SLORR_FLAG_SEPARATE_NORM 1024 /* 16-bit iterates: take ||W||_F and write X_0 in two
-                                       passes over W.  By default one pass does both:
-                                       it stores W rounded to 16 bits and the first
-                                       Gram and Update epilogues apply 1/(||W||_F+eps)
-                                       (a matrix with max |w| > 2^15, or ||W||_F < 1 in
-                                       fp16, is re-cast with the scale); tuning          */
 
 /* Fill *opt with the defaults listed beside each field above (App. C.1: T = 6,
  * ell = 1e-3, degree 5; eps, lambda and grad_scale as in Listing 1 / Alg. 2). */
