@@ -131,6 +131,21 @@ def test_ragged_shapes(compute, variant):
     check(Ws, variant, compute, lam=0.7, grad_scale=2.0)
 
 
+@pytest.mark.parametrize("compute", ["fp32", "fp16", "bf16"])
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_flat_tiles_with_tails(compute, dtype):
+    """Rows a multiple of 128 elements: the memory passes take flat runs of
+    8192 elements.  The shapes end in partial runs (m n not a multiple of
+    8192), include m > n (X^T stored, padding rows zero-filled by the flat
+    cast), a matrix smaller than one run, and (fp32 storage) a gradient
+    accumulated onto an existing one: in bf16 storage the existing values'
+    own rounding would dominate the comparison."""
+    shapes = [(130, 768), (1000, 384), (77, 128), (200, 1280), (3, 256), (640, 1024)]
+    Ws = [workloads.random_matrix(s, seed=40 + i, std=0.05) for i, s in enumerate(shapes)]
+    G0 = [workloads.random_matrix(s, seed=60 + i, std=0.01) for i, s in enumerate(shapes)]
+    check(Ws, "hoyer", compute, lam=0.3, dtype=dtype, grads0=G0 if dtype == "f32" else None)
+
+
 @pytest.mark.parametrize("compute", ["fp16", "bf16"])
 @pytest.mark.parametrize("variant", ["hoyer", "nuclear"])
 def test_resnet18_weight_set(compute, variant):
