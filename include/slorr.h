@@ -141,6 +141,12 @@ typedef struct slorr_options {
                                        workspace).  Ignored while timing is on; a stream
                                        that is being captured gets the launches.  Saves
                                        the launch gaps of small sets                    */
+#define SLORR_FLAG_WIDE_UPDATE 8192  /* CTA-pair Update with 256 x 512 tiles: one 128 x 512
+                                       accumulator per SM (all 512 TMEM columns, so no
+                                       epilogue overlap), two N = 256 UMMAs per K slice
+                                       and 4 stages of 48 KB; each SM copies 48 KB per
+                                       K block for twice the FLOPs of the 32 KB of a
+                                       256 x 256 tile (tuning)                          */
 
 /* Fill *opt with the defaults listed beside each field above (App. C.1: T = 6,
  * ell = 1e-3, degree 5; eps, lambda and grad_scale as in Listing 1 / Alg. 2). */

@@ -105,6 +105,11 @@ bool tc_pair(const slorr_handle* h) {
     return (h->opt.flags & (SLORR_FLAG_TC_SINGLE_CTA | SLORR_FLAG_TC_BK32 | SLORR_FLAG_TC_M128)) == 0;
 }
 
+// CTA-pair Update with 256 x 512 tiles (the 4-CTA kernel keeps 256 x 256).
+bool wide_update(const slorr_handle* h) {
+    return tc_pair(h) && (h->opt.flags & SLORR_FLAG_WIDE_UPDATE) && !(h->opt.flags & SLORR_FLAG_TC_QUAD);
+}
+
 // Programmatic dependent launch of the memory passes and the pair kernel.
 bool use_pdl(const slorr_handle* h) { return (h->opt.flags & SLORR_FLAG_NO_PDL) == 0; }
 
@@ -280,17 +285,18 @@ void build_plan(slorr_handle* h) {
         g.xtile_count = xseq;
         tile_base += seq;
         xtile_base += xseq;
-        // tensor-core tiles: msz x nsz with msz <= 128 mt, nsz <= 256.  The Gram
-        // and Poly outputs are symmetric: tiles lying strictly below the
-        // diagonal (in 128 x 128 blocks) are skipped; the kernel mirrors the
-        // blocks they need.
+        // tensor-core tiles: msz x nsz with msz <= 128 mt, nsz <= 256 (512 for
+        // the wide CTA-pair Update).  The Gram and Poly outputs are symmetric:
+        // tiles lying strictly below the diagonal (in 128 x 128 blocks) are
+        // skipped; the kernel mirrors the blocks they need.
         for (int ph = 0; ph < 3; ++ph) {
             const int mt = tc_mt(h, ph);
             const int N = ph == kUpdate ? g.Qpad : g.Ppad;
+            const int bn = ph == kUpdate && wide_update(h) ? 512 : 256;
             for (int tm = 0; tm * 128 * mt < g.Ppad; ++tm) {
                 const int msz = std::min(128 * mt, g.Ppad - tm * 128 * mt);
-                for (int tn = 0; tn * 256 < N; ++tn) {
-                    const int nsz = std::min(256, N - tn * 256);
+                for (int tn = 0; tn * bn < N; ++tn) {
+                    const int nsz = std::min(bn, N - tn * bn);
                     if (ph != kUpdate && (2 * tn + nsz / 128 - 1) < tm * mt) continue;
                     h->tc_items[ph].push_back(
                         GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), uint16_t(nsz), uint16_t(msz), 0});
@@ -732,6 +738,7 @@ slorr_status launch_all(slorr_handle* h, uint8_t* ws, float* loss, float* per, i
     const bool pair = tc_pair(h);
     const bool quad = pair && (h->opt.flags & SLORR_FLAG_TC_QUAD) != 0;
     g.pair_slots = (h->opt.flags & SLORR_FLAG_PAIR_ONE_SLOT) ? 1 : 2;
+    g.wide_update = wide_update(h) ? 1 : 0;
     g.pdl = (use_pdl(h) && pair && !quad) ? 1 : 0;
     g.scalars = reinterpret_cast<const MatScalars*>(ws + h->off_scalars);
     g.split_part = reinterpret_cast<float*>(ws + h->off_split_part);

@@ -127,6 +127,7 @@ struct GemmLaunch {
     int32_t mt;                // 128-row M tiles per CTA tile: 1 or 2 (256 x 256 tiles)
     int32_t test_stall;        // 1: the MMA thread first waits on a barrier nothing arrives on
     int32_t pair_slots;        // CTA-pair kernel: accumulators per CTA (1 or 2)
+    int32_t wide_update;       // CTA-pair Update tiles are 256 x 512 (one 512-column accumulator)
     int32_t pdl;               // launch with programmatic dependent launch
     // x0_scaled = 1 (first step after the fused norm pass, which stores X_0
     // as W rounded to 16 bits): the Gram epilogue multiplies by

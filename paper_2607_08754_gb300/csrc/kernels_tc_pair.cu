@@ -45,21 +45,26 @@ namespace {
 
 using namespace tc;
 
-template <int STAGES_, int SLOTS_, int EPIW_>
+template <int STAGES_, int SLOTS_, int EPIW_, int BN_ = kBNMax>
 struct PairCfg {
     static constexpr int BK = 64;
     static constexpr int STAGES = STAGES_;
     static constexpr int kSlots = SLOTS_;                 // accumulators per CTA in TMEM
+    static constexpr int kBN = BN_;                       // tile columns: 256, or 512 (two UMMAs)
+    static_assert(BN_ == 256 || BN_ == 512, "tile width");
+    static constexpr int kSubs = BN_ / 256;               // N <= 256 UMMAs per K slice
     static constexpr int kBoxBytes = 64 * BK * 2;         // one 64 x 64 box
     static constexpr int kABytes = kBM * BK * 2;          // this CTA's 128 rows of A
-    static constexpr int kBBytes = (kBNMax / 2) * BK * 2; // this CTA's half of B (<= 128 rows)
+    static constexpr int kSubBBytes = 128 * BK * 2;       // this CTA's half of one UMMA's B (<= 128 rows)
+    static constexpr int kBBytes = kSubs * kSubBBytes;
+    static constexpr int kAccCols = BN_;                  // fp32 TMEM columns of one accumulator
     static constexpr int kStageBytes = kABytes + kBBytes;
     static constexpr int kEpiWarps = EPIW_;               // 4, or 8: two per TMEM lane quadrant
     static_assert(EPIW_ == 4 || EPIW_ == 8, "epilogue warps");
     static constexpr int kThreads = 64 + 32 * kEpiWarps;
     static constexpr uint32_t kKLayout = 2u;              // SWIZZLE_128B
     static constexpr uint32_t kKSbo = 8 * BK * 2;
-    static constexpr uint32_t kTmemCols = uint32_t(kSlots) * kAccCols;
+    static constexpr uint32_t kTmemCols = uint32_t(kSlots) * uint32_t(kAccCols);
     static constexpr size_t kBarrierBytes = 512;
     static constexpr size_t kSmemBytes = size_t(STAGES) * kStageBytes + 1024 /*align*/ + kBarrierBytes;
     static_assert((2 * STAGES + 2 * kSlots + 1) * 8 + 16 <= kBarrierBytes, "barrier area");
@@ -76,6 +81,8 @@ struct PairCfg {
 using PairCfg1 = PairCfg<SLORR_PAIR_STAGES, 1, 4>;   // one accumulator per CTA: no overlap
 using PairCfg2 = PairCfg<SLORR_PAIR_STAGES, 2, 4>;
 using PairCfg2Wide = PairCfg<SLORR_PAIR_STAGES, 2, 8>;
+// 256 x 512 Update tiles: one 128 x 512 accumulator per CTA, 4 stages of 48 KB.
+using PairCfgN512 = PairCfg<4, 1, 8, 512>;
 
 struct PairSmem {
     uint8_t* stages;
@@ -123,7 +130,6 @@ __device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, 
         const PhaseInfo pi = phase_info<C>(p, it);
         const bool load_a = rank * kBM < it.msz;
         const bool load_b = !shared_operand(p, it);
-        const int bhalf = it.nsz / 2;  // 64 or 128 rows of B per CTA
         int kb_begin, kb_end;
         split_range(it, pi.nkb, &kb_begin, &kb_end);
         for (int kb = kb_begin; kb < kb_end; ++kb) {
@@ -141,9 +147,15 @@ __device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, 
                     const int mn = it.tm * (2 * kBM) + rank * kBM + b * 64;
                     ptx::tma_load_2d_pair(sa + b * C::kBoxBytes, pi.mapA, bar, pi.a_mn ? mn : k, pi.a_mn ? k : mn);
                 }
-            for (int j = 0; load_b && j < bhalf / 64; ++j) {
-                const int mn = it.tn * kBNMax + rank * bhalf + j * 64;
-                ptx::tma_load_2d_pair(sb + j * C::kBoxBytes, pi.mapB, bar, pi.b_mn ? mn : k, pi.b_mn ? k : mn);
+            // B columns of UMMA u (tile columns [256 u, 256 u + nu)): this
+            // CTA's half, nu / 2 = 64 or 128 rows, in its own 128-row region
+            for (int u = 0; load_b && u * 256 < it.nsz; ++u) {
+                const int bhalf = min(256, it.nsz - u * 256) / 2;
+                for (int j = 0; j < bhalf / 64; ++j) {
+                    const int mn = it.tn * C::kBN + u * 256 + rank * bhalf + j * 64;
+                    ptx::tma_load_2d_pair(sb + u * C::kSubBBytes + j * C::kBoxBytes, pi.mapB, bar, pi.b_mn ? mn : k,
+                                          pi.b_mn ? k : mn);
+                }
             }
             if (++stage == C::STAGES) {
                 stage = 0;
@@ -210,7 +222,9 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
     for (int idx = pair; idx < p.num_items && ok; idx += npairs, ++local) {
         const GemmItem it = p.items[idx];
         const PhaseInfo pi = phase_info<C>(p, it);
-        const uint32_t idesc = ptx::idesc_f16(2 * kBM, it.nsz, BF16, pi.a_mn, pi.b_mn);
+        const int n0 = min(256, int(it.nsz));  // columns of UMMA 0; UMMA 1 (512-wide tiles) takes the rest
+        const uint32_t idesc0 = ptx::idesc_f16(2 * kBM, n0, BF16, pi.a_mn, pi.b_mn);
+        const uint32_t idesc1 = it.nsz > 256 ? ptx::idesc_f16(2 * kBM, it.nsz - 256, BF16, pi.a_mn, pi.b_mn) : 0u;
         const int slot = local % C::kSlots;
         const uint32_t tphase = uint32_t(local / C::kSlots) & 1u;
         if (!ptx::mbar_wait<true>(&s.tempty[slot], tphase ^ 1u, s.abort, p.timeout_ns)) {
@@ -219,7 +233,7 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
             break;
         }
         ptx::tc_fence_after();
-        const uint32_t d_tmem = tmem_base + uint32_t(slot * kAccCols);
+        const uint32_t d_tmem = tmem_base + uint32_t(slot * C::kAccCols);
         int kb_begin, kb_end;
         split_range(it, pi.nkb, &kb_begin, &kb_end);
         for (int kb = kb_begin; kb < kb_end; ++kb) {
@@ -239,9 +253,14 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
             const uint32_t a0 = ptx::smem_u32(s.stages + size_t(stage) * C::kStageBytes);
             const uint32_t b0 = shared_operand(p, it) ? a0 : a0 + C::kABytes;
 #pragma unroll
-            for (int kk = 0; kk < C::BK / 16; ++kk)
-                ptx::umma_f16_pair(d_tmem, operand_desc<C>(a0, kk, pi.a_mn), operand_desc<C>(b0, kk, pi.b_mn), idesc,
-                                   (kb != kb_begin || kk != 0) ? 1u : 0u);
+            for (int kk = 0; kk < C::BK / 16; ++kk) {
+                const uint64_t adesc = operand_desc<C>(a0, kk, pi.a_mn);
+                const uint32_t acc = (kb != kb_begin || kk != 0) ? 1u : 0u;
+                ptx::umma_f16_pair(d_tmem, adesc, operand_desc<C>(b0, kk, pi.b_mn), idesc0, acc);
+                if (C::kSubs > 1 && it.nsz > 256)
+                    ptx::umma_f16_pair(d_tmem + 256u, adesc, operand_desc<C>(b0 + C::kSubBBytes, kk, pi.b_mn), idesc1,
+                                       acc);
+            }
             issued_any = true;
             ptx::umma_commit_pair_mc(&s.empty[stage], 0x3);
             if (++stage == C::STAGES) {
@@ -288,11 +307,11 @@ __device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t t
         ptx::tc_fence_after();
         if (rank * kBM < it.msz) {
             const int row0 = it.tm * (2 * kBM) + rank * kBM;
-            const uint32_t t_row = tmem_base + (uint32_t(quad * 32) << 16) + uint32_t(slot * kAccCols);
+            const uint32_t t_row = tmem_base + (uint32_t(quad * 32) << 16) + uint32_t(slot * C::kAccCols);
             const int per = it.nsz / 32 / ngroups;  // 32-column chunks per warp
             const int parts = it.ksplit >> 8;
             if (parts <= 1) {
-                store_rows<BF16, 2>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per);
+                store_rows<BF16, 2, C::kBN>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per);
             } else if constexpr (C::kEpiWarps == 4) {  // split K: Gram only, one warp per lane quadrant
                 if (split_partial_is_last(p, it, rank, quad, lane, t_row, 0, per))
                     store_rows<BF16, 2>(p, it, md, row0, t_row, quad, lane, 0, per,
@@ -410,6 +429,9 @@ cudaError_t launch_pair_cfg(const GemmLaunch& p, int num_sms, cudaStream_t st) {
 cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t st) {
     if (p.num_items == 0) return cudaSuccess;
     const bool bf = elem == kBF16;
+    if (p.wide_update && p.phase == kUpdate)
+        return bf ? launch_pair_cfg<true, PairCfgN512>(p, num_sms, st)
+                  : launch_pair_cfg<false, PairCfgN512>(p, num_sms, st);
     if (p.pair_slots == 2 && p.phase == kPoly)
         return bf ? launch_pair_cfg<true, PairCfg2Wide>(p, num_sms, st)
                   : launch_pair_cfg<false, PairCfg2Wide>(p, num_sms, st);

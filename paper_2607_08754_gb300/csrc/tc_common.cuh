@@ -143,7 +143,7 @@ __device__ __forceinline__ bool split_partial_is_last(const GemmLaunch& p, const
 
 // Epilogue of one 128-row block of a finished tile: this warp's 32 TMEM lanes
 // (rows row0 + 32 quad + [0, 32)) and the tile's 32-column chunks
-// [ch_begin, ch_end) (chunk c: columns tn * 256 + 32 c, TMEM columns t_row + 32 c).
+// [ch_begin, ch_end) (chunk c: columns tn * BN + 32 c, TMEM columns t_row + 32 c).
 //   Update: X' rows, stored in W's orientation (transposed iterates take one
 //           coalesced 64-byte segment per column);
 //   Gram / Poly: c * acc (+ b A + a I for Poly) into the Ppad x Ppad output,
@@ -154,7 +154,7 @@ __device__ __forceinline__ bool split_partial_is_last(const GemmLaunch& p, const
 // With split K (Gram), the accumulator is replaced by the sum, in part
 // order, of the `parts` fp32 partials at split_tile (row row_t of the tile;
 // this warp's own part among them).
-template <bool BF16, int MT>
+template <bool BF16, int MT, int BN = kBNMax>
 __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& it, const MatDev& md, int row0,
                                            uint32_t t_row, int quad, int lane, int ch_begin, int ch_end,
                                            const float* split_tile = nullptr, int parts = 1, int row_t = 0) {
@@ -168,7 +168,7 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
             uint32_t r[32];
             ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
             ptx::tmem_ld_wait();
-            const int col0 = it.tn * kBNMax + ch * 32;
+            const int col0 = it.tn * BN + ch * 32;
             if (md.transposed) {
                 // X^T[q][p]: for each column the warp's 32 rows are contiguous
                 uint16_t* dst = out + int64_t(col0) * ld + row;

@@ -37,6 +37,7 @@ FLAG_NO_PDL = 512
 FLAG_SEPARATE_NORM = 1024
 FLAG_NO_SPLIT_K = 2048
 FLAG_GRAPH = 4096
+FLAG_WIDE_UPDATE = 8192
 
 
 class SlorrError(RuntimeError):

@@ -6,8 +6,9 @@ Shapes are chosen to reach every tile case of the pair kernel: a last row tile
 with only 128 rows (the odd CTA's half idle), last column tiles of 128 columns
 (64 B rows per CTA), K-major and MN-major operands (m <= n and m > n), a
 matrix smaller than one tile, and more tiles than pairs.  Test ids carry
-"one_slot" (one accumulator per SM) or "two_slot" (two, the overlapped
-epilogue).
+"one_slot" (one accumulator per SM), "two_slot" (two, the overlapped
+epilogue) or "wide" (256 x 512 Update tiles, two UMMAs per K slice; the
+Update column tiles of these shapes are 128, 256, 384 and 512 wide).
 
 Tolerances are those of the tensor-core-vs-CUDA-core test: 4 ulp of the
 operand type per step (at most 6 steps' worth), and the oracle parity bounds
@@ -23,7 +24,7 @@ torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
 EPS = 1e-7
-MODES = {"one_slot": 128, "two_slot": 0}   # SLORR_FLAG_PAIR_ONE_SLOT, default
+MODES = {"one_slot": 128, "two_slot": 0, "wide": 8192}   # PAIR_ONE_SLOT, default, WIDE_UPDATE
 SHAPES = [(256, 768), (768, 256), (320, 1280), (384, 384), (640, 1000), (64, 64), (130, 700), (1000, 130)]
 
 
@@ -83,7 +84,7 @@ def test_pair_forward_backward_matches_oracle(mode, variant):
         assert rel(g[i].double().cpu().numpy(), ref_inc[i]) <= 2e-2, (i, shapes[i])
 
 
-@pytest.mark.parametrize("mode", ["two_slot"])
+@pytest.mark.parametrize("mode", ["two_slot", "wide"])
 def test_pair_vit_l16_layers_match_single_cta_kernel(mode):
     """Paper-sized matrices (one ViT-L/16 block): the pair kernel and the one-CTA
     kernels give the same iterates up to 16-bit rounding."""

@@ -265,3 +265,30 @@ def test_split_k_plan(lib):
         slorr.slorr_gemm_items(slorr.Regularizer(rn, compute="fp32", flags=slorr.FLAG_NO_SPLIT_K).handle, 0)
     with pytest.raises(slorr.SlorrError):
         slorr.slorr_gemm_items(split.handle, 3)
+
+
+def test_wide_update_plan(lib):
+    """SLORR_FLAG_WIDE_UPDATE plans the CTA-pair Update in 256 x 512 tiles:
+    ceil(Qpad / 512) column tiles per 256-row band instead of Qpad / 256,
+    the last one 128, 256, 384 or 512 wide.  Gram and Poly keep their tiles,
+    the executed FLOPs do not change, and the one-CTA and 4-CTA kernels
+    ignore the flag."""
+    import workloads
+    vl = workloads.shapes("vit_l16")
+    base = slorr.Regularizer(vl)
+    wide = slorr.Regularizer(vl, flags=slorr.FLAG_WIDE_UPDATE)
+    # per block: P = 1024 (4 bands) and Q = 3072, 1024, 4096, 4096
+    assert slorr.slorr_gemm_items(base.handle, 2) == 24 * 4 * (12 + 4 + 16 + 16)
+    assert slorr.slorr_gemm_items(wide.handle, 2) == 24 * 4 * (6 + 2 + 8 + 8)
+    for ph in (0, 1):
+        assert slorr.slorr_gemm_items(wide.handle, ph) == slorr.slorr_gemm_items(base.handle, ph)
+    assert slorr.slorr_executed_flops(wide.handle) == slorr.slorr_executed_flops(base.handle)
+    # Qpad = 128, 384, 640, 768, 1024: 1, 1, 2, 2, 2 column tiles per band
+    shapes = [(64, 64), (256, 384), (256, 640), (130, 700), (1000, 130)]
+    w = slorr.Regularizer(shapes, flags=slorr.FLAG_WIDE_UPDATE)
+    assert slorr.slorr_gemm_items(w.handle, 2) == 1 + 1 + 2 + 2 + 2
+    assert slorr.slorr_executed_flops(w.handle) == slorr.slorr_executed_flops(slorr.Regularizer(shapes).handle)
+    for other in (slorr.FLAG_TC_SINGLE_CTA, slorr.FLAG_TC_QUAD):
+        a = slorr.Regularizer(vl, flags=other | slorr.FLAG_WIDE_UPDATE)
+        b = slorr.Regularizer(vl, flags=other)
+        assert slorr.slorr_gemm_items(a.handle, 2) == slorr.slorr_gemm_items(b.handle, 2)
