@@ -66,7 +66,8 @@ struct PairCfg {
     static constexpr uint32_t kKSbo = 8 * BK * 2;
     static constexpr uint32_t kTmemCols = uint32_t(kSlots) * uint32_t(kAccCols);
     static constexpr size_t kBarrierBytes = 512;
-    static constexpr size_t kSmemBytes = size_t(STAGES) * kStageBytes + 1024 /*align*/ + kBarrierBytes;
+    static constexpr size_t kEpiBytes = size_t(kEpiWarps) * kStageWarpBytes;  // epilogue staging
+    static constexpr size_t kSmemBytes = size_t(STAGES) * kStageBytes + 1024 /*align*/ + kBarrierBytes + kEpiBytes;
     static_assert((2 * STAGES + 2 * kSlots + 1) * 8 + 16 <= kBarrierBytes, "barrier area");
     static_assert(kSmemBytes <= 232448, "shared memory budget");
     static_assert(kTmemCols <= 512, "tensor memory budget");
@@ -86,6 +87,7 @@ using PairCfgN512 = PairCfg<4, 1, 8, 512>;
 
 struct PairSmem {
     uint8_t* stages;
+    uint8_t* epi;      // kStageWarpBytes per epilogue warp
     uint64_t* full;    // even CTA: both CTAs' copies of the stage landed
     uint64_t* empty;   // stage consumed by the pair UMMAs (multicast commit)
     uint64_t* tfull;   // accumulator slot complete (multicast commit)
@@ -290,6 +292,7 @@ __device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t t
     const int quad = warp & 3;             // TMEM lanes [32 quad, 32 quad + 32) (hardware rule)
     const int ngroups = C::kEpiWarps / 4;  // warps per lane quadrant, splitting the columns
     const int group = (warp - 2) / 4;
+    uint8_t* sbuf = s.epi + (warp - 2) * kStageWarpBytes;
     int local = 0;
     const uint32_t even_tempty = ptx::mapa(ptx::smem_u32(s.tempty), 0);
     for (int idx = pair; idx < p.num_items; idx += npairs, ++local) {
@@ -311,8 +314,11 @@ __device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t t
             const int per = it.nsz / 32 / ngroups;  // 32-column chunks per warp
             const int parts = it.ksplit >> 8;
             if (parts <= 1) {
-                store_rows<BF16, 2, C::kBN>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per);
+                store_rows<BF16, 2, C::kBN, true>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per,
+                                                  nullptr, 1, 0, sbuf);
             } else if constexpr (C::kEpiWarps == 4) {  // split K: Gram only, one warp per lane quadrant
+                // direct stores: the last part's sum is a serial step, which
+                // the staging round trip lengthens (small sets, ResNet-18 Gram +7%)
                 if (split_partial_is_last(p, it, rank, quad, lane, t_row, 0, per))
                     store_rows<BF16, 2>(p, it, md, row0, t_row, quad, lane, 0, per,
                                         p.split_part + size_t(it.sid) * 65536, parts, rank * kBM + quad * 32 + lane);
@@ -335,6 +341,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(C::kThreads, 1)
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     PairSmem s;
     s.stages = base;
+    s.epi = base + size_t(C::STAGES) * C::kStageBytes + C::kBarrierBytes;
     s.full = reinterpret_cast<uint64_t*>(base + size_t(C::STAGES) * C::kStageBytes);
     s.empty = s.full + C::STAGES;
     s.tfull = s.empty + C::STAGES;

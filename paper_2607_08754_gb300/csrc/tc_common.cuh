@@ -141,6 +141,72 @@ __device__ __forceinline__ bool split_partial_is_last(const GemmLaunch& p, const
     return last != 0;
 }
 
+// Staged epilogue stores (CTA-pair kernel).  A TMEM load gives each lane one
+// row of a 32 x 32 chunk, so a lane's own 16-byte stores would touch 32 rows
+// per instruction, half a 32-byte sector each.  Instead the warp stages the
+// chunk in its own shared-memory buffer (rows kStageRow bytes apart: the
+// 16-byte row writes of any 8 lanes fall in 8 different bank groups) and
+// stores it as 8 rows x 64 bytes per instruction, or transposed (column c of
+// the chunk as a row of the output) as 8 columns x 64 bytes.
+constexpr int kStageRow = 80;
+constexpr int kStageWarpBytes = 32 * kStageRow;
+
+__device__ __forceinline__ void stage_chunk(uint8_t* buf, int lane, const uint4 (&o)[4]) {
+    uint4* dst = reinterpret_cast<uint4*>(buf + lane * kStageRow);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) dst[q] = o[q];
+    __syncwarp();
+}
+
+// out[(r0 + r) * ld + c0 + c] = chunk[r][c]
+__device__ __forceinline__ void put_rows(const uint8_t* buf, int lane, uint16_t* out, int64_t ld, int r0, int c0) {
+    const int seg = lane & 3;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int r = i * 8 + (lane >> 2);
+        const uint4 v = *reinterpret_cast<const uint4*>(buf + r * kStageRow + seg * 16);
+        *reinterpret_cast<uint4*>(out + int64_t(r0 + r) * ld + c0 + seg * 8) = v;
+    }
+}
+
+// out[(c0 + c) * ld + r0 + r] = chunk[r][c]
+__device__ __forceinline__ void put_cols(const uint8_t* buf, int lane, uint16_t* out, int64_t ld, int r0, int c0) {
+    const int seg = lane & 3;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int c = i * 8 + (lane >> 2);
+        const uint8_t* src = buf + (seg * 8) * kStageRow + c * 2;
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const uint32_t lo = *reinterpret_cast<const uint16_t*>(src + (2 * e) * kStageRow);
+            const uint32_t hi = *reinterpret_cast<const uint16_t*>(src + (2 * e + 1) * kStageRow);
+            w[e] = lo | (hi << 16);
+        }
+        *reinterpret_cast<uint4*>(out + int64_t(c0 + c) * ld + r0 + seg * 8) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
+// The 32 x 32 chunk at src[(r0 + r) * ld + c0 + c] in the put_rows order:
+// v[i] holds row 8 i + lane / 4, columns 8 (lane % 4) .. + 7.
+__device__ __forceinline__ void get_rows(const uint16_t* src, int64_t ld, int r0, int c0, int lane, uint4 (&v)[4]) {
+    const int seg = lane & 3;
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+        v[i] = *reinterpret_cast<const uint4*>(src + int64_t(r0 + i * 8 + (lane >> 2)) * ld + c0 + seg * 8);
+}
+
+// A chunk from get_rows, through the staging buffer, as this lane's row.
+__device__ __forceinline__ void own_row(uint8_t* buf, int lane, const uint4 (&v)[4], uint4 (&row)[4]) {
+    const int seg = lane & 3;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) *reinterpret_cast<uint4*>(buf + (i * 8 + (lane >> 2)) * kStageRow + seg * 16) = v[i];
+    __syncwarp();
+#pragma unroll
+    for (int q = 0; q < 4; ++q) row[q] = *reinterpret_cast<const uint4*>(buf + lane * kStageRow + q * 16);
+    __syncwarp();
+}
+
 // Epilogue of one 128-row block of a finished tile: this warp's 32 TMEM lanes
 // (rows row0 + 32 quad + [0, 32)) and the tile's 32-column chunks
 // [ch_begin, ch_end) (chunk c: columns tn * BN + 32 c, TMEM columns t_row + 32 c).
@@ -153,12 +219,15 @@ __device__ __forceinline__ bool split_partial_is_last(const GemmLaunch& p, const
 // is W itself: the Gram scales acc by x0_scale^2 and the Update by x0_scale.
 // With split K (Gram), the accumulator is replaced by the sum, in part
 // order, of the `parts` fp32 partials at split_tile (row row_t of the tile;
-// this warp's own part among them).
-template <bool BF16, int MT, int BN = kBNMax>
+// this warp's own part among them).  STAGED: the stores go through the
+// warp's staging buffer sbuf (kStageWarpBytes of shared memory).
+template <bool BF16, int MT, int BN = kBNMax, bool STAGED = false>
 __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& it, const MatDev& md, int row0,
                                            uint32_t t_row, int quad, int lane, int ch_begin, int ch_end,
-                                           const float* split_tile = nullptr, int parts = 1, int row_t = 0) {
-    const int row = row0 + quad * 32 + lane;
+                                           const float* split_tile = nullptr, int parts = 1, int row_t = 0,
+                                           uint8_t* sbuf = nullptr) {
+    const int row_w = row0 + quad * 32;  // the warp's first row
+    const int row = row_w + lane;
     const int nch = ch_end;
     const float xs = p.x0_scaled ? p.scalars[it.mat].x0_scale : 1.f;
     if (p.phase == kUpdate) {
@@ -169,7 +238,20 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
             ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
             ptx::tmem_ld_wait();
             const int col0 = it.tn * BN + ch * 32;
-            if (md.transposed) {
+            if constexpr (STAGED) {
+                uint4 o[4];
+                uint32_t* ow = reinterpret_cast<uint32_t*>(o);
+#pragma unroll
+                for (int j = 0; j < 16; ++j)
+                    ow[j] = pack2<BF16>(xs * __uint_as_float(r[2 * j]), xs * __uint_as_float(r[2 * j + 1]));
+                stage_chunk(sbuf, lane, o);
+                // transposed iterates: X^T[q][p], the chunk's columns are rows of the buffer
+                if (md.transposed)
+                    put_cols(sbuf, lane, out, ld, row_w, col0);
+                else
+                    put_rows(sbuf, lane, out, ld, row_w, col0);
+                __syncwarp();
+            } else if (md.transposed) {
                 // X^T[q][p]: for each column the warp's 32 rows are contiguous
                 uint16_t* dst = out + int64_t(col0) * ld + row;
 #pragma unroll
@@ -192,25 +274,35 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
         const bool poly = p.phase == kPoly;
         const float cacc = poly ? p.c : xs * xs;
         // Poly reads b A at the output position: loads for the next chunk are
-        // issued before the current chunk is processed.
+        // issued before the current chunk is processed (staged: coalesced
+        // loads, turned into this lane's row through the staging buffer).
         uint4 e_next[4];
         if (poly) {
-            const uint4* src =
-                reinterpret_cast<const uint4*>(amat + int64_t(row) * ld + it.tn * kBNMax + ch_begin * 32);
+            if constexpr (STAGED) {
+                get_rows(amat, ld, row_w, it.tn * kBNMax + ch_begin * 32, lane, e_next);
+            } else {
+                const uint4* src =
+                    reinterpret_cast<const uint4*>(amat + int64_t(row) * ld + it.tn * kBNMax + ch_begin * 32);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) e_next[q] = src[q];
+                for (int q = 0; q < 4; ++q) e_next[q] = src[q];
+            }
         }
         for (int ch = ch_begin; ch < nch; ++ch) {
             const int col0 = it.tn * kBNMax + ch * 32;
             const int64_t off = int64_t(row) * ld + col0;
             uint4 e[4];
             if (poly) {
+                if constexpr (STAGED) {
+                    own_row(sbuf, lane, e_next, e);
+                    if (ch + 1 < nch) get_rows(amat, ld, row_w, col0 + 32, lane, e_next);
+                } else {
 #pragma unroll
-                for (int q = 0; q < 4; ++q) e[q] = e_next[q];
-                if (ch + 1 < nch) {
-                    const uint4* src = reinterpret_cast<const uint4*>(amat + off + 32);
+                    for (int q = 0; q < 4; ++q) e[q] = e_next[q];
+                    if (ch + 1 < nch) {
+                        const uint4* src = reinterpret_cast<const uint4*>(amat + off + 32);
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) e_next[q] = src[q];
+                        for (int q = 0; q < 4; ++q) e_next[q] = src[q];
+                    }
                 }
             }
             uint32_t r[32];
@@ -257,16 +349,24 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
                 }
                 ow[j] = pack2<BF16>(lo, hi);
             }
-            uint4* dst = reinterpret_cast<uint4*>(out + off);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) dst[q] = o[q];
             // The output is symmetric and strictly-lower tiles are skipped:
             // write the transpose of this 128 x 128 block (I, J), J > I, when
             // the tile that holds (J, I) is not computed.  The mirrored copy
             // uses the same rounded 16-bit values, so the stored matrix is
             // exactly symmetric.
             const int I = row0 / kBM, J = col0 / kBM;
-            if (J > I && !sym_tile_computed(J / MT, I / 2, md.Ppad, MT)) {
+            const bool mirror = J > I && !sym_tile_computed(J / MT, I / 2, md.Ppad, MT);
+            if constexpr (STAGED) {
+                stage_chunk(sbuf, lane, o);
+                put_rows(sbuf, lane, out, ld, row_w, col0);
+                if (mirror) put_cols(sbuf, lane, out, ld, row_w, col0);
+                __syncwarp();
+                continue;
+            }
+            uint4* dst = reinterpret_cast<uint4*>(out + off);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) dst[q] = o[q];
+            if (mirror) {
                 uint16_t* tdst = out + int64_t(col0) * ld + row;
 #pragma unroll
                 for (int j = 0; j < 16; ++j) {
