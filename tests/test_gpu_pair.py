@@ -209,3 +209,23 @@ def test_split_k_is_deterministic():
     for o in outs[1:]:
         for a, b in zip(outs[0], o):
             assert torch.equal(a, b)
+
+
+@pytest.mark.parametrize("compute", ["fp16", "bf16"])
+def test_wide_update_is_bit_identical(compute):
+    """256 x 512 Update tiles (SLORR_FLAG_WIDE_UPDATE) issue, for every output
+    column, the same N = 256 UMMA slices in the same K order as 256 x 256
+    tiles; only the tile a column belongs to changes.  The iterates are
+    equal bit for bit, including Update tiles 128, 256, 384 and 512 wide."""
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_WIDE_UPDATE
+    Ws = [workloads.random_matrix(s, seed=700 + i, std=0.02) for i, s in enumerate(SHAPES)]
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    wide = Regularizer(SHAPES, compute=compute, flags=FLAG_WIDE_UPDATE)
+    base = Regularizer(SHAPES, compute=compute)
+    for k in (1, 2, 6):
+        wide.run_steps(w, k)
+        base.run_steps(w, k)
+        torch.cuda.synchronize()
+        assert wide.status() == 0 and base.status() == 0
+        for i in range(len(SHAPES)):
+            assert torch.equal(wide.iterate(i, k).cpu(), base.iterate(i, k).cpu()), (k, i, SHAPES[i])

@@ -53,7 +53,10 @@ def test_quad_iterates_match_simt_and_pair(compute):
             b = st.iterate(i, k).double().cpu().numpy()
             c = pr.iterate(i, k).double().cpu().numpy()
             assert rel(a, b) <= 4 * ulp * (k if k < 6 else 6), (k, i, SHAPES[i], rel(a, b))
-            # same tiles, same K order: the quad and pair kernels agree exactly
+            # same tiles, same K order: the quad and pair kernels agree exactly.  The pair
+            # kernel stages its epilogue chunks in shared memory and the quad kernel stores
+            # them directly, so this also checks the staging (rows, transposed iterates,
+            # mirrored blocks, Poly's b A)
             assert np.array_equal(a, c), (k, i, SHAPES[i], rel(a, c))
 
 
