@@ -3,7 +3,9 @@
 // "Computing the polar factor"): Gram A = X X^T, Poly M = a I + b A + c A A,
 // Update X' = M X, over every matrix of the weight set in one launch.
 //
-// A cluster of two CTAs on two SMs computes one 256 x 256 tile.  CTA r of the
+// A cluster of two CTAs on two SMs computes one 256 x 256 tile (or, for the
+// Update under SLORR_FLAG_WIDE_UPDATE, one 256 x 512 tile as two N = 256
+// UMMAs per K slice into a single 512-column accumulator).  CTA r of the
 // pair holds rows [128 r, 128 r + 128) of the tile's A operand and columns
 // [nsz/2 r, nsz/2 (r + 1)) of its B operand in shared memory, and rows
 // [128 r, 128 r + 128) of the fp32 accumulator in its own tensor memory; one
@@ -25,8 +27,10 @@
 //                   each stage release and each tile completion to both CTAs;
 //   warps 2..       epilogue (both CTAs): 128 rows of the tile from TMEM, one
 //                   warp (two for Poly, each taking half of the columns) per
-//                   32-row TMEM lane quadrant; then release the accumulator
-//                   slot on the even CTA's barrier.
+//                   32-row TMEM lane quadrant, each 32 x 32 chunk staged in
+//                   the warp's shared-memory buffer so that global stores (and
+//                   Poly's loads of A) move 8 rows x 64 bytes per instruction;
+//                   then release the accumulator slot on the even CTA's barrier.
 // A stage is released only by a commit the MMA thread issues after arming the
 // stage's next phase, so every copy of either CTA is counted on a phase the
 // MMA thread armed; on a timeout that thread waits (bounded) for the last
