@@ -273,6 +273,14 @@ SLORR_API slorr_status slorr_executed_flops(const slorr_handle* h, double* out);
  * kernel a pair of tiles; for the CUDA-core kernel a 64 x 64 tile. */
 SLORR_API slorr_status slorr_gemm_items(const slorr_handle* h, int32_t phase, int32_t* items);
 
+/* Balance of one tensor-core GEMM launch (host-only): the launch hands item i
+ * of the plan to CTA pair (or CTA) i mod npairs.  *max_k is the largest total
+ * K (the K range of each item, summed over one pair's items) and *total_k the
+ * sum over all items, so total_k / npairs is the ideal.  The CTA-pair plan is
+ * ordered to balance npairs = 76 (152 SMs). */
+SLORR_API slorr_status slorr_gemm_pair_load(const slorr_handle* h, int32_t phase, int32_t npairs, int64_t* max_k,
+                                            int64_t* total_k);
+
 /* Per-kernel timing (tracing).  While enabled, every kernel this handle
  * launches is bracketed by a pair of CUDA events recorded on the caller's
  * stream (events are created on the host; no device memory is allocated).

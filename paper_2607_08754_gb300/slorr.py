@@ -96,6 +96,7 @@ def load_library(path: str | None = None) -> ctypes.CDLL:
                                   ctypes.POINTER(i32)]),
         "slorr_executed_flops": (i32, [vp, ctypes.POINTER(dbl)]),
         "slorr_gemm_items": (i32, [vp, i32, ctypes.POINTER(i32)]),
+        "slorr_gemm_pair_load": (i32, [vp, i32, i32, ctypes.POINTER(i64), ctypes.POINTER(i64)]),
         "slorr_set_timing": (i32, [vp, i32]),
         "slorr_read_timing": (i32, [vp, ctypes.POINTER(dbl), ctypes.POINTER(i64), i32]),
         "slorr_frob_sq_noalloc": (i32, [vp, i64, i64, i32, vp, vp]),
@@ -225,6 +226,14 @@ def slorr_executed_flops(handle) -> float:
     out = ctypes.c_double()
     _check(load_library().slorr_executed_flops(handle, ctypes.byref(out)))
     return out.value
+
+
+def slorr_gemm_pair_load(handle, phase: int, npairs: int = 76) -> tuple:
+    """(largest per-pair total K, total K) of one tensor-core GEMM launch when
+    item i goes to pair i mod npairs."""
+    mx, tot = ctypes.c_int64(0), ctypes.c_int64(0)
+    _check(load_library().slorr_gemm_pair_load(handle, int(phase), int(npairs), ctypes.byref(mx), ctypes.byref(tot)))
+    return int(mx.value), int(tot.value)
 
 
 def slorr_gemm_items(handle, phase: int) -> int:

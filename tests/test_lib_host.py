@@ -292,3 +292,28 @@ def test_wide_update_plan(lib):
         a = slorr.Regularizer(vl, flags=other | slorr.FLAG_WIDE_UPDATE)
         b = slorr.Regularizer(vl, flags=other)
         assert slorr.slorr_gemm_items(a.handle, 2) == slorr.slorr_gemm_items(b.handle, 2)
+
+
+def test_pair_plan_is_balanced(lib):
+    """The CTA-pair kernel hands item i to pair i mod npairs; the plan orders
+    its items so that the 76 pairs of a GB300 get nearly equal total K.
+    ViT-L/16's Gram has 960 tiles (10 per 1024-row matrix) with K = 4096, 3072
+    and 1024: sorted round-robin gives one pair 40960, the balanced order at
+    most one K = 1024 tile above the ideal total / 76.  The totals match an
+    independent count from the shapes, and equal-K phases reach the whole-tile
+    optimum ceil(tiles / 76) * K."""
+    import math
+    import workloads
+    vl = workloads.shapes("vit_l16")
+    pair = slorr.Regularizer(vl)
+    mx, tot = slorr.slorr_gemm_pair_load(pair.handle, 0)
+    assert tot == sum(10 * max(s) for s in vl)
+    assert mx <= math.ceil(tot / 76) + 1024
+    one = slorr.Regularizer(vl, flags=slorr.FLAG_TC_SINGLE_CTA)   # the same tiles, sorted, not balanced
+    mx1, tot1 = slorr.slorr_gemm_pair_load(one.handle, 0, 76)
+    assert tot1 == tot and mx1 == 40960 and mx < mx1
+    for ph, tiles in ((1, 960), (2, 4608)):
+        m, t = slorr.slorr_gemm_pair_load(pair.handle, ph)
+        assert t == tiles * 1024 and m == math.ceil(tiles / 76) * 1024
+    with pytest.raises(slorr.SlorrError):
+        slorr.slorr_gemm_pair_load(pair.handle, 0, 0)
