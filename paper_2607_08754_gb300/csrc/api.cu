@@ -209,12 +209,15 @@ constexpr int kPlanPairs = 76;
 // keeps the number of items that round-robin gives it; items go to the
 // least-loaded pair with room (longest processing time first), then swaps
 // between the most-loaded pair and the others lower the largest load.  Pair
-// p's j-th item is placed at index j kPlanPairs + p.  Any npairs processes
-// every item; kPlanPairs (GB300's 152 SMs as pairs) is the one it balances.
+// p's j-th item is placed at index j kPlanPairs + p, unless that does not
+// lower the largest load of the input order.  Any npairs processes every
+// item; kPlanPairs (GB300's 152 SMs as pairs) is the one it balances.
 void balance_pairs(std::vector<GemmItem>& v, const std::vector<int64_t>& cost) {
     const int n = kPlanPairs;
     const size_t N = v.size();
     if (N <= size_t(n)) return;
+    std::vector<int64_t> rr(n, 0);  // the input order's loads
+    for (size_t i = 0; i < N; ++i) rr[i % n] += cost[i];
     std::vector<std::vector<int>> lists(n);
     std::vector<int64_t> load(n, 0);
     std::vector<size_t> cap(n);
@@ -256,6 +259,7 @@ void balance_pairs(std::vector<GemmItem>& v, const std::vector<int64_t>& cost) {
         load[p] += cost[by] - cost[bx];
         load[bq] += cost[bx] - cost[by];
     }
+    if (*std::max_element(load.begin(), load.end()) >= *std::max_element(rr.begin(), rr.end())) return;
     std::vector<GemmItem> out(N);
     std::vector<char> used(N, 0);
     for (int p = 0; p < n; ++p) {

@@ -317,3 +317,23 @@ def test_pair_plan_is_balanced(lib):
         assert t == tiles * 1024 and m == math.ceil(tiles / 76) * 1024
     with pytest.raises(slorr.SlorrError):
         slorr.slorr_gemm_pair_load(pair.handle, 0, 0)
+
+
+def test_pair_plan_balance_on_random_sets(lib):
+    """On random weight sets (1 to 40 matrices, sides 1 to 3000) the CTA-pair
+    plan's Gram and Update items are the one-CTA plan's tiles (same total K
+    over every npairs: a permutation) and its largest per-pair total over 76
+    pairs is not above that of the sorted order the one-CTA plan keeps.  The
+    planner weighs each tile as its K plus one K block (64) for its fixed
+    cost, so in pure K the bound holds to within that one block."""
+    rng = np.random.default_rng(2607)
+    for _ in range(25):
+        count = int(rng.integers(1, 41))
+        shapes = [(int(rng.integers(1, 3001)), int(rng.integers(1, 3001))) for _ in range(count)]
+        pair = slorr.Regularizer(shapes, flags=slorr.FLAG_NO_SPLIT_K)
+        one = slorr.Regularizer(shapes, flags=slorr.FLAG_TC_SINGLE_CTA)
+        for ph in (0, 2):
+            for npairs in (1, 7, 76):
+                assert slorr.slorr_gemm_pair_load(pair.handle, ph, npairs)[1] == \
+                    slorr.slorr_gemm_pair_load(one.handle, ph, npairs)[1]
+            assert slorr.slorr_gemm_pair_load(pair.handle, ph)[0] <= slorr.slorr_gemm_pair_load(one.handle, ph)[0] + 64
