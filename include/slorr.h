@@ -273,11 +273,13 @@ SLORR_API slorr_status slorr_executed_flops(const slorr_handle* h, double* out);
  * kernel a pair of tiles; for the CUDA-core kernel a 64 x 64 tile. */
 SLORR_API slorr_status slorr_gemm_items(const slorr_handle* h, int32_t phase, int32_t* items);
 
-/* Balance of one tensor-core GEMM launch (host-only): the launch hands item i
- * of the plan to CTA pair (or CTA) i mod npairs.  *max_k is the largest total
- * K (the K range of each item, summed over one pair's items) and *total_k the
- * sum over all items, so total_k / npairs is the ideal.  The CTA-pair plan is
- * ordered to balance npairs = 76 (152 SMs). */
+/* Balance of one tensor-core GEMM launch (host-only) of the CTA-pair or
+ * one-CTA plan (not the 4-CTA kernel's super-tiles): the launch hands item i
+ * to CTA pair (or CTA) i mod npairs.  *max_k is the largest total K (the K
+ * range of each item, summed over one pair's items) and *total_k the sum over
+ * all items, so total_k / npairs is the ideal.  The CTA-pair plan is ordered
+ * to balance npairs = 76 (152 SMs).  Errors: SLORR_ERR_INVALID_ARG for a NULL
+ * pointer, a phase outside 0..2 or npairs < 1. */
 SLORR_API slorr_status slorr_gemm_pair_load(const slorr_handle* h, int32_t phase, int32_t npairs, int64_t* max_k,
                                             int64_t* total_k);
 
