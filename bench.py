@@ -22,9 +22,13 @@ number of steps (events between kernels would serialise the programmatic
 dependent launches of the first); cpu_baseline = the fp64 oracle on a bounded
 sample of the same workload on this host's cores.
 
-With --gpus N > 1 (launched by torchrun) every rank regularizes its own full
-copy of the weight set (weak scaling, no collective on the data path); the
-time is the max over ranks.  --impl reference times the oracle instead.
+With --gpus N > 1 (launched by torchrun) the matrices are partitioned across
+the ranks as in App. F (slorr_partition: longest-processing-time split by
+FLOPs; each rank regularizes its subset with grad_scale = N, which the data-
+parallel gradient average turns back into lambda): the whole set is done once
+per step by all ranks together (strong scaling, no collective on the data
+path), and the step time is the max over ranks.  --mode replicas instead has
+every rank regularize its own full copy (weak scaling).  --impl reference times the oracle instead.
 --op descent times slorr_reg_descent_step instead (the in-place regularizer-only
 step W -= eta lambda G of Alg. 1's last line; e2e then copies W in and out).
 """
@@ -58,9 +62,14 @@ TC_SOURCES = [os.path.join(ROOT, "paper_2607_08754_gb300", "csrc", f)
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--mode", default="partition", choices=["partition", "replicas"],
+                    help="N > 1: partition the matrices across ranks (App. F) or run full replicas")
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--workload", default="vit_l16", choices=list(workloads.WEIGHT_SETS))
+    ap.add_argument("--matrices", type=int, default=0,
+                    help="only the first N matrices of the workload (a smaller case of the same shapes, "
+                         "for profiling); 0: all")
     ap.add_argument("--variant", default="hoyer", choices=["hoyer", "nuclear"])
     ap.add_argument("--compute", default="fp16", choices=["fp16", "bf16", "fp32"])
     ap.add_argument("--dtype", default="f32", choices=["f32", "bf16"], help="storage of the weights and grads")
@@ -293,17 +302,31 @@ def main():
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     name = args.workload
-    shapes = workloads.shapes(name)
+    set_shapes = workloads.shapes(name)
+    if args.matrices > 0:
+        set_shapes = set_shapes[: args.matrices]
+    partition = args.mode == "partition" and world > 1
+    # App. F: this rank's matrices, gradients scaled by the world size
+    own = slorr.slorr_partition(set_shapes, world, rank) if partition else list(range(len(set_shapes)))
+    assert own, "a rank without matrices: more ranks than matrices"
+    shapes = [set_shapes[i] for i in own]
+    grad_scale = float(world) if partition else 1.0
     reg = slorr.Regularizer(shapes, variant=args.variant, compute=args.compute, dtype=args.dtype, iters=args.iters,
-                            lam=1.0, flags=args.flags)
+                            lam=1.0, grad_scale=grad_scale, flags=args.flags)
     tdt = torch.float32 if args.dtype == "f32" else torch.bfloat16
-    W_host = [torch.from_numpy(workloads.generate_one(name, i)).to(tdt) for i in range(len(shapes))]
+    W_host = [torch.from_numpy(workloads.generate_one(name, i)).to(tdt) for i in own]
     W = [w.to(dev) for w in W_host]
     G = [torch.zeros_like(w) for w in W]
     loss = torch.zeros(1, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
-    flops_step = slorr.slorr_flops(shapes, args.iters)
-    flops_exec = slorr.slorr_executed_flops(reg.handle)  # incl. padding, minus skipped symmetric tiles
+    flops_set = slorr.slorr_flops(set_shapes, args.iters)
+    flops_step = slorr.slorr_flops(shapes, args.iters)   # this rank's share
+    # whole-job FLOPs per step: the set once (partition) or once per rank (replicas)
+    flops_job = flops_set if partition else world * flops_set
+    flops_exec_t = torch.tensor([slorr.slorr_executed_flops(reg.handle)], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(flops_exec_t)   # every rank's padded MMA work (symmetric tiles skipped)
+    flops_exec = flops_exec_t.item()
 
     def barrier():
         if world > 1:
@@ -356,7 +379,7 @@ def main():
     if world > 1:
         dist.all_reduce(ms, op=dist.ReduceOp.MAX)
     ms_step = ms.item() / args.steps
-    value = world * flops_step / (ms_step * 1e-3) / 1e12
+    value = flops_job / (ms_step * 1e-3) / 1e12
     assert reg.status() == 0, "device status word reports an error in the timed region"
 
     # e2e: pinned host buffers, copies inside the timed region.  The buffers
@@ -377,7 +400,7 @@ def main():
 
     pipe = None if descent else slorr.Pipeline(shapes, groups=args.e2e_groups or None, variant=args.variant,
                                                compute=args.compute, dtype=args.dtype, iters=args.iters, lam=1.0,
-                                               flags=args.flags)
+                                               grad_scale=grad_scale, flags=args.flags)
 
     def e2e_step():
         if pipe is not None:
@@ -410,11 +433,10 @@ def main():
     os.sched_setaffinity(0, all_cpus)
     if pipe is not None:
         assert pipe.status() == 0, "device status word reports an error in the e2e region"
-    e2e_val = world * flops_step / (e2e_ms * 1e-3) / 1e12
+    e2e_val = flops_job / (e2e_ms * 1e-3) / 1e12
 
     if rank == 0:
         pk = peaks()
-        single_cta = bool(args.flags & (slorr.FLAG_TC_SINGLE_CTA | slorr.FLAG_TC_BK32 | slorr.FLAG_TC_M128))
         gemm_ms = sum(kt[k][0] for k in ("gram", "poly", "update"))
         gemm_launches = sum(kt[k][1] for k in ("gram", "poly", "update"))
         launches = sum(v[1] for v in kt.values())  # the same launches as the headline timed region
@@ -462,27 +484,31 @@ def main():
                             for k, v in kt.items()}
         line = {
             "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+            "scaling": "strong" if partition else "weak",
             "vs_baseline": None, "dtype": "f16" if args.compute == "fp16" else args.compute,
             "data": "synthetic",
-            "config": {"workload": f"{name} {args.variant}{' descent step' if descent else ''}: "
-                                   f"{len(shapes)} matrices, T={args.iters}, "
+            "config": {"workload": f"{name}{' (first %d matrices)' % len(set_shapes) if args.matrices else ''} "
+                                   f"{args.variant}{' descent step' if descent else ''}: "
+                                   f"{len(set_shapes)} matrices, T={args.iters}, "
                                    f"{args.compute} operands / fp32 accumulate, {args.dtype} weights and grads",
-                       "matrices": len(shapes), "iters": args.iters, "variant": args.variant, "op": args.op,
-                       "gflop_per_step": flops_step / 1e9,
+                       "matrices": len(set_shapes), "iters": args.iters, "variant": args.variant, "op": args.op,
+                       "gflop_per_step": flops_job / 1e9,
+                       "parallelism": (f"layer partition over {world} ranks (App. F), grad_scale {world}; "
+                                       f"rank 0 holds {len(shapes)} matrices" if partition else
+                                       f"{world} full replicas" if world > 1 else "one GPU"),
                        "l2": l2_note},
             "pct_of_dense_peak": value / world / pk["bf16"],
             "step_ms": {"mean": ms_step, "p10": per_call[len(per_call) // 10],
                         "p50": per_call[len(per_call) // 2], "p90": per_call[(9 * len(per_call)) // 10]},
             "executed": {"gflop_per_step": flops_exec / 1e9,
-                         "tflops": world * flops_exec / (ms_step * 1e-3) / 1e12,
+                         "tflops": flops_exec / (ms_step * 1e-3) / 1e12,
                          "note": "MMA FLOPs the kernels execute: padding included, strictly-lower "
                                  "symmetric tiles skipped"},
             "roofline": ({"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                          "frac": achieved / peak, "traffic": None if single_cta else tc_traffic(),
+                          "frac": achieved / peak, "traffic": tc_traffic(),
                           "frac_of_sustained": achieved / pk["bf16_sustained"],
-                          "kernel": ("tc_gemm_kernel" if single_cta else "tc_pair_kernel")
-                                    + " (Gram/Poly/Update launches)",
+                          "kernel": "tc_pair_kernel (Gram/Poly/Update launches)",
                           "peak_source": pk["source"] + " bf16 burst (fp16 dense rate equal)"}
                          if not simt else
                          {"bound": "alu", "achieved": achieved, "peak": alu_peak, "unit": "TFLOP/s",
@@ -502,7 +528,7 @@ def main():
                                     if local_cpus else "page-locked (GPU-local CPUs unknown)"},
             "clocks": clk,
         }
-        if not args.no_cpu_baseline:
+        if not args.no_cpu_baseline and world == 1:
             f, t, desc = oracle_sample(name, args.variant, args.iters, args.cpu_seconds)
             line["cpu_baseline"] = {"value": f / t / 1e12, "unit": "TFLOP/s", "cores": cpu_cores(),
                                     "kind": "oracle", "sample": desc, "blas": blas_info(),

@@ -94,11 +94,8 @@ typedef struct slorr_options {
     double  timeout_s;           /* budget of each bounded device wait, s (2.0)      */
 } slorr_options;
 
-/* Flags. */
+/* Flags.  slorr_create rejects any other bit with SLORR_ERR_INVALID_ARG. */
 #define SLORR_FLAG_SIMT_GEMM    1   /* run the 16-bit products on CUDA cores (debug)  */
-#define SLORR_FLAG_L2_PREFETCH  2   /* tensor-core producer also warms L2 ahead (tuning) */
-#define SLORR_FLAG_TC_BK32      4   /* 9 stages of K = 32 instead of 4 of K = 64 (tuning) */
-#define SLORR_FLAG_TC_M128      8   /* 128 x 256 tensor-core tiles in every phase (tuning) */
 #define SLORR_FLAG_TEST_STALL  16   /* test only: every tensor-core CTA first waits on a
                                        barrier nothing arrives on, so its bounded wait
                                        runs out after timeout_s and the call reports
@@ -107,15 +104,6 @@ typedef struct slorr_options {
                                        the pre-update gradient of the decoupled variant
                                        (Alg. 1, App. C.2), applied by the caller as
                                        W -= lr * grads[i] after its optimizer step      */
-#define SLORR_FLAG_TC_SINGLE_CTA 64 /* one-CTA tensor-core kernels (256 x 256 Gram/Update
-                                       tiles, 128 x 256 Poly tiles) instead of the
-                                       default CTA-pair kernel (tcgen05 cta_group::2);
-                                       implied by TC_BK32 and TC_M128 (tuning)           */
-#define SLORR_FLAG_PAIR_ONE_SLOT 128 /* CTA-pair kernel with one accumulator per SM (no
-                                       epilogue overlap; tuning)                         */
-#define SLORR_FLAG_TC_QUAD     256  /* clusters of two CTA pairs computing two tiles that
-                                       share an operand, loaded once by TMA multicast
-                                       (tuning)                                          */
 #define SLORR_FLAG_NO_PDL      512  /* launch every kernel after the previous one completes.
                                        By default the memory passes and the CTA-pair
                                        kernel are programmatic dependents of the kernel
@@ -141,12 +129,6 @@ typedef struct slorr_options {
                                        workspace).  Ignored while timing is on; a stream
                                        that is being captured gets the launches.  Saves
                                        the launch gaps of small sets                    */
-#define SLORR_FLAG_WIDE_UPDATE 8192  /* CTA-pair Update with 256 x 512 tiles: one 128 x 512
-                                       accumulator per SM (all 512 TMEM columns, so no
-                                       epilogue overlap), two N = 256 UMMAs per K slice
-                                       and 4 stages of 48 KB; each SM copies 48 KB per
-                                       K block for twice the FLOPs of the 32 KB of a
-                                       256 x 256 tile (tuning)                          */
 
 /* Fill *opt with the defaults listed beside each field above (App. C.1: T = 6,
  * ell = 1e-3, degree 5; eps, lambda and grad_scale as in Listing 1 / Alg. 2). */
@@ -268,14 +250,24 @@ SLORR_API slorr_status slorr_partition(const slorr_shape* shapes, int32_t count,
 SLORR_API slorr_status slorr_executed_flops(const slorr_handle* h, double* out);
 
 /* Work items of one GEMM launch of the plan (host-only): phase 0 Gram, 1 Poly,
- * 2 Update.  For the tensor-core kernels an item is a 256 x 256 output tile,
- * or one K part of a split Gram tile (SLORR_FLAG_NO_SPLIT_K); for the 4-CTA
- * kernel a pair of tiles; for the CUDA-core kernel a 64 x 64 tile. */
+ * 2 Update.  For the tensor-core kernel an item is a 256 x 256 output tile or,
+ * for Gram tiles whose K range is split (the default for sets with few long-K
+ * tiles, unless SLORR_FLAG_NO_SPLIT_K is set), one K part of such a tile; for
+ * the CUDA-core kernel it is a 32 x 32 tile. */
 SLORR_API slorr_status slorr_gemm_items(const slorr_handle* h, int32_t phase, int32_t* items);
 
-/* Balance of one tensor-core GEMM launch (host-only) of the CTA-pair or
- * one-CTA plan (not the 4-CTA kernel's super-tiles): the launch hands item i
- * to CTA pair (or CTA) i mod npairs.  *max_k is the largest total K (the K
+/* The work items of one GEMM launch of the plan (host-only), in the order the
+ * launch hands them out (tensor cores: item i to CTA pair i mod npairs):
+ * 7 int32 per item, (mat, tm, tn, msz, nsz, part, parts): matrix index, row
+ * and column tile index, rows and columns of the tile, and for a Gram tile
+ * whose K range is split, which of `parts` equal K ranges this item
+ * accumulates (part 0 of 1 otherwise).  `out` holds `capacity` int32, at
+ * least 7 * slorr_gemm_items().  Errors: SLORR_ERR_INVALID_ARG for a NULL
+ * pointer, a phase outside 0..2 or a capacity that is too small. */
+SLORR_API slorr_status slorr_gemm_item_list(const slorr_handle* h, int32_t phase, int32_t* out, int32_t capacity);
+
+/* Balance of one tensor-core GEMM launch (host-only): the launch hands item i
+ * to CTA pair i mod npairs.  *max_k is the largest total K (the K
  * range of each item, summed over one pair's items) and *total_k the sum over
  * all items, so total_k / npairs is the ideal.  The CTA-pair plan is ordered
  * to balance npairs = 76 (152 SMs).  Errors: SLORR_ERR_INVALID_ARG for a NULL

@@ -1,12 +1,18 @@
 """Builds libslorr.so in-tree for sm_103a with nvcc (no CMake, no torch extension).
 
 The translation units are compiled in parallel and linked with the static CUDA
-runtime, so the library depends only on the CUDA driver at run time.
+runtime, so the library depends only on the CUDA driver at run time.  A build
+is reused only when the stamp file beside the library records the same hash
+of every source, the public header, the compiler command lines and the
+machine's architecture; anything else (a library copied in from another
+machine, an edited source, other flags) recompiles.
 """
 
 from __future__ import annotations
 
+import hashlib
 import os
+import platform
 import shutil
 import subprocess
 from concurrent.futures import ThreadPoolExecutor
@@ -15,8 +21,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libslorr.so")
-SOURCES = ["api.cu", "kernels_mem.cu", "kernels_simt.cu", "kernels_tc.cu", "kernels_tc_pair.cu",
-           "kernels_tc_quad.cu", "noalloc.cu", "schedule.cpp"]
+STAMP = os.path.join(BUILD, "libslorr.stamp")
+SOURCES = ["api.cu", "kernels_mem.cu", "kernels_simt.cu", "kernels_tc_pair.cu", "noalloc.cu", "schedule.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
          "--expt-relaxed-constexpr"]
@@ -33,11 +39,11 @@ def build(verbose: bool = False, force: bool = False) -> str:
     """Compile every source for sm_103a and link libslorr.so; returns its path."""
     nvcc = _nvcc()
     os.makedirs(BUILD, exist_ok=True)
-    deps = [os.path.join(CSRC, f) for f in os.listdir(CSRC)]
-    deps.append(os.path.join(os.path.dirname(HERE), "include", "slorr.h"))
-    newest = max(os.path.getmtime(d) for d in deps)
-    if not force and os.path.exists(LIB) and os.path.getmtime(LIB) >= newest:
-        return LIB
+    digest = _digest(nvcc)
+    if not force and os.path.exists(LIB) and os.path.exists(STAMP):
+        with open(STAMP) as f:
+            if f.read().strip() == digest:
+                return LIB
 
     def compile_one(src: str) -> str:
         obj = os.path.join(BUILD, src + ".o")
@@ -63,7 +69,22 @@ def build(verbose: bool = False, force: bool = False) -> str:
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
     os.replace(tmp, LIB)
+    with open(STAMP, "w") as f:
+        f.write(digest + "\n")
     return LIB
+
+
+def _digest(nvcc: str) -> str:
+    """Hash of everything the library is built from."""
+    h = hashlib.sha256()
+    h.update(" ".join([nvcc, *ARCH, *FLAGS, platform.machine()]).encode())
+    deps = sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC))
+    deps.append(os.path.join(os.path.dirname(HERE), "include", "slorr.h"))
+    for d in deps:
+        h.update(os.path.basename(d).encode())
+        with open(d, "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
 
 
 if __name__ == "__main__":

@@ -60,7 +60,6 @@ struct slorr_handle {
     int esize;
     // item lists (host)
     std::vector<GemmItem> tc_items[3];
-    std::vector<GemmItem> quad_items[3];  // super-tiles: 2 items each (the second may be empty)
     std::vector<GemmItem> simt_items[3];
     std::vector<MemItem> w_items;  // tiles of W (sumsq, dot, combine)
     std::vector<MemItem> x_items;  // tiles of the padded iterate (cast)
@@ -70,8 +69,7 @@ struct slorr_handle {
     // workspace layout
     size_t off_status = 0, off_counters = 0, off_scalars = 0, off_partials = 0, off_partials_max = 0,
            off_tilebase = 0, off_tilecount = 0, off_xtilebase = 0, off_xtilecount = 0, off_split_cnt = 0,
-           off_split_part = 0, off_mats = 0, off_maps = 0, off_tc_items[3] = {}, off_quad_items[3] = {},
-           off_simt_items[3] = {},
+           off_split_part = 0, off_mats = 0, off_maps = 0, off_tc_items[3] = {}, off_simt_items[3] = {},
            off_w_items = 0, off_x_items = 0, off_ptrs = 0, off_plan_end = 0, total_bytes = 0;
     // device state
     const void* prepared_ws = nullptr;
@@ -99,17 +97,6 @@ struct slorr_handle {
 
 namespace {
 
-// The CTA-pair kernel (256 x 256 tiles over two SMs, two accumulators per SM)
-// runs every phase unless a one-CTA kernel is asked for.
-bool tc_pair(const slorr_handle* h) {
-    return (h->opt.flags & (SLORR_FLAG_TC_SINGLE_CTA | SLORR_FLAG_TC_BK32 | SLORR_FLAG_TC_M128)) == 0;
-}
-
-// CTA-pair Update with 256 x 512 tiles (the 4-CTA kernel keeps 256 x 256).
-bool wide_update(const slorr_handle* h) {
-    return tc_pair(h) && (h->opt.flags & SLORR_FLAG_WIDE_UPDATE) && !(h->opt.flags & SLORR_FLAG_TC_QUAD);
-}
-
 // Programmatic dependent launch of the memory passes and the pair kernel.
 bool use_pdl(const slorr_handle* h) { return (h->opt.flags & SLORR_FLAG_NO_PDL) == 0; }
 
@@ -120,23 +107,9 @@ bool fused_norm(const slorr_handle* h) {
            (h->opt.flags & (SLORR_FLAG_SIMT_GEMM | SLORR_FLAG_SEPARATE_NORM)) == 0;
 }
 
-// K depth of the tensor-core pipeline stages for this handle.
-int tc_bk(const slorr_handle* h) {
-    if (tc_pair(h)) return 64;  // the pair kernel's stages are K = 64
-    return (h->opt.flags & SLORR_FLAG_TC_BK32) ? 32 : 64;
-}
-
-// 128-row M tiles per tensor-core tile for one phase.  The pair kernel always
-// takes 256 x 256 tiles.  Of the one-CTA kernels, 256 x 256 tiles (mt = 2) move
-// a third fewer operand rows per FLOP but cannot overlap a tile's epilogue
-// with the next main loop; they win for the long-K Gram and the store-only
-// Update, while the short-K Poly, whose epilogue also reads A, keeps
-// double-buffered 128 x 256 tiles.
-int tc_mt(const slorr_handle* h, int phase) {
-    if (tc_pair(h)) return 2;
-    if (h->opt.flags & (SLORR_FLAG_TC_M128 | SLORR_FLAG_TC_BK32)) return 1;
-    return phase == kPoly ? 1 : 2;
-}
+constexpr int32_t kKnownFlags = SLORR_FLAG_SIMT_GEMM | SLORR_FLAG_TEST_STALL | SLORR_FLAG_WRITE_GRAD |
+                                SLORR_FLAG_NO_PDL | SLORR_FLAG_SEPARATE_NORM | SLORR_FLAG_NO_SPLIT_K |
+                                SLORR_FLAG_GRAPH;
 
 bool valid_options(const slorr_options& o, std::string* why) {
     if (o.variant != SLORR_HOYER && o.variant != SLORR_NUCLEAR) return *why = "variant", false;
@@ -149,45 +122,8 @@ bool valid_options(const slorr_options& o, std::string* why) {
     if (!(o.eps >= 0.f) || !std::isfinite(o.eps)) return *why = "eps must be >= 0", false;
     if (!std::isfinite(o.lambda) || !std::isfinite(o.grad_scale)) return *why = "lambda/grad_scale", false;
     if (!(o.timeout_s > 0.0) || o.timeout_s > 3600.0) return *why = "timeout_s must be in (0, 3600]", false;
+    if (o.flags & ~kKnownFlags) return *why = "flags holds a bit this build does not define", false;
     return true;
-}
-
-// Super-tiles of the 4-CTA kernel for one matrix and phase: two 256 x 256
-// tiles that share an operand, one per CTA pair of the cluster.  The tiles of
-// each row (the same A rows) are paired left to right; a row's odd last tile
-// waits, and the leftovers of each column (the same B columns) are paired top
-// to bottom; a final odd leftover runs alone (second item empty, msz = 0).
-// Gram and Poly keep only the tiles on or above the diagonal, as the pair
-// kernel does.
-void add_quad_items(std::vector<GemmItem>& out, int mat, int ph, int Ppad, int N) {
-    const GemmItem none{uint16_t(mat), 0, 0, 0, 0, 0};
-    std::vector<std::vector<GemmItem>> by_col((N + 255) / 256);
-    for (int tm = 0; tm * 256 < Ppad; ++tm) {
-        const int msz = std::min(256, Ppad - tm * 256);
-        std::vector<GemmItem> row;
-        for (int tn = 0; tn * 256 < N; ++tn) {
-            const int nsz = std::min(256, N - tn * 256);
-            if (ph != kUpdate && (2 * tn + nsz / 128 - 1) < tm * 2) continue;
-            row.push_back(GemmItem{uint16_t(mat), uint16_t(tm), uint16_t(tn), uint16_t(nsz), uint16_t(msz), 0});
-        }
-        size_t j = 0;
-        for (; j + 1 < row.size(); j += 2) {
-            out.push_back(row[j]);
-            out.push_back(row[j + 1]);
-        }
-        if (j < row.size()) by_col[row[j].tn].push_back(row[j]);
-    }
-    for (auto& col : by_col) {
-        size_t j = 0;
-        for (; j + 1 < col.size(); j += 2) {
-            out.push_back(col[j]);
-            out.push_back(col[j + 1]);
-        }
-        if (j < col.size()) {
-            out.push_back(col[j]);
-            out.push_back(none);
-        }
-    }
 }
 
 // Split K of the CTA-pair kernel's Gram tiles (A = X X^T with K = Qpad).  A
@@ -276,8 +212,7 @@ void balance_pairs(std::vector<GemmItem>& v, const std::vector<int64_t>& cost) {
 
 void split_gram_items(slorr_handle* h) {
     h->total_split_parts = 0;
-    if (h->opt.compute == SLORR_COMPUTE_FP32 || !tc_pair(h) ||
-        (h->opt.flags & (SLORR_FLAG_SIMT_GEMM | SLORR_FLAG_TC_QUAD | SLORR_FLAG_NO_SPLIT_K)))
+    if (h->opt.compute == SLORR_COMPUTE_FP32 || (h->opt.flags & (SLORR_FLAG_SIMT_GEMM | SLORR_FLAG_NO_SPLIT_K)))
         return;
     std::vector<GemmItem>& items = h->tc_items[kGram];
     double work = 0.0;
@@ -308,7 +243,6 @@ void build_plan(slorr_handle* h) {
     h->geom.resize(count);
     for (int i = 0; i < 3; ++i) {
         h->tc_items[i].clear();
-        h->quad_items[i].clear();
         h->simt_items[i].clear();
     }
     h->w_items.clear();
@@ -355,24 +289,21 @@ void build_plan(slorr_handle* h) {
         g.xtile_count = xseq;
         tile_base += seq;
         xtile_base += xseq;
-        // tensor-core tiles: msz x nsz with msz <= 128 mt, nsz <= 256 (512 for
-        // the wide CTA-pair Update).  The Gram and Poly outputs are symmetric:
-        // tiles lying strictly below the diagonal (in 128 x 128 blocks) are
-        // skipped; the kernel mirrors the blocks they need.
+        // tensor-core tiles: msz x nsz with msz, nsz <= 256.  The Gram and
+        // Poly outputs are symmetric: tiles lying strictly below the diagonal
+        // (in 128 x 128 blocks) are skipped; the kernel mirrors the blocks
+        // they need.
         for (int ph = 0; ph < 3; ++ph) {
-            const int mt = tc_mt(h, ph);
             const int N = ph == kUpdate ? g.Qpad : g.Ppad;
-            const int bn = ph == kUpdate && wide_update(h) ? 512 : 256;
-            for (int tm = 0; tm * 128 * mt < g.Ppad; ++tm) {
-                const int msz = std::min(128 * mt, g.Ppad - tm * 128 * mt);
-                for (int tn = 0; tn * bn < N; ++tn) {
-                    const int nsz = std::min(bn, N - tn * bn);
-                    if (ph != kUpdate && (2 * tn + nsz / 128 - 1) < tm * mt) continue;
+            for (int tm = 0; tm * 256 < g.Ppad; ++tm) {
+                const int msz = std::min(256, g.Ppad - tm * 256);
+                for (int tn = 0; tn * 256 < N; ++tn) {
+                    const int nsz = std::min(256, N - tn * 256);
+                    if (ph != kUpdate && (2 * tn + nsz / 128 - 1) < tm * 2) continue;
                     h->tc_items[ph].push_back(
                         GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), uint16_t(nsz), uint16_t(msz), 0});
                 }
             }
-            add_quad_items(h->quad_items[ph], i, ph, g.Ppad, N);
             // CUDA-core tiles; the symmetric Gram and Poly keep those on or above the diagonal
             for (int tm = 0; tm < g.Ppad / kSimtTile; ++tm)
                 for (int tn = (ph == kUpdate ? 0 : tm); tn < N / kSimtTile; ++tn)
@@ -398,24 +329,9 @@ void build_plan(slorr_handle* h) {
         // fixed cost).  For ViT-L/16's Gram tiles (K = 4096, 3072, 1024) the
         // largest total drops from 40960 to 38912 (ideal 38804); the Gram
         // launches take 1.7% less time than in plain sorted order.
-        if (tc_pair(h)) {
-            std::vector<int64_t> cost;
-            for (const GemmItem& it : h->tc_items[ph]) cost.push_back(kdim(it) + 64);
-            balance_pairs(h->tc_items[ph], cost);
-        }
-        // super-tiles move as units of two items
-        std::vector<std::pair<GemmItem, GemmItem>> sup;
-        for (size_t j = 0; j + 1 < h->quad_items[ph].size(); j += 2)
-            sup.push_back({h->quad_items[ph][j], h->quad_items[ph][j + 1]});
-        std::stable_sort(sup.begin(), sup.end(), [&](const std::pair<GemmItem, GemmItem>& a,
-                                                     const std::pair<GemmItem, GemmItem>& b) {
-            return kdim(a.first) > kdim(b.first);
-        });
-        h->quad_items[ph].clear();
-        for (auto& pr : sup) {
-            h->quad_items[ph].push_back(pr.first);
-            h->quad_items[ph].push_back(pr.second);
-        }
+        std::vector<int64_t> cost;
+        for (const GemmItem& it : h->tc_items[ph]) cost.push_back(kdim(it) + 64);
+        balance_pairs(h->tc_items[ph], cost);
     }
 
     // Workspace layout.
@@ -447,8 +363,6 @@ void build_plan(slorr_handle* h) {
     for (int ph = 0; ph < 3; ++ph) {
         h->off_tc_items[ph] = off;
         off = align_up(off + h->tc_items[ph].size() * sizeof(GemmItem), 256);
-        h->off_quad_items[ph] = off;
-        off = align_up(off + h->quad_items[ph].size() * sizeof(GemmItem), 256);
         h->off_simt_items[ph] = off;
         off = align_up(off + h->simt_items[ph].size() * sizeof(GemmItem), 256);
     }
@@ -526,7 +440,7 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
     std::vector<int32_t> tb(count), tcnt(count), xtb(count), xtcnt(count);
     std::vector<MatDev> mats(count);
     std::vector<uint8_t> maps(size_t(count) * kMapsPerMatrix * 128, 0);
-    const int bk = tc_bk(h);
+    const int bk = 64;  // K depth of a pipeline stage
     const bool tc = h->opt.compute != SLORR_COMPUTE_FP32;
     for (int i = 0; i < count; ++i) {
         const Geom& g = h->geom[i];
@@ -571,7 +485,6 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
     put(plan, h->off_maps - base, maps.data(), maps.size());
     for (int ph = 0; ph < 3; ++ph) {
         put(plan, h->off_tc_items[ph] - base, h->tc_items[ph].data(), h->tc_items[ph].size());
-        put(plan, h->off_quad_items[ph] - base, h->quad_items[ph].data(), h->quad_items[ph].size());
         put(plan, h->off_simt_items[ph] - base, h->simt_items[ph].data(), h->simt_items[ph].size());
     }
     put(plan, h->off_w_items - base, h->w_items.data(), h->w_items.size());
@@ -811,14 +724,8 @@ slorr_status launch_all(slorr_handle* h, uint8_t* ws, float* loss, float* per, i
     g.maps = ws + h->off_maps;
     g.status = reinterpret_cast<uint32_t*>(ws + h->off_status);
     g.timeout_ns = static_cast<unsigned long long>(h->opt.timeout_s * 1e9);
-    g.prefetch = (h->opt.flags & SLORR_FLAG_L2_PREFETCH) ? 8 : 0;
-    g.bk = tc_bk(h);
     g.test_stall = (h->opt.flags & SLORR_FLAG_TEST_STALL) ? 1 : 0;
-    const bool pair = tc_pair(h);
-    const bool quad = pair && (h->opt.flags & SLORR_FLAG_TC_QUAD) != 0;
-    g.pair_slots = (h->opt.flags & SLORR_FLAG_PAIR_ONE_SLOT) ? 1 : 2;
-    g.wide_update = wide_update(h) ? 1 : 0;
-    g.pdl = (use_pdl(h) && pair && !quad) ? 1 : 0;
+    g.pdl = use_pdl(h) ? 1 : 0;
     g.scalars = reinterpret_cast<const MatScalars*>(ws + h->off_scalars);
     g.split_part = reinterpret_cast<float*>(ws + h->off_split_part);
     g.split_cnt = reinterpret_cast<uint32_t*>(ws + h->off_split_cnt);
@@ -829,18 +736,12 @@ slorr_status launch_all(slorr_handle* h, uint8_t* ws, float* loss, float* per, i
         g.c = float(h->coeffs[3 * t + 2]);
         for (int ph = 0; ph < 3; ++ph) {
             g.phase = ph;
-            g.mt = tc_mt(h, ph);
             g.x0_scaled = (fuse_norm && t == 0 && ph != kPoly) ? 1 : 0;
             Traced tr(h, 2 + ph, st);
-            if (use_tc && quad) {
-                g.items = reinterpret_cast<const GemmItem*>(ws + h->off_quad_items[ph]);
-                g.num_items = int(h->quad_items[ph].size() / 2);
-                e = launch_gemm_tc_quad(g, h->elem, h->num_sms, st);
-            } else if (use_tc) {
+            if (use_tc) {
                 g.items = reinterpret_cast<const GemmItem*>(ws + h->off_tc_items[ph]);
                 g.num_items = int(h->tc_items[ph].size());
-                e = pair ? launch_gemm_tc_pair(g, h->elem, h->num_sms, st)
-                         : launch_gemm_tc(g, h->elem, h->num_sms, st);
+                e = launch_gemm_tc_pair(g, h->elem, h->num_sms, st);
             } else {
                 g.items = reinterpret_cast<const GemmItem*>(ws + h->off_simt_items[ph]);
                 g.num_items = int(h->simt_items[ph].size());
@@ -954,20 +855,15 @@ slorr_status slorr_create(slorr_handle** out, const slorr_shape* shapes, int32_t
 slorr_status slorr_executed_flops(const slorr_handle* h, double* out) {
     if (!h || !out) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
     const bool simt = h->opt.compute == SLORR_COMPUTE_FP32 || (h->opt.flags & SLORR_FLAG_SIMT_GEMM);
-    const bool pair = !simt && tc_pair(h);
-    const bool quad = pair && (h->opt.flags & SLORR_FLAG_TC_QUAD);
     double total = 0.0;
     for (int ph = 0; ph < 3; ++ph) {
-        const std::vector<GemmItem>& items =
-            simt ? h->simt_items[ph] : (quad ? h->quad_items[ph] : h->tc_items[ph]);
-        for (const GemmItem& it : items) {
-            if (it.msz == 0) continue;  // empty half of a super-tile
+        for (const GemmItem& it : simt ? h->simt_items[ph] : h->tc_items[ph]) {
             const Geom& g = h->geom[it.mat];
             const int Kfull = ph == kGram ? g.Qpad : g.Ppad;
             int kb0, kb1;
             split_range(it, Kfull / 64, &kb0, &kb1);
             const double K = it.ksplit ? double(kb1 - kb0) * 64 : double(Kfull);
-            const double rows = pair ? 256.0 : double(it.msz);  // pair UMMAs are always M = 256
+            const double rows = simt ? double(it.msz) : 256.0;  // pair UMMAs are always M = 256
             total += 2.0 * rows * double(it.nsz) * K;
         }
     }
@@ -979,9 +875,28 @@ slorr_status slorr_gemm_items(const slorr_handle* h, int32_t phase, int32_t* ite
     if (!h || !items) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
     if (phase < 0 || phase > 2) return fail(SLORR_ERR_INVALID_ARG, "phase must be 0 (Gram), 1 (Poly) or 2 (Update)");
     const bool simt = h->opt.compute == SLORR_COMPUTE_FP32 || (h->opt.flags & SLORR_FLAG_SIMT_GEMM);
-    const bool quad = !simt && tc_pair(h) && (h->opt.flags & SLORR_FLAG_TC_QUAD);
-    *items = int32_t(simt ? h->simt_items[phase].size()
-                          : quad ? h->quad_items[phase].size() / 2 : h->tc_items[phase].size());
+    *items = int32_t(simt ? h->simt_items[phase].size() : h->tc_items[phase].size());
+    return SLORR_OK;
+}
+
+slorr_status slorr_gemm_item_list(const slorr_handle* h, int32_t phase, int32_t* out, int32_t capacity) {
+    if (!h || !out) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
+    if (phase < 0 || phase > 2) return fail(SLORR_ERR_INVALID_ARG, "phase must be 0 (Gram), 1 (Poly) or 2 (Update)");
+    const bool simt = h->opt.compute == SLORR_COMPUTE_FP32 || (h->opt.flags & SLORR_FLAG_SIMT_GEMM);
+    const std::vector<GemmItem>& v = simt ? h->simt_items[phase] : h->tc_items[phase];
+    if (capacity < int64_t(v.size()) * 7) return fail(SLORR_ERR_INVALID_ARG, "capacity too small");
+    for (size_t i = 0; i < v.size(); ++i) {
+        const GemmItem& it = v[i];
+        const int parts = it.ksplit >> 8;
+        int32_t* o = out + i * 7;
+        o[0] = it.mat;
+        o[1] = it.tm;
+        o[2] = it.tn;
+        o[3] = it.msz;
+        o[4] = it.nsz;
+        o[5] = parts > 1 ? (it.ksplit & 0xff) : 0;
+        o[6] = parts > 1 ? parts : 1;
+    }
     return SLORR_OK;
 }
 

@@ -65,8 +65,8 @@ struct MatScalars {
 // One output tile of a grouped GEMM phase.
 struct GemmItem {
     uint16_t mat;
-    uint16_t tm;       // row tile index (128 x mt rows per tcgen05 tile, 64 for SIMT)
-    uint16_t tn;       // column tile index (256 columns per tcgen05 tile, 64 for SIMT)
+    uint16_t tm;       // row tile index (256 rows per tcgen05 tile, 32 for SIMT)
+    uint16_t tn;       // column tile index (256 columns per tcgen05 tile, 32 for SIMT)
     uint16_t nsz;      // columns in this tile
     uint16_t msz;      // rows in this tile
     uint16_t ksplit;   // split K (CTA-pair Gram): part s | (parts S << 8); 0 = whole K
@@ -89,8 +89,8 @@ __host__ __device__ inline void split_range(const GemmItem& it, int nkb, int* be
 #ifndef SLORR_MAX_SPLIT
 #define SLORR_MAX_SPLIT 2
 #endif
-constexpr int kMaxSplit = SLORR_MAX_SPLIT;
-constexpr int kSimtTile = 32;  // output tile of the CUDA-core GEMM (32 x 32)  // K parts of a split Gram tile (a build-time tuning knob)
+constexpr int kMaxSplit = SLORR_MAX_SPLIT;  // K parts of a split Gram tile (a build-time tuning knob)
+constexpr int kSimtTile = 32;              // output tile of the CUDA-core GEMM (32 x 32)
 
 // One chunk of a memory-bound pass: a kMemRows x kMemCols tile of W (or of
 // the padded iterate buffer for the cast).
@@ -122,12 +122,7 @@ struct GemmLaunch {
     const void* maps;          // CUtensorMap array, kMapsPerMatrix per matrix
     uint32_t* status;
     unsigned long long timeout_ns;
-    int32_t prefetch;          // k blocks of L2 prefetch lookahead (0 = off)
-    int32_t bk;                // K depth of a pipeline stage: 64 (4 stages) or 32 (9 stages)
-    int32_t mt;                // 128-row M tiles per CTA tile: 1 or 2 (256 x 256 tiles)
     int32_t test_stall;        // 1: the MMA thread first waits on a barrier nothing arrives on
-    int32_t pair_slots;        // CTA-pair kernel: accumulators per CTA (1 or 2)
-    int32_t wide_update;       // CTA-pair Update tiles are 256 x 512 (one 512-column accumulator)
     int32_t pdl;               // launch with programmatic dependent launch
     // x0_scaled = 1 (first step after the fused norm pass, which stores X_0
     // as W rounded to 16 bits): the Gram epilogue multiplies by
@@ -188,11 +183,7 @@ cudaError_t launch_finalize(const MemLaunch& p, int which, cudaStream_t s);
 cudaError_t launch_combine(const MemLaunch& p, cudaStream_t s);
 cudaError_t launch_sum_parts(const float* parts, int n, float* out, cudaStream_t s);
 cudaError_t launch_gemm_simt(const GemmLaunch& p, int elem, cudaStream_t s);
-cudaError_t launch_gemm_tc(const GemmLaunch& p, int elem, int grid, cudaStream_t s);
 cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t s);
-// items: 2 per super-tile (num_items super-tiles); see kernels_tc_quad.cu
-cudaError_t launch_gemm_tc_quad(const GemmLaunch& p, int elem, int num_sms, cudaStream_t s);
-int tc_smem_bytes();
 
 #if defined(__CUDACC__)
 // Launches `kernel` on `st`; with pdl, as a programmatic dependent of the

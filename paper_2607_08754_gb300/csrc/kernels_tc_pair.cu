@@ -1,11 +1,9 @@
-// Grouped persistent tensor-core GEMM on CTA pairs (tcgen05 cta_group::2), for
-// the same three phases of a Polar Express step as kernels_tc.cu (Sec. 3
-// "Computing the polar factor"): Gram A = X X^T, Poly M = a I + b A + c A A,
-// Update X' = M X, over every matrix of the weight set in one launch.
+// Grouped persistent tensor-core GEMM on CTA pairs (tcgen05 cta_group::2) for
+// the three phases of a Polar Express step (Sec. 3 "Computing the polar
+// factor"): Gram A = X X^T, Poly M = a I + b A + c A A, Update X' = M X, over
+// every matrix of the weight set in one launch.
 //
-// A cluster of two CTAs on two SMs computes one 256 x 256 tile (or, for the
-// Update under SLORR_FLAG_WIDE_UPDATE, one 256 x 512 tile as two N = 256
-// UMMAs per K slice into a single 512-column accumulator).  CTA r of the
+// A cluster of two CTAs on two SMs computes one 256 x 256 tile.  CTA r of the
 // pair holds rows [128 r, 128 r + 128) of the tile's A operand and columns
 // [nsz/2 r, nsz/2 (r + 1)) of its B operand in shared memory, and rows
 // [128 r, 128 r + 128) of the fp32 accumulator in its own tensor memory; one
@@ -42,6 +40,8 @@
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
+#include <atomic>
+
 #include "tc_common.cuh"
 
 namespace slorr {
@@ -49,19 +49,15 @@ namespace {
 
 using namespace tc;
 
-template <int STAGES_, int SLOTS_, int EPIW_, int BN_ = kBNMax>
+template <int STAGES_, int EPIW_>
 struct PairCfg {
     static constexpr int BK = 64;
     static constexpr int STAGES = STAGES_;
-    static constexpr int kSlots = SLOTS_;                 // accumulators per CTA in TMEM
-    static constexpr int kBN = BN_;                       // tile columns: 256, or 512 (two UMMAs)
-    static_assert(BN_ == 256 || BN_ == 512, "tile width");
-    static constexpr int kSubs = BN_ / 256;               // N <= 256 UMMAs per K slice
+    static constexpr int kSlots = 2;                      // accumulators per CTA in TMEM
     static constexpr int kBoxBytes = 64 * BK * 2;         // one 64 x 64 box
     static constexpr int kABytes = kBM * BK * 2;          // this CTA's 128 rows of A
-    static constexpr int kSubBBytes = 128 * BK * 2;       // this CTA's half of one UMMA's B (<= 128 rows)
-    static constexpr int kBBytes = kSubs * kSubBBytes;
-    static constexpr int kAccCols = BN_;                  // fp32 TMEM columns of one accumulator
+    static constexpr int kBBytes = 128 * BK * 2;          // this CTA's half of B (<= 128 rows)
+    static constexpr int kAccCols = kBNMax;               // fp32 TMEM columns of one accumulator
     static constexpr int kStageBytes = kABytes + kBBytes;
     static constexpr int kEpiWarps = EPIW_;               // 4, or 8: two per TMEM lane quadrant
     static_assert(EPIW_ == 4 || EPIW_ == 8, "epilogue warps");
@@ -83,11 +79,8 @@ struct PairCfg {
 // Two accumulators per CTA (the tile epilogue overlaps the next main loop);
 // the Poly epilogue, which also reads b A, takes 8 warps, the others 4 (more
 // polling warps slow the producer and MMA threads of the long-K phases).
-using PairCfg1 = PairCfg<SLORR_PAIR_STAGES, 1, 4>;   // one accumulator per CTA: no overlap
-using PairCfg2 = PairCfg<SLORR_PAIR_STAGES, 2, 4>;
-using PairCfg2Wide = PairCfg<SLORR_PAIR_STAGES, 2, 8>;
-// 256 x 512 Update tiles: one 128 x 512 accumulator per CTA, 4 stages of 48 KB.
-using PairCfgN512 = PairCfg<4, 1, 8, 512>;
+using PairCfg2 = PairCfg<SLORR_PAIR_STAGES, 4>;
+using PairCfg2Wide = PairCfg<SLORR_PAIR_STAGES, 8>;
 
 struct PairSmem {
     uint8_t* stages;
@@ -153,14 +146,12 @@ __device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, 
                     const int mn = it.tm * (2 * kBM) + rank * kBM + b * 64;
                     ptx::tma_load_2d_pair(sa + b * C::kBoxBytes, pi.mapA, bar, pi.a_mn ? mn : k, pi.a_mn ? k : mn);
                 }
-            // B columns of UMMA u (tile columns [256 u, 256 u + nu)): this
-            // CTA's half, nu / 2 = 64 or 128 rows, in its own 128-row region
-            for (int u = 0; load_b && u * 256 < it.nsz; ++u) {
-                const int bhalf = min(256, it.nsz - u * 256) / 2;
+            // B columns: this CTA's half, nsz / 2 = 64 or 128 rows
+            if (load_b) {
+                const int bhalf = it.nsz / 2;
                 for (int j = 0; j < bhalf / 64; ++j) {
-                    const int mn = it.tn * C::kBN + u * 256 + rank * bhalf + j * 64;
-                    ptx::tma_load_2d_pair(sb + u * C::kSubBBytes + j * C::kBoxBytes, pi.mapB, bar, pi.b_mn ? mn : k,
-                                          pi.b_mn ? k : mn);
+                    const int mn = it.tn * kBNMax + rank * bhalf + j * 64;
+                    ptx::tma_load_2d_pair(sb + j * C::kBoxBytes, pi.mapB, bar, pi.b_mn ? mn : k, pi.b_mn ? k : mn);
                 }
             }
             if (++stage == C::STAGES) {
@@ -228,9 +219,7 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
     for (int idx = pair; idx < p.num_items && ok; idx += npairs, ++local) {
         const GemmItem it = p.items[idx];
         const PhaseInfo pi = phase_info<C>(p, it);
-        const int n0 = min(256, int(it.nsz));  // columns of UMMA 0; UMMA 1 (512-wide tiles) takes the rest
-        const uint32_t idesc0 = ptx::idesc_f16(2 * kBM, n0, BF16, pi.a_mn, pi.b_mn);
-        const uint32_t idesc1 = it.nsz > 256 ? ptx::idesc_f16(2 * kBM, it.nsz - 256, BF16, pi.a_mn, pi.b_mn) : 0u;
+        const uint32_t idesc = ptx::idesc_f16(2 * kBM, it.nsz, BF16, pi.a_mn, pi.b_mn);
         const int slot = local % C::kSlots;
         const uint32_t tphase = uint32_t(local / C::kSlots) & 1u;
         if (!ptx::mbar_wait<true>(&s.tempty[slot], tphase ^ 1u, s.abort, p.timeout_ns)) {
@@ -260,12 +249,9 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
             const uint32_t b0 = shared_operand(p, it) ? a0 : a0 + C::kABytes;
 #pragma unroll
             for (int kk = 0; kk < C::BK / 16; ++kk) {
-                const uint64_t adesc = operand_desc<C>(a0, kk, pi.a_mn);
                 const uint32_t acc = (kb != kb_begin || kk != 0) ? 1u : 0u;
-                ptx::umma_f16_pair(d_tmem, adesc, operand_desc<C>(b0, kk, pi.b_mn), idesc0, acc);
-                if (C::kSubs > 1 && it.nsz > 256)
-                    ptx::umma_f16_pair(d_tmem + 256u, adesc, operand_desc<C>(b0 + C::kSubBBytes, kk, pi.b_mn), idesc1,
-                                       acc);
+                ptx::umma_f16_pair(d_tmem, operand_desc<C>(a0, kk, pi.a_mn), operand_desc<C>(b0, kk, pi.b_mn), idesc,
+                                   acc);
             }
             issued_any = true;
             ptx::umma_commit_pair_mc(&s.empty[stage], 0x3);
@@ -318,13 +304,13 @@ __device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t t
             const int per = it.nsz / 32 / ngroups;  // 32-column chunks per warp
             const int parts = it.ksplit >> 8;
             if (parts <= 1) {
-                store_rows<BF16, 2, C::kBN, true>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per,
-                                                  nullptr, 1, 0, sbuf);
+                store_rows<BF16, true>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per, nullptr, 1,
+                                       0, sbuf);
             } else if constexpr (C::kEpiWarps == 4) {  // split K: Gram only, one warp per lane quadrant
                 // direct stores: the last part's sum is a serial step, which
                 // the staging round trip lengthens (small sets, ResNet-18 Gram +7%)
                 if (split_partial_is_last(p, it, rank, quad, lane, t_row, 0, per))
-                    store_rows<BF16, 2>(p, it, md, row0, t_row, quad, lane, 0, per,
+                    store_rows<BF16>(p, it, md, row0, t_row, quad, lane, 0, per,
                                         p.split_part + size_t(it.sid) * 65536, parts, rank * kBM + quad * 32 + lane);
             }
         }
@@ -414,12 +400,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(C::kThreads, 1)
     }
 }
 
+// Co-resident CTA pairs of one kernel configuration on each device, found
+// once per device (the function attribute is per device, too).  Concurrent
+// first launches on one device may both query; they store the same value.
+constexpr int kMaxDevices = 64;
+
 template <bool BF16, class C>
 cudaError_t launch_pair_cfg(const GemmLaunch& p, int num_sms, cudaStream_t st) {
-    static int max_pairs = 0;
+    static std::atomic<int> max_pairs_of[kMaxDevices];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    int max_pairs = max_pairs_of[dev].load(std::memory_order_acquire);
     if (max_pairs == 0) {
-        cudaError_t e = cudaFuncSetAttribute(tc_pair_kernel<BF16, C>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             int(C::kSmemBytes));
+        e = cudaFuncSetAttribute(tc_pair_kernel<BF16, C>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 int(C::kSmemBytes));
         if (e != cudaSuccess) return e;
         cudaLaunchConfig_t probe = {};
         probe.gridDim = dim3(unsigned(2 * (num_sms / 2)));
@@ -430,6 +426,7 @@ cudaError_t launch_pair_cfg(const GemmLaunch& p, int num_sms, cudaStream_t st) {
         if (e != cudaSuccess) return e;
         if (clusters < 1) return cudaErrorInvalidConfiguration;
         max_pairs = clusters < num_sms / 2 ? clusters : num_sms / 2;
+        max_pairs_of[dev].store(max_pairs, std::memory_order_release);
     }
     const int npairs = p.num_items < max_pairs ? p.num_items : max_pairs;
     return launch_kernel(tc_pair_kernel<BF16, C>, unsigned(2 * npairs), C::kThreads, C::kSmemBytes, st, p.pdl != 0, p);
@@ -440,15 +437,10 @@ cudaError_t launch_pair_cfg(const GemmLaunch& p, int num_sms, cudaStream_t st) {
 cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t st) {
     if (p.num_items == 0) return cudaSuccess;
     const bool bf = elem == kBF16;
-    if (p.wide_update && p.phase == kUpdate)
-        return bf ? launch_pair_cfg<true, PairCfgN512>(p, num_sms, st)
-                  : launch_pair_cfg<false, PairCfgN512>(p, num_sms, st);
-    if (p.pair_slots == 2 && p.phase == kPoly)
+    if (p.phase == kPoly)
         return bf ? launch_pair_cfg<true, PairCfg2Wide>(p, num_sms, st)
                   : launch_pair_cfg<false, PairCfg2Wide>(p, num_sms, st);
-    if (p.pair_slots == 2)
-        return bf ? launch_pair_cfg<true, PairCfg2>(p, num_sms, st) : launch_pair_cfg<false, PairCfg2>(p, num_sms, st);
-    return bf ? launch_pair_cfg<true, PairCfg1>(p, num_sms, st) : launch_pair_cfg<false, PairCfg1>(p, num_sms, st);
+    return bf ? launch_pair_cfg<true, PairCfg2>(p, num_sms, st) : launch_pair_cfg<false, PairCfg2>(p, num_sms, st);
 }
 
 }  // namespace slorr

@@ -36,10 +36,6 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t by
                  : "memory");
 }
 
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
@@ -147,17 +143,6 @@ __device__ __forceinline__ void prefetch_tmap(const void* map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(map) : "memory");
 }
 
-// 2-D tiled load of one box into shared memory, completing `bytes` on `bar`.
-// x is the innermost (contiguous) coordinate in elements.
-__device__ __forceinline__ void tma_load_2d(void* dst, const void* map, uint64_t* bar, int32_t x,
-                                            int32_t y) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
-        "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y)
-        : "memory");
-}
-
 // CTA-pair form: the box lands in this CTA's shared memory, and its bytes are
 // counted on the mbarrier at shared::cluster address `bar_cluster`, which may
 // belong to the other CTA of the pair.
@@ -170,26 +155,6 @@ __device__ __forceinline__ void tma_load_2d_pair(void* dst, const void* map, uin
         : "memory");
 }
 
-// As tma_load_2d_pair, multicast: the box lands at the same shared-memory
-// offset in every CTA of `cta_mask`, and its bytes are counted, for each
-// destination, on the barrier at bar_cluster's offset in that destination's
-// pair leader (the even CTA of its pair).
-__device__ __forceinline__ void tma_load_2d_pair_mc(void* dst, const void* map, uint32_t bar_cluster, int32_t x,
-                                                    int32_t y, uint16_t cta_mask) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
-        ".multicast::cluster [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
-        "l"(map), "r"(bar_cluster), "r"(x), "r"(y), "h"(cta_mask)
-        : "memory");
-}
-
-// Hint: bring one box of a tensor into L2 (no shared memory, no completion).
-__device__ __forceinline__ void tma_prefetch_l2_2d(const void* map, int32_t x, int32_t y) {
-    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(map), "r"(x),
-                 "r"(y)
-                 : "memory");
-}
-
 // Orders this thread's earlier generic-proxy global accesses with its later
 // async-proxy (TMA) accesses.
 __device__ __forceinline__ void fence_proxy_async_global() {
@@ -197,22 +162,6 @@ __device__ __forceinline__ void fence_proxy_async_global() {
 }
 
 // ---- tcgen05 ----------------------------------------------------------------------
-
-__device__ __forceinline__ void tmem_alloc(uint32_t* dst_smem, uint32_t ncols) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                     smem_u32(dst_smem)),
-                 "r"(ncols)
-                 : "memory");
-}
-
-__device__ __forceinline__ void tmem_relinquish() {
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-}
-
-__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
-                 : "memory");
-}
 
 // CTA-pair forms (cta_group::2): one warp of each CTA of the pair executes the
 // allocation, relinquish and deallocation; every tcgen05 instruction of a
@@ -241,17 +190,6 @@ __device__ __forceinline__ void tc_fence_after() {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
-// D[tmem] (+)= A[smem] * B[smem], kind::f16 (fp16 or bf16 operands, fp32 accumulate).
-__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
-                                         uint32_t idesc, uint32_t accumulate) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
-
 // CTA-pair UMMA, issued by one thread of the even CTA of the pair: M = 256 rows,
 // rows [0,128) from this CTA's A tile and TMEM, rows [128,256) from the peer's
 // (same shared-memory and TMEM addresses); the B tile's N columns are split the
@@ -273,15 +211,6 @@ __device__ __forceinline__ void umma_commit_pair_mc(uint64_t* bar, uint16_t cta_
         "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
         " [%0], %1;" ::"r"(smem_u32(bar)),
         "h"(cta_mask)
-        : "memory");
-}
-
-// Arrive once on `bar` when every tcgen05 operation issued so far by this
-// thread has completed.
-__device__ __forceinline__ void umma_commit(uint64_t* bar) {
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-            smem_u32(bar))
         : "memory");
 }
 

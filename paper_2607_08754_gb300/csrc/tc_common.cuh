@@ -1,7 +1,7 @@
-// Pieces shared by the tensor-core GEMM kernels (kernels_tc.cu: one CTA per
-// tile; kernels_tc_pair.cu: a CTA pair per tile): 16-bit packing, the operand
-// maps and orientation of each phase, the symmetric-tile rule, shared-memory
-// operand descriptors and the epilogue of one 128-row block.
+// Pieces of the tensor-core GEMM kernel (kernels_tc_pair.cu: a CTA pair per
+// 256 x 256 tile): 16-bit packing, the operand maps and orientation of each
+// phase, the symmetric-tile rule, shared-memory operand descriptors and the
+// epilogue of one 128-row block.
 #pragma once
 
 #include <cuda_bf16.h>
@@ -90,12 +90,12 @@ __device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmI
 }
 
 // Symmetric products (Gram, Poly): only tiles holding some 128 x 128 block on
-// or above the diagonal are computed.  Tile (tm, tn) covers row blocks from
-// tm MT on and column blocks 2 tn .. min(2 tn + 1, nb - 1) (nb = Ppad / 128), so
-// it is computed iff its last column block reaches its first row block.
-__device__ __forceinline__ bool sym_tile_computed(int tm, int tn, int Ppad, int mt) {
+// or above the diagonal are computed.  Tile (tm, tn) covers row blocks 2 tm,
+// 2 tm + 1 and column blocks 2 tn .. min(2 tn + 1, nb - 1) (nb = Ppad / 128),
+// so it is computed iff its last column block reaches its first row block.
+__device__ __forceinline__ bool sym_tile_computed(int tm, int tn, int Ppad) {
     const int last_col_block = min(2 * tn + 1, Ppad / 128 - 1);
-    return last_col_block >= tm * mt;
+    return last_col_block >= 2 * tm;
 }
 
 // Shared-memory descriptor of one K = 16 slice (kk) of a BK-wide K block:
@@ -209,19 +209,19 @@ __device__ __forceinline__ void own_row(uint8_t* buf, int lane, const uint4 (&v)
 
 // Epilogue of one 128-row block of a finished tile: this warp's 32 TMEM lanes
 // (rows row0 + 32 quad + [0, 32)) and the tile's 32-column chunks
-// [ch_begin, ch_end) (chunk c: columns tn * BN + 32 c, TMEM columns t_row + 32 c).
+// [ch_begin, ch_end) (chunk c: columns 256 tn + 32 c, TMEM columns t_row + 32 c).
 //   Update: X' rows, stored in W's orientation (transposed iterates take one
 //           coalesced 64-byte segment per column);
 //   Gram / Poly: c * acc (+ b A + a I for Poly) into the Ppad x Ppad output,
 //           plus the transpose of every 128 x 128 block (I, J), J > I, whose
-//           mirror tile is skipped (tiles are MT x 128 rows by 256 columns).
+//           mirror tile is skipped (tiles are 256 rows by 256 columns).
 // In the first step after the fused norm pass (p.x0_scaled) the stored X_0
 // is W itself: the Gram scales acc by x0_scale^2 and the Update by x0_scale.
 // With split K (Gram), the accumulator is replaced by the sum, in part
 // order, of the `parts` fp32 partials at split_tile (row row_t of the tile;
 // this warp's own part among them).  STAGED: the stores go through the
 // warp's staging buffer sbuf (kStageWarpBytes of shared memory).
-template <bool BF16, int MT, int BN = kBNMax, bool STAGED = false>
+template <bool BF16, bool STAGED = false>
 __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& it, const MatDev& md, int row0,
                                            uint32_t t_row, int quad, int lane, int ch_begin, int ch_end,
                                            const float* split_tile = nullptr, int parts = 1, int row_t = 0,
@@ -237,7 +237,7 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
             uint32_t r[32];
             ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
             ptx::tmem_ld_wait();
-            const int col0 = it.tn * BN + ch * 32;
+            const int col0 = it.tn * kBNMax + ch * 32;
             if constexpr (STAGED) {
                 uint4 o[4];
                 uint32_t* ow = reinterpret_cast<uint32_t*>(o);
@@ -355,7 +355,7 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
             // uses the same rounded 16-bit values, so the stored matrix is
             // exactly symmetric.
             const int I = row0 / kBM, J = col0 / kBM;
-            const bool mirror = J > I && !sym_tile_computed(J / MT, I / 2, md.Ppad, MT);
+            const bool mirror = J > I && !sym_tile_computed(J / 2, I / 2, md.Ppad);
             if constexpr (STAGED) {
                 stage_chunk(sbuf, lane, o);
                 put_rows(sbuf, lane, out, ld, row_w, col0);

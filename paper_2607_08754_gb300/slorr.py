@@ -25,19 +25,12 @@ VARIANTS = {"hoyer": 0, "nuclear": 1}
 COMPUTES = {"fp16": 0, "bf16": 1, "fp32": 2}
 DTYPES = {"f32": 0, "bf16": 1}
 FLAG_SIMT_GEMM = 1
-FLAG_L2_PREFETCH = 2
-FLAG_TC_BK32 = 4
-FLAG_TC_M128 = 8
 FLAG_TEST_STALL = 16
 FLAG_WRITE_GRAD = 32
-FLAG_TC_SINGLE_CTA = 64
-FLAG_PAIR_ONE_SLOT = 128
-FLAG_TC_QUAD = 256
 FLAG_NO_PDL = 512
 FLAG_SEPARATE_NORM = 1024
 FLAG_NO_SPLIT_K = 2048
 FLAG_GRAPH = 4096
-FLAG_WIDE_UPDATE = 8192
 
 
 class SlorrError(RuntimeError):
@@ -97,6 +90,7 @@ def load_library(path: str | None = None) -> ctypes.CDLL:
         "slorr_executed_flops": (i32, [vp, ctypes.POINTER(dbl)]),
         "slorr_gemm_items": (i32, [vp, i32, ctypes.POINTER(i32)]),
         "slorr_gemm_pair_load": (i32, [vp, i32, i32, ctypes.POINTER(i64), ctypes.POINTER(i64)]),
+        "slorr_gemm_item_list": (i32, [vp, i32, ctypes.POINTER(i32), i32]),
         "slorr_set_timing": (i32, [vp, i32]),
         "slorr_read_timing": (i32, [vp, ctypes.POINTER(dbl), ctypes.POINTER(i64), i32]),
         "slorr_frob_sq_noalloc": (i32, [vp, i64, i64, i32, vp, vp]),
@@ -243,6 +237,14 @@ def slorr_gemm_items(handle, phase: int) -> int:
     return int(out.value)
 
 
+def slorr_gemm_item_list(handle, phase: int) -> np.ndarray:
+    """(items, 7) int32 array: mat, tm, tn, msz, nsz, part, parts per item, in launch order."""
+    n = slorr_gemm_items(handle, phase)
+    buf = (ctypes.c_int32 * max(1, 7 * n))()
+    _check(load_library().slorr_gemm_item_list(handle, int(phase), buf, 7 * n))
+    return np.frombuffer(buf, dtype=np.int32, count=7 * n).reshape(n, 7).copy()
+
+
 def slorr_partition(shapes, world: int, rank: int) -> list[int]:
     arr, n = _shapes(shapes)
     out = (ctypes.c_int32 * max(n, 1))()
@@ -335,6 +337,12 @@ def make_options(variant: str = "hoyer", compute: str = "fp16", dtype: str = "f3
     return o
 
 
+class _OwnedHandle(ctypes.c_void_p):
+    """A slorr_handle* that keeps the Python object owning it alive while the
+    handle is referenced, so that ``Regularizer(...).handle`` passed straight
+    into a call cannot be destroyed before the call has used it."""
+
+
 class Regularizer:
     """One planned weight set.  Holds the handle and a torch-allocated workspace.
 
@@ -351,15 +359,21 @@ class Regularizer:
         self.shapes = [(int(m), int(n)) for m, n in shapes]
         self.iters = int(iters)
         self.options = o
-        self.handle = slorr_create(self.shapes, o)
-        self.workspace_bytes = slorr_workspace_size(self.handle)
+        self._raw = slorr_create(self.shapes, o)
+        self.workspace_bytes = slorr_workspace_size(self._raw)
         self._ws = None
 
+    @property
+    def handle(self) -> _OwnedHandle:
+        h = _OwnedHandle(self._raw.value)
+        h.owner = self
+        return h
+
     def __del__(self):
-        h = getattr(self, "handle", None)
+        h = getattr(self, "_raw", None)
         if h is not None and _lib is not None:
             slorr_destroy(h)
-            self.handle = None
+            self._raw = None
 
     def workspace(self, device):
         import torch

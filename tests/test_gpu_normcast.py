@@ -27,7 +27,11 @@ torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
 EPS = 1e-7
-TOL = {"fp16": (2e-2, 2e-2), "bf16": (2e-2, 5e-2)}
+TOL = {"fp16": (2e-2, 2e-2), "bf16": (2e-2, 2e-2)}
+# bf16-operand SLORR-Hoyer gradients do not meet the 2e-2 target (2.1e-2 to
+# 4.1e-2 measured on the paper-shaped sets; tests/test_gpu_parity.py's module
+# docstring gives the reason): they are held to their measured floor with margin
+BF16_HOYER_GRAD = 5e-2
 SHAPES = [(256, 768), (768, 256), (130, 700), (64, 147), (1000, 130), (384, 384)]
 
 
@@ -58,6 +62,8 @@ def run(Ws, compute, flags=0, variant="hoyer"):
 def check_oracle(Ws, out, compute, variant="hoyer"):
     loss, per, grads = out[:3]
     tl, tg = TOL[compute]
+    if compute == "bf16" and variant == "hoyer":
+        tg = BF16_HOYER_GRAD
     W64 = [W.astype(np.float32).astype(np.float64) for W in Ws]
     ref_loss, ref_per, ref_inc = oracle.reg_forward_backward(W64, variant, oracle.pe_coefficients(6), 1.0, EPS)
     assert abs(loss - ref_loss) <= tl * abs(ref_loss)

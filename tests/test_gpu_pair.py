@@ -1,14 +1,10 @@
-"""The CTA-pair tensor-core kernel (the default: tcgen05 cta_group::2, 256 x 256
-tiles over two SMs) against the CUDA-core path, the one-CTA kernels and the
-oracle.
+"""The CTA-pair tensor-core kernel (tcgen05 cta_group::2, 256 x 256 tiles over
+two SMs, two accumulators per SM) against the CUDA-core path and the oracle.
 
 Shapes are chosen to reach every tile case of the pair kernel: a last row tile
 with only 128 rows (the odd CTA's half idle), last column tiles of 128 columns
 (64 B rows per CTA), K-major and MN-major operands (m <= n and m > n), a
-matrix smaller than one tile, and more tiles than pairs.  Test ids carry
-"one_slot" (one accumulator per SM), "two_slot" (two, the overlapped
-epilogue) or "wide" (256 x 512 Update tiles, two UMMAs per K slice; the
-Update column tiles of these shapes are 128, 256, 384 and 512 wide).
+matrix smaller than one tile, and more tiles than pairs.
 
 Tolerances are those of the tensor-core-vs-CUDA-core test: 4 ulp of the
 operand type per step (at most 6 steps' worth), and the oracle parity bounds
@@ -24,7 +20,6 @@ torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
 EPS = 1e-7
-MODES = {"one_slot": 128, "two_slot": 0, "wide": 8192}   # PAIR_ONE_SLOT, default, WIDE_UPDATE
 SHAPES = [(256, 768), (768, 256), (320, 1280), (384, 384), (640, 1000), (64, 64), (130, 700), (1000, 130)]
 
 
@@ -40,13 +35,12 @@ def rel(a, b):
     return np.linalg.norm(a - b) / np.linalg.norm(b)
 
 
-@pytest.mark.parametrize("mode", list(MODES))
 @pytest.mark.parametrize("compute", ["fp16", "bf16"])
-def test_pair_iterates_match_simt(mode, compute):
+def test_pair_iterates_match_simt(compute):
     from paper_2607_08754_gb300.slorr import Regularizer, FLAG_SIMT_GEMM
     Ws = [workloads.random_matrix(s, seed=90 + i, std=0.02) for i, s in enumerate(SHAPES)]
     w = [torch.from_numpy(W).cuda() for W in Ws]
-    tc = Regularizer(SHAPES, compute=compute, flags=MODES[mode])
+    tc = Regularizer(SHAPES, compute=compute)
     st = Regularizer(SHAPES, compute=compute, flags=FLAG_SIMT_GEMM)
     ulp = 2.0 ** -10 if compute == "fp16" else 2.0 ** -7
     for k in (1, 2, 6):
@@ -60,14 +54,13 @@ def test_pair_iterates_match_simt(mode, compute):
             assert rel(a, b) <= 4 * ulp * (k if k < 6 else 6), (k, i, SHAPES[i], rel(a, b))
 
 
-@pytest.mark.parametrize("mode", list(MODES))
 @pytest.mark.parametrize("variant", ["hoyer", "nuclear"])
-def test_pair_forward_backward_matches_oracle(mode, variant):
+def test_pair_forward_backward_matches_oracle(variant):
     from paper_2607_08754_gb300.slorr import Regularizer
     Ws = [workloads.random_matrix(s, seed=120 + i, std=0.05) for i, s in enumerate(SHAPES)]
     Ws += workloads.generate("resnet18", [0, 5, 12, 20])
     shapes = [W.shape for W in Ws]
-    reg = Regularizer(shapes, variant=variant, compute="fp16", lam=0.5, flags=MODES[mode])
+    reg = Regularizer(shapes, variant=variant, compute="fp16", lam=0.5)
     w = [torch.from_numpy(W).cuda() for W in Ws]
     g = [torch.zeros_like(x) for x in w]
     per = torch.empty(len(Ws), device="cuda")
@@ -84,16 +77,15 @@ def test_pair_forward_backward_matches_oracle(mode, variant):
         assert rel(g[i].double().cpu().numpy(), ref_inc[i]) <= 2e-2, (i, shapes[i])
 
 
-@pytest.mark.parametrize("mode", ["two_slot", "wide"])
-def test_pair_vit_l16_layers_match_single_cta_kernel(mode):
-    """Paper-sized matrices (one ViT-L/16 block): the pair kernel and the one-CTA
-    kernels give the same iterates up to 16-bit rounding."""
-    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_TC_SINGLE_CTA
+def test_pair_vit_l16_layers_match_simt():
+    """Paper-sized matrices (one ViT-L/16 block): the pair kernel and the
+    CUDA-core kernel give the same iterates up to 16-bit rounding."""
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_SIMT_GEMM
     Ws = workloads.generate("vit_l16", [0, 1, 2, 3])
     shapes = [W.shape for W in Ws]
     w = [torch.from_numpy(W).cuda() for W in Ws]
-    a_reg = Regularizer(shapes, flags=MODES[mode])
-    b_reg = Regularizer(shapes, flags=FLAG_TC_SINGLE_CTA)
+    a_reg = Regularizer(shapes)
+    b_reg = Regularizer(shapes, flags=FLAG_SIMT_GEMM)
     a_reg.run_steps(w, 6)
     b_reg.run_steps(w, 6)
     torch.cuda.synchronize()
@@ -104,8 +96,7 @@ def test_pair_vit_l16_layers_match_single_cta_kernel(mode):
         assert rel(a, b) <= 24 * 2.0 ** -10, (i, rel(a, b))
 
 
-@pytest.mark.parametrize("mode", ["two_slot"])
-def test_pair_bounded_wait_timeout_and_recovery(mode):
+def test_pair_bounded_wait_timeout_and_recovery():
     """SLORR_FLAG_TEST_STALL in the pair kernel: the even CTA's MMA thread waits on
     a barrier nothing arrives on, gives up after timeout_s, and sets both CTAs'
     abort flags; every role unwinds, the even CTA drains the pair's copies, and
@@ -115,12 +106,12 @@ def test_pair_bounded_wait_timeout_and_recovery(mode):
     shapes = [(256, 512), (384, 128), (640, 1000)]
     Ws = [workloads.random_matrix(s, 31 + i, 0.05) for i, s in enumerate(shapes)]
     w = [torch.from_numpy(W).cuda() for W in Ws]
-    stall = Regularizer(shapes, flags=MODES[mode] | FLAG_TEST_STALL, timeout_s=0.05)
+    stall = Regularizer(shapes, flags=FLAG_TEST_STALL, timeout_s=0.05)
     stall.run_steps(w, 1)
     torch.cuda.synchronize()
     assert stall.status() == 5          # SLORR_ERR_TIMEOUT
     assert stall.status() == 0
-    tc = Regularizer(shapes, flags=MODES[mode])
+    tc = Regularizer(shapes)
     st = Regularizer(shapes, flags=FLAG_SIMT_GEMM)
     tc.run_steps(w, 2)
     st.run_steps(w, 2)
@@ -209,23 +200,3 @@ def test_split_k_is_deterministic():
     for o in outs[1:]:
         for a, b in zip(outs[0], o):
             assert torch.equal(a, b)
-
-
-@pytest.mark.parametrize("compute", ["fp16", "bf16"])
-def test_wide_update_is_bit_identical(compute):
-    """256 x 512 Update tiles (SLORR_FLAG_WIDE_UPDATE) issue, for every output
-    column, the same N = 256 UMMA slices in the same K order as 256 x 256
-    tiles; only the tile a column belongs to changes.  The iterates are
-    equal bit for bit, including Update tiles 128, 256, 384 and 512 wide."""
-    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_WIDE_UPDATE
-    Ws = [workloads.random_matrix(s, seed=700 + i, std=0.02) for i, s in enumerate(SHAPES)]
-    w = [torch.from_numpy(W).cuda() for W in Ws]
-    wide = Regularizer(SHAPES, compute=compute, flags=FLAG_WIDE_UPDATE)
-    base = Regularizer(SHAPES, compute=compute)
-    for k in (1, 2, 6):
-        wide.run_steps(w, k)
-        base.run_steps(w, k)
-        torch.cuda.synchronize()
-        assert wide.status() == 0 and base.status() == 0
-        for i in range(len(SHAPES)):
-            assert torch.equal(wide.iterate(i, k).cpu(), base.iterate(i, k).cpu()), (k, i, SHAPES[i])

@@ -2,13 +2,20 @@
 seeded inputs (Sec. 3, Eq. 1, Listing 1, Alg. 2).
 
 Tolerances (relative, on the loss and on each matrix's gradient in Frobenius
-norm):
+norm), the stated targets:
 * fp32 compute mode: 1e-5;
 * fp16-operand mode (tensor cores, the default): 2e-2;
-* bf16-operand mode: 2e-2 on the loss, 5e-2 on the gradient.  bf16 keeps 8
-  significand bits against fp16's 11, and the measured fp16 gradient errors on
-  the paper-shaped sets stay below 4.5e-3, so 8 x that bound (3.6e-2) plus
-  margin gives 5e-2; the loss is a smooth trace and stays within 2e-2.
+* bf16-operand mode: 2e-2.
+Weights and gradients stored in bf16 add one rounding of the stored gradient
+(2^-9 relative).
+
+One exception, which does NOT meet the 2e-2 target: the SLORR-Hoyer gradient
+with bf16 operands.  It is the difference of two nearly equal terms, and
+rounding the iterate to bf16 (8 significand bits) after every step leaves
+2.1e-2 to 4.1e-2 on the paper-shaped sets (fp16, 11 bits, at the same tensor
+rate: 2.7e-3 to 5.1e-3).  Those gradients are held to BF16_HOYER_GRAD = 5e-2,
+their measured floor with margin, so that the option stays tested; the bf16
+loss and the bf16 SLORR-Nuc gradient are held to 2e-2.
 
 The Hoyer gradient is the difference of two terms, 2 reg P_hat / frob and
 2 reg n_hat W / frob^3 (Listing 1).  When they cancel almost completely (rank
@@ -26,8 +33,14 @@ import workloads
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
-TOL = {"fp32": (1e-5, 1e-5), "fp16": (2e-2, 2e-2), "bf16": (2e-2, 5e-2)}
+TOL = {"fp32": (1e-5, 1e-5), "fp16": (2e-2, 2e-2), "bf16": (2e-2, 2e-2)}
+BF16_HOYER_GRAD = 5e-2   # outside the 2e-2 target: see the module docstring
+BF16_STORAGE = 2.0 ** -9  # one rounding of a gradient stored in bf16
 EPS = 1e-7
+
+
+def grad_tol(compute, variant):
+    return BF16_HOYER_GRAD if (compute == "bf16" and variant == "hoyer") else TOL[compute][1]
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -82,7 +95,7 @@ def check(Ws, variant, compute, lam=1.0, grad_scale=1.0, dtype="f32", iters=6, g
     assert status == 0
     co = oracle.pe_coefficients(T=iters)
     ref_loss, ref_per, ref_inc = oracle.reg_forward_backward(w_used, variant, co, lam, EPS, grad_scale)
-    tl, tg = TOL[compute]
+    tl, tg = TOL[compute][0], grad_tol(compute, variant)
     assert abs(loss - ref_loss) <= tl * abs(ref_loss) + 1e-6, (loss, ref_loss)
     for i in range(len(Ws)):
         assert abs(per[i] - ref_per[i]) <= tl * abs(ref_per[i]) + 1e-6, (i, per[i], ref_per[i])
@@ -91,7 +104,7 @@ def check(Ws, variant, compute, lam=1.0, grad_scale=1.0, dtype="f32", iters=6, g
         err = grad_err(grads[i] - base, ref_inc[i], w_used[i], variant, lam, grad_scale)
         if dtype == "bf16":
             # the accumulated gradient is stored in bf16: one extra rounding
-            assert err <= tg + 8e-3, (i, err)
+            assert err <= tg + BF16_STORAGE, (i, err)
         else:
             assert err <= tg, (i, err)
             assert np.all(np.isfinite(grads[i])) and grads[i].shape == ref_g.shape
@@ -162,13 +175,11 @@ def test_decoder_560m_layer_fp16():
 
 # ---- tensor cores vs CUDA cores on the same 16-bit arithmetic -------------------
 
-@pytest.mark.parametrize("compute,flags", [("fp16", 0), ("bf16", 0), ("fp16", 64), ("bf16", 64), ("fp16", 4),
-                                           ("fp16", 8), ("bf16", 8)])
+@pytest.mark.parametrize("compute,flags", [("fp16", 0), ("bf16", 0), ("fp16", 2048)])
 def test_tensor_core_iterates_match_simt(compute, flags):
-    """Default: the CTA-pair kernel (256 x 256 tiles); 64 = SLORR_FLAG_TC_SINGLE_CTA
-    (one-CTA kernels: 256 x 256 Gram/Update, 128 x 256 Poly); 4 =
-    SLORR_FLAG_TC_BK32 (9-stage, 64-byte-swizzle pipeline); 8 =
-    SLORR_FLAG_TC_M128 (128 x 256 tiles everywhere)."""
+    """The CTA-pair tensor-core kernel (256 x 256 tiles; 2048 =
+    SLORR_FLAG_NO_SPLIT_K) against the CUDA-core kernel on the same 16-bit
+    iterates."""
     from paper_2607_08754_gb300.slorr import Regularizer, FLAG_SIMT_GEMM
     shapes = [(256, 768), (768, 256), (320, 1280), (384, 384), (640, 1000)]
     Ws = [workloads.random_matrix(s, seed=70 + i, std=0.02) for i, s in enumerate(shapes)]
@@ -273,7 +284,7 @@ def full_set_sampled(name, samples, variant="hoyer", compute="fp16"):
     per = per.double().cpu().numpy()
     assert loss == pytest.approx(per.sum(), rel=1e-6)
     co = oracle.pe_coefficients(6)
-    tl, tg = TOL[compute]
+    tl, tg = TOL[compute][0], grad_tol(compute, variant)
     for i in samples:
         W = workloads.generate_one(name, i).astype(np.float64)
         L, G, _, _ = oracle.reg_single(W, variant, co, EPS)
@@ -295,6 +306,20 @@ def test_vit_b16_full_size_sampled_bf16():
     full_set_sampled("vit_b16", (0, 1, 2, 3, 47), compute="bf16")
 
 
+def test_vit_l16_full_size_sampled_nuclear():
+    """ViT-L/16 set, SLORR-Nuc (the configuration names Hoyer and nuclear)."""
+    full_set_sampled("vit_l16", (0, 1, 2, 3, 93), variant="nuclear")
+
+
+@pytest.mark.parametrize("variant", ["hoyer", "nuclear"])
+def test_vit_l16_full_size_sampled_bf16(variant):
+    full_set_sampled("vit_l16", (0, 1, 2, 3, 95), variant=variant, compute="bf16")
+
+
+def test_decoder_560m_full_size_sampled_bf16():
+    full_set_sampled("decoder_560m", (0, 1, 2, 4, 6, 164), compute="bf16")
+
+
 # ---- failure detection: a bounded device wait runs out -----------------------------
 
 def test_bounded_wait_timeout_reports_status_and_context_survives():
@@ -302,11 +327,10 @@ def test_bounded_wait_timeout_reports_status_and_context_survives():
     arrives on; with timeout_s = 0.05 each wait gives up, the kernel records
     SLORR_ERR_TIMEOUT in the status word, drains and returns.  The same process
     then runs a normal call that must still match the oracle."""
-    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_TEST_STALL, FLAG_TC_SINGLE_CTA
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_TEST_STALL
     Ws = [workloads.random_matrix((256, 512), 21, 0.05), workloads.random_matrix((384, 128), 22, 0.05)]
     w = [torch.from_numpy(W).cuda() for W in Ws]
-    # the one-CTA kernel here; tests/test_gpu_pair.py stalls the pair kernel
-    stall = Regularizer([W.shape for W in Ws], flags=FLAG_TEST_STALL | FLAG_TC_SINGLE_CTA, timeout_s=0.05)
+    stall = Regularizer([W.shape for W in Ws], flags=FLAG_TEST_STALL, timeout_s=0.05)
     stall.run_steps(w, 1)
     torch.cuda.synchronize()
     assert stall.status() == 5          # SLORR_ERR_TIMEOUT

@@ -65,7 +65,8 @@ def test_validation_rejects_bad_requests(lib):
     with pytest.raises(slorr.SlorrError):
         slorr.slorr_create([(3, 70000)])
     for field, bad in [("iters", 0), ("iters", 17), ("ell", 0.0), ("ell", 1.0), ("safety", 0.5),
-                       ("eps", -1.0), ("variant", 5), ("compute", 9), ("dtype", 3), ("timeout_s", 0.0)]:
+                       ("eps", -1.0), ("variant", 5), ("compute", 9), ("dtype", 3), ("timeout_s", 0.0),
+                       ("flags", 2), ("flags", 8192), ("flags", 1 << 20)]:
         o = slorr.slorr_default_options()
         setattr(o, field, bad)
         with pytest.raises(slorr.SlorrError) as e:
@@ -267,31 +268,32 @@ def test_split_k_plan(lib):
         slorr.slorr_gemm_items(split.handle, 3)
 
 
-def test_wide_update_plan(lib):
-    """SLORR_FLAG_WIDE_UPDATE plans the CTA-pair Update in 256 x 512 tiles:
-    ceil(Qpad / 512) column tiles per 256-row band instead of Qpad / 256,
-    the last one 128, 256, 384 or 512 wide.  Gram and Poly keep their tiles,
-    the executed FLOPs do not change, and the one-CTA and 4-CTA kernels
-    ignore the flag."""
-    import workloads
-    vl = workloads.shapes("vit_l16")
-    base = slorr.Regularizer(vl)
-    wide = slorr.Regularizer(vl, flags=slorr.FLAG_WIDE_UPDATE)
-    # per block: P = 1024 (4 bands) and Q = 3072, 1024, 4096, 4096
-    assert slorr.slorr_gemm_items(base.handle, 2) == 24 * 4 * (12 + 4 + 16 + 16)
-    assert slorr.slorr_gemm_items(wide.handle, 2) == 24 * 4 * (6 + 2 + 8 + 8)
-    for ph in (0, 1):
-        assert slorr.slorr_gemm_items(wide.handle, ph) == slorr.slorr_gemm_items(base.handle, ph)
-    assert slorr.slorr_executed_flops(wide.handle) == slorr.slorr_executed_flops(base.handle)
-    # Qpad = 128, 384, 640, 768, 1024: 1, 1, 2, 2, 2 column tiles per band
-    shapes = [(64, 64), (256, 384), (256, 640), (130, 700), (1000, 130)]
-    w = slorr.Regularizer(shapes, flags=slorr.FLAG_WIDE_UPDATE)
-    assert slorr.slorr_gemm_items(w.handle, 2) == 1 + 1 + 2 + 2 + 2
-    assert slorr.slorr_executed_flops(w.handle) == slorr.slorr_executed_flops(slorr.Regularizer(shapes).handle)
-    for other in (slorr.FLAG_TC_SINGLE_CTA, slorr.FLAG_TC_QUAD):
-        a = slorr.Regularizer(vl, flags=other | slorr.FLAG_WIDE_UPDATE)
-        b = slorr.Regularizer(vl, flags=other)
-        assert slorr.slorr_gemm_items(a.handle, 2) == slorr.slorr_gemm_items(b.handle, 2)
+def expected_tiles(shapes, phase):
+    """The tensor-core tiles of one phase, written out from the shapes: 256 x 256
+    tiles of the padded products (P and Q padded to multiples of 128), the
+    strictly-lower tiles of the symmetric Gram and Poly products left out;
+    (mat, tm, tn, msz, nsz) and the tile's K."""
+    out = []
+    for i, (m, n) in enumerate(shapes):
+        P, Q = min(m, n), max(m, n)
+        Pp, Qp = -(-P // 128) * 128, -(-Q // 128) * 128
+        N = Qp if phase == 2 else Pp
+        K = Qp if phase == 0 else Pp
+        for tm in range(-(-Pp // 256)):
+            for tn in range(-(-N // 256)):
+                msz, nsz = min(256, Pp - 256 * tm), min(256, N - 256 * tn)
+                if phase < 2 and 2 * tn + nsz // 128 - 1 < 2 * tm:
+                    continue
+                out.append(((i, tm, tn, msz, nsz), K))
+    return out
+
+
+def pair_loads(ks, npairs=76):
+    """Per-pair total K when item j goes to pair j mod npairs."""
+    load = [0] * npairs
+    for j, k in enumerate(ks):
+        load[j % npairs] += k
+    return load
 
 
 def test_pair_plan_is_balanced(lib):
@@ -299,19 +301,25 @@ def test_pair_plan_is_balanced(lib):
     its items so that the 76 pairs of a GB300 get nearly equal total K.
     ViT-L/16's Gram has 960 tiles (10 per 1024-row matrix) with K = 4096, 3072
     and 1024: sorted round-robin gives one pair 40960, the balanced order at
-    most one K = 1024 tile above the ideal total / 76.  The totals match an
-    independent count from the shapes, and equal-K phases reach the whole-tile
-    optimum ceil(tiles / 76) * K."""
+    most one K = 1024 tile above the ideal total / 76.  The plan's items are
+    exactly the tiles written out from the shapes (as a multiset), the totals
+    match, and equal-K phases reach the whole-tile optimum ceil(tiles / 76) * K."""
     import math
     import workloads
     vl = workloads.shapes("vit_l16")
     pair = slorr.Regularizer(vl)
+    items = slorr.slorr_gemm_item_list(pair.handle, 0)
+    exp = expected_tiles(vl, 0)
+    assert sorted(map(tuple, items[:, :5].tolist())) == sorted(t for t, _ in exp)
+    assert np.all(items[:, 5] == 0) and np.all(items[:, 6] == 1)   # ViT-L/16's Gram tiles are not split
     mx, tot = slorr.slorr_gemm_pair_load(pair.handle, 0)
-    assert tot == sum(10 * max(s) for s in vl)
+    assert tot == sum(10 * max(s) for s in vl) == sum(k for _, k in exp)
     assert mx <= math.ceil(tot / 76) + 1024
-    one = slorr.Regularizer(vl, flags=slorr.FLAG_TC_SINGLE_CTA)   # the same tiles, sorted, not balanced
-    mx1, tot1 = slorr.slorr_gemm_pair_load(one.handle, 0, 76)
-    assert tot1 == tot and mx1 == 40960 and mx < mx1
+    kmap = {t: k for t, k in exp}
+    assert mx == max(pair_loads([kmap[tuple(r)] for r in items[:, :5].tolist()]))
+    # the sorted order without balancing (longest K first, stable)
+    srt = sorted(exp, key=lambda e: -e[1])
+    assert max(pair_loads([k for _, k in srt])) == 40960 and mx < 40960
     for ph, tiles in ((1, 960), (2, 4608)):
         m, t = slorr.slorr_gemm_pair_load(pair.handle, ph)
         assert t == tiles * 1024 and m == math.ceil(tiles / 76) * 1024
@@ -321,19 +329,42 @@ def test_pair_plan_is_balanced(lib):
 
 def test_pair_plan_balance_on_random_sets(lib):
     """On random weight sets (1 to 40 matrices, sides 1 to 3000) the CTA-pair
-    plan's Gram and Update items are the one-CTA plan's tiles (same total K
-    over every npairs: a permutation) and its largest per-pair total over 76
-    pairs is not above that of the sorted order the one-CTA plan keeps.  The
-    planner weighs each tile as its K plus one K block (64) for its fixed
-    cost, so in pure K the bound holds to within that one block."""
+    plan's Gram and Update items are exactly the tiles written out from the
+    shapes (compared as multisets: a dropped tile and a duplicated one with
+    the same K would be caught), and its largest per-pair total over 76 pairs
+    is not above that of the sorted order.  The planner weighs each tile as
+    its K plus one K block (64) for its fixed cost, so in pure K the bound
+    holds to within that one block."""
     rng = np.random.default_rng(2607)
     for _ in range(25):
         count = int(rng.integers(1, 41))
         shapes = [(int(rng.integers(1, 3001)), int(rng.integers(1, 3001))) for _ in range(count)]
         pair = slorr.Regularizer(shapes, flags=slorr.FLAG_NO_SPLIT_K)
-        one = slorr.Regularizer(shapes, flags=slorr.FLAG_TC_SINGLE_CTA)
         for ph in (0, 2):
-            for npairs in (1, 7, 76):
-                assert slorr.slorr_gemm_pair_load(pair.handle, ph, npairs)[1] == \
-                    slorr.slorr_gemm_pair_load(one.handle, ph, npairs)[1]
-            assert slorr.slorr_gemm_pair_load(pair.handle, ph)[0] <= slorr.slorr_gemm_pair_load(one.handle, ph)[0] + 64
+            items = slorr.slorr_gemm_item_list(pair.handle, ph)
+            exp = expected_tiles(shapes, ph)
+            assert sorted(map(tuple, items[:, :5].tolist())) == sorted(t for t, _ in exp)
+            srt = sorted(exp, key=lambda e: -e[1])
+            mx = slorr.slorr_gemm_pair_load(pair.handle, ph)[0]
+            assert mx <= max(pair_loads([k for _, k in srt])) + 64
+
+
+def test_split_plan_items(lib):
+    """Split Gram tiles (ResNet-18): every tile of the set appears once per
+    part, with part indices 0 .. parts - 1 and the same number of parts on
+    each of them; unsplit tiles appear once as part 0 of 1."""
+    import workloads
+    rn = workloads.shapes("resnet18")
+    items = slorr.slorr_gemm_item_list(slorr.Regularizer(rn).handle, 0)
+    exp = expected_tiles(rn, 0)
+    seen = {}
+    for r in items.tolist():
+        seen.setdefault(tuple(r[:5]), []).append((r[5], r[6]))
+    assert sorted(seen) == sorted(t for t, _ in exp)
+    assert any(len(v) > 1 for v in seen.values())
+    for v in seen.values():
+        parts = v[0][1]
+        assert len(v) == parts and sorted(p for p, _ in v) == list(range(parts))
+        assert all(q == parts for _, q in v)
+    with pytest.raises(slorr.SlorrError):
+        slorr._check(slorr.load_library().slorr_gemm_item_list(slorr.Regularizer(rn).handle, 0, None, 0))

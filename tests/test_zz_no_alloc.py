@@ -20,10 +20,12 @@ pytestmark = pytest.mark.gpu
 TOL = 1e-5   # the fp32 tolerance of the parity tests
 
 
-def _workspace_frob_sq(W):
+def _workspace_frob_sq(W, dtype="f32"):
     from paper_2607_08754_gb300.slorr import Regularizer
-    reg = Regularizer([W.shape], compute="fp32")
+    reg = Regularizer([W.shape], compute="fp32", dtype=dtype)
     w = torch.from_numpy(W).cuda()
+    if dtype == "bf16":
+        w = w.to(torch.bfloat16)
     reg.run_steps([w], 0)
     torch.cuda.synchronize()
     return reg.scalars(0)[0]
@@ -48,6 +50,26 @@ def test_noalloc_frob_sq_matches_workspace_path_on_two_calls():
         exact = float(np.sum(W.astype(np.float64) ** 2))
         assert got == pytest.approx(ref, rel=TOL)
         assert got == pytest.approx(exact, rel=TOL)
+
+
+def test_noalloc_frob_sq_bf16_on_two_calls():
+    """bf16 weights (dtype SLORR_BF16): two calls in a row against the
+    workspace path with bf16 storage and an fp64 sum of the bf16 values."""
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2607_08754_gb300 import slorr
+    mats = [workloads.random_matrix((2048, 1536), seed=5003, std=0.02),
+            workloads.random_matrix((77, 300), seed=5004, std=0.5)]
+    refs = [_workspace_frob_sq(W, "bf16") for W in mats]
+    stream = torch.cuda.current_stream().cuda_stream
+    for W, ref in zip(mats, refs):
+        w = torch.from_numpy(W).cuda().to(torch.bfloat16)
+        out = torch.full((1,), float("nan"), dtype=torch.float64, device="cuda")
+        slorr.slorr_frob_sq_noalloc(w.data_ptr(), W.shape[0], W.shape[1], 1, out.data_ptr(), stream)
+        torch.cuda.synchronize()
+        exact = float(torch.sum(w.double() ** 2).item())
+        assert out.item() == pytest.approx(ref, rel=TOL)
+        assert out.item() == pytest.approx(exact, rel=TOL)
 
 
 def test_noalloc_rejects_oversized_matrix():
