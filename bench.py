@@ -437,11 +437,11 @@ def main():
 
     if rank == 0:
         pk = peaks()
-        gemm_ms = sum(kt[k][0] for k in ("gram", "poly", "update"))
-        gemm_launches = sum(kt[k][1] for k in ("gram", "poly", "update"))
+        gemm_ms = sum(kt[k][0] for k in ("gram", "poly", "update", "gemm"))
+        gemm_launches = sum(kt[k][1] for k in ("gram", "poly", "update", "gemm"))
         launches = sum(v[1] for v in kt.values())  # the same launches as the headline timed region
         per_launch_ms = gemm_ms / max(gemm_launches, 1)
-        flops_per_launch = flops_step / (3 * args.iters)
+        flops_per_launch = flops_step * args.steps / max(gemm_launches, 1)
         achieved = flops_per_launch / (per_launch_ms * 1e-3) / 1e12
         peak = pk["bf16"]  # fp16 and bf16 share the dense tensor rate (nominal ratio 1)
         # CUDA-core GEMM (fp32 mode, or the 16-bit check path): bound by FP32
@@ -508,7 +508,9 @@ def main():
             "roofline": ({"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                           "frac": achieved / peak, "traffic": tc_traffic(),
                           "frac_of_sustained": achieved / pk["bf16_sustained"],
-                          "kernel": "tc_pair_kernel (Gram/Poly/Update launches)",
+                          "kernel": "tc_pair_kernel (" + ("one dataflow launch per call: every Gram, Poly and "
+                                                          "Update of the T steps" if kt["gemm"][1] else
+                                                          "Gram/Poly/Update launches") + ")",
                           "peak_source": pk["source"] + " bf16 burst (fp16 dense rate equal)"}
                          if not simt else
                          {"bound": "alu", "achieved": achieved, "peak": alu_peak, "unit": "TFLOP/s",

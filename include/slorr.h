@@ -129,6 +129,20 @@ typedef struct slorr_options {
                                        workspace).  Ignored while timing is on; a stream
                                        that is being captured gets the launches.  Saves
                                        the launch gaps of small sets                    */
+#define SLORR_FLAG_PHASE_LAUNCHES 16384 /* tensor-core GEMMs as 3 T launches, one per phase
+                                       and step, each waiting for the previous one     */
+#define SLORR_FLAG_DATAFLOW    32768 /* tensor-core GEMMs as one dataflow launch: every
+                                       phase of every step, a matrix's Poly tiles
+                                       starting as soon as that matrix's Gram tiles are
+                                       stored, and so on, with no grid-wide barrier, so
+                                       the phases of different matrices overlap.
+                                       Without either flag the plan takes the dataflow
+                                       launch for sets of up to about 3 ms of GEMM work
+                                       on GB300 (measured faster there: fewer launch
+                                       tails) and per-phase launches for larger ones
+                                       (measured faster there: lighter epilogues).
+                                       Both give the same results bit for bit; the two
+                                       flags exclude each other                         */
 
 /* Fill *opt with the defaults listed beside each field above (App. C.1: T = 6,
  * ell = 1e-3, degree 5; eps, lambda and grad_scale as in Listing 1 / Alg. 2). */
@@ -266,6 +280,26 @@ SLORR_API slorr_status slorr_gemm_items(const slorr_handle* h, int32_t phase, in
  * pointer, a phase outside 0..2 or a capacity that is too small. */
 SLORR_API slorr_status slorr_gemm_item_list(const slorr_handle* h, int32_t phase, int32_t* out, int32_t capacity);
 
+/* The dataflow plan of the tensor-core GEMMs (host-only): every Gram, Poly and
+ * Update item of the T steps in one launch.  CTA pair q runs its items in
+ * order; an item may start once its matrix's completion count (each epilogue
+ * warp of both CTAs adds 1 per item it finishes: 16 per item) reaches the
+ * item's threshold, i.e. once every item of the matrix's earlier (step, phase)
+ * groups is stored.  *npairs receives the pairs the plan is made for (76 for
+ * GB300's 152 SMs until a call re-plans for the current device) and *count
+ * the items.  Unless `out` is NULL, it receives 10 int32 per item, pair by
+ * pair: (pair, seq, step, phase, mat, tm, tn, part, parts, wait), where seq
+ * is the item's rank when all items are ordered by their planned start
+ * (every item comes after every item it waits for), step is 0-based, phase 0
+ * Gram, 1 Poly, 2 Update, and part/parts as for slorr_gemm_item_list.
+ * `capacity` counts int32.  *makespan_k (if not NULL) receives the planned
+ * duration in K blocks of a 256 x 256 tile.  Errors: SLORR_ERR_INVALID_ARG
+ * for a NULL handle or count, a capacity below 10 x items, or a handle that
+ * runs per-phase launches (SLORR_FLAG_PHASE_LAUNCHES, a set above the size
+ * for which the dataflow launch is chosen, fp32 or CUDA-core). */
+SLORR_API slorr_status slorr_dataflow_items(const slorr_handle* h, int32_t* out, int32_t capacity, int32_t* npairs,
+                                            int32_t* count, double* makespan_k);
+
 /* Balance of one tensor-core GEMM launch (host-only): the launch hands item i
  * to CTA pair i mod npairs.  *max_k is the largest total K (the K
  * range of each item, summed over one pair's items) and *total_k the sum over
@@ -282,9 +316,11 @@ SLORR_API slorr_status slorr_gemm_pair_load(const slorr_handle* h, int32_t phase
  * milliseconds and kernel launch counts per kind into ms[k] / launches[k]
  * (k < kinds, kinds <= SLORR_NUM_KERNEL_KINDS; kinds are sumsq, cast, gram,
  * poly, update, dot, combine, normcast: the 16-bit iterates' single pass
- * for the norm and X_0, which replaces sumsq and cast; sumsq, normcast and
- * dot each include their finalize kernel) and forgets them. */
-#define SLORR_NUM_KERNEL_KINDS 8
+ * for the norm and X_0, which replaces sumsq and cast; gemm: the dataflow
+ * launch of every Gram, Poly and Update of a call, which replaces the gram,
+ * poly and update launches; sumsq, normcast and dot each include their
+ * finalize kernel) and forgets them. */
+#define SLORR_NUM_KERNEL_KINDS 9
 SLORR_API slorr_status slorr_set_timing(slorr_handle* h, int32_t enable);
 SLORR_API slorr_status slorr_read_timing(slorr_handle* h, double* ms, int64_t* launches, int32_t kinds);
 

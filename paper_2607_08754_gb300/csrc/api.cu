@@ -1,12 +1,14 @@
 // libslorr C ABI: planning, workspace layout, tensor maps and the launch
 // sequence of one regularizer forward + backward (Listing 1, Alg. 2):
-//   sumsq -> cast -> T x (Gram, Poly, Update) -> dot -> combine
+//   normcast (or sumsq, cast) -> the T steps' Gram, Poly and Update tiles in
+//   one dataflow launch (or 3 T per-phase launches) -> dot -> combine
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
 #include <cmath>
+#include <queue>
 #include <cstdio>
 #include <cstring>
 #include <numeric>
@@ -61,6 +63,13 @@ struct slorr_handle {
     // item lists (host)
     std::vector<GemmItem> tc_items[3];
     std::vector<GemmItem> simt_items[3];
+    // dataflow plan: every (step, phase, tile) item, pair by pair
+    std::vector<GemmItem> df_items;
+    std::vector<int32_t> df_pair_begin;  // df_pairs + 1 offsets into df_items
+    std::vector<int32_t> df_seq;         // each df item's rank in the plan's global start order
+    int df_pairs = 0;
+    double df_makespan = 0.0;            // simulated, in K blocks of a 256 x 256 tile
+    bool df = false;                     // the GEMMs run as the dataflow launch
     std::vector<MemItem> w_items;  // tiles of W (sumsq, dot, combine)
     std::vector<MemItem> x_items;  // tiles of the padded iterate (cast)
     int total_w_tiles = 0;
@@ -70,6 +79,7 @@ struct slorr_handle {
     size_t off_status = 0, off_counters = 0, off_scalars = 0, off_partials = 0, off_partials_max = 0,
            off_tilebase = 0, off_tilecount = 0, off_xtilebase = 0, off_xtilecount = 0, off_split_cnt = 0,
            off_split_part = 0, off_mats = 0, off_maps = 0, off_tc_items[3] = {}, off_simt_items[3] = {},
+           off_done = 0, off_df_items = 0, off_df_pair_begin = 0,
            off_w_items = 0, off_x_items = 0, off_ptrs = 0, off_plan_end = 0, total_bytes = 0;
     // device state
     const void* prepared_ws = nullptr;
@@ -97,6 +107,15 @@ struct slorr_handle {
 
 namespace {
 
+// Tensor-core GEMM phases as one dataflow launch, or one launch per phase and
+// step (build_plan decides; see kDataflowMaxWork).
+bool dataflow(const slorr_handle* h) { return h->df; }
+
+bool dataflow_possible(const slorr_handle* h) {
+    return h->opt.compute != SLORR_COMPUTE_FP32 &&
+           (h->opt.flags & (SLORR_FLAG_SIMT_GEMM | SLORR_FLAG_PHASE_LAUNCHES)) == 0;
+}
+
 // Programmatic dependent launch of the memory passes and the pair kernel.
 bool use_pdl(const slorr_handle* h) { return (h->opt.flags & SLORR_FLAG_NO_PDL) == 0; }
 
@@ -109,7 +128,7 @@ bool fused_norm(const slorr_handle* h) {
 
 constexpr int32_t kKnownFlags = SLORR_FLAG_SIMT_GEMM | SLORR_FLAG_TEST_STALL | SLORR_FLAG_WRITE_GRAD |
                                 SLORR_FLAG_NO_PDL | SLORR_FLAG_SEPARATE_NORM | SLORR_FLAG_NO_SPLIT_K |
-                                SLORR_FLAG_GRAPH;
+                                SLORR_FLAG_GRAPH | SLORR_FLAG_PHASE_LAUNCHES | SLORR_FLAG_DATAFLOW;
 
 bool valid_options(const slorr_options& o, std::string* why) {
     if (o.variant != SLORR_HOYER && o.variant != SLORR_NUCLEAR) return *why = "variant", false;
@@ -123,6 +142,8 @@ bool valid_options(const slorr_options& o, std::string* why) {
     if (!std::isfinite(o.lambda) || !std::isfinite(o.grad_scale)) return *why = "lambda/grad_scale", false;
     if (!(o.timeout_s > 0.0) || o.timeout_s > 3600.0) return *why = "timeout_s must be in (0, 3600]", false;
     if (o.flags & ~kKnownFlags) return *why = "flags holds a bit this build does not define", false;
+    if ((o.flags & SLORR_FLAG_PHASE_LAUNCHES) && (o.flags & SLORR_FLAG_DATAFLOW))
+        return *why = "SLORR_FLAG_PHASE_LAUNCHES and SLORR_FLAG_DATAFLOW exclude each other", false;
     return true;
 }
 
@@ -238,6 +259,182 @@ void split_gram_items(slorr_handle* h) {
     items.swap(out);
 }
 
+// Dataflow plan.  The T steps' Gram, Poly and Update tiles of every matrix
+// run in one launch; a matrix's phases are strictly ordered (each phase reads
+// what the previous one wrote: Gram X_t -> A, Poly A -> M, Update M, X_t ->
+// X_{t+1}), and different matrices are independent.  The items are assigned
+// to CTA pairs by list scheduling over a simulated clock: whenever a pair is
+// free it takes, among the items whose matrix has finished the previous phase,
+// the one with the longest remaining chain of phases below it (the sum, over
+// the matrix's remaining phases, of their longest tile plus the latency of a
+// dependency), longest tile first among equals.  Each pair runs its items in
+// the order of their simulated start times; an item's simulated start is
+// later than every start of the items it depends on, so ordering all items by
+// start time puts each one after its dependencies, and the earliest item not
+// yet finished can always run: the launch cannot deadlock whatever the real
+// timings are, provided every pair is resident.
+//
+// Costs are in K blocks (64) of a 256 x 256 tile: the tile's K blocks, scaled
+// by its width (an N = 128 UMMA moves 3/4 of the bytes of an N = 256 one), plus
+// one block for its start and epilogue (overlapped with the next tile); Poly
+// tiles count 1.6 x (their epilogue reads A and writes M and its mirror:
+// measured 0.82 against 1.37 PFLOP/s of MMA work on ViT-L/16-shaped tiles);
+// the last part of a split tile adds the parts.  A dependency adds 4 blocks
+// (the last increments, the producer's wake-up, the first copies landing).
+constexpr double kDepLatency = 4.0;
+
+// Which launch a set gets by default.  Measured on GB300 (bench, one box, both
+// modes back to back): the dataflow launch is faster for sets of up to about
+// 3 ms of GEMM work (ViT-S -20%, ViT-B/16 -8%, the first 48 ViT-L/16 matrices
+// -4%, cfg1 -15%), equal around the first 64 ViT-L/16 matrices and ViT-B
+// with 24 blocks, and slower beyond (ViT-L/16 +1.5%, 560M decoder and ViT-H
+// +5%): per item it runs 8 epilogue warps in every phase and mixes phases and
+// matrices on each pair, which costs more than the 3 T launch tails it saves
+// once each phase fills the pairs many times over.  The crossover, in the
+// planner's units (K blocks of a 256 x 256 tile on 76 pairs), is put at 7000.
+constexpr double kDataflowMaxWork = 7000.0;
+
+double df_cost(const slorr_handle* h, const GemmItem& it) {
+    const Geom& g = h->geom[it.mat];
+    const int K = it.phase == kGram ? g.Qpad : g.Ppad;
+    int b, e;
+    split_range(it, K / 64, &b, &e);
+    const double kb = double(e - b) * (0.5 + 0.5 * double(it.nsz) / 256.0);
+    double c = (it.phase == kPoly ? 1.6 * kb : kb) + 1.0;
+    if (it.ksplit) c += 2.0;
+    return c;
+}
+
+void build_dataflow(slorr_handle* h, int npairs) {
+    h->df_items.clear();
+    h->df_seq.clear();
+    h->df_pair_begin.assign(size_t(npairs) + 1, 0);
+    h->df_pairs = npairs;
+    h->df_makespan = 0.0;
+    const int count = int(h->shapes.size());
+    const int T = h->opt.iters;
+    // items of each (matrix, phase), in the per-phase plan's order
+    std::vector<std::vector<int>> of(size_t(count) * 3);
+    std::vector<double> maxcost(size_t(count) * 3, 0.0);
+    for (int ph = 0; ph < 3; ++ph)
+        for (size_t i = 0; i < h->tc_items[ph].size(); ++i) {
+            const GemmItem& it = h->tc_items[ph][i];
+            of[size_t(it.mat) * 3 + ph].push_back(int(i));
+            maxcost[size_t(it.mat) * 3 + ph] = std::max(maxcost[size_t(it.mat) * 3 + ph], df_cost(h, it));
+        }
+    // group g = (mat, t, ph), g = (mat * T + t) * 3 + ph; its successor is g + 1
+    // (the matrix's next phase; Update of step t is followed by Gram of t + 1)
+    const size_t G = size_t(count) * T * 3;
+    auto gmat = [&](size_t g) { return int(g / (size_t(T) * 3)); };
+    auto gstep = [&](size_t g) { return int(g / 3 % size_t(T)); };
+    auto gph = [&](size_t g) { return int(g % 3); };
+    std::vector<double> level(G, 0.0), gend(G, 0.0);
+    std::vector<int> left(G, 0);
+    std::vector<uint32_t> base(G, 0);
+    for (int m = 0; m < count; ++m) {
+        double acc = 0.0;
+        for (int k = T * 3 - 1; k >= 0; --k) {
+            acc += maxcost[size_t(m) * 3 + k % 3] + kDepLatency;
+            level[size_t(m) * T * 3 + k] = acc;
+        }
+        uint32_t done = 0;
+        for (int k = 0; k < T * 3; ++k) {
+            base[size_t(m) * T * 3 + k] = done;
+            left[size_t(m) * T * 3 + k] = int(of[size_t(m) * 3 + k % 3].size());
+            done += uint32_t(of[size_t(m) * 3 + k % 3].size()) * kDoneIncPerItem;
+        }
+    }
+    struct Ready {
+        double level, cost;
+        int mat, order;
+        size_t g;
+        int src;
+        bool operator<(const Ready& o) const {  // max-heap: higher level, then longer, then lower index
+            if (level != o.level) return level < o.level;
+            if (cost != o.cost) return cost < o.cost;
+            if (mat != o.mat) return mat > o.mat;
+            return order > o.order;
+        }
+    };
+    std::priority_queue<Ready> ready;
+    using TimedGroup = std::pair<double, size_t>;  // (ready time, group)
+    std::priority_queue<TimedGroup, std::vector<TimedGroup>, std::greater<TimedGroup>> pending;
+    using Free = std::pair<double, int>;  // (free time, pair)
+    std::priority_queue<Free, std::vector<Free>, std::greater<Free>> pairs;
+    for (int q = 0; q < npairs; ++q) pairs.push({0.0, q});
+    auto release = [&](size_t g) {
+        const std::vector<int>& v = of[size_t(gmat(g)) * 3 + gph(g)];
+        for (size_t k = 0; k < v.size(); ++k) {
+            const GemmItem& it = h->tc_items[gph(g)][size_t(v[k])];
+            ready.push(Ready{level[g], df_cost(h, it), gmat(g), int(k), g, v[k]});
+        }
+    };
+    // every matrix has at least one tile in every phase, so each group is
+    // released when its predecessor's last item is assigned
+    size_t total = 0;
+    for (int m = 0; m < count; ++m) {
+        const size_t g0 = size_t(m) * T * 3;
+        for (int k = 0; k < T * 3; ++k) total += size_t(left[g0 + k]);
+        pending.push({0.0, g0});
+    }
+    struct Assigned {
+        double start;
+        int pair;
+        size_t g;
+        int src;
+    };
+    std::vector<Assigned> out;
+    out.reserve(total);
+    while (out.size() < total) {
+        Free f = pairs.top();
+        pairs.pop();
+        while (!pending.empty() && pending.top().first <= f.first) {
+            release(pending.top().second);
+            pending.pop();
+        }
+        if (ready.empty()) {
+            if (pending.empty()) break;  // not reachable: every group is released once its predecessor ends
+            pairs.push({pending.top().first, f.second});
+            continue;
+        }
+        const Ready r = ready.top();
+        ready.pop();
+        const double end = f.first + r.cost;
+        out.push_back(Assigned{f.first, f.second, r.g, r.src});
+        gend[r.g] = std::max(gend[r.g], end);
+        h->df_makespan = std::max(h->df_makespan, end);
+        // the matrix's next (step, phase) becomes ready when this one ends
+        if (--left[r.g] == 0 && r.g % (size_t(T) * 3) + 1 < size_t(T) * 3)
+            pending.push({gend[r.g] + kDepLatency, r.g + 1});
+        pairs.push({end, f.second});
+    }
+    // global order: by simulated start, then pair
+    std::vector<size_t> order(out.size());
+    std::iota(order.begin(), order.end(), size_t(0));
+    std::stable_sort(order.begin(), order.end(), [&](size_t a, size_t b) {
+        if (out[a].start != out[b].start) return out[a].start < out[b].start;
+        return out[a].pair < out[b].pair;
+    });
+    std::vector<int32_t> rank(out.size());
+    for (size_t k = 0; k < order.size(); ++k) rank[order[k]] = int32_t(k);
+    // pair-major layout; each pair's items are already in start order
+    std::vector<std::vector<size_t>> per(static_cast<size_t>(npairs));
+    for (size_t k = 0; k < out.size(); ++k) per[size_t(out[k].pair)].push_back(k);
+    for (int q = 0; q < npairs; ++q) {
+        h->df_pair_begin[size_t(q)] = int32_t(h->df_items.size());
+        for (size_t k : per[size_t(q)]) {
+            const Assigned& a = out[k];
+            GemmItem it = h->tc_items[gph(a.g)][size_t(a.src)];
+            it.step = uint8_t(gstep(a.g));
+            it.phase = uint8_t(gph(a.g));
+            it.wait = base[a.g];
+            h->df_items.push_back(it);
+            h->df_seq.push_back(rank[k]);
+        }
+    }
+    h->df_pair_begin[size_t(npairs)] = int32_t(h->df_items.size());
+}
+
 void build_plan(slorr_handle* h) {
     const int count = int(h->shapes.size());
     h->geom.resize(count);
@@ -302,13 +499,16 @@ void build_plan(slorr_handle* h) {
                     if (ph != kUpdate && (2 * tn + nsz / 128 - 1) < tm * 2) continue;
                     h->tc_items[ph].push_back(
                         GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), uint16_t(nsz), uint16_t(msz), 0});
+                    h->tc_items[ph].back().phase = uint8_t(ph);
                 }
             }
             // CUDA-core tiles; the symmetric Gram and Poly keep those on or above the diagonal
             for (int tm = 0; tm < g.Ppad / kSimtTile; ++tm)
-                for (int tn = (ph == kUpdate ? 0 : tm); tn < N / kSimtTile; ++tn)
+                for (int tn = (ph == kUpdate ? 0 : tm); tn < N / kSimtTile; ++tn) {
                     h->simt_items[ph].push_back(
                         GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), kSimtTile, kSimtTile, 0});
+                    h->simt_items[ph].back().phase = uint8_t(ph);
+                }
         }
     }
     h->total_w_tiles = tile_base;
@@ -333,13 +533,29 @@ void build_plan(slorr_handle* h) {
         for (const GemmItem& it : h->tc_items[ph]) cost.push_back(kdim(it) + 64);
         balance_pairs(h->tc_items[ph], cost);
     }
+    // the dataflow plan for GB300's 76 pairs (prepare() re-plans for a device
+    // that holds another number of pairs at once), kept for sets below the
+    // measured crossover or when asked for
+    h->df = false;
+    if (dataflow_possible(h)) {
+        build_dataflow(h, kPlanPairs);
+        h->df = (h->opt.flags & SLORR_FLAG_DATAFLOW) || h->df_makespan < kDataflowMaxWork;
+        if (!h->df) {
+            h->df_items.clear();
+            h->df_seq.clear();
+            h->df_pair_begin.clear();
+            h->df_pairs = 0;
+        }
+    }
 
     // Workspace layout.
     size_t off = 0;
     h->off_status = off;
     off += 256;
     h->off_counters = off;
-    off = align_up(off + size_t(count + 1) * 4, 256);
+    off += size_t(count + 1) * 4;
+    h->off_done = off;  // zeroed together with the counters at the start of each call
+    off = align_up(off + size_t(count) * 4, 256);
     h->off_scalars = off;
     off = align_up(off + size_t(count) * sizeof(MatScalars), 256);
     h->off_partials = off;
@@ -347,7 +563,7 @@ void build_plan(slorr_handle* h) {
     h->off_partials_max = off;
     off = align_up(off + size_t(h->total_x_tiles) * 4, 256);
     h->off_split_cnt = off;
-    off = align_up(off + size_t(h->total_split_parts) * 8 * 4, 256);
+    off = align_up(off + size_t(h->total_split_parts) * 16 * 4, 256);
     h->off_tilebase = off;
     off = align_up(off + size_t(count) * 4, 256);
     h->off_tilecount = off;
@@ -366,6 +582,10 @@ void build_plan(slorr_handle* h) {
         h->off_simt_items[ph] = off;
         off = align_up(off + h->simt_items[ph].size() * sizeof(GemmItem), 256);
     }
+    h->off_df_items = off;
+    off = align_up(off + h->df_items.size() * sizeof(GemmItem), 256);
+    h->off_df_pair_begin = off;
+    off = align_up(off + size_t(dataflow(h) ? kMaxPlanPairs + 1 : 0) * 4, 256);
     h->off_w_items = off;
     off = align_up(off + h->w_items.size() * sizeof(MemItem), 256);
     h->off_x_items = off;
@@ -435,6 +655,16 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
         if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, dev);
         if (e != cudaSuccess) return cuda_fail(e, "device query");
     }
+    if (dataflow(h)) {
+        // every pair of the dataflow launch must be resident at once: plan for
+        // as many pairs as this device holds (76 on a GB300)
+        int cap = 0;
+        cudaError_t e = tc_pair_dataflow_capacity(h->elem, h->num_sms, &cap);
+        if (e != cudaSuccess) return cuda_fail(e, "occupancy query");
+        const int npairs = std::min(std::min(cap, h->num_sms / 2), kMaxPlanPairs);
+        if (npairs < 1) return fail(SLORR_ERR_UNSUPPORTED, "no CTA pair of the tensor-core kernel fits this device");
+        if (npairs != h->df_pairs) build_dataflow(h, npairs);
+    }
     std::vector<uint8_t> plan(h->off_plan_end - h->off_tilebase, 0);
     const size_t base = h->off_tilebase;
     std::vector<int32_t> tb(count), tcnt(count), xtb(count), xtcnt(count);
@@ -487,6 +717,8 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
         put(plan, h->off_tc_items[ph] - base, h->tc_items[ph].data(), h->tc_items[ph].size());
         put(plan, h->off_simt_items[ph] - base, h->simt_items[ph].data(), h->simt_items[ph].size());
     }
+    put(plan, h->off_df_items - base, h->df_items.data(), h->df_items.size());
+    put(plan, h->off_df_pair_begin - base, h->df_pair_begin.data(), h->df_pair_begin.size());
     put(plan, h->off_w_items - base, h->w_items.data(), h->w_items.size());
     put(plan, h->off_x_items - base, h->x_items.data(), h->x_items.size());
     cudaError_t e = cudaMemcpyAsync(ws + base, plan.data(), plan.size(), cudaMemcpyHostToDevice, st);
@@ -685,11 +917,11 @@ slorr_status run(slorr_handle* h, const void* const* weights, void* const* grads
 // plan is in the workspace and the pointer arrays are uploaded).
 slorr_status launch_all(slorr_handle* h, uint8_t* ws, float* loss, float* per, int steps, bool finish,
                         cudaStream_t st, bool descent, float eta) {
-    cudaError_t e = cudaMemsetAsync(ws + h->off_counters, 0, (h->shapes.size() + 1) * 4, st);
+    cudaError_t e = cudaMemsetAsync(ws + h->off_counters, 0, (2 * h->shapes.size() + 1) * 4, st);
     // split-K part counts: each Gram's last parts leave them at zero, but a
     // call that timed out may not have
     if (e == cudaSuccess && h->total_split_parts > 0)
-        e = cudaMemsetAsync(ws + h->off_split_cnt, 0, size_t(h->total_split_parts) * 8 * 4, st);
+        e = cudaMemsetAsync(ws + h->off_split_cnt, 0, size_t(h->total_split_parts) * 16 * 4, st);
     if (e != cudaSuccess) return cuda_fail(e, "counter reset");
 
     const bool use_tc = h->opt.compute != SLORR_COMPUTE_FP32 && !(h->opt.flags & SLORR_FLAG_SIMT_GEMM);
@@ -726,29 +958,41 @@ slorr_status launch_all(slorr_handle* h, uint8_t* ws, float* loss, float* per, i
     g.timeout_ns = static_cast<unsigned long long>(h->opt.timeout_s * 1e9);
     g.test_stall = (h->opt.flags & SLORR_FLAG_TEST_STALL) ? 1 : 0;
     g.pdl = use_pdl(h) ? 1 : 0;
+    g.fused_norm = fuse_norm ? 1 : 0;
     g.scalars = reinterpret_cast<const MatScalars*>(ws + h->off_scalars);
     g.split_part = reinterpret_cast<float*>(ws + h->off_split_part);
     g.split_cnt = reinterpret_cast<uint32_t*>(ws + h->off_split_cnt);
-    for (int t = 0; t < steps; ++t) {
-        g.cur = t & 1;
-        g.a = float(h->coeffs[3 * t + 0]);
-        g.b = float(h->coeffs[3 * t + 1]);
-        g.c = float(h->coeffs[3 * t + 2]);
-        for (int ph = 0; ph < 3; ++ph) {
-            g.phase = ph;
-            g.x0_scaled = (fuse_norm && t == 0 && ph != kPoly) ? 1 : 0;
-            Traced tr(h, 2 + ph, st);
-            if (use_tc) {
-                g.items = reinterpret_cast<const GemmItem*>(ws + h->off_tc_items[ph]);
-                g.num_items = int(h->tc_items[ph].size());
-                e = launch_gemm_tc_pair(g, h->elem, h->num_sms, st);
-            } else {
-                g.items = reinterpret_cast<const GemmItem*>(ws + h->off_simt_items[ph]);
-                g.num_items = int(h->simt_items[ph].size());
-                e = launch_gemm_simt(g, h->elem, st);
+    for (int t = 0; t < h->opt.iters; ++t)
+        for (int k = 0; k < 3; ++k) g.coef[t][k] = float(h->coeffs[3 * t + k]);
+    if (use_tc && dataflow(h) && steps > 0) {
+        // every phase of every step in one launch, ordered by completion counts
+        g.items = reinterpret_cast<const GemmItem*>(ws + h->off_df_items);
+        g.num_items = int(h->df_items.size());
+        g.step = -1;
+        g.steps = steps;
+        g.pair_begin = reinterpret_cast<const int32_t*>(ws + h->off_df_pair_begin);
+        g.done = reinterpret_cast<uint32_t*>(ws + h->off_done);
+        Traced tr(h, 8, st);
+        e = launch_gemm_tc_pair(g, h->elem, h->num_sms, st, kDataflowEpiWarps, h->df_pairs);
+        if (e != cudaSuccess) return cuda_fail(e, "gemm launch");
+        tr.done();
+    } else {
+        for (int t = 0; t < steps; ++t) {
+            g.step = t;
+            for (int ph = 0; ph < 3; ++ph) {
+                Traced tr(h, 2 + ph, st);
+                if (use_tc) {
+                    g.items = reinterpret_cast<const GemmItem*>(ws + h->off_tc_items[ph]);
+                    g.num_items = int(h->tc_items[ph].size());
+                    e = launch_gemm_tc_pair(g, h->elem, h->num_sms, st, ph == kPoly ? 8 : 4, 0);
+                } else {
+                    g.items = reinterpret_cast<const GemmItem*>(ws + h->off_simt_items[ph]);
+                    g.num_items = int(h->simt_items[ph].size());
+                    e = launch_gemm_simt(g, h->elem, st);
+                }
+                if (e != cudaSuccess) return cuda_fail(e, "gemm launch");
+                tr.done();
             }
-            if (e != cudaSuccess) return cuda_fail(e, "gemm launch");
-            tr.done();
         }
     }
     if (!finish) return SLORR_OK;
@@ -897,6 +1141,34 @@ slorr_status slorr_gemm_item_list(const slorr_handle* h, int32_t phase, int32_t*
         o[5] = parts > 1 ? (it.ksplit & 0xff) : 0;
         o[6] = parts > 1 ? parts : 1;
     }
+    return SLORR_OK;
+}
+
+slorr_status slorr_dataflow_items(const slorr_handle* h, int32_t* out, int32_t capacity, int32_t* npairs,
+                                  int32_t* count, double* makespan_k) {
+    if (!h || !npairs || !count) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
+    if (!dataflow(h)) return fail(SLORR_ERR_INVALID_ARG, "this handle runs per-phase launches");
+    *npairs = h->df_pairs;
+    *count = int32_t(h->df_items.size());
+    if (makespan_k) *makespan_k = h->df_makespan;
+    if (!out) return SLORR_OK;
+    if (int64_t(capacity) < int64_t(h->df_items.size()) * 10) return fail(SLORR_ERR_INVALID_ARG, "capacity too small");
+    for (int q = 0; q < h->df_pairs; ++q)
+        for (int32_t i = h->df_pair_begin[size_t(q)]; i < h->df_pair_begin[size_t(q) + 1]; ++i) {
+            const GemmItem& it = h->df_items[size_t(i)];
+            const int parts = it.ksplit >> 8;
+            int32_t* o = out + size_t(i) * 10;
+            o[0] = q;
+            o[1] = h->df_seq[size_t(i)];
+            o[2] = it.step;
+            o[3] = it.phase;
+            o[4] = it.mat;
+            o[5] = it.tm;
+            o[6] = it.tn;
+            o[7] = parts > 1 ? (it.ksplit & 0xff) : 0;
+            o[8] = parts > 1 ? parts : 1;
+            o[9] = int32_t(it.wait);
+        }
     return SLORR_OK;
 }
 

@@ -6,8 +6,7 @@
 // orientation -- row-major [m][n], i.e. as X^T when m > n -- so that the norm,
 // cast, dot and gradient passes are elementwise; the tensor-core kernel reads
 // it as a K-major or MN-major operand as each phase needs.  Both dimensions
-// are zero-padded: P to Ppad (a multiple of 128) and Q to Qpad (a multiple of
-// 64).  Zero padding is exact: zero rows/columns of X give zero rows/columns
+// are zero-padded: P to Ppad and Q to Qpad (multiples of 128).  Zero padding is exact: zero rows/columns of X give zero rows/columns
 // of A = X X^T; M = a I + b A + c A^2 is a I on the padded block, which only
 // ever multiplies zero rows of X; and the odd polynomial maps zero to zero
 // (App. B, "zero singular values stay zero").
@@ -71,6 +70,10 @@ struct GemmItem {
     uint16_t msz;      // rows in this tile
     uint16_t ksplit;   // split K (CTA-pair Gram): part s | (parts S << 8); 0 = whole K
     uint32_t sid;      // split K: the tile's first 256 x 256 partial slot (parts sid .. sid + S - 1)
+    uint8_t step;      // Polar Express step t of this item (dataflow launch; 0 in per-phase lists)
+    uint8_t phase;     // kGram, kPoly or kUpdate
+    uint16_t pad_;
+    uint32_t wait;     // dataflow launch: the item may start once done[mat] >= wait
 };
 
 // K blocks [begin, end) of an item's nkb: part s of S takes an equal share.
@@ -112,27 +115,41 @@ constexpr uint16_t kFlatTile = 0xffff;
 // X <- M X with M = a I + b A + c A^2, the same product as a X + (b A + c A^2) X).
 enum Phase : int32_t { kGram = 0, kPoly = 1, kUpdate = 2 };
 
+// Dataflow launch (the default): every Gram, Poly and Update tile of every
+// step in one launch.  CTA pair q runs items [pair_begin[q], pair_begin[q + 1])
+// in order; each epilogue warp of both CTAs adds 1 to done[mat] once its part
+// of an item is stored, and an item's TMA producer waits until done[mat]
+// reaches the item's `wait`: the count after every earlier (step, phase) of
+// its matrix.  Per-phase launches (pair_begin == nullptr) hand item i to pair
+// i mod npairs and run the single step `step`.
+constexpr int kDataflowEpiWarps = 8;   // epilogue warps per CTA of the dataflow kernel
+constexpr int kDoneIncPerItem = 2 * kDataflowEpiWarps;
+constexpr int kMaxPlanPairs = 512;
+
 struct GemmLaunch {
     const GemmItem* items;
     int32_t num_items;
-    int32_t phase;
-    int32_t cur;               // index of the current iterate buffer (0/1)
-    float a, b, c;             // step coefficients (a_t, b_t, c_t)
+    int32_t step;              // per-phase launch: the step t; dataflow: -1 (each item's own)
+    int32_t steps;             // dataflow: items of steps >= steps are skipped
+    float coef[kMaxIters][3];  // (a_t, b_t, c_t) for t = 0 .. T - 1
+    const int32_t* pair_begin; // dataflow: each pair's range of items (npairs + 1 offsets)
+    uint32_t* done;            // dataflow: per-matrix completion counts (zeroed before the launch)
     const MatDev* mats;
     const void* maps;          // CUtensorMap array, kMapsPerMatrix per matrix
     uint32_t* status;
     unsigned long long timeout_ns;
     int32_t test_stall;        // 1: the MMA thread first waits on a barrier nothing arrives on
     int32_t pdl;               // launch with programmatic dependent launch
-    // x0_scaled = 1 (first step after the fused norm pass, which stores X_0
-    // as W rounded to 16 bits): the Gram epilogue multiplies by
+    // fused_norm = 1 (16-bit iterates after the fused norm pass, which stores
+    // X_0 as W rounded to 16 bits): in step 0 the Gram epilogue multiplies by
     // scalars[i].x0_scale^2 and the Update epilogue by scalars[i].x0_scale.
-    int32_t x0_scaled;
+    int32_t fused_norm;
     const MatScalars* scalars;
     // split K (CTA-pair Gram): part s of a split tile leaves its fp32 partial
     // at split_part + ((sid + s) * 256 + column) * 256 + row (tile
-    // coordinates), and counts it in split_cnt[sid * 8 + rank * 4 + quad];
-    // the epilogue warp that counts last adds the parts and stores the tile.
+    // coordinates), and counts it in split_cnt[sid * 16 + rank * 8 + group * 4
+    // + quad]; the epilogue warp that counts last adds the parts and stores
+    // the tile.
     float* split_part;
     uint32_t* split_cnt;
 };
@@ -183,7 +200,14 @@ cudaError_t launch_finalize(const MemLaunch& p, int which, cudaStream_t s);
 cudaError_t launch_combine(const MemLaunch& p, cudaStream_t s);
 cudaError_t launch_sum_parts(const float* parts, int n, float* out, cudaStream_t s);
 cudaError_t launch_gemm_simt(const GemmLaunch& p, int elem, cudaStream_t s);
-cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t s);
+// Per-phase launches (p.pair_begin == nullptr; npairs ignored) or the
+// dataflow launch over `npairs` CTA pairs, with 4 or 8 epilogue warps per CTA
+// (Poly and the dataflow launch, which mixes phases, take 8).
+cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t s, int epi_warps,
+                                int npairs);
+// CTA pairs of the dataflow kernel that can be resident at once on the
+// current device (0 and an error when the query fails).
+cudaError_t tc_pair_dataflow_capacity(int elem, int num_sms, int* pairs);
 
 #if defined(__CUDACC__)
 // Launches `kernel` on `st`; with pdl, as a programmatic dependent of the

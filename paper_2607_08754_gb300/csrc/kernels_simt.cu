@@ -51,7 +51,9 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const GemmLaunch p) {
     __shared__ float Bs[2][kBK][kT + 1];  // [buffer][k][j]
     const GemmItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
-    const T* X = reinterpret_cast<const T*>(md.x[p.cur]);
+    const int ph = it.phase, cur = p.step & 1;  // one launch per phase and step
+    const float ca = p.coef[p.step][0], cb = p.coef[p.step][1], cc = p.coef[p.step][2];
+    const T* X = reinterpret_cast<const T*>(md.x[cur]);
     const T* Am = reinterpret_cast<const T*>(md.a);
     const T* Bm = reinterpret_cast<const T*>(md.b);
     // X(p, q) lives at xb[p * sp + q * sq] (the buffer is in W's orientation).
@@ -61,9 +63,9 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const GemmLaunch p) {
     const T* opB;
     int64_t sa_i, sa_k, sb_j, sb_k;
     int K;
-    if (p.phase == kGram) {          // A = X X^T
+    if (ph == kGram) {               // A = X X^T
         opA = X; sa_i = sp; sa_k = sq; opB = X; sb_j = sp; sb_k = sq; K = md.Qpad;
-    } else if (p.phase == kPoly) {   // A A
+    } else if (ph == kPoly) {        // A A
         opA = Am; sa_i = md.Ppad; sa_k = 1; opB = Am; sb_j = md.Ppad; sb_k = 1; K = md.Ppad;
     } else {                         // M X
         opA = Bm; sa_i = md.Ppad; sa_k = 1; opB = X; sb_j = sq; sb_k = sp; K = md.Ppad;
@@ -128,26 +130,26 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const GemmLaunch p) {
         __syncthreads();
         buf ^= 1;
     }
-    const bool mirror = p.phase != kUpdate && it.tn > it.tm;
+    const bool mirror = ph != kUpdate && it.tn > it.tm;
 #pragma unroll
     for (int u = 0; u < 2; ++u) {
 #pragma unroll
         for (int v = 0; v < 2; ++v) {
             const int i = m0 + ty * 2 + u, j = n0 + tx * 2 + v;
             const float acc_uv = acc[u][v] + cmp[u][v];
-            if (p.phase == kGram) {
+            if (ph == kGram) {
                 T* a = reinterpret_cast<T*>(md.a);
                 st_f<T>(a + static_cast<int64_t>(i) * md.Ppad + j, acc_uv);
                 if (mirror) st_f<T>(a + static_cast<int64_t>(j) * md.Ppad + i, acc_uv);
-            } else if (p.phase == kPoly) {      // M = c A^2 + b A + a I (A is stored symmetric)
+            } else if (ph == kPoly) {           // M = c A^2 + b A + a I (A is stored symmetric)
                 const int64_t idx = static_cast<int64_t>(i) * md.Ppad + j;
-                float val = fmaf(p.b, ld_f<T>(Am + idx), p.c * acc_uv);
-                if (i == j) val += p.a;
+                float val = fmaf(cb, ld_f<T>(Am + idx), cc * acc_uv);
+                if (i == j) val += ca;
                 T* m = reinterpret_cast<T*>(md.b);
                 st_f<T>(m + idx, val);
                 if (mirror) st_f<T>(m + static_cast<int64_t>(j) * md.Ppad + i, val);
             } else {                            // X' = M X
-                st_f<T>(reinterpret_cast<T*>(md.x[p.cur ^ 1]) + static_cast<int64_t>(i) * sp +
+                st_f<T>(reinterpret_cast<T*>(md.x[cur ^ 1]) + static_cast<int64_t>(i) * sp +
                             static_cast<int64_t>(j) * sq, acc_uv);
             }
         }

@@ -1,7 +1,21 @@
 // Grouped persistent tensor-core GEMM on CTA pairs (tcgen05 cta_group::2) for
 // the three phases of a Polar Express step (Sec. 3 "Computing the polar
 // factor"): Gram A = X X^T, Poly M = a I + b A + c A A, Update X' = M X, over
-// every matrix of the weight set in one launch.
+// every matrix of the weight set.  Two launch modes:
+//   per-phase   one launch per phase and step (3 T launches); pair q runs
+//               items q, q + npairs, ...; the launch boundary orders phases.
+//   dataflow    one launch for every phase of every step.  Pair q runs its
+//               own list of the host's plan, in order.  Each epilogue warp of
+//               both CTAs adds 1 to its matrix's completion count once its
+//               part of an item is stored (after a GPU-scope fence), and a TMA
+//               producer waits (acquire, bounded) until the count reaches the
+//               item's threshold -- every item of the matrix's earlier (step,
+//               phase) groups -- before copying its operands.  So a matrix's
+//               Poly tiles start as soon as its own Gram tiles are stored,
+//               and the phases of different matrices overlap.  The plan lists
+//               each pair's items in an order in which every item comes after
+//               the items it waits for (see build_dataflow in api.cu), and all
+//               pairs are resident, so the launch cannot deadlock.
 //
 // A cluster of two CTAs on two SMs computes one 256 x 256 tile.  CTA r of the
 // pair holds rows [128 r, 128 r + 128) of the tile's A operand and columns
@@ -13,7 +27,7 @@
 // 256 TMEM columns per SM: two of them fit, so a tile's epilogue overlaps the
 // next tile's main loop.
 //
-// Roles (192 threads per CTA; 320 for Poly):
+// Roles (192 threads per CTA; 320 for Poly and the dataflow launch):
 //   warp 0 lane 0   TMA producer (both CTAs): waits for a stage to be free and
 //                   loads its CTA's A rows and B half into its own shared
 //                   memory, counting the bytes on the even CTA's stage barrier
@@ -28,7 +42,8 @@
 //                   32-row TMEM lane quadrant, each 32 x 32 chunk staged in
 //                   the warp's shared-memory buffer so that global stores (and
 //                   Poly's loads of A) move 8 rows x 64 bytes per instruction;
-//                   then release the accumulator slot on the even CTA's barrier.
+//                   then release the accumulator slot on the even CTA's barrier
+//                   (and, in the dataflow launch, count the item as done).
 // A stage is released only by a commit the MMA thread issues after arming the
 // stage's next phase, so every copy of either CTA is counted on a phase the
 // MMA thread armed; on a timeout that thread waits (bounded) for the last
@@ -81,6 +96,7 @@ struct PairCfg {
 // polling warps slow the producer and MMA threads of the long-K phases).
 using PairCfg2 = PairCfg<SLORR_PAIR_STAGES, 4>;
 using PairCfg2Wide = PairCfg<SLORR_PAIR_STAGES, 8>;
+static_assert(PairCfg2Wide::kEpiWarps == kDataflowEpiWarps, "the dataflow plan counts 2 x 8 warps per item");
 
 struct PairSmem {
     uint8_t* stages;
@@ -102,33 +118,109 @@ __device__ __forceinline__ void record_timeout(const GemmLaunch& p, const PairSm
     atomicOr(p.status, kStatusTimeout);
 }
 
+// The items a CTA pair runs, in order: its range of the dataflow plan, or
+// every npairs-th item of a per-phase launch.  A dataflow launch of fewer
+// steps than the plan (slorr_run_steps) skips the later steps' items; every
+// role skips the same ones.
+struct PairItems {
+    int first, end, stride;
+    __device__ PairItems(const GemmLaunch& p, int pair, int npairs) {
+        if (p.pair_begin != nullptr) {
+            first = p.pair_begin[pair];
+            end = p.pair_begin[pair + 1];
+            stride = 1;
+        } else {
+            first = pair;
+            end = p.num_items;
+            stride = npairs;
+        }
+    }
+};
+
+__device__ __forceinline__ bool item_runs(const GemmLaunch& p, const GemmItem& it) {
+    return p.pair_begin == nullptr || int(it.step) < p.steps;
+}
+
+// The first index >= idx (in steps of `stride`, below `end`) whose item runs.
+__device__ __forceinline__ int next_running(const GemmLaunch& p, int idx, int end, int stride) {
+    while (idx < end && !item_runs(p, p.items[idx])) idx += stride;
+    return idx;
+}
+
+// Dataflow launch: waits until the completion count of the item's matrix
+// reaches the item's threshold.  The acquire load makes every store the
+// counted epilogue warps made before their (fenced) increments visible to
+// this thread.  Gives up on this CTA's abort flag, on a timeout recorded
+// anywhere in the launch (the status word), or after the launch's budget.
+// *seen receives the count that satisfied the wait.
+__device__ __forceinline__ bool wait_done(const GemmLaunch& p, const PairSmem& s, const GemmItem& it,
+                                          uint32_t* seen = nullptr) {
+    if (p.done == nullptr || it.wait == 0) return true;
+    const uint32_t* c = p.done + it.mat;
+    uint32_t v = ptx::ld_acquire_gpu(c);
+    if (v >= it.wait) {
+        if (seen) *seen = v;
+        return true;
+    }
+    const uint64_t t0 = ptx::globaltimer();
+    for (uint32_t i = 1;; ++i) {
+        __nanosleep(32);
+        v = ptx::ld_acquire_gpu(c);
+        if (v >= it.wait) {
+            if (seen) *seen = v;
+            return true;
+        }
+        if ((i & 15u) == 0u) {
+            if (*s.abort) return false;
+            if (ptx::ld_relaxed_gpu(p.status) & kStatusTimeout) return false;
+            if (ptx::globaltimer() - t0 > p.timeout_ns) return false;
+        }
+    }
+}
+
 // Diagonal tiles of the symmetric products (Gram A = X X^T, Poly A A): with
 // tm == tn and a full 256 x 256 tile, each CTA's A rows and B columns are the
 // same 128 rows of the same matrix, so they are copied once and both UMMA
 // operands read them (the B descriptor points at the A half).
-__device__ __forceinline__ bool shared_operand(const GemmLaunch& p, const GemmItem& it) {
-    return p.phase != kUpdate && it.tm == it.tn && it.msz == 2 * kBM && it.nsz == kBNMax;
+__device__ __forceinline__ bool shared_operand(const GemmItem& it) {
+    return it.phase != kUpdate && it.tm == it.tn && it.msz == 2 * kBM && it.nsz == kBNMax;
 }
 
 // Bytes one CTA of the pair copies per stage of a tile: its A rows, unless they
 // lie beyond the matrix (the UMMA rows they would feed are never stored), and
 // its half of the B columns, unless they are its A rows (shared_operand).
 template <class C>
-__device__ __forceinline__ uint32_t pair_stage_bytes(const GemmLaunch& p, const GemmItem& it, int rank) {
+__device__ __forceinline__ uint32_t pair_stage_bytes(const GemmItem& it, int rank) {
     const uint32_t a = rank * kBM < it.msz ? uint32_t(C::kABytes) : 0u;
-    return shared_operand(p, it) ? a : a + uint32_t(it.nsz / 2) * C::BK * 2;
+    return shared_operand(it) ? a : a + uint32_t(it.nsz / 2) * C::BK * 2;
 }
 
 template <class C>
-__device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, int pair, int npairs) {
+__device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, const PairItems& seq) {
     int stage = 0;
     uint32_t phase = 0;
     const uint32_t even_full = ptx::mapa(ptx::smem_u32(s.full), 0);
-    for (int idx = pair; idx < p.num_items; idx += npairs) {
+    // the last completion count this thread acquired, and of which matrix:
+    // an item it already covers needs no new acquire
+    int seen_mat = -1;
+    uint32_t seen = 0;
+    for (int idx = next_running(p, seq.first, seq.end, seq.stride); idx < seq.end;
+         idx = next_running(p, idx + seq.stride, seq.end, seq.stride)) {
         const GemmItem it = p.items[idx];
+        // Dataflow: the item's operands are complete once its matrix's earlier
+        // phases are; the proxy fence orders those generic-proxy stores, now
+        // visible to this thread, before its tensor copies read them.
+        if (p.done != nullptr && it.wait != 0 && !(int(it.mat) == seen_mat && seen >= it.wait)) {
+            if (!wait_done(p, s, it, &seen)) {
+                record_timeout(p, s);
+                return;
+            }
+            ptx::fence_proxy_async_global();
+            seen_mat = it.mat;
+        }
         const PhaseInfo pi = phase_info<C>(p, it);
         const bool load_a = rank * kBM < it.msz;
-        const bool load_b = !shared_operand(p, it);
+        const bool load_b = !shared_operand(it);
         int kb_begin, kb_end;
         split_range(it, pi.nkb, &kb_begin, &kb_end);
         for (int kb = kb_begin; kb < kb_end; ++kb) {
@@ -167,38 +259,39 @@ __device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, 
 template <class C>
 struct KCursor {
     const GemmLaunch* p;
-    int idx, kb, nkb, step;
+    int idx, end, stride, kb, nkb;
     uint32_t bytes;  // bytes both CTAs copy for the current K block
     __device__ void load() {
-        if (idx < p->num_items) {
+        idx = next_running(*p, idx, end, stride);
+        if (idx < end) {
             const GemmItem it = p->items[idx];
             int b, e;
             split_range(it, phase_info<C>(*p, it).nkb, &b, &e);
             nkb = e - b;
-            bytes = pair_stage_bytes<C>(*p, it, 0) + pair_stage_bytes<C>(*p, it, 1);
+            bytes = pair_stage_bytes<C>(it, 0) + pair_stage_bytes<C>(it, 1);
         }
     }
-    __device__ KCursor(const GemmLaunch& gp, int first, int stride) : p(&gp), idx(first), kb(0), nkb(0), step(stride),
-                                                                      bytes(0) {
+    __device__ KCursor(const GemmLaunch& gp, const PairItems& seq)
+        : p(&gp), idx(seq.first), end(seq.end), stride(seq.stride), kb(0), nkb(0), bytes(0) {
         load();
     }
-    __device__ bool valid() const { return idx < p->num_items; }
+    __device__ bool valid() const { return idx < end; }
     __device__ void next() {
         if (++kb == nkb) {
             kb = 0;
-            idx += step;
+            idx += stride;
             load();
         }
     }
 };
 
 template <bool BF16, class C>
-__device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_base, int pair, int npairs) {
+__device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_base, const PairItems& seq) {
     int armed_parity[C::STAGES];
 #pragma unroll
     for (int i = 0; i < C::STAGES; ++i) armed_parity[i] = -1;
     // Arm the first ring: phase 0 of every stage the sequence reaches.
-    KCursor<C> arm(p, pair, npairs);
+    KCursor<C> arm(p, seq);
     for (int i = 0; i < C::STAGES && arm.valid(); ++i, arm.next()) {
         ptx::mbar_arrive_expect_tx(&s.full[i], arm.bytes);
         armed_parity[i] = 0;
@@ -216,7 +309,8 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
             ok = false;
         }
     }
-    for (int idx = pair; idx < p.num_items && ok; idx += npairs, ++local) {
+    for (int idx = next_running(p, seq.first, seq.end, seq.stride); idx < seq.end && ok;
+         idx = next_running(p, idx + seq.stride, seq.end, seq.stride), ++local) {
         const GemmItem it = p.items[idx];
         const PhaseInfo pi = phase_info<C>(p, it);
         const uint32_t idesc = ptx::idesc_f16(2 * kBM, it.nsz, BF16, pi.a_mn, pi.b_mn);
@@ -246,7 +340,7 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
             }
             ptx::tc_fence_after();
             const uint32_t a0 = ptx::smem_u32(s.stages + size_t(stage) * C::kStageBytes);
-            const uint32_t b0 = shared_operand(p, it) ? a0 : a0 + C::kABytes;
+            const uint32_t b0 = shared_operand(it) ? a0 : a0 + C::kABytes;
 #pragma unroll
             for (int kk = 0; kk < C::BK / 16; ++kk) {
                 const uint32_t acc = (kb != kb_begin || kk != 0) ? 1u : 0u;
@@ -277,21 +371,27 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
 }
 
 template <bool BF16, class C>
-__device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_base, int rank, int pair,
-                              int npairs, int warp, int lane) {
+__device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_base, int rank,
+                              const PairItems& seq, int warp, int lane) {
     const int quad = warp & 3;             // TMEM lanes [32 quad, 32 quad + 32) (hardware rule)
     const int ngroups = C::kEpiWarps / 4;  // warps per lane quadrant, splitting the columns
     const int group = (warp - 2) / 4;
     uint8_t* sbuf = s.epi + (warp - 2) * kStageWarpBytes;
     int local = 0;
     const uint32_t even_tempty = ptx::mapa(ptx::smem_u32(s.tempty), 0);
-    for (int idx = pair; idx < p.num_items; idx += npairs, ++local) {
+    for (int idx = next_running(p, seq.first, seq.end, seq.stride); idx < seq.end;
+         idx = next_running(p, idx + seq.stride, seq.end, seq.stride), ++local) {
         const GemmItem it = p.items[idx];
         const MatDev& md = p.mats[it.mat];
         const int slot = local % C::kSlots;
         const uint32_t tphase = uint32_t(local / C::kSlots) & 1u;
         int ok = 1;
-        if (lane == 0) ok = ptx::mbar_wait(&s.tfull[slot], tphase, s.abort, p.timeout_ns) ? 1 : 0;
+        if (lane == 0) {
+            ok = ptx::mbar_wait(&s.tfull[slot], tphase, s.abort, p.timeout_ns) ? 1 : 0;
+            // Poly reads b A with plain loads: acquire A's completion count in
+            // this thread too (the producer already saw it reached).
+            if (ok && it.phase == kPoly && !wait_done(p, s, it)) ok = 0;
+        }
         ok = __shfl_sync(0xffffffffu, ok, 0);
         if (!ok) {
             if (lane == 0) record_timeout(p, s);
@@ -306,12 +406,12 @@ __device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t t
             if (parts <= 1) {
                 store_rows<BF16, true>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per, nullptr, 1,
                                        0, sbuf);
-            } else if constexpr (C::kEpiWarps == 4) {  // split K: Gram only, one warp per lane quadrant
-                // direct stores: the last part's sum is a serial step, which
-                // the staging round trip lengthens (small sets, ResNet-18 Gram +7%)
-                if (split_partial_is_last(p, it, rank, quad, lane, t_row, 0, per))
-                    store_rows<BF16>(p, it, md, row0, t_row, quad, lane, 0, per,
-                                        p.split_part + size_t(it.sid) * 65536, parts, rank * kBM + quad * 32 + lane);
+            } else if (split_partial_is_last(p, it, rank, quad, group, lane, t_row, group * per, (group + 1) * per)) {
+                // split K (Gram): direct stores, since the last part's sum is a
+                // serial step, which the staging round trip lengthens (small
+                // sets, ResNet-18 Gram +7%)
+                store_rows<BF16>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per,
+                                 p.split_part + size_t(it.sid) * 65536, parts, rank * kBM + quad * 32 + lane);
             }
         }
         // The slot may be overwritten once this warp's TMEM loads are done
@@ -319,7 +419,15 @@ __device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t t
         // next UMMAs, so the arrive is relaxed.
         ptx::tc_fence_before();
         __syncwarp();
-        if (lane == 0) ptx::mbar_arrive_cluster_relaxed(even_tempty + uint32_t(slot * 8));
+        if (lane == 0) {
+            ptx::mbar_arrive_cluster_relaxed(even_tempty + uint32_t(slot * 8));
+            // Dataflow: publish this warp's part of the item (every lane's
+            // stores happen before the fence through the warp barrier above).
+            if (p.done != nullptr) {
+                __threadfence();
+                atomicAdd(p.done + it.mat, 1u);
+            }
+        }
     }
 }
 
@@ -344,6 +452,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(C::kThreads, 1)
     s.peer = uint32_t(rank ^ 1);
     const int pair = blockIdx.x / 2, npairs = gridDim.x / 2;
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const PairItems seq(p, pair, npairs);
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < C::STAGES; ++i) {
@@ -359,8 +468,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(C::kThreads, 1)
         *s.never = 0;
         ptx::fence_mbar_init();
     }
-    if (warp == 0 && lane == 0 && pair < p.num_items) {
-        const PhaseInfo pi = phase_info<C>(p, p.items[pair]);
+    if (warp == 0 && lane == 0 && seq.first < seq.end) {
+        const PhaseInfo pi = phase_info<C>(p, p.items[seq.first]);
         ptx::prefetch_tmap(pi.mapA);
         ptx::prefetch_tmap(pi.mapB);
     }
@@ -383,13 +492,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(C::kThreads, 1)
     if (peer_base != tmem_base) {
         if (threadIdx.x == 0) atomicOr(p.status, kStatusInternal);
     } else if (warp == 0) {
-        if (lane == 0) pair_producer<C>(p, s, rank, pair, npairs);
+        if (lane == 0) pair_producer<C>(p, s, rank, seq);
         __syncwarp();
     } else if (warp == 1) {
-        if (lane == 0 && rank == 0) pair_mma<BF16, C>(p, s, tmem_base, pair, npairs);
+        if (lane == 0 && rank == 0) pair_mma<BF16, C>(p, s, tmem_base, seq);
         __syncwarp();
     } else {
-        pair_epilogue<BF16, C>(p, s, tmem_base, rank, pair, npairs, warp, lane);
+        pair_epilogue<BF16, C>(p, s, tmem_base, rank, seq, warp, lane);
     }
     ptx::tc_fence_before();
     __syncthreads();
@@ -402,17 +511,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(C::kThreads, 1)
 
 // Co-resident CTA pairs of one kernel configuration on each device, found
 // once per device (the function attribute is per device, too).  Concurrent
-// first launches on one device may both query; they store the same value.
+// first queries on one device may both run; they store the same value.
 constexpr int kMaxDevices = 64;
 
 template <bool BF16, class C>
-cudaError_t launch_pair_cfg(const GemmLaunch& p, int num_sms, cudaStream_t st) {
-    static std::atomic<int> max_pairs_of[kMaxDevices];
+cudaError_t max_pairs_of(int num_sms, int* out) {
+    static std::atomic<int> cache[kMaxDevices];
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-    int max_pairs = max_pairs_of[dev].load(std::memory_order_acquire);
+    int max_pairs = cache[dev].load(std::memory_order_acquire);
     if (max_pairs == 0) {
         e = cudaFuncSetAttribute(tc_pair_kernel<BF16, C>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  int(C::kSmemBytes));
@@ -426,21 +535,46 @@ cudaError_t launch_pair_cfg(const GemmLaunch& p, int num_sms, cudaStream_t st) {
         if (e != cudaSuccess) return e;
         if (clusters < 1) return cudaErrorInvalidConfiguration;
         max_pairs = clusters < num_sms / 2 ? clusters : num_sms / 2;
-        max_pairs_of[dev].store(max_pairs, std::memory_order_release);
+        cache[dev].store(max_pairs, std::memory_order_release);
     }
-    const int npairs = p.num_items < max_pairs ? p.num_items : max_pairs;
+    *out = max_pairs;
+    return cudaSuccess;
+}
+
+// Per-phase launches: min(items, co-resident pairs) pairs.  Dataflow launch:
+// exactly the plan's `npairs` pairs, which must all be resident at once (a
+// pair may wait for items of any other), so a plan for more pairs than fit is
+// refused.
+template <bool BF16, class C>
+cudaError_t launch_pair_cfg(const GemmLaunch& p, int num_sms, cudaStream_t st, int npairs) {
+    int max_pairs = 0;
+    cudaError_t e = max_pairs_of<BF16, C>(num_sms, &max_pairs);
+    if (e != cudaSuccess) return e;
+    if (p.pair_begin != nullptr) {
+        if (npairs < 1 || npairs > max_pairs) return cudaErrorInvalidConfiguration;
+    } else {
+        npairs = p.num_items < max_pairs ? p.num_items : max_pairs;
+    }
     return launch_kernel(tc_pair_kernel<BF16, C>, unsigned(2 * npairs), C::kThreads, C::kSmemBytes, st, p.pdl != 0, p);
 }
 
 }  // namespace
 
-cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t st) {
+cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t st, int epi_warps,
+                                int npairs) {
     if (p.num_items == 0) return cudaSuccess;
     const bool bf = elem == kBF16;
-    if (p.phase == kPoly)
-        return bf ? launch_pair_cfg<true, PairCfg2Wide>(p, num_sms, st)
-                  : launch_pair_cfg<false, PairCfg2Wide>(p, num_sms, st);
-    return bf ? launch_pair_cfg<true, PairCfg2>(p, num_sms, st) : launch_pair_cfg<false, PairCfg2>(p, num_sms, st);
+    if (epi_warps == 8)
+        return bf ? launch_pair_cfg<true, PairCfg2Wide>(p, num_sms, st, npairs)
+                  : launch_pair_cfg<false, PairCfg2Wide>(p, num_sms, st, npairs);
+    return bf ? launch_pair_cfg<true, PairCfg2>(p, num_sms, st, npairs)
+              : launch_pair_cfg<false, PairCfg2>(p, num_sms, st, npairs);
+}
+
+cudaError_t tc_pair_dataflow_capacity(int elem, int num_sms, int* pairs) {
+    *pairs = 0;
+    return elem == kBF16 ? max_pairs_of<true, PairCfg2Wide>(num_sms, pairs)
+                         : max_pairs_of<false, PairCfg2Wide>(num_sms, pairs);
 }
 
 }  // namespace slorr

@@ -80,6 +80,23 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
     }
 }
 
+// ---- global memory flags -----------------------------------------------------------
+
+// Load with acquire semantics at GPU scope: every write that was released
+// before the value read (by any thread of the GPU) is visible afterwards.
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// Relaxed load at GPU scope (a flag polled for a change, ordering nothing).
+__device__ __forceinline__ uint32_t ld_relaxed_gpu(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
 // ---- programmatic dependent launch -------------------------------------------------
 
 // Blocks until every grid this one depends on programmatically has completed

@@ -47,6 +47,12 @@ __device__ __forceinline__ float2 unpack2(uint32_t u) {
     }
 }
 
+// The Polar Express step an item belongs to: its own (dataflow launch) or the
+// launch's (per-phase launches).
+__device__ __forceinline__ int item_step(const GemmLaunch& p, const GemmItem& it) {
+    return p.step >= 0 ? p.step : int(it.step);
+}
+
 struct PhaseInfo {
     const void* mapA;
     const void* mapB;
@@ -66,14 +72,15 @@ __device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmI
     const MatDev& md = p.mats[it.mat];
     const uint8_t* maps = reinterpret_cast<const uint8_t*>(p.maps) + size_t(it.mat) * kMapsPerMatrix * 128;
     const bool tr = md.transposed != 0;
+    const int cur = item_step(p, it) & 1;
     PhaseInfo pi;
-    if (p.phase == kGram) {
+    if (it.phase == kGram) {
         pi.a_mn = tr;
         pi.b_mn = tr;
-        pi.mapA = xmap(maps, p.cur, tr);
+        pi.mapA = xmap(maps, cur, tr);
         pi.mapB = pi.mapA;
         pi.nkb = md.Qpad / C::BK;
-    } else if (p.phase == kPoly) {
+    } else if (it.phase == kPoly) {
         pi.a_mn = false;
         pi.b_mn = false;
         pi.mapA = maps + 4 * 128;
@@ -83,7 +90,7 @@ __device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmI
         pi.a_mn = false;
         pi.b_mn = !tr;
         pi.mapA = maps + 5 * 128;
-        pi.mapB = xmap(maps, p.cur, pi.b_mn);
+        pi.mapB = xmap(maps, cur, pi.b_mn);
         pi.nkb = md.Ppad / C::BK;
     }
     return pi;
@@ -110,14 +117,16 @@ __device__ __forceinline__ uint64_t operand_desc(uint32_t base, int kk, bool mn)
 }
 
 // Split K, one part of a tile: this warp stores its 32 rows of the part's
-// fp32 accumulator (columns [32 ch_begin, 32 ch_end) of the tile) in the
-// part's 256 x 256 slot, split_part + (sid + s) * 65536, column-major so that
-// each column's 32 rows are one coalesced segment, and counts them in
-// split_cnt[sid * 8 + rank * 4 + quad].  Returns true in the warp that
-// counts last for its rows (the other parts' rows are then visible to it);
-// that warp resets the count for the next launch.
+// fp32 accumulator (columns [32 ch_begin, 32 ch_end) of the tile, the share
+// of epilogue warp group `group`) in the part's 256 x 256 slot, split_part +
+// (sid + s) * 65536, column-major so that each column's 32 rows are one
+// coalesced segment, and counts them in split_cnt[sid * 16 + rank * 8 +
+// group * 4 + quad].  Returns true in the warp that counts last for its rows
+// and columns (the other parts' values there are then visible to it); that
+// warp resets the count for the next use.
 __device__ __forceinline__ bool split_partial_is_last(const GemmLaunch& p, const GemmItem& it, int rank, int quad,
-                                                      int lane, uint32_t t_row, int ch_begin, int ch_end) {
+                                                      int group, int lane, uint32_t t_row, int ch_begin,
+                                                      int ch_end) {
     const int parts = it.ksplit >> 8, own = it.ksplit & 0xff;
     const int row_t = rank * kBM + quad * 32 + lane;
     float* dst = p.split_part + (size_t(it.sid) + own) * 65536 + row_t;
@@ -130,7 +139,7 @@ __device__ __forceinline__ bool split_partial_is_last(const GemmLaunch& p, const
     }
     __threadfence();
     __syncwarp();
-    uint32_t* cnt = p.split_cnt + size_t(it.sid) * 8 + rank * 4 + quad;
+    uint32_t* cnt = p.split_cnt + size_t(it.sid) * 16 + rank * 8 + group * 4 + quad;
     int last = 0;
     if (lane == 0) {
         last = atomicAdd(cnt, 1u) == uint32_t(parts - 1) ? 1 : 0;
@@ -188,12 +197,13 @@ __device__ __forceinline__ void put_cols(const uint8_t* buf, int lane, uint16_t*
 }
 
 // The 32 x 32 chunk at src[(r0 + r) * ld + c0 + c] in the put_rows order:
-// v[i] holds row 8 i + lane / 4, columns 8 (lane % 4) .. + 7.
+// v[i] holds row 8 i + lane / 4, columns 8 (lane % 4) .. + 7.  The loads
+// bypass L1 (the chunk was written by other SMs in the same launch).
 __device__ __forceinline__ void get_rows(const uint16_t* src, int64_t ld, int r0, int c0, int lane, uint4 (&v)[4]) {
     const int seg = lane & 3;
 #pragma unroll
     for (int i = 0; i < 4; ++i)
-        v[i] = *reinterpret_cast<const uint4*>(src + int64_t(r0 + i * 8 + (lane >> 2)) * ld + c0 + seg * 8);
+        v[i] = __ldcg(reinterpret_cast<const uint4*>(src + int64_t(r0 + i * 8 + (lane >> 2)) * ld + c0 + seg * 8));
 }
 
 // A chunk from get_rows, through the staging buffer, as this lane's row.
@@ -215,7 +225,7 @@ __device__ __forceinline__ void own_row(uint8_t* buf, int lane, const uint4 (&v)
 //   Gram / Poly: c * acc (+ b A + a I for Poly) into the Ppad x Ppad output,
 //           plus the transpose of every 128 x 128 block (I, J), J > I, whose
 //           mirror tile is skipped (tiles are 256 rows by 256 columns).
-// In the first step after the fused norm pass (p.x0_scaled) the stored X_0
+// In the first step after the fused norm pass (p.fused_norm) the stored X_0
 // is W itself: the Gram scales acc by x0_scale^2 and the Update by x0_scale.
 // With split K (Gram), the accumulator is replaced by the sum, in part
 // order, of the `parts` fp32 partials at split_tile (row row_t of the tile;
@@ -229,9 +239,10 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
     const int row_w = row0 + quad * 32;  // the warp's first row
     const int row = row_w + lane;
     const int nch = ch_end;
-    const float xs = p.x0_scaled ? p.scalars[it.mat].x0_scale : 1.f;
-    if (p.phase == kUpdate) {
-        uint16_t* out = reinterpret_cast<uint16_t*>(md.x[p.cur ^ 1]);
+    const int t = item_step(p, it);
+    const float xs = (p.fused_norm && t == 0) ? p.scalars[it.mat].x0_scale : 1.f;
+    if (it.phase == kUpdate) {
+        uint16_t* out = reinterpret_cast<uint16_t*>(md.x[(t & 1) ^ 1]);
         const int64_t ld = md.ld;
         for (int ch = ch_begin; ch < nch; ++ch) {
             uint32_t r[32];
@@ -268,11 +279,12 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
             }
         }
     } else {
-        uint16_t* out = reinterpret_cast<uint16_t*>(p.phase == kGram ? md.a : md.b);
+        uint16_t* out = reinterpret_cast<uint16_t*>(it.phase == kGram ? md.a : md.b);
         const uint16_t* amat = reinterpret_cast<const uint16_t*>(md.a);
         const int64_t ld = md.Ppad;
-        const bool poly = p.phase == kPoly;
-        const float cacc = poly ? p.c : xs * xs;
+        const bool poly = it.phase == kPoly;
+        const float ca = p.coef[t][0], cb = p.coef[t][1];
+        const float cacc = poly ? p.coef[t][2] : xs * xs;
         // Poly reads b A at the output position: loads for the next chunk are
         // issued before the current chunk is processed (staged: coalesced
         // loads, turned into this lane's row through the staging buffer).
@@ -284,7 +296,7 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
                 const uint4* src =
                     reinterpret_cast<const uint4*>(amat + int64_t(row) * ld + it.tn * kBNMax + ch_begin * 32);
 #pragma unroll
-                for (int q = 0; q < 4; ++q) e_next[q] = src[q];
+                for (int q = 0; q < 4; ++q) e_next[q] = __ldcg(src + q);
             }
         }
         for (int ch = ch_begin; ch < nch; ++ch) {
@@ -301,7 +313,7 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
                     if (ch + 1 < nch) {
                         const uint4* src = reinterpret_cast<const uint4*>(amat + off + 32);
 #pragma unroll
-                        for (int q = 0; q < 4; ++q) e_next[q] = src[q];
+                        for (int q = 0; q < 4; ++q) e_next[q] = __ldcg(src + q);
                     }
                 }
             }
@@ -310,27 +322,18 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
                 ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
                 ptx::tmem_ld_wait();
             } else {
-                // every part from memory, in part order, two parts' loads in
-                // flight at a time: the sum does not depend on which part
-                // finished last
+                // every part from memory, in part order: the sum does not
+                // depend on which part finished last
                 const float* src = split_tile + size_t(ch * 32) * 256 + row_t;
 #pragma unroll
                 for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(__ldcg(src + size_t(j) * 256));
-                for (int q = 1; q < parts; q += 2) {
+                for (int q = 1; q < parts; ++q) {
                     const float* s1 = src + size_t(q) * 65536;
-                    float a[32], b[32];
+                    float a[32];
 #pragma unroll
                     for (int j = 0; j < 32; ++j) a[j] = __ldcg(s1 + size_t(j) * 256);
-                    if (q + 1 < parts) {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) b[j] = __ldcg(s1 + 65536 + size_t(j) * 256);
-                    }
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        float v = __uint_as_float(r[j]) + a[j];
-                        if (q + 1 < parts) v += b[j];
-                        r[j] = __float_as_uint(v);
-                    }
+                    for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(__uint_as_float(r[j]) + a[j]);
                 }
             }
             uint4 o[4];
@@ -344,8 +347,8 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
                 if (poly) {
                     // M = c A^2 + b A + a I
                     const float2 x = unpack2<BF16>(ew[j]);
-                    lo = fmaf(p.b, x.x, lo) + (2 * j == d ? p.a : 0.f);
-                    hi = fmaf(p.b, x.y, hi) + (2 * j + 1 == d ? p.a : 0.f);
+                    lo = fmaf(cb, x.x, lo) + (2 * j == d ? ca : 0.f);
+                    hi = fmaf(cb, x.y, hi) + (2 * j + 1 == d ? ca : 0.f);
                 }
                 ow[j] = pack2<BF16>(lo, hi);
             }

@@ -31,6 +31,8 @@ FLAG_NO_PDL = 512
 FLAG_SEPARATE_NORM = 1024
 FLAG_NO_SPLIT_K = 2048
 FLAG_GRAPH = 4096
+FLAG_PHASE_LAUNCHES = 16384
+FLAG_DATAFLOW = 32768
 
 
 class SlorrError(RuntimeError):
@@ -91,6 +93,8 @@ def load_library(path: str | None = None) -> ctypes.CDLL:
         "slorr_gemm_items": (i32, [vp, i32, ctypes.POINTER(i32)]),
         "slorr_gemm_pair_load": (i32, [vp, i32, i32, ctypes.POINTER(i64), ctypes.POINTER(i64)]),
         "slorr_gemm_item_list": (i32, [vp, i32, ctypes.POINTER(i32), i32]),
+        "slorr_dataflow_items": (i32, [vp, ctypes.POINTER(i32), i32, ctypes.POINTER(i32), ctypes.POINTER(i32),
+                                       ctypes.POINTER(dbl)]),
         "slorr_set_timing": (i32, [vp, i32]),
         "slorr_read_timing": (i32, [vp, ctypes.POINTER(dbl), ctypes.POINTER(i64), i32]),
         "slorr_frob_sq_noalloc": (i32, [vp, i64, i64, i32, vp, vp]),
@@ -245,6 +249,18 @@ def slorr_gemm_item_list(handle, phase: int) -> np.ndarray:
     return np.frombuffer(buf, dtype=np.int32, count=7 * n).reshape(n, 7).copy()
 
 
+def slorr_dataflow_items(handle):
+    """(items, npairs, makespan_k): the dataflow plan as an (n, 10) int32 array
+    of (pair, seq, step, phase, mat, tm, tn, part, parts, wait), pair by pair."""
+    lib = load_library()
+    npairs, count, mk = ctypes.c_int32(), ctypes.c_int32(), ctypes.c_double()
+    _check(lib.slorr_dataflow_items(handle, None, 0, ctypes.byref(npairs), ctypes.byref(count), ctypes.byref(mk)))
+    n = count.value
+    buf = (ctypes.c_int32 * max(1, 10 * n))()
+    _check(lib.slorr_dataflow_items(handle, buf, 10 * n, ctypes.byref(npairs), ctypes.byref(count), None))
+    return np.frombuffer(buf, dtype=np.int32, count=10 * n).reshape(n, 10).copy(), npairs.value, mk.value
+
+
 def slorr_partition(shapes, world: int, rank: int) -> list[int]:
     arr, n = _shapes(shapes)
     out = (ctypes.c_int32 * max(n, 1))()
@@ -253,7 +269,7 @@ def slorr_partition(shapes, world: int, rank: int) -> list[int]:
     return [int(out[i]) for i in range(cnt.value)]
 
 
-KERNEL_KINDS = ("sumsq", "cast", "gram", "poly", "update", "dot", "combine", "normcast")
+KERNEL_KINDS = ("sumsq", "cast", "gram", "poly", "update", "dot", "combine", "normcast", "gemm")
 
 
 def slorr_set_timing(handle, enable: bool) -> None:

@@ -96,22 +96,27 @@ def test_pair_vit_l16_layers_match_simt():
         assert rel(a, b) <= 24 * 2.0 ** -10, (i, rel(a, b))
 
 
-def test_pair_bounded_wait_timeout_and_recovery():
+@pytest.mark.parametrize("mode", ["dataflow", "phase_launches"])
+def test_pair_bounded_wait_timeout_and_recovery(mode):
     """SLORR_FLAG_TEST_STALL in the pair kernel: the even CTA's MMA thread waits on
     a barrier nothing arrives on, gives up after timeout_s, and sets both CTAs'
     abort flags; every role unwinds, the even CTA drains the pair's copies, and
-    the call reports SLORR_ERR_TIMEOUT.  A normal pair call afterwards matches
-    the CUDA-core path."""
-    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_TEST_STALL, FLAG_SIMT_GEMM
+    the call reports SLORR_ERR_TIMEOUT.  In the dataflow launch the other pairs'
+    producers, waiting for completions that never come, see the timeout in the
+    status word and unwind too.  A normal pair call afterwards matches the
+    CUDA-core path."""
+    from paper_2607_08754_gb300.slorr import (Regularizer, FLAG_TEST_STALL, FLAG_SIMT_GEMM, FLAG_PHASE_LAUNCHES,
+                                              FLAG_DATAFLOW)
     shapes = [(256, 512), (384, 128), (640, 1000)]
     Ws = [workloads.random_matrix(s, 31 + i, 0.05) for i, s in enumerate(shapes)]
     w = [torch.from_numpy(W).cuda() for W in Ws]
-    stall = Regularizer(shapes, flags=FLAG_TEST_STALL, timeout_s=0.05)
+    extra = FLAG_PHASE_LAUNCHES if mode == "phase_launches" else FLAG_DATAFLOW
+    stall = Regularizer(shapes, flags=FLAG_TEST_STALL | extra, timeout_s=0.05)
     stall.run_steps(w, 1)
     torch.cuda.synchronize()
     assert stall.status() == 5          # SLORR_ERR_TIMEOUT
     assert stall.status() == 0
-    tc = Regularizer(shapes)
+    tc = Regularizer(shapes, flags=extra)
     st = Regularizer(shapes, flags=FLAG_SIMT_GEMM)
     tc.run_steps(w, 2)
     st.run_steps(w, 2)
@@ -200,3 +205,41 @@ def test_split_k_is_deterministic():
     for o in outs[1:]:
         for a, b in zip(outs[0], o):
             assert torch.equal(a, b)
+
+
+@pytest.mark.parametrize("compute", ["fp16", "bf16"])
+def test_dataflow_launch_is_bit_identical_to_phase_launches(compute):
+    """The dataflow launch (every Gram, Poly and Update tile of the T steps in
+    one launch, ordered by per-matrix completion counts) computes
+    each tile exactly as the per-phase launches (SLORR_FLAG_PHASE_LAUNCHES)
+    do: the same K order, split-K parts and epilogue arithmetic.  Iterates
+    after 1, 2 and 6 steps (slorr_run_steps skips the later steps' items of
+    the dataflow plan), per-matrix values, gradients and the loss are equal
+    bit for bit, on a set with every tile case and split-K Gram tiles."""
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_PHASE_LAUNCHES, FLAG_DATAFLOW, slorr_gemm_item_list
+    Ws = [workloads.random_matrix(s, seed=800 + i, std=0.02) for i, s in enumerate(SHAPES)]
+    Ws += [workloads.random_matrix(s, seed=820 + i, std=0.02) for i, s in enumerate([(512, 4608), (4608, 384)])]
+    Ws += workloads.generate("resnet18", [0, 7, 15, 20])
+    shapes = [W.shape for W in Ws]
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    df = Regularizer(shapes, compute=compute, flags=FLAG_DATAFLOW)
+    ph = Regularizer(shapes, compute=compute, flags=FLAG_PHASE_LAUNCHES)
+    assert (slorr_gemm_item_list(df.handle, 0)[:, 6] > 1).any()   # some Gram tiles are split
+    for k in (1, 2, 6):
+        df.run_steps(w, k)
+        ph.run_steps(w, k)
+        torch.cuda.synchronize()
+        assert df.status() == 0 and ph.status() == 0
+        for i in range(len(shapes)):
+            assert torch.equal(df.iterate(i, k).cpu(), ph.iterate(i, k).cpu()), (k, i, shapes[i])
+    out = []
+    for reg in (df, ph):
+        g = [torch.zeros_like(x) for x in w]
+        per = torch.empty(len(shapes), device="cuda")
+        loss = reg(w, g, per_matrix=per)
+        torch.cuda.synchronize()
+        assert reg.status() == 0
+        out.append((loss.cpu(), per.cpu(), [x.cpu() for x in g]))
+    assert torch.equal(out[0][0], out[1][0]) and torch.equal(out[0][1], out[1][1])
+    for a, b in zip(out[0][2], out[1][2]):
+        assert torch.equal(a, b)

@@ -368,3 +368,97 @@ def test_split_plan_items(lib):
         assert all(q == parts for _, q in v)
     with pytest.raises(slorr.SlorrError):
         slorr._check(slorr.load_library().slorr_gemm_item_list(slorr.Regularizer(rn).handle, 0, None, 0))
+
+
+def _df_cost(shapes, phase, nsz, K):
+    """The planner's cost of one item in K blocks (written out again here)."""
+    kb = (K // 64) * (0.5 + 0.5 * nsz / 256.0)
+    return (1.6 * kb if phase == 1 else kb) + 1.0
+
+
+@pytest.mark.parametrize("name", ["cfg1", "resnet18", "vit_b16", "vit_l16"])
+def test_dataflow_plan(lib, name):
+    """The dataflow plan (every Gram, Poly and Update tile of the T steps in
+    one launch): each step's items are exactly the per-phase tiles; each pair's
+    items are in planned start order; every item of a matrix's (step, phase)
+    group starts after every item of the group before it (so the launch cannot
+    deadlock); each item waits for 16 completions per item of its matrix's
+    earlier groups; and the planned duration is within 15% of the larger of
+    the two lower bounds, total work / 76 pairs and the longest chain of one
+    matrix's phases."""
+    import workloads
+    shapes = workloads.shapes(name)
+    T = 6
+    reg = slorr.Regularizer(shapes, iters=T, flags=slorr.FLAG_DATAFLOW)
+    items, npairs, makespan = slorr.slorr_dataflow_items(reg.handle)
+    assert npairs == 76
+    pair, seq, step, phase, mat = (items[:, k] for k in range(5))
+    # the per-phase tiles, T times
+    for ph in range(3):
+        ref = sorted(map(tuple, slorr.slorr_gemm_item_list(reg.handle, ph)[:, [0, 1, 2, 5, 6]].tolist()))
+        for t in range(T):
+            sel = items[(step == t) & (phase == ph)]
+            assert sorted(map(tuple, sel[:, [4, 5, 6, 7, 8]].tolist())) == ref
+    assert sorted(seq.tolist()) == list(range(len(items)))
+    for q in range(npairs):
+        s = seq[pair == q]
+        assert np.all(np.diff(s) > 0)
+    counts = {}
+    for ph in range(3):
+        for r in slorr.slorr_gemm_item_list(reg.handle, ph).tolist():
+            counts[(r[0], ph)] = counts.get((r[0], ph), 0) + 1
+    for m in range(len(shapes)):
+        g = (step * 3 + phase)[mat == m]
+        s = seq[mat == m]
+        w = items[mat == m][:, 9]
+        done = 0
+        for k in range(3 * T):
+            assert np.all(w[g == k] == done)
+            if k + 1 < 3 * T:
+                assert s[g == k].max() < s[g == k + 1].min()
+            done += 16 * counts[(m, k % 3)]
+    # planned duration against the lower bounds (the same cost model)
+    cost = {}
+    total = 0.0
+    for ph in range(3):
+        for r in slorr.slorr_gemm_item_list(reg.handle, ph).tolist():
+            P, Q = min(shapes[r[0]]), max(shapes[r[0]])
+            Pp, Qp = -(-P // 128) * 128, -(-Q // 128) * 128
+            K = (Qp if ph == 0 else Pp) // r[6]
+            c = _df_cost(shapes, ph, r[4], K) + (2.0 if r[6] > 1 else 0.0)
+            total += T * c
+            cost[(r[0], ph)] = max(cost.get((r[0], ph), 0.0), c)
+    chain = max(T * sum(cost[(m, ph)] + 4.0 for ph in range(3)) - 4.0 for m in range(len(shapes)))
+    bound = max(total / 76, chain)
+    assert bound <= makespan <= 1.15 * bound, (makespan, total / 76, chain)
+
+
+def test_dataflow_plan_is_absent_for_phase_launches(lib):
+    for kw in ({"flags": slorr.FLAG_PHASE_LAUNCHES}, {"compute": "fp32"}, {"flags": slorr.FLAG_SIMT_GEMM}):
+        r = slorr.Regularizer([(256, 512)], **kw)
+        with pytest.raises(slorr.SlorrError):
+            slorr.slorr_dataflow_items(r.handle)
+    with pytest.raises(slorr.SlorrError):
+        slorr.Regularizer([(256, 512)], flags=slorr.FLAG_PHASE_LAUNCHES | slorr.FLAG_DATAFLOW)
+
+
+def test_launch_mode_is_chosen_by_set_size(lib):
+    """Without a flag the plan takes the dataflow launch for sets of up to
+    about 3 ms of GEMM work (7000 K blocks of a 256 x 256 tile over 76 pairs,
+    the measured crossover) and per-phase launches above; SLORR_FLAG_DATAFLOW
+    forces the dataflow launch."""
+    import workloads
+    for name, df in (("cfg1", True), ("resnet18", True), ("vit_b16", True), ("vit_ladder_vit_s", True),
+                     ("vit_l16", False), ("decoder_560m", False), ("vit_ladder_vit_h", False)):
+        shapes = workloads.shapes(name)
+        r = slorr.Regularizer(shapes)
+        forced = slorr.Regularizer(shapes, flags=slorr.FLAG_DATAFLOW)
+        mk = slorr.slorr_dataflow_items(forced.handle)[2]
+        assert (mk < 7000) == df, (name, mk)
+        if df:
+            assert slorr.slorr_dataflow_items(r.handle)[2] == mk
+        else:
+            with pytest.raises(slorr.SlorrError):
+                slorr.slorr_dataflow_items(r.handle)
+        # the workspace holds the dataflow plan only when it is used
+        assert (forced.workspace_bytes > r.workspace_bytes) == (not df)
