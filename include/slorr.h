@@ -137,10 +137,13 @@ typedef struct slorr_options {
                                        stored, and so on, with no grid-wide barrier, so
                                        the phases of different matrices overlap.
                                        Without either flag the plan takes the dataflow
-                                       launch for sets of up to about 3 ms of GEMM work
-                                       on GB300 (measured faster there: fewer launch
-                                       tails) and per-phase launches for larger ones
-                                       (measured faster there: lighter epilogues).
+                                       launch for sets with enough independent work to
+                                       overlap (no matrix's chain of phases longer than
+                                       3/4 of the work per pair) whose per-phase
+                                       launches would be short (fewer than 7 Gram tiles
+                                       per CTA pair): measured faster there (fewer
+                                       launch tails); per-phase launches otherwise
+                                       (measured faster: lighter epilogues).
                                        Both give the same results bit for bit; the two
                                        flags exclude each other                         */
 

@@ -69,6 +69,8 @@ struct slorr_handle {
     std::vector<int32_t> df_seq;         // each df item's rank in the plan's global start order
     int df_pairs = 0;
     double df_makespan = 0.0;            // simulated, in K blocks of a 256 x 256 tile
+    double df_work = 0.0;                // total cost / pairs (a lower bound of the makespan)
+    double df_chain = 0.0;               // the longest chain of one matrix's phases (the other bound)
     bool df = false;                     // the GEMMs run as the dataflow launch
     std::vector<MemItem> w_items;  // tiles of W (sumsq, dot, combine)
     std::vector<MemItem> x_items;  // tiles of the padded iterate (cast)
@@ -79,7 +81,7 @@ struct slorr_handle {
     size_t off_status = 0, off_counters = 0, off_scalars = 0, off_partials = 0, off_partials_max = 0,
            off_tilebase = 0, off_tilecount = 0, off_xtilebase = 0, off_xtilecount = 0, off_split_cnt = 0,
            off_split_part = 0, off_mats = 0, off_maps = 0, off_tc_items[3] = {}, off_simt_items[3] = {},
-           off_done = 0, off_df_items = 0, off_df_pair_begin = 0,
+           off_done = 0, off_df_items = 0, off_df_pair_begin = 0, off_coef = 0,
            off_w_items = 0, off_x_items = 0, off_ptrs = 0, off_plan_end = 0, total_bytes = 0;
     // device state
     const void* prepared_ws = nullptr;
@@ -283,16 +285,22 @@ void split_gram_items(slorr_handle* h) {
 // (the last increments, the producer's wake-up, the first copies landing).
 constexpr double kDepLatency = 4.0;
 
-// Which launch a set gets by default.  Measured on GB300 (bench, one box, both
-// modes back to back): the dataflow launch is faster for sets of up to about
-// 3 ms of GEMM work (ViT-S -20%, ViT-B/16 -8%, the first 48 ViT-L/16 matrices
-// -4%, cfg1 -15%), equal around the first 64 ViT-L/16 matrices and ViT-B
-// with 24 blocks, and slower beyond (ViT-L/16 +1.5%, 560M decoder and ViT-H
-// +5%): per item it runs 8 epilogue warps in every phase and mixes phases and
-// matrices on each pair, which costs more than the 3 T launch tails it saves
-// once each phase fills the pairs many times over.  The crossover, in the
-// planner's units (K blocks of a 256 x 256 tile on 76 pairs), is put at 7000.
-constexpr double kDataflowMaxWork = 7000.0;
+// Which launch a set gets by default.  Per tile the dataflow launch is a few
+// per cent slower than the phase-specialised per-phase kernels (8 epilogue
+// warps in every phase, phases and matrices mixed on each pair, a dependency
+// hand-off through global memory), and what it saves is the tail of each of
+// the 3 T per-phase launches.  Measured on GB300 (bench, one box, both modes
+// back to back), it is faster when two things hold:
+// - the set is work-bound: its longest chain of one matrix's phases is
+//   shorter than the work per pair (chain-bound sets -- ResNet-18 +7%, cfg1
+//   +2.6% -- wait on dependency hand-offs instead);
+// - the per-phase launches are short: fewer than 7 Gram (or Poly) tiles per
+//   pair, so a launch tail is a large share (ViT-S -12%, ViT-512 -7%,
+//   ViT-B/16 -4.4%, the 560M decoder's first 4 blocks -4.7%, the first 32 and
+//   48 ViT-L/16 matrices -3% and -2%; ViT-B with 24 blocks, 7.6 tiles per
+//   pair, +2%; ViT-L/16, 12.6, +3%; 560M, 25.6, +5%).
+constexpr double kDataflowMaxChainShare = 0.75;
+constexpr double kDataflowMaxRounds = 7.0;
 
 double df_cost(const slorr_handle* h, const GemmItem& it) {
     const Geom& g = h->geom[it.mat];
@@ -311,6 +319,8 @@ void build_dataflow(slorr_handle* h, int npairs) {
     h->df_pair_begin.assign(size_t(npairs) + 1, 0);
     h->df_pairs = npairs;
     h->df_makespan = 0.0;
+    h->df_work = 0.0;
+    h->df_chain = 0.0;
     const int count = int(h->shapes.size());
     const int T = h->opt.iters;
     // items of each (matrix, phase), in the per-phase plan's order
@@ -369,6 +379,10 @@ void build_dataflow(slorr_handle* h, int npairs) {
             ready.push(Ready{level[g], df_cost(h, it), gmat(g), int(k), g, v[k]});
         }
     };
+    // the two lower bounds of the makespan
+    for (int m = 0; m < count; ++m) h->df_chain = std::max(h->df_chain, level[size_t(m) * T * 3] - kDepLatency);
+    for (int ph = 0; ph < 3; ++ph)
+        for (const GemmItem& it : h->tc_items[ph]) h->df_work += T * df_cost(h, it) / npairs;
     // every matrix has at least one tile in every phase, so each group is
     // released when its predecessor's last item is assigned
     size_t total = 0;
@@ -539,7 +553,9 @@ void build_plan(slorr_handle* h) {
     h->df = false;
     if (dataflow_possible(h)) {
         build_dataflow(h, kPlanPairs);
-        h->df = (h->opt.flags & SLORR_FLAG_DATAFLOW) || h->df_makespan < kDataflowMaxWork;
+        const double rounds = double(std::min(h->tc_items[kGram].size(), h->tc_items[kPoly].size())) / kPlanPairs;
+        h->df = (h->opt.flags & SLORR_FLAG_DATAFLOW) ||
+                (h->df_chain < kDataflowMaxChainShare * h->df_work && rounds < kDataflowMaxRounds);
         if (!h->df) {
             h->df_items.clear();
             h->df_seq.clear();
@@ -582,6 +598,8 @@ void build_plan(slorr_handle* h) {
         h->off_simt_items[ph] = off;
         off = align_up(off + h->simt_items[ph].size() * sizeof(GemmItem), 256);
     }
+    h->off_coef = off;
+    off = align_up(off + size_t(3 * h->opt.iters) * sizeof(float), 256);
     h->off_df_items = off;
     off = align_up(off + h->df_items.size() * sizeof(GemmItem), 256);
     h->off_df_pair_begin = off;
@@ -717,6 +735,8 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
         put(plan, h->off_tc_items[ph] - base, h->tc_items[ph].data(), h->tc_items[ph].size());
         put(plan, h->off_simt_items[ph] - base, h->simt_items[ph].data(), h->simt_items[ph].size());
     }
+    std::vector<float> coef(h->coeffs.begin(), h->coeffs.end());
+    put(plan, h->off_coef - base, coef.data(), coef.size());
     put(plan, h->off_df_items - base, h->df_items.data(), h->df_items.size());
     put(plan, h->off_df_pair_begin - base, h->df_pair_begin.data(), h->df_pair_begin.size());
     put(plan, h->off_w_items - base, h->w_items.data(), h->w_items.size());
@@ -962,8 +982,7 @@ slorr_status launch_all(slorr_handle* h, uint8_t* ws, float* loss, float* per, i
     g.scalars = reinterpret_cast<const MatScalars*>(ws + h->off_scalars);
     g.split_part = reinterpret_cast<float*>(ws + h->off_split_part);
     g.split_cnt = reinterpret_cast<uint32_t*>(ws + h->off_split_cnt);
-    for (int t = 0; t < h->opt.iters; ++t)
-        for (int k = 0; k < 3; ++k) g.coef[t][k] = float(h->coeffs[3 * t + k]);
+    g.coef = reinterpret_cast<const float*>(ws + h->off_coef);
     if (use_tc && dataflow(h) && steps > 0) {
         // every phase of every step in one launch, ordered by completion counts
         g.items = reinterpret_cast<const GemmItem*>(ws + h->off_df_items);
@@ -973,7 +992,7 @@ slorr_status launch_all(slorr_handle* h, uint8_t* ws, float* loss, float* per, i
         g.pair_begin = reinterpret_cast<const int32_t*>(ws + h->off_df_pair_begin);
         g.done = reinterpret_cast<uint32_t*>(ws + h->off_done);
         Traced tr(h, 8, st);
-        e = launch_gemm_tc_pair(g, h->elem, h->num_sms, st, kDataflowEpiWarps, h->df_pairs);
+        e = launch_gemm_tc_pair(g, h->elem, h->num_sms, st, -1, h->df_pairs);
         if (e != cudaSuccess) return cuda_fail(e, "gemm launch");
         tr.done();
     } else {
@@ -984,7 +1003,7 @@ slorr_status launch_all(slorr_handle* h, uint8_t* ws, float* loss, float* per, i
                 if (use_tc) {
                     g.items = reinterpret_cast<const GemmItem*>(ws + h->off_tc_items[ph]);
                     g.num_items = int(h->tc_items[ph].size());
-                    e = launch_gemm_tc_pair(g, h->elem, h->num_sms, st, ph == kPoly ? 8 : 4, 0);
+                    e = launch_gemm_tc_pair(g, h->elem, h->num_sms, st, ph, 0);
                 } else {
                     g.items = reinterpret_cast<const GemmItem*>(ws + h->off_simt_items[ph]);
                     g.num_items = int(h->simt_items[ph].size());

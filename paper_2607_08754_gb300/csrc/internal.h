@@ -131,7 +131,7 @@ struct GemmLaunch {
     int32_t num_items;
     int32_t step;              // per-phase launch: the step t; dataflow: -1 (each item's own)
     int32_t steps;             // dataflow: items of steps >= steps are skipped
-    float coef[kMaxIters][3];  // (a_t, b_t, c_t) for t = 0 .. T - 1
+    const float* coef;         // (a_t, b_t, c_t) for t = 0 .. T - 1, 3 T floats (workspace)
     const int32_t* pair_begin; // dataflow: each pair's range of items (npairs + 1 offsets)
     uint32_t* done;            // dataflow: per-matrix completion counts (zeroed before the launch)
     const MatDev* mats;
@@ -200,10 +200,11 @@ cudaError_t launch_finalize(const MemLaunch& p, int which, cudaStream_t s);
 cudaError_t launch_combine(const MemLaunch& p, cudaStream_t s);
 cudaError_t launch_sum_parts(const float* parts, int n, float* out, cudaStream_t s);
 cudaError_t launch_gemm_simt(const GemmLaunch& p, int elem, cudaStream_t s);
-// Per-phase launches (p.pair_begin == nullptr; npairs ignored) or the
-// dataflow launch over `npairs` CTA pairs, with 4 or 8 epilogue warps per CTA
-// (Poly and the dataflow launch, which mixes phases, take 8).
-cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t s, int epi_warps,
+// One per-phase launch (phase = kGram, kPoly or kUpdate; npairs ignored) or
+// the dataflow launch (phase = -1) over `npairs` CTA pairs.  Gram and Update
+// take 4 epilogue warps per CTA, Poly and the dataflow launch, which mixes
+// phases, 8.
+cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t s, int phase,
                                 int npairs);
 // CTA pairs of the dataflow kernel that can be resident at once on the
 // current device (0 and an error when the query fails).

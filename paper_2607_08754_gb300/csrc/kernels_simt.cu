@@ -52,7 +52,7 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const GemmLaunch p) {
     const GemmItem it = p.items[blockIdx.x];
     const MatDev md = p.mats[it.mat];
     const int ph = it.phase, cur = p.step & 1;  // one launch per phase and step
-    const float ca = p.coef[p.step][0], cb = p.coef[p.step][1], cc = p.coef[p.step][2];
+    const float ca = p.coef[3 * p.step], cb = p.coef[3 * p.step + 1], cc = p.coef[3 * p.step + 2];
     const T* X = reinterpret_cast<const T*>(md.x[cur]);
     const T* Am = reinterpret_cast<const T*>(md.a);
     const T* Bm = reinterpret_cast<const T*>(md.b);

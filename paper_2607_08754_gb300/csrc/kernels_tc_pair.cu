@@ -122,10 +122,11 @@ __device__ __forceinline__ void record_timeout(const GemmLaunch& p, const PairSm
 // every npairs-th item of a per-phase launch.  A dataflow launch of fewer
 // steps than the plan (slorr_run_steps) skips the later steps' items; every
 // role skips the same ones.
+template <int PH>
 struct PairItems {
     int first, end, stride;
     __device__ PairItems(const GemmLaunch& p, int pair, int npairs) {
-        if (p.pair_begin != nullptr) {
+        if constexpr (PH == kAnyPhase) {
             first = p.pair_begin[pair];
             end = p.pair_begin[pair + 1];
             stride = 1;
@@ -137,13 +138,11 @@ struct PairItems {
     }
 };
 
-__device__ __forceinline__ bool item_runs(const GemmLaunch& p, const GemmItem& it) {
-    return p.pair_begin == nullptr || int(it.step) < p.steps;
-}
-
 // The first index >= idx (in steps of `stride`, below `end`) whose item runs.
+template <int PH>
 __device__ __forceinline__ int next_running(const GemmLaunch& p, int idx, int end, int stride) {
-    while (idx < end && !item_runs(p, p.items[idx])) idx += stride;
+    if constexpr (PH == kAnyPhase)
+        while (idx < end && int(p.items[idx].step) >= p.steps) idx += stride;
     return idx;
 }
 
@@ -155,7 +154,7 @@ __device__ __forceinline__ int next_running(const GemmLaunch& p, int idx, int en
 // *seen receives the count that satisfied the wait.
 __device__ __forceinline__ bool wait_done(const GemmLaunch& p, const PairSmem& s, const GemmItem& it,
                                           uint32_t* seen = nullptr) {
-    if (p.done == nullptr || it.wait == 0) return true;
+    if (it.wait == 0) return true;
     const uint32_t* c = p.done + it.mat;
     uint32_t v = ptx::ld_acquire_gpu(c);
     if (v >= it.wait) {
@@ -182,21 +181,22 @@ __device__ __forceinline__ bool wait_done(const GemmLaunch& p, const PairSmem& s
 // tm == tn and a full 256 x 256 tile, each CTA's A rows and B columns are the
 // same 128 rows of the same matrix, so they are copied once and both UMMA
 // operands read them (the B descriptor points at the A half).
+template <int PH>
 __device__ __forceinline__ bool shared_operand(const GemmItem& it) {
-    return it.phase != kUpdate && it.tm == it.tn && it.msz == 2 * kBM && it.nsz == kBNMax;
+    return item_phase<PH>(it) != kUpdate && it.tm == it.tn && it.msz == 2 * kBM && it.nsz == kBNMax;
 }
 
 // Bytes one CTA of the pair copies per stage of a tile: its A rows, unless they
 // lie beyond the matrix (the UMMA rows they would feed are never stored), and
 // its half of the B columns, unless they are its A rows (shared_operand).
-template <class C>
+template <class C, int PH>
 __device__ __forceinline__ uint32_t pair_stage_bytes(const GemmItem& it, int rank) {
     const uint32_t a = rank * kBM < it.msz ? uint32_t(C::kABytes) : 0u;
-    return shared_operand(it) ? a : a + uint32_t(it.nsz / 2) * C::BK * 2;
+    return shared_operand<PH>(it) ? a : a + uint32_t(it.nsz / 2) * C::BK * 2;
 }
 
-template <class C>
-__device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, const PairItems& seq) {
+template <class C, int PH>
+__device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, const PairItems<PH>& seq) {
     int stage = 0;
     uint32_t phase = 0;
     const uint32_t even_full = ptx::mapa(ptx::smem_u32(s.full), 0);
@@ -204,23 +204,25 @@ __device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, 
     // an item it already covers needs no new acquire
     int seen_mat = -1;
     uint32_t seen = 0;
-    for (int idx = next_running(p, seq.first, seq.end, seq.stride); idx < seq.end;
-         idx = next_running(p, idx + seq.stride, seq.end, seq.stride)) {
+    for (int idx = next_running<PH>(p, seq.first, seq.end, seq.stride); idx < seq.end;
+         idx = next_running<PH>(p, idx + seq.stride, seq.end, seq.stride)) {
         const GemmItem it = p.items[idx];
         // Dataflow: the item's operands are complete once its matrix's earlier
         // phases are; the proxy fence orders those generic-proxy stores, now
         // visible to this thread, before its tensor copies read them.
-        if (p.done != nullptr && it.wait != 0 && !(int(it.mat) == seen_mat && seen >= it.wait)) {
-            if (!wait_done(p, s, it, &seen)) {
-                record_timeout(p, s);
-                return;
+        if constexpr (PH == kAnyPhase) {
+            if (it.wait != 0 && !(int(it.mat) == seen_mat && seen >= it.wait)) {
+                if (!wait_done(p, s, it, &seen)) {
+                    record_timeout(p, s);
+                    return;
+                }
+                ptx::fence_proxy_async_global();
+                seen_mat = it.mat;
             }
-            ptx::fence_proxy_async_global();
-            seen_mat = it.mat;
         }
-        const PhaseInfo pi = phase_info<C>(p, it);
+        const PhaseInfo pi = phase_info<C, PH>(p, it);
         const bool load_a = rank * kBM < it.msz;
-        const bool load_b = !shared_operand(it);
+        const bool load_b = !shared_operand<PH>(it);
         int kb_begin, kb_end;
         split_range(it, pi.nkb, &kb_begin, &kb_end);
         for (int kb = kb_begin; kb < kb_end; ++kb) {
@@ -256,22 +258,22 @@ __device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, 
 
 // Walks this pair's (tile, K block) sequence; the MMA thread keeps one cursor
 // STAGES K blocks ahead of the one it consumes, to arm stage barriers.
-template <class C>
+template <class C, int PH>
 struct KCursor {
     const GemmLaunch* p;
     int idx, end, stride, kb, nkb;
     uint32_t bytes;  // bytes both CTAs copy for the current K block
     __device__ void load() {
-        idx = next_running(*p, idx, end, stride);
+        idx = next_running<PH>(*p, idx, end, stride);
         if (idx < end) {
             const GemmItem it = p->items[idx];
             int b, e;
-            split_range(it, phase_info<C>(*p, it).nkb, &b, &e);
+            split_range(it, phase_info<C, PH>(*p, it).nkb, &b, &e);
             nkb = e - b;
-            bytes = pair_stage_bytes<C>(it, 0) + pair_stage_bytes<C>(it, 1);
+            bytes = pair_stage_bytes<C, PH>(it, 0) + pair_stage_bytes<C, PH>(it, 1);
         }
     }
-    __device__ KCursor(const GemmLaunch& gp, const PairItems& seq)
+    __device__ KCursor(const GemmLaunch& gp, const PairItems<PH>& seq)
         : p(&gp), idx(seq.first), end(seq.end), stride(seq.stride), kb(0), nkb(0), bytes(0) {
         load();
     }
@@ -285,13 +287,13 @@ struct KCursor {
     }
 };
 
-template <bool BF16, class C>
-__device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_base, const PairItems& seq) {
+template <bool BF16, class C, int PH>
+__device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_base, const PairItems<PH>& seq) {
     int armed_parity[C::STAGES];
 #pragma unroll
     for (int i = 0; i < C::STAGES; ++i) armed_parity[i] = -1;
     // Arm the first ring: phase 0 of every stage the sequence reaches.
-    KCursor<C> arm(p, seq);
+    KCursor<C, PH> arm(p, seq);
     for (int i = 0; i < C::STAGES && arm.valid(); ++i, arm.next()) {
         ptx::mbar_arrive_expect_tx(&s.full[i], arm.bytes);
         armed_parity[i] = 0;
@@ -309,10 +311,10 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
             ok = false;
         }
     }
-    for (int idx = next_running(p, seq.first, seq.end, seq.stride); idx < seq.end && ok;
-         idx = next_running(p, idx + seq.stride, seq.end, seq.stride), ++local) {
+    for (int idx = next_running<PH>(p, seq.first, seq.end, seq.stride); idx < seq.end && ok;
+         idx = next_running<PH>(p, idx + seq.stride, seq.end, seq.stride), ++local) {
         const GemmItem it = p.items[idx];
-        const PhaseInfo pi = phase_info<C>(p, it);
+        const PhaseInfo pi = phase_info<C, PH>(p, it);
         const uint32_t idesc = ptx::idesc_f16(2 * kBM, it.nsz, BF16, pi.a_mn, pi.b_mn);
         const int slot = local % C::kSlots;
         const uint32_t tphase = uint32_t(local / C::kSlots) & 1u;
@@ -340,7 +342,7 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
             }
             ptx::tc_fence_after();
             const uint32_t a0 = ptx::smem_u32(s.stages + size_t(stage) * C::kStageBytes);
-            const uint32_t b0 = shared_operand(it) ? a0 : a0 + C::kABytes;
+            const uint32_t b0 = shared_operand<PH>(it) ? a0 : a0 + C::kABytes;
 #pragma unroll
             for (int kk = 0; kk < C::BK / 16; ++kk) {
                 const uint32_t acc = (kb != kb_begin || kk != 0) ? 1u : 0u;
@@ -370,17 +372,17 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
     }
 }
 
-template <bool BF16, class C>
+template <bool BF16, class C, int PH>
 __device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_base, int rank,
-                              const PairItems& seq, int warp, int lane) {
+                              const PairItems<PH>& seq, int warp, int lane) {
     const int quad = warp & 3;             // TMEM lanes [32 quad, 32 quad + 32) (hardware rule)
     const int ngroups = C::kEpiWarps / 4;  // warps per lane quadrant, splitting the columns
     const int group = (warp - 2) / 4;
     uint8_t* sbuf = s.epi + (warp - 2) * kStageWarpBytes;
     int local = 0;
     const uint32_t even_tempty = ptx::mapa(ptx::smem_u32(s.tempty), 0);
-    for (int idx = next_running(p, seq.first, seq.end, seq.stride); idx < seq.end;
-         idx = next_running(p, idx + seq.stride, seq.end, seq.stride), ++local) {
+    for (int idx = next_running<PH>(p, seq.first, seq.end, seq.stride); idx < seq.end;
+         idx = next_running<PH>(p, idx + seq.stride, seq.end, seq.stride), ++local) {
         const GemmItem it = p.items[idx];
         const MatDev& md = p.mats[it.mat];
         const int slot = local % C::kSlots;
@@ -390,7 +392,8 @@ __device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t t
             ok = ptx::mbar_wait(&s.tfull[slot], tphase, s.abort, p.timeout_ns) ? 1 : 0;
             // Poly reads b A with plain loads: acquire A's completion count in
             // this thread too (the producer already saw it reached).
-            if (ok && it.phase == kPoly && !wait_done(p, s, it)) ok = 0;
+            if constexpr (PH == kAnyPhase)
+                if (ok && it.phase == kPoly && !wait_done(p, s, it)) ok = 0;
         }
         ok = __shfl_sync(0xffffffffu, ok, 0);
         if (!ok) {
@@ -404,13 +407,14 @@ __device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t t
             const int per = it.nsz / 32 / ngroups;  // 32-column chunks per warp
             const int parts = it.ksplit >> 8;
             if (parts <= 1) {
-                store_rows<BF16, true>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per, nullptr, 1,
-                                       0, sbuf);
-            } else if (split_partial_is_last(p, it, rank, quad, group, lane, t_row, group * per, (group + 1) * per)) {
+                store_rows<BF16, PH, true>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per, nullptr,
+                                           1, 0, sbuf);
+            } else if (PH != kPoly && PH != kUpdate &&
+                       split_partial_is_last(p, it, rank, quad, group, lane, t_row, group * per, (group + 1) * per)) {
                 // split K (Gram): direct stores, since the last part's sum is a
                 // serial step, which the staging round trip lengthens (small
                 // sets, ResNet-18 Gram +7%)
-                store_rows<BF16>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per,
+                store_rows<BF16, PH>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per,
                                  p.split_part + size_t(it.sid) * 65536, parts, rank * kBM + quad * 32 + lane);
             }
         }
@@ -423,7 +427,7 @@ __device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t t
             ptx::mbar_arrive_cluster_relaxed(even_tempty + uint32_t(slot * 8));
             // Dataflow: publish this warp's part of the item (every lane's
             // stores happen before the fence through the warp barrier above).
-            if (p.done != nullptr) {
+            if constexpr (PH == kAnyPhase) {
                 __threadfence();
                 atomicAdd(p.done + it.mat, 1u);
             }
@@ -431,7 +435,7 @@ __device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t t
     }
 }
 
-template <bool BF16, class C>
+template <bool BF16, class C, int PH>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(C::kThreads, 1)
     tc_pair_kernel(const __grid_constant__ GemmLaunch p) {
     extern __shared__ uint8_t smem_raw[];
@@ -452,7 +456,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(C::kThreads, 1)
     s.peer = uint32_t(rank ^ 1);
     const int pair = blockIdx.x / 2, npairs = gridDim.x / 2;
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    const PairItems seq(p, pair, npairs);
+    const PairItems<PH> seq(p, pair, npairs);
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < C::STAGES; ++i) {
@@ -469,7 +473,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(C::kThreads, 1)
         ptx::fence_mbar_init();
     }
     if (warp == 0 && lane == 0 && seq.first < seq.end) {
-        const PhaseInfo pi = phase_info<C>(p, p.items[seq.first]);
+        const PhaseInfo pi = phase_info<C, PH>(p, p.items[seq.first]);
         ptx::prefetch_tmap(pi.mapA);
         ptx::prefetch_tmap(pi.mapB);
     }
@@ -492,13 +496,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(C::kThreads, 1)
     if (peer_base != tmem_base) {
         if (threadIdx.x == 0) atomicOr(p.status, kStatusInternal);
     } else if (warp == 0) {
-        if (lane == 0) pair_producer<C>(p, s, rank, seq);
+        if (lane == 0) pair_producer<C, PH>(p, s, rank, seq);
         __syncwarp();
     } else if (warp == 1) {
-        if (lane == 0 && rank == 0) pair_mma<BF16, C>(p, s, tmem_base, seq);
+        if (lane == 0 && rank == 0) pair_mma<BF16, C, PH>(p, s, tmem_base, seq);
         __syncwarp();
     } else {
-        pair_epilogue<BF16, C>(p, s, tmem_base, rank, seq, warp, lane);
+        pair_epilogue<BF16, C, PH>(p, s, tmem_base, rank, seq, warp, lane);
     }
     ptx::tc_fence_before();
     __syncthreads();
@@ -514,7 +518,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(C::kThreads, 1)
 // first queries on one device may both run; they store the same value.
 constexpr int kMaxDevices = 64;
 
-template <bool BF16, class C>
+template <bool BF16, class C, int PH>
 cudaError_t max_pairs_of(int num_sms, int* out) {
     static std::atomic<int> cache[kMaxDevices];
     int dev = 0;
@@ -523,7 +527,7 @@ cudaError_t max_pairs_of(int num_sms, int* out) {
     if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
     int max_pairs = cache[dev].load(std::memory_order_acquire);
     if (max_pairs == 0) {
-        e = cudaFuncSetAttribute(tc_pair_kernel<BF16, C>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(tc_pair_kernel<BF16, C, PH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  int(C::kSmemBytes));
         if (e != cudaSuccess) return e;
         cudaLaunchConfig_t probe = {};
@@ -531,7 +535,7 @@ cudaError_t max_pairs_of(int num_sms, int* out) {
         probe.blockDim = dim3(C::kThreads);
         probe.dynamicSmemBytes = C::kSmemBytes;
         int clusters = 0;
-        e = cudaOccupancyMaxActiveClusters(&clusters, tc_pair_kernel<BF16, C>, &probe);
+        e = cudaOccupancyMaxActiveClusters(&clusters, tc_pair_kernel<BF16, C, PH>, &probe);
         if (e != cudaSuccess) return e;
         if (clusters < 1) return cudaErrorInvalidConfiguration;
         max_pairs = clusters < num_sms / 2 ? clusters : num_sms / 2;
@@ -545,36 +549,43 @@ cudaError_t max_pairs_of(int num_sms, int* out) {
 // exactly the plan's `npairs` pairs, which must all be resident at once (a
 // pair may wait for items of any other), so a plan for more pairs than fit is
 // refused.
-template <bool BF16, class C>
+template <bool BF16, class C, int PH>
 cudaError_t launch_pair_cfg(const GemmLaunch& p, int num_sms, cudaStream_t st, int npairs) {
     int max_pairs = 0;
-    cudaError_t e = max_pairs_of<BF16, C>(num_sms, &max_pairs);
+    cudaError_t e = max_pairs_of<BF16, C, PH>(num_sms, &max_pairs);
     if (e != cudaSuccess) return e;
-    if (p.pair_begin != nullptr) {
+    if constexpr (PH == kAnyPhase) {
         if (npairs < 1 || npairs > max_pairs) return cudaErrorInvalidConfiguration;
     } else {
         npairs = p.num_items < max_pairs ? p.num_items : max_pairs;
     }
-    return launch_kernel(tc_pair_kernel<BF16, C>, unsigned(2 * npairs), C::kThreads, C::kSmemBytes, st, p.pdl != 0, p);
+    return launch_kernel(tc_pair_kernel<BF16, C, PH>, unsigned(2 * npairs), C::kThreads, C::kSmemBytes, st,
+                         p.pdl != 0, p);
+}
+
+template <bool BF16>
+cudaError_t launch_pair_bf(const GemmLaunch& p, int num_sms, cudaStream_t st, int phase, int npairs) {
+    switch (phase) {
+        case kGram: return launch_pair_cfg<BF16, PairCfg2, kGram>(p, num_sms, st, npairs);
+        case kPoly: return launch_pair_cfg<BF16, PairCfg2Wide, kPoly>(p, num_sms, st, npairs);
+        case kUpdate: return launch_pair_cfg<BF16, PairCfg2, kUpdate>(p, num_sms, st, npairs);
+        default: return launch_pair_cfg<BF16, PairCfg2Wide, kAnyPhase>(p, num_sms, st, npairs);
+    }
 }
 
 }  // namespace
 
-cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t st, int epi_warps,
+cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t st, int phase,
                                 int npairs) {
     if (p.num_items == 0) return cudaSuccess;
-    const bool bf = elem == kBF16;
-    if (epi_warps == 8)
-        return bf ? launch_pair_cfg<true, PairCfg2Wide>(p, num_sms, st, npairs)
-                  : launch_pair_cfg<false, PairCfg2Wide>(p, num_sms, st, npairs);
-    return bf ? launch_pair_cfg<true, PairCfg2>(p, num_sms, st, npairs)
-              : launch_pair_cfg<false, PairCfg2>(p, num_sms, st, npairs);
+    return elem == kBF16 ? launch_pair_bf<true>(p, num_sms, st, phase, npairs)
+                         : launch_pair_bf<false>(p, num_sms, st, phase, npairs);
 }
 
 cudaError_t tc_pair_dataflow_capacity(int elem, int num_sms, int* pairs) {
     *pairs = 0;
-    return elem == kBF16 ? max_pairs_of<true, PairCfg2Wide>(num_sms, pairs)
-                         : max_pairs_of<false, PairCfg2Wide>(num_sms, pairs);
+    return elem == kBF16 ? max_pairs_of<true, PairCfg2Wide, kAnyPhase>(num_sms, pairs)
+                         : max_pairs_of<false, PairCfg2Wide, kAnyPhase>(num_sms, pairs);
 }
 
 }  // namespace slorr

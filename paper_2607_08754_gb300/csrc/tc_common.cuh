@@ -47,10 +47,27 @@ __device__ __forceinline__ float2 unpack2(uint32_t u) {
     }
 }
 
+// The kernel template's phase: kGram, kPoly or kUpdate for a per-phase launch
+// (its epilogue and operand code compile for that phase alone), kAnyPhase for
+// the dataflow launch (each item's own phase).
+constexpr int kAnyPhase = -1;
+
+template <int PH>
+__device__ __forceinline__ int item_phase(const GemmItem& it) {
+    if constexpr (PH >= 0)
+        return PH;
+    else
+        return int(it.phase);
+}
+
 // The Polar Express step an item belongs to: its own (dataflow launch) or the
 // launch's (per-phase launches).
+template <int PH>
 __device__ __forceinline__ int item_step(const GemmLaunch& p, const GemmItem& it) {
-    return p.step >= 0 ? p.step : int(it.step);
+    if constexpr (PH >= 0)
+        return p.step;
+    else
+        return int(it.step);
 }
 
 struct PhaseInfo {
@@ -67,20 +84,21 @@ __device__ __forceinline__ const void* xmap(const uint8_t* maps, int buf, bool m
     return maps + (mn ? 2 + buf : buf) * 128;
 }
 
-template <class C>
+template <class C, int PH>
 __device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmItem& it) {
     const MatDev& md = p.mats[it.mat];
     const uint8_t* maps = reinterpret_cast<const uint8_t*>(p.maps) + size_t(it.mat) * kMapsPerMatrix * 128;
     const bool tr = md.transposed != 0;
-    const int cur = item_step(p, it) & 1;
+    const int cur = item_step<PH>(p, it) & 1;
+    const int phase = item_phase<PH>(it);
     PhaseInfo pi;
-    if (it.phase == kGram) {
+    if (phase == kGram) {
         pi.a_mn = tr;
         pi.b_mn = tr;
         pi.mapA = xmap(maps, cur, tr);
         pi.mapB = pi.mapA;
         pi.nkb = md.Qpad / C::BK;
-    } else if (it.phase == kPoly) {
+    } else if (phase == kPoly) {
         pi.a_mn = false;
         pi.b_mn = false;
         pi.mapA = maps + 4 * 128;
@@ -231,7 +249,7 @@ __device__ __forceinline__ void own_row(uint8_t* buf, int lane, const uint4 (&v)
 // order, of the `parts` fp32 partials at split_tile (row row_t of the tile;
 // this warp's own part among them).  STAGED: the stores go through the
 // warp's staging buffer sbuf (kStageWarpBytes of shared memory).
-template <bool BF16, bool STAGED = false>
+template <bool BF16, int PH, bool STAGED = false>
 __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& it, const MatDev& md, int row0,
                                            uint32_t t_row, int quad, int lane, int ch_begin, int ch_end,
                                            const float* split_tile = nullptr, int parts = 1, int row_t = 0,
@@ -239,9 +257,10 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
     const int row_w = row0 + quad * 32;  // the warp's first row
     const int row = row_w + lane;
     const int nch = ch_end;
-    const int t = item_step(p, it);
+    const int t = item_step<PH>(p, it);
+    const int phase = item_phase<PH>(it);
     const float xs = (p.fused_norm && t == 0) ? p.scalars[it.mat].x0_scale : 1.f;
-    if (it.phase == kUpdate) {
+    if (phase == kUpdate) {
         uint16_t* out = reinterpret_cast<uint16_t*>(md.x[(t & 1) ^ 1]);
         const int64_t ld = md.ld;
         for (int ch = ch_begin; ch < nch; ++ch) {
@@ -279,12 +298,12 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
             }
         }
     } else {
-        uint16_t* out = reinterpret_cast<uint16_t*>(it.phase == kGram ? md.a : md.b);
+        uint16_t* out = reinterpret_cast<uint16_t*>(phase == kGram ? md.a : md.b);
         const uint16_t* amat = reinterpret_cast<const uint16_t*>(md.a);
         const int64_t ld = md.Ppad;
-        const bool poly = it.phase == kPoly;
-        const float ca = p.coef[t][0], cb = p.coef[t][1];
-        const float cacc = poly ? p.coef[t][2] : xs * xs;
+        const bool poly = phase == kPoly;
+        const float ca = poly ? p.coef[3 * t] : 0.f, cb = poly ? p.coef[3 * t + 1] : 0.f;
+        const float cacc = poly ? p.coef[3 * t + 2] : xs * xs;
         // Poly reads b A at the output position: loads for the next chunk are
         // issued before the current chunk is processed (staged: coalesced
         // loads, turned into this lane's row through the staging buffer).

@@ -442,19 +442,25 @@ def test_dataflow_plan_is_absent_for_phase_launches(lib):
         slorr.Regularizer([(256, 512)], flags=slorr.FLAG_PHASE_LAUNCHES | slorr.FLAG_DATAFLOW)
 
 
-def test_launch_mode_is_chosen_by_set_size(lib):
-    """Without a flag the plan takes the dataflow launch for sets of up to
-    about 3 ms of GEMM work (7000 K blocks of a 256 x 256 tile over 76 pairs,
-    the measured crossover) and per-phase launches above; SLORR_FLAG_DATAFLOW
-    forces the dataflow launch."""
+def test_launch_mode_is_chosen_by_set_shape(lib):
+    """Without a flag the plan takes the dataflow launch for work-bound sets
+    whose per-phase launches would be short (fewer than 7 Gram tiles per
+    pair), the measured winners, and per-phase launches for chain-bound sets
+    (cfg1, ResNet-18) and for sets with many tiles per pair (ViT-L/16, 560M,
+    ViT-H, ViT-B with 24 blocks); SLORR_FLAG_DATAFLOW forces the dataflow
+    launch."""
     import workloads
-    for name, df in (("cfg1", True), ("resnet18", True), ("vit_b16", True), ("vit_ladder_vit_s", True),
-                     ("vit_l16", False), ("decoder_560m", False), ("vit_ladder_vit_h", False)):
+    for name, m, df in (("cfg1", 0, False), ("resnet18", 0, False), ("vit_ladder_vit_ti", 0, False),
+                        ("vit_ladder_vit_s", 0, True), ("vit_ladder_vit_512", 0, True), ("vit_b16", 0, True),
+                        ("vit_l16", 32, True), ("vit_l16", 48, True), ("decoder_560m", 28, True),
+                        ("vit_ladder_vit_b24", 0, False), ("vit_l16", 64, False), ("decoder_560m", 56, False),
+                        ("vit_l16", 0, False), ("decoder_560m", 0, False), ("vit_ladder_vit_h", 0, False)):
         shapes = workloads.shapes(name)
+        if m:
+            shapes = shapes[:m]
         r = slorr.Regularizer(shapes)
         forced = slorr.Regularizer(shapes, flags=slorr.FLAG_DATAFLOW)
         mk = slorr.slorr_dataflow_items(forced.handle)[2]
-        assert (mk < 7000) == df, (name, mk)
         if df:
             assert slorr.slorr_dataflow_items(r.handle)[2] == mk
         else:
