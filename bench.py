@@ -52,6 +52,9 @@ sys.path.insert(0, ROOT)
 import workloads  # noqa: E402
 
 METRIC = "regularizer fwd+bwd ms/step & TFLOP/s (% GB300 dense peak) per weight set"
+# nominal dense tf32 over bf16 tensor rate on GB300 (1.1 and 2.25 PFLOP/s): the
+# tf32 peak is the measured bf16 peak times this ratio
+TF32_RATIO = 1.1 / 2.25
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 PROFILE_FILE = os.path.join(ROOT, "profiles", "tc_pair_vit_l16.txt")
 # the default tensor-core GEMM (the CTA-pair kernel) and the headers it is built from
@@ -448,7 +451,8 @@ def main():
         # instruction issue.  128 FP32 lanes per SM at the maximum SM clock; the
         # compensated (Dot2) multiply-add of fp32 mode takes 10 FP32 operations
         # (product, its FMA error, two-sum, two error adds), the plain one 1.
-        simt = args.compute == "fp32" or bool(args.flags & slorr.FLAG_SIMT_GEMM)
+        simt = bool(args.flags & slorr.FLAG_SIMT_GEMM)
+        tf32 = args.compute == "fp32" and not simt
         ops_per_mac = 10 if args.compute == "fp32" else 1
         sm_max = (clk or {}).get("sm_max_mhz") or 2070.0
         nsm = torch.cuda.get_device_properties(dev).multi_processor_count
@@ -486,7 +490,8 @@ def main():
             "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
             "scaling": "strong" if partition else "weak",
-            "vs_baseline": None, "dtype": "f16" if args.compute == "fp16" else args.compute,
+            "vs_baseline": None,
+            "dtype": {"fp16": "f16", "bf16": "bf16"}.get(args.compute, "tf32x3" if tf32 else "f32"),
             "data": "synthetic",
             "config": {"workload": f"{name}{' (first %d matrices)' % len(set_shapes) if args.matrices else ''} "
                                    f"{args.variant}{' descent step' if descent else ''}: "
@@ -505,7 +510,15 @@ def main():
                          "tflops": flops_exec / (ms_step * 1e-3) / 1e12,
                          "note": "MMA FLOPs the kernels execute: padding included, strictly-lower "
                                  "symmetric tiles skipped"},
-            "roofline": ({"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+            "roofline": ({"bound": "tensor", "achieved": 3 * achieved, "peak": peak * TF32_RATIO, "unit": "TFLOP/s",
+                          "frac": 3 * achieved / (peak * TF32_RATIO), "traffic": None,
+                          "frac_of_sustained": 3 * achieved / (pk["bf16_sustained"] * TF32_RATIO),
+                          "kernel": "tf32_gemm_kernel (Gram/Poly/Update launches: three tf32 products per fp32 "
+                                    "product, counted in achieved)",
+                          "peak_source": pk["source"] + " bf16 burst x %.4f (nominal dense tf32 / bf16: "
+                                                        "1.1 / 2.25 PFLOP/s)" % TF32_RATIO}
+                         if tf32 else
+                         {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                           "frac": achieved / peak, "traffic": tc_traffic(),
                           "frac_of_sustained": achieved / pk["bf16_sustained"],
                           "kernel": "tc_pair_kernel (" + ("one dataflow launch per call: every Gram, Poly and "

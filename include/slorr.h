@@ -71,7 +71,10 @@ typedef enum slorr_dtype {       /* storage type of the weights and of their gra
 typedef enum slorr_compute {     /* operand type of the Polar Express matrix products */
     SLORR_COMPUTE_FP16 = 0,      /* fp16 operands, fp32 accumulation (tensor cores)  */
     SLORR_COMPUTE_BF16 = 1,      /* bf16 operands, fp32 accumulation (tensor cores)  */
-    SLORR_COMPUTE_FP32 = 2       /* fp32 operands and accumulation (CUDA cores)      */
+    SLORR_COMPUTE_FP32 = 2       /* fp32 operands: three tf32 tensor-core products per
+                                    product, short-K fp32 accumulations added with
+                                    compensated sums (CUDA cores, compensated dot
+                                    products, with SLORR_FLAG_SIMT_GEMM)              */
 } slorr_compute;
 
 typedef struct slorr_shape {
@@ -95,7 +98,7 @@ typedef struct slorr_options {
 } slorr_options;
 
 /* Flags.  slorr_create rejects any other bit with SLORR_ERR_INVALID_ARG. */
-#define SLORR_FLAG_SIMT_GEMM    1   /* run the 16-bit products on CUDA cores (debug)  */
+#define SLORR_FLAG_SIMT_GEMM    1   /* run the products on CUDA cores (a checker)      */
 #define SLORR_FLAG_TEST_STALL  16   /* test only: every tensor-core CTA first waits on a
                                        barrier nothing arrives on, so its bounded wait
                                        runs out after timeout_s and the call reports

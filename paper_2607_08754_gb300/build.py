@@ -22,7 +22,8 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libslorr.so")
 STAMP = os.path.join(BUILD, "libslorr.stamp")
-SOURCES = ["api.cu", "kernels_mem.cu", "kernels_simt.cu", "kernels_tc_pair.cu", "noalloc.cu", "schedule.cpp"]
+SOURCES = ["api.cu", "kernels_mem.cu", "kernels_simt.cu", "kernels_tc_pair.cu", "kernels_tf32.cu", "noalloc.cu",
+           "schedule.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
          "--expt-relaxed-constexpr"]

@@ -47,6 +47,7 @@ namespace {
 struct Geom {
     int m, n, P, Q, Ppad, Qpad, transposed, rows, ld;
     size_t off_x[2], off_a, off_b;
+    size_t off_tf32[10];            // fp32 tensor-core mode: xg[2][2], xu[2][2], a lo, m lo
     int tile_base, tile_count;      // tiles of W (sumsq, dot, combine)
     int xtile_base, xtile_count;    // tiles of the padded iterate (cast, normcast)
 };
@@ -63,6 +64,7 @@ struct slorr_handle {
     // item lists (host)
     std::vector<GemmItem> tc_items[3];
     std::vector<GemmItem> simt_items[3];
+    std::vector<GemmItem> tf32_items[3];  // fp32 mode on the tensor cores: 128 x 64 tiles
     // dataflow plan: every (step, phase, tile) item, pair by pair
     std::vector<GemmItem> df_items;
     std::vector<int32_t> df_pair_begin;  // df_pairs + 1 offsets into df_items
@@ -77,11 +79,13 @@ struct slorr_handle {
     int total_w_tiles = 0;
     int total_x_tiles = 0;
     int total_split_parts = 0;  // 256 x 256 fp32 partial slots of split-K Gram tiles
+    int tf32_split_tiles = 0;   // 32 x 32 tiles of the largest padded iterate (fp32 tensor-core mode)
     // workspace layout
     size_t off_status = 0, off_counters = 0, off_scalars = 0, off_partials = 0, off_partials_max = 0,
            off_tilebase = 0, off_tilecount = 0, off_xtilebase = 0, off_xtilecount = 0, off_split_cnt = 0,
            off_split_part = 0, off_mats = 0, off_maps = 0, off_tc_items[3] = {}, off_simt_items[3] = {},
-           off_done = 0, off_df_items = 0, off_df_pair_begin = 0, off_coef = 0,
+           off_done = 0, off_df_items = 0, off_df_pair_begin = 0, off_coef = 0, off_tf32_mats = 0,
+           off_tf32_maps = 0, off_tf32_items[3] = {},
            off_w_items = 0, off_x_items = 0, off_ptrs = 0, off_plan_end = 0, total_bytes = 0;
     // device state
     const void* prepared_ws = nullptr;
@@ -116,6 +120,12 @@ bool dataflow(const slorr_handle* h) { return h->df; }
 bool dataflow_possible(const slorr_handle* h) {
     return h->opt.compute != SLORR_COMPUTE_FP32 &&
            (h->opt.flags & (SLORR_FLAG_SIMT_GEMM | SLORR_FLAG_PHASE_LAUNCHES)) == 0;
+}
+
+// fp32 mode runs its products on the tensor cores as three tf32 products
+// (kernels_tf32.cu) unless the CUDA-core kernel is asked for.
+bool tf32_tc(const slorr_handle* h) {
+    return h->opt.compute == SLORR_COMPUTE_FP32 && (h->opt.flags & SLORR_FLAG_SIMT_GEMM) == 0;
 }
 
 // Programmatic dependent launch of the memory passes and the pair kernel.
@@ -455,6 +465,7 @@ void build_plan(slorr_handle* h) {
     for (int i = 0; i < 3; ++i) {
         h->tc_items[i].clear();
         h->simt_items[i].clear();
+        h->tf32_items[i].clear();
     }
     h->w_items.clear();
     h->x_items.clear();
@@ -516,6 +527,15 @@ void build_plan(slorr_handle* h) {
                     h->tc_items[ph].back().phase = uint8_t(ph);
                 }
             }
+            // fp32 tensor-core tiles (128 x 64); the symmetric Gram and Poly keep
+            // those that reach the diagonal
+            if (tf32_tc(h))
+                for (int tm = 0; tm < g.Ppad / 128; ++tm)
+                    for (int tn = 0; tn < N / 64; ++tn) {
+                        if (ph != kUpdate && (tn + 1) * 64 <= tm * 128) continue;
+                        h->tf32_items[ph].push_back(GemmItem{uint16_t(i), uint16_t(tm), uint16_t(tn), 64, 128, 0});
+                        h->tf32_items[ph].back().phase = uint8_t(ph);
+                    }
             // CUDA-core tiles; the symmetric Gram and Poly keep those on or above the diagonal
             for (int tm = 0; tm < g.Ppad / kSimtTile; ++tm)
                 for (int tn = (ph == kUpdate ? 0 : tm); tn < N / kSimtTile; ++tn) {
@@ -527,6 +547,9 @@ void build_plan(slorr_handle* h) {
     }
     h->total_w_tiles = tile_base;
     h->total_x_tiles = xtile_base;
+    h->tf32_split_tiles = 0;
+    if (tf32_tc(h))
+        for (const Geom& g : h->geom) h->tf32_split_tiles = std::max(h->tf32_split_tiles, (g.Ppad / 32) * (g.Qpad / 32));
     split_gram_items(h);
     // Longest K first (stable: keeps a matrix's tiles together).
     for (int ph = 0; ph < 3; ++ph) {
@@ -598,6 +621,15 @@ void build_plan(slorr_handle* h) {
         h->off_simt_items[ph] = off;
         off = align_up(off + h->simt_items[ph].size() * sizeof(GemmItem), 256);
     }
+    for (int ph = 0; ph < 3; ++ph) {
+        h->off_tf32_items[ph] = off;
+        off = align_up(off + h->tf32_items[ph].size() * sizeof(GemmItem), 256);
+    }
+    const bool tf32 = tf32_tc(h);
+    h->off_tf32_mats = off;
+    off = align_up(off + (tf32 ? size_t(count) * sizeof(MatTf32) : 0), 256);
+    h->off_tf32_maps = off;
+    off = align_up(off + (tf32 ? size_t(count) * kTf32MapsPerMatrix * 128 : 0), 256);
     h->off_coef = off;
     off = align_up(off + size_t(3 * h->opt.iters) * sizeof(float), 256);
     h->off_df_items = off;
@@ -625,6 +657,17 @@ void build_plan(slorr_handle* h) {
         off = align_up(off + pbytes, 1024);
         g.off_b = off;
         off = align_up(off + pbytes, 1024);
+        if (tf32) {
+            // xg[b][h] (Ppad x Qpad) and xu[b][h] (Qpad x Ppad), then the lo halves of A and M
+            for (int k = 0; k < 8; ++k) {
+                g.off_tf32[k] = off;
+                off = align_up(off + size_t(g.Ppad) * g.Qpad * 4, 1024);
+            }
+            for (int k = 8; k < 10; ++k) {
+                g.off_tf32[k] = off;
+                off = align_up(off + pbytes, 1024);
+            }
+        }
     }
     h->total_bytes = off;
 }
@@ -659,6 +702,21 @@ bool encode_map(CUtensorMap* map, void* base, int rows, int cols, bool bf16, int
     return r == CUDA_SUCCESS;
 }
 
+// Row-major rows x cols fp32 matrix read by the fp32 tensor-core kernel in
+// boxes of 32 (contiguous, 128 bytes, 128-byte swizzle) x 64 rows.
+bool encode_map_f32(CUtensorMap* map, void* base, int rows, int cols) {
+    auto enc = get_encode();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {cuuint64_t(cols), cuuint64_t(rows)};
+    cuuint64_t strides[1] = {cuuint64_t(cols) * 4};
+    cuuint32_t box[2] = {32, 64};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 template <typename T>
 void put(std::vector<uint8_t>& buf, size_t off, const T* src, size_t n) {
     if (n) std::memcpy(buf.data() + off, src, n * sizeof(T));
@@ -688,6 +746,9 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
     std::vector<int32_t> tb(count), tcnt(count), xtb(count), xtcnt(count);
     std::vector<MatDev> mats(count);
     std::vector<uint8_t> maps(size_t(count) * kMapsPerMatrix * 128, 0);
+    const bool tf32 = tf32_tc(h);
+    std::vector<MatTf32> tmats(tf32 ? size_t(count) : 0);
+    std::vector<uint8_t> tmaps(tf32 ? size_t(count) * kTf32MapsPerMatrix * 128 : 0, 0);
     const int bk = 64;  // K depth of a pipeline stage
     const bool tc = h->opt.compute != SLORR_COMPUTE_FP32;
     for (int i = 0; i < count; ++i) {
@@ -724,6 +785,30 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
             ok = ok && encode_map(mp + 5, md.b, g.Ppad, g.Ppad, bf, bk, 64);
             if (!ok) return fail(SLORR_ERR_CUDA, "cuTensorMapEncodeTiled failed");
         }
+        if (tf32) {
+            MatTf32& mt = tmats[i];
+            for (int b = 0; b < 2; ++b)
+                for (int hl = 0; hl < 2; ++hl) {
+                    mt.xg[b][hl] = ws + g.off_tf32[2 * b + hl];
+                    mt.xu[b][hl] = ws + g.off_tf32[4 + 2 * b + hl];
+                }
+            mt.a[0] = md.a;
+            mt.a[1] = ws + g.off_tf32[8];
+            mt.m[0] = md.b;
+            mt.m[1] = ws + g.off_tf32[9];
+            CUtensorMap* mp = reinterpret_cast<CUtensorMap*>(tmaps.data() + size_t(i) * kTf32MapsPerMatrix * 128);
+            bool ok = true;
+            for (int b = 0; b < 2; ++b)
+                for (int hl = 0; hl < 2; ++hl) {
+                    ok = ok && encode_map_f32(mp + 2 * b + hl, mt.xg[b][hl], g.Ppad, g.Qpad);
+                    ok = ok && encode_map_f32(mp + 4 + 2 * b + hl, mt.xu[b][hl], g.Qpad, g.Ppad);
+                }
+            for (int hl = 0; hl < 2; ++hl) {
+                ok = ok && encode_map_f32(mp + 8 + hl, mt.a[hl], g.Ppad, g.Ppad);
+                ok = ok && encode_map_f32(mp + 10 + hl, mt.m[hl], g.Ppad, g.Ppad);
+            }
+            if (!ok) return fail(SLORR_ERR_CUDA, "cuTensorMapEncodeTiled failed (fp32 operands)");
+        }
     }
     put(plan, h->off_tilebase - base, tb.data(), tb.size());
     put(plan, h->off_tilecount - base, tcnt.data(), tcnt.size());
@@ -731,9 +816,12 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
     put(plan, h->off_xtilecount - base, xtcnt.data(), xtcnt.size());
     put(plan, h->off_mats - base, mats.data(), mats.size());
     put(plan, h->off_maps - base, maps.data(), maps.size());
+    put(plan, h->off_tf32_mats - base, tmats.data(), tmats.size());
+    put(plan, h->off_tf32_maps - base, tmaps.data(), tmaps.size());
     for (int ph = 0; ph < 3; ++ph) {
         put(plan, h->off_tc_items[ph] - base, h->tc_items[ph].data(), h->tc_items[ph].size());
         put(plan, h->off_simt_items[ph] - base, h->simt_items[ph].data(), h->simt_items[ph].size());
+        put(plan, h->off_tf32_items[ph] - base, h->tf32_items[ph].data(), h->tf32_items[ph].size());
     }
     std::vector<float> coef(h->coeffs.begin(), h->coeffs.end());
     put(plan, h->off_coef - base, coef.data(), coef.size());
@@ -968,7 +1056,16 @@ slorr_status launch_all(slorr_handle* h, uint8_t* ws, float* loss, float* per, i
         }
         Traced tr(h, 1, st);
         if ((e = launch_cast(cp, st)) != cudaSuccess) return cuda_fail(e, "cast launch");
-        tr.done();
+        if (tf32_tc(h)) {
+            // fp32 mode on the tensor cores: X_0 into hi/lo operand pairs, both orientations
+            e = launch_tf32_split(reinterpret_cast<const MatDev*>(ws + h->off_mats),
+                                  reinterpret_cast<const MatTf32*>(ws + h->off_tf32_mats), int(h->shapes.size()),
+                                  h->tf32_split_tiles, st);
+            if (e != cudaSuccess) return cuda_fail(e, "split launch");
+            tr.done(2);
+        } else {
+            tr.done();
+        }
     }
 
     GemmLaunch g{};
@@ -983,6 +1080,8 @@ slorr_status launch_all(slorr_handle* h, uint8_t* ws, float* loss, float* per, i
     g.split_part = reinterpret_cast<float*>(ws + h->off_split_part);
     g.split_cnt = reinterpret_cast<uint32_t*>(ws + h->off_split_cnt);
     g.coef = reinterpret_cast<const float*>(ws + h->off_coef);
+    g.tf32 = reinterpret_cast<const MatTf32*>(ws + h->off_tf32_mats);
+    g.tf32_maps = ws + h->off_tf32_maps;
     if (use_tc && dataflow(h) && steps > 0) {
         // every phase of every step in one launch, ordered by completion counts
         g.items = reinterpret_cast<const GemmItem*>(ws + h->off_df_items);
@@ -1004,6 +1103,10 @@ slorr_status launch_all(slorr_handle* h, uint8_t* ws, float* loss, float* per, i
                     g.items = reinterpret_cast<const GemmItem*>(ws + h->off_tc_items[ph]);
                     g.num_items = int(h->tc_items[ph].size());
                     e = launch_gemm_tc_pair(g, h->elem, h->num_sms, st, ph, 0);
+                } else if (tf32_tc(h)) {
+                    g.items = reinterpret_cast<const GemmItem*>(ws + h->off_tf32_items[ph]);
+                    g.num_items = int(h->tf32_items[ph].size());
+                    e = launch_gemm_tf32(g, ph, st);
                 } else {
                     g.items = reinterpret_cast<const GemmItem*>(ws + h->off_simt_items[ph]);
                     g.num_items = int(h->simt_items[ph].size());
@@ -1117,17 +1220,18 @@ slorr_status slorr_create(slorr_handle** out, const slorr_shape* shapes, int32_t
 
 slorr_status slorr_executed_flops(const slorr_handle* h, double* out) {
     if (!h || !out) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
-    const bool simt = h->opt.compute == SLORR_COMPUTE_FP32 || (h->opt.flags & SLORR_FLAG_SIMT_GEMM);
+    const bool tf32 = tf32_tc(h);
+    const bool simt = !tf32 && (h->opt.compute == SLORR_COMPUTE_FP32 || (h->opt.flags & SLORR_FLAG_SIMT_GEMM));
     double total = 0.0;
     for (int ph = 0; ph < 3; ++ph) {
-        for (const GemmItem& it : simt ? h->simt_items[ph] : h->tc_items[ph]) {
+        for (const GemmItem& it : tf32 ? h->tf32_items[ph] : simt ? h->simt_items[ph] : h->tc_items[ph]) {
             const Geom& g = h->geom[it.mat];
             const int Kfull = ph == kGram ? g.Qpad : g.Ppad;
             int kb0, kb1;
             split_range(it, Kfull / 64, &kb0, &kb1);
             const double K = it.ksplit ? double(kb1 - kb0) * 64 : double(Kfull);
-            const double rows = simt ? double(it.msz) : 256.0;  // pair UMMAs are always M = 256
-            total += 2.0 * rows * double(it.nsz) * K;
+            const double rows = (simt || tf32) ? double(it.msz) : 256.0;  // pair UMMAs are always M = 256
+            total += (tf32 ? 3.0 : 1.0) * 2.0 * rows * double(it.nsz) * K;  // tf32: three products
         }
     }
     *out = total * double(h->opt.iters);
@@ -1138,7 +1242,8 @@ slorr_status slorr_gemm_items(const slorr_handle* h, int32_t phase, int32_t* ite
     if (!h || !items) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
     if (phase < 0 || phase > 2) return fail(SLORR_ERR_INVALID_ARG, "phase must be 0 (Gram), 1 (Poly) or 2 (Update)");
     const bool simt = h->opt.compute == SLORR_COMPUTE_FP32 || (h->opt.flags & SLORR_FLAG_SIMT_GEMM);
-    *items = int32_t(simt ? h->simt_items[phase].size() : h->tc_items[phase].size());
+    *items = int32_t(tf32_tc(h) ? h->tf32_items[phase].size()
+                                : simt ? h->simt_items[phase].size() : h->tc_items[phase].size());
     return SLORR_OK;
 }
 
@@ -1146,7 +1251,8 @@ slorr_status slorr_gemm_item_list(const slorr_handle* h, int32_t phase, int32_t*
     if (!h || !out) return fail(SLORR_ERR_INVALID_ARG, "NULL argument");
     if (phase < 0 || phase > 2) return fail(SLORR_ERR_INVALID_ARG, "phase must be 0 (Gram), 1 (Poly) or 2 (Update)");
     const bool simt = h->opt.compute == SLORR_COMPUTE_FP32 || (h->opt.flags & SLORR_FLAG_SIMT_GEMM);
-    const std::vector<GemmItem>& v = simt ? h->simt_items[phase] : h->tc_items[phase];
+    const std::vector<GemmItem>& v =
+        tf32_tc(h) ? h->tf32_items[phase] : simt ? h->simt_items[phase] : h->tc_items[phase];
     if (capacity < int64_t(v.size()) * 7) return fail(SLORR_ERR_INVALID_ARG, "capacity too small");
     for (size_t i = 0; i < v.size(); ++i) {
         const GemmItem& it = v[i];

@@ -48,6 +48,21 @@ struct MatDev {
     int32_t pad_;
 };
 
+// fp32 mode on the tensor cores (three-pass TF32): every product operand is
+// kept as a pair (hi, lo) of fp32 arrays holding tf32 values, hi = tf32(v) and
+// lo = tf32(v - hi), both rounded to nearest.  All operands are K-major: the
+// iterate is kept both in the Gram orientation (P x Q, for the Gram product)
+// and transposed (Q x P, the B operand of the update M X).
+struct MatTf32 {
+    void* xg[2][2];    // [buffer][hi, lo]: X, Ppad x Qpad row-major
+    void* xu[2][2];    // [buffer][hi, lo]: X^T, Qpad x Ppad row-major
+    void* a[2];        // [hi, lo]: A, Ppad x Ppad
+    void* m[2];        // [hi, lo]: M, Ppad x Ppad
+};
+// Tensor maps per matrix of the fp32 tensor-core path (32 x 64-element boxes):
+// xg[b][h] at 2 b + h, xu[b][h] at 4 + 2 b + h, a[h] at 8 + h, m[h] at 10 + h.
+constexpr int kTf32MapsPerMatrix = 12;
+
 // Per-matrix scalars (workspace).
 struct MatScalars {
     double frob_sq;    // ||W||_F^2
@@ -152,6 +167,9 @@ struct GemmLaunch {
     // the tile.
     float* split_part;
     uint32_t* split_cnt;
+    // fp32 mode on the tensor cores: the hi/lo operand arrays and their maps
+    const MatTf32* tf32;
+    const void* tf32_maps;
 };
 
 // Tensor maps per matrix: X0 K-major, X1 K-major, X0 MN-major, X1 MN-major,
@@ -206,6 +224,12 @@ cudaError_t launch_gemm_simt(const GemmLaunch& p, int elem, cudaStream_t s);
 // phases, 8.
 cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t s, int phase,
                                 int npairs);
+// fp32 mode on the tensor cores: one phase of one step (p.step), one CTA per
+// 128 x 64 output tile (kernels_tf32.cu).
+cudaError_t launch_gemm_tf32(const GemmLaunch& p, int phase, cudaStream_t s);
+// fp32 mode on the tensor cores: splits X_0 (the fp32 iterate buffer x[0], in
+// W's orientation) into the hi/lo arrays of both orientations.
+cudaError_t launch_tf32_split(const MatDev* mats, const MatTf32* tf32, int count, int max_tiles, cudaStream_t s);
 // CTA pairs of the dataflow kernel that can be resident at once on the
 // current device (0 and an error when the query fails).
 cudaError_t tc_pair_dataflow_capacity(int elem, int num_sms, int* pairs);

@@ -62,6 +62,10 @@ __device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t pa
     return ok != 0;
 }
 
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
 // Wait until the phase of `bar` with the given parity has completed.  Gives up
 // (returns false) when *abort becomes non-zero or after `budget_ns` of
 // %globaltimer time; the caller then records the timeout and unwinds.
@@ -160,6 +164,16 @@ __device__ __forceinline__ void prefetch_tmap(const void* map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(map) : "memory");
 }
 
+// 2-D tiled load of one box into this CTA's shared memory, completing its bytes
+// on `bar`.  x is the innermost (contiguous) coordinate in elements.
+__device__ __forceinline__ void tma_load_2d(void* dst, const void* map, uint64_t* bar, int32_t x, int32_t y) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
+        "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y)
+        : "memory");
+}
+
 // CTA-pair form: the box lands in this CTA's shared memory, and its bytes are
 // counted on the mbarrier at shared::cluster address `bar_cluster`, which may
 // belong to the other CTA of the pair.
@@ -179,6 +193,40 @@ __device__ __forceinline__ void fence_proxy_async_global() {
 }
 
 // ---- tcgen05 ----------------------------------------------------------------------
+
+// One-CTA forms (cta_group::1): one warp allocates, relinquishes and frees.
+__device__ __forceinline__ void tmem_alloc(uint32_t* dst_smem, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst_smem)),
+                 "r"(ncols)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tmem_relinquish() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+// D[tmem] (+)= A[smem] * B[smem], kind::tf32 (tf32 operands read from 32-bit
+// containers, fp32 accumulation), issued by one thread for this CTA alone.
+__device__ __forceinline__ void umma_tf32(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// Arrive once on `bar` when every tcgen05 operation this thread issued so far
+// has completed (one-CTA form).
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+                 : "memory");
+}
 
 // CTA-pair forms (cta_group::2): one warp of each CTA of the pair executes the
 // allocation, relinquish and deallocation; every tcgen05 instruction of a
@@ -265,6 +313,22 @@ __device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo_bytes, ui
     d |= static_cast<uint64_t>(1) << 46;
     d |= static_cast<uint64_t>(layout & 7u) << 61;
     return d;
+}
+
+// fp32 -> tf32, round to nearest (ties away from zero); the result is an fp32
+// bit pattern whose 13 low significand bits are zero.
+__device__ __forceinline__ float cvt_rna_tf32(float x) {
+    uint32_t r;
+    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
+    return __uint_as_float(r);
+}
+
+// Instruction descriptor for kind::tf32 with fp32 accumulation: D format F32
+// (1) in [4,6), A and B format TF32 (2) in [7,10) and [10,13), both K-major
+// (bits 15, 16 clear), N >> 3 in [17,23), M >> 4 in [24,29).
+__host__ __device__ constexpr uint32_t idesc_tf32(int M, int N) {
+    return (1u << 4) | (2u << 7) | (2u << 10) | (static_cast<uint32_t>(N >> 3) << 17) |
+           (static_cast<uint32_t>(M >> 4) << 24);
 }
 
 // Instruction descriptor for kind::f16 with fp32 accumulation:

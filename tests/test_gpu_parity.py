@@ -397,3 +397,51 @@ def test_vit_ladder_vit_h_sampled():
         L, G, _, _ = oracle.reg_single(W, "hoyer", co, EPS)
         assert abs(per[i] - L) <= 2e-2 * L
         assert rel(g[i].double().cpu().numpy(), G) <= 2e-2
+
+
+# ---- fp32 mode on the tensor cores (three tf32 products per product) ----------------
+
+@pytest.mark.parametrize("variant", ["hoyer", "nuclear"])
+def test_fp32_tensor_cores_long_k(variant):
+    """fp32 mode runs its products as three tf32 tensor-core products with short-K
+    accumulations added by compensated sums; K up to 4608 (the truncating
+    tensor-core accumulation would otherwise bias a long K) against the
+    oracle at the fp32 tolerance."""
+    shapes = [(320, 1280), (512, 4608), (4608, 384), (1000, 512), (130, 70)]
+    Ws = [workloads.random_matrix(s, seed=610 + i, std=0.03) for i, s in enumerate(shapes)]
+    check(Ws, variant, "fp32", lam=0.4)
+
+
+def test_fp32_tensor_cores_match_compensated_cuda_cores():
+    """The tf32 tensor-core iterates stay within the fp32 tolerance of the
+    CUDA-core kernel's compensated fp32 dot products after 1, 3 and 6 steps."""
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_SIMT_GEMM
+    shapes = [(256, 768), (768, 256), (320, 1280), (384, 384)]
+    Ws = [workloads.random_matrix(s, seed=630 + i, std=0.02) for i, s in enumerate(shapes)]
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    tc = Regularizer(shapes, compute="fp32")
+    st = Regularizer(shapes, compute="fp32", flags=FLAG_SIMT_GEMM)
+    for k in (1, 3, 6):
+        tc.run_steps(w, k)
+        st.run_steps(w, k)
+        torch.cuda.synchronize()
+        assert tc.status() == 0 and st.status() == 0
+        for i in range(len(shapes)):
+            a = tc.iterate(i, k).double().cpu().numpy()
+            b = st.iterate(i, k).double().cpu().numpy()
+            assert rel(a, b) <= 1e-5, (k, i, rel(a, b))
+
+
+def test_fp32_tensor_core_bounded_wait_timeout():
+    """SLORR_FLAG_TEST_STALL in the tf32 kernel: the MMA thread's bounded wait
+    runs out, the call reports SLORR_ERR_TIMEOUT, and a normal fp32 call
+    afterwards matches the oracle."""
+    from paper_2607_08754_gb300.slorr import Regularizer, FLAG_TEST_STALL
+    Ws = [workloads.random_matrix((256, 512), 641, 0.05), workloads.random_matrix((384, 128), 642, 0.05)]
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    stall = Regularizer([W.shape for W in Ws], compute="fp32", flags=FLAG_TEST_STALL, timeout_s=0.05)
+    stall.run_steps(w, 1)
+    torch.cuda.synchronize()
+    assert stall.status() == 5
+    assert stall.status() == 0
+    check(Ws, "hoyer", "fp32")
