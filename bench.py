@@ -235,18 +235,22 @@ def tc_source_hash() -> str:
     return h.hexdigest()
 
 
-def tc_traffic():
+def tc_traffic(workload: str, matrices: int, per_phase: bool):
     """dram bytes per launch of the tensor-core GEMM from the committed ncu
-    summary, or None when the kernel source changed since it was taken."""
+    summary, or None when the kernel source changed since it was taken, or when
+    this run's weight set, matrix count or launch mode is not the one captured."""
     try:
         src = tc_source_hash()
         vals = {}
         with open(PROFILE_FILE) as f:
             for line in f:
-                if ":" in line:
+                if ":" in line and not line.startswith("#"):
                     k, v = line.split(":", 1)
                     vals[k.strip()] = v.strip()
         if vals.get("source_sha256") != src:
+            return None
+        if (vals.get("workload") != workload or int(vals.get("matrices", -1)) != matrices
+                or vals.get("launch_mode") != ("per-phase" if per_phase else "dataflow")):
             return None
         return float(vals["dram_bytes_per_launch_scaled"])
     except Exception:
@@ -519,7 +523,7 @@ def main():
                                                         "1.1 / 2.25 PFLOP/s)" % TF32_RATIO}
                          if tf32 else
                          {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                          "frac": achieved / peak, "traffic": tc_traffic(),
+                          "frac": achieved / peak, "traffic": tc_traffic(args.workload, len(shapes), not kt["gemm"][1]),
                           "frac_of_sustained": achieved / pk["bf16_sustained"],
                           "kernel": "tc_pair_kernel (" + ("one dataflow launch per call: every Gram, Poly and "
                                                           "Update of the T steps" if kt["gemm"][1] else
