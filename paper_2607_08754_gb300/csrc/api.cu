@@ -255,7 +255,7 @@ void split_gram_items(slorr_handle* h) {
     for (const GemmItem& it : items) {
         const int K = h->geom[it.mat].Qpad;
         int parts = int(std::ceil(K / target));
-        parts = std::min(std::min(parts, kMaxSplit), K / 64);
+        parts = std::min(std::min(parts, kMaxSplit), K / kPairBK);
         if (parts <= 1) {
             out.push_back(it);
             continue;
@@ -557,8 +557,8 @@ void build_plan(slorr_handle* h) {
             const Geom& g = h->geom[it.mat];
             const int K = ph == kGram ? g.Qpad : g.Ppad;
             int b, e;
-            split_range(it, K / 64, &b, &e);
-            return it.ksplit ? (e - b) * 64 : K;
+            split_range(it, K / kPairBK, &b, &e);
+            return it.ksplit ? (e - b) * kPairBK : K;
         };
         std::stable_sort(h->tc_items[ph].begin(), h->tc_items[ph].end(),
                          [&](const GemmItem& a, const GemmItem& b) { return kdim(a) > kdim(b); });
@@ -685,19 +685,20 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
     return fn;
 }
 
-// Row-major rows x cols 16-bit matrix read in boxes of box_inner (contiguous)
-// x box_outer elements.  A 128-byte inner box uses the 128-byte swizzle, a
-// 64-byte one the 64-byte swizzle (the kernel's descriptors match).
-bool encode_map(CUtensorMap* map, void* base, int rows, int cols, bool bf16, int box_inner, int box_outer) {
+// Row-major rows x cols 16-bit matrix seen as a 3-D tensor of 64-element
+// chunks: x = the element within a chunk, y = the row, z = the chunk along
+// the row (128 bytes apart).  One box is 128 rows of two chunks (32 KB,
+// 128-byte swizzle): the K-major half of a CTA-pair operand (rows MN, chunks
+// K) or its MN-major half (rows K, chunks MN) for a 128-wide K block.
+bool encode_map(CUtensorMap* map, void* base, int rows, int cols, bool bf16) {
     auto enc = get_encode();
     if (!enc) return false;
-    cuuint64_t dims[2] = {cuuint64_t(cols), cuuint64_t(rows)};
-    cuuint64_t strides[1] = {cuuint64_t(cols) * 2};
-    cuuint32_t box[2] = {cuuint32_t(box_inner), cuuint32_t(box_outer)};
-    cuuint32_t estr[2] = {1, 1};
-    const CUtensorMapSwizzle sw = box_inner * 2 == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
-    CUresult r = enc(map, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, base,
-                     dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
+    cuuint64_t dims[3] = {64u, cuuint64_t(rows), cuuint64_t(cols / 64)};
+    cuuint64_t strides[2] = {cuuint64_t(cols) * 2, 128u};
+    cuuint32_t box[3] = {64u, 128u, cuuint32_t(kPairBK / 64)};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = enc(map, bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, base,
+                     dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
@@ -749,7 +750,6 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
     const bool tf32 = tf32_tc(h);
     std::vector<MatTf32> tmats(tf32 ? size_t(count) : 0);
     std::vector<uint8_t> tmaps(tf32 ? size_t(count) * kTf32MapsPerMatrix * 128 : 0, 0);
-    const int bk = 64;  // K depth of a pipeline stage
     const bool tc = h->opt.compute != SLORR_COMPUTE_FP32;
     for (int i = 0; i < count; ++i) {
         const Geom& g = h->geom[i];
@@ -775,14 +775,10 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
         if (tc) {
             const bool bf = h->opt.compute == SLORR_COMPUTE_BF16;
             CUtensorMap* mp = reinterpret_cast<CUtensorMap*>(maps.data() + size_t(i) * kMapsPerMatrix * 128);
-            // K-major boxes: bk (k) x 64 rows; MN-major boxes: 64 (mn) x bk rows
             bool ok = true;
-            for (int b = 0; b < 2; ++b) {
-                ok = ok && encode_map(mp + b, md.x[b], g.rows, g.ld, bf, bk, 64);
-                ok = ok && encode_map(mp + 2 + b, md.x[b], g.rows, g.ld, bf, 64, bk);
-            }
-            ok = ok && encode_map(mp + 4, md.a, g.Ppad, g.Ppad, bf, bk, 64);
-            ok = ok && encode_map(mp + 5, md.b, g.Ppad, g.Ppad, bf, bk, 64);
+            for (int b = 0; b < 2; ++b) ok = ok && encode_map(mp + b, md.x[b], g.rows, g.ld, bf);
+            ok = ok && encode_map(mp + 2, md.a, g.Ppad, g.Ppad, bf);
+            ok = ok && encode_map(mp + 3, md.b, g.Ppad, g.Ppad, bf);
             if (!ok) return fail(SLORR_ERR_CUDA, "cuTensorMapEncodeTiled failed");
         }
         if (tf32) {
@@ -1228,8 +1224,8 @@ slorr_status slorr_executed_flops(const slorr_handle* h, double* out) {
             const Geom& g = h->geom[it.mat];
             const int Kfull = ph == kGram ? g.Qpad : g.Ppad;
             int kb0, kb1;
-            split_range(it, Kfull / 64, &kb0, &kb1);
-            const double K = it.ksplit ? double(kb1 - kb0) * 64 : double(Kfull);
+            split_range(it, Kfull / kPairBK, &kb0, &kb1);
+            const double K = it.ksplit ? double(kb1 - kb0) * kPairBK : double(Kfull);
             const double rows = (simt || tf32) ? double(it.msz) : 256.0;  // pair UMMAs are always M = 256
             total += (tf32 ? 3.0 : 1.0) * 2.0 * rows * double(it.nsz) * K;  // tf32: three products
         }
@@ -1308,8 +1304,8 @@ slorr_status slorr_gemm_pair_load(const slorr_handle* h, int32_t phase, int32_t 
         const Geom& g = h->geom[v[i].mat];
         const int K = phase == kGram ? g.Qpad : g.Ppad;
         int b, e;
-        split_range(v[i], K / 64, &b, &e);
-        load[i % size_t(npairs)] += int64_t(e - b) * 64;
+        split_range(v[i], K / kPairBK, &b, &e);
+        load[i % size_t(npairs)] += int64_t(e - b) * kPairBK;
     }
     *max_k = *std::max_element(load.begin(), load.end());
     *total_k = std::accumulate(load.begin(), load.end(), int64_t(0));

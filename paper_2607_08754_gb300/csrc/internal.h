@@ -25,6 +25,9 @@ constexpr int kMaxMatrices = 4096;
 constexpr int kMaxIters = 16;
 constexpr int kPadRows = 128;   // Ppad granularity (tcgen05 tile M)
 constexpr int kPadCols = 128;   // Qpad granularity (a CTA pair splits a tile's 2 x 64 columns)
+// K block of one stage of the CTA-pair GEMM: two 128-byte swizzle atoms of
+// 16-bit elements (Ppad and Qpad are multiples of it)
+constexpr int kPairBK = 128;
 
 // Element type of the iterate buffers X, A, B.
 enum Elem : int32_t { kF32 = 0, kF16 = 1, kBF16 = 2 };
@@ -172,9 +175,9 @@ struct GemmLaunch {
     const void* tf32_maps;
 };
 
-// Tensor maps per matrix: X0 K-major, X1 K-major, X0 MN-major, X1 MN-major,
-// A K-major, M K-major.
-constexpr int kMapsPerMatrix = 6;
+// Tensor maps per matrix: X0, X1, A, M (each read as K-major or MN-major
+// halves through the same 3-D map).
+constexpr int kMapsPerMatrix = 4;
 
 // Where the combine pass puts lambda * grad_scale * G_i.
 enum OutMode : int32_t {

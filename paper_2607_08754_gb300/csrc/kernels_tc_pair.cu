@@ -66,19 +66,20 @@ using namespace tc;
 
 template <int STAGES_, int EPIW_>
 struct PairCfg {
-    static constexpr int BK = 64;
+    static constexpr int BK = kPairBK;                    // two 128-byte swizzle atoms of K
     static constexpr int STAGES = STAGES_;
     static constexpr int kSlots = 2;                      // accumulators per CTA in TMEM
-    static constexpr int kBoxBytes = 64 * BK * 2;         // one 64 x 64 box
     static constexpr int kABytes = kBM * BK * 2;          // this CTA's 128 rows of A
-    static constexpr int kBBytes = 128 * BK * 2;          // this CTA's half of B (<= 128 rows)
+    static constexpr int kBBytes = 128 * BK * 2;          // this CTA's half of B (a 128-row box, <= 128 used)
+    static constexpr uint32_t kAtomBytes = 128 * 128;     // one 128-row swizzle atom column (64 elements wide)
+    static constexpr uint32_t kMnLbo = uint32_t(BK) * 128;  // MN-major: 64-element MN chunks this far apart
     static constexpr int kAccCols = kBNMax;               // fp32 TMEM columns of one accumulator
     static constexpr int kStageBytes = kABytes + kBBytes;
     static constexpr int kEpiWarps = EPIW_;               // 4, or 8: two per TMEM lane quadrant
     static_assert(EPIW_ == 4 || EPIW_ == 8, "epilogue warps");
     static constexpr int kThreads = 64 + 32 * kEpiWarps;
     static constexpr uint32_t kKLayout = 2u;              // SWIZZLE_128B
-    static constexpr uint32_t kKSbo = 8 * BK * 2;
+    static constexpr uint32_t kKSbo = 8 * 128;            // 8-row groups of 128-byte rows
     static constexpr uint32_t kTmemCols = uint32_t(kSlots) * uint32_t(kAccCols);
     static constexpr size_t kBarrierBytes = 512;
     static constexpr size_t kEpiBytes = size_t(kEpiWarps) * kStageWarpBytes;  // epilogue staging
@@ -87,9 +88,9 @@ struct PairCfg {
     static_assert(kSmemBytes <= 232448, "shared memory budget");
     static_assert(kTmemCols <= 512, "tensor memory budget");
 };
-// Ring depth (a build-time tuning knob): 6 stages of 32 KB; 7 still fit.
+// Ring depth (a build-time tuning knob): 3 stages of 64 KB.
 #ifndef SLORR_PAIR_STAGES
-#define SLORR_PAIR_STAGES 6
+#define SLORR_PAIR_STAGES 3
 #endif
 // Two accumulators per CTA (the tile epilogue overlaps the next main loop);
 // the Poly epilogue, which also reads b A, takes 8 warps, the others 4 (more
@@ -192,7 +193,7 @@ __device__ __forceinline__ bool shared_operand(const GemmItem& it) {
 template <class C, int PH>
 __device__ __forceinline__ uint32_t pair_stage_bytes(const GemmItem& it, int rank) {
     const uint32_t a = rank * kBM < it.msz ? uint32_t(C::kABytes) : 0u;
-    return shared_operand<PH>(it) ? a : a + uint32_t(it.nsz / 2) * C::BK * 2;
+    return shared_operand<PH>(it) ? a : a + uint32_t(C::kBBytes);
 }
 
 template <class C, int PH>
@@ -234,19 +235,24 @@ __device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, 
             uint8_t* sb = sa + C::kABytes;
             const int k = kb * C::BK;
             const uint32_t bar = even_full + uint32_t(stage * 8);
-            // box coordinates are (inner, outer): (k, mn) for K-major, (mn, k) for MN-major
-            if (load_a)
-                for (int b = 0; b < 2; ++b) {
-                    const int mn = it.tm * (2 * kBM) + rank * kBM + b * 64;
-                    ptx::tma_load_2d_pair(sa + b * C::kBoxBytes, pi.mapA, bar, pi.a_mn ? mn : k, pi.a_mn ? k : mn);
-                }
-            // B columns: this CTA's half, nsz / 2 = 64 or 128 rows
+            // one 3-D box per operand half: 128 rows (y) of two 64-element
+            // chunks (z) of each row.  K-major: rows are MN, chunks are K;
+            // MN-major: rows are K, chunks are MN.
+            if (load_a) {
+                const int mn = it.tm * (2 * kBM) + rank * kBM;
+                if (!pi.a_mn)
+                    ptx::tma_load_3d_pair(sa, pi.mapA, bar, 0, mn, k / 64);
+                else
+                    ptx::tma_load_3d_pair(sa, pi.mapA, bar, 0, k, mn / 64);
+            }
+            // B columns: this CTA's half, nsz / 2 = 64 or 128 (a 64-wide half
+            // takes the same box; the UMMA reads its first 64)
             if (load_b) {
-                const int bhalf = it.nsz / 2;
-                for (int j = 0; j < bhalf / 64; ++j) {
-                    const int mn = it.tn * kBNMax + rank * bhalf + j * 64;
-                    ptx::tma_load_2d_pair(sb + j * C::kBoxBytes, pi.mapB, bar, pi.b_mn ? mn : k, pi.b_mn ? k : mn);
-                }
+                const int mn = it.tn * kBNMax + rank * (it.nsz / 2);
+                if (!pi.b_mn)
+                    ptx::tma_load_3d_pair(sb, pi.mapB, bar, 0, mn, k / 64);
+                else
+                    ptx::tma_load_3d_pair(sb, pi.mapB, bar, 0, k, mn / 64);
             }
             if (++stage == C::STAGES) {
                 stage = 0;

@@ -186,6 +186,16 @@ __device__ __forceinline__ void tma_load_2d_pair(void* dst, const void* map, uin
         : "memory");
 }
 
+// 3-D form of tma_load_2d_pair: box (x, y, z) with x the contiguous coordinate.
+__device__ __forceinline__ void tma_load_3d_pair(void* dst, const void* map, uint32_t bar_cluster, int32_t x,
+                                                 int32_t y, int32_t z) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
+        "l"(map), "r"(bar_cluster), "r"(x), "r"(y), "r"(z)
+        : "memory");
+}
+
 // Orders this thread's earlier generic-proxy global accesses with its later
 // async-proxy (TMA) accesses.
 __device__ __forceinline__ void fence_proxy_async_global() {

@@ -78,11 +78,9 @@ struct PhaseInfo {
     bool b_mn;   // B operand MN-major (else K-major)
 };
 
-// Tensor maps per matrix (kMapsPerMatrix of them, 128 bytes each):
-// X0 K-major, X1 K-major, X0 MN-major, X1 MN-major, A K-major, M K-major.
-__device__ __forceinline__ const void* xmap(const uint8_t* maps, int buf, bool mn) {
-    return maps + (mn ? 2 + buf : buf) * 128;
-}
+// Tensor maps per matrix (kMapsPerMatrix of them, 128 bytes each): X0, X1,
+// A, M.
+__device__ __forceinline__ const void* xmap(const uint8_t* maps, int buf) { return maps + buf * 128; }
 
 template <class C, int PH>
 __device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmItem& it) {
@@ -95,20 +93,20 @@ __device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmI
     if (phase == kGram) {
         pi.a_mn = tr;
         pi.b_mn = tr;
-        pi.mapA = xmap(maps, cur, tr);
+        pi.mapA = xmap(maps, cur);
         pi.mapB = pi.mapA;
         pi.nkb = md.Qpad / C::BK;
     } else if (phase == kPoly) {
         pi.a_mn = false;
         pi.b_mn = false;
-        pi.mapA = maps + 4 * 128;
+        pi.mapA = maps + 2 * 128;
         pi.mapB = pi.mapA;
         pi.nkb = md.Ppad / C::BK;
     } else {
         pi.a_mn = false;
         pi.b_mn = !tr;
-        pi.mapA = maps + 5 * 128;
-        pi.mapB = xmap(maps, cur, pi.b_mn);
+        pi.mapA = maps + 3 * 128;
+        pi.mapB = xmap(maps, cur);
         pi.nkb = md.Ppad / C::BK;
     }
     return pi;
@@ -124,14 +122,15 @@ __device__ __forceinline__ bool sym_tile_computed(int tm, int tn, int Ppad) {
 }
 
 // Shared-memory descriptor of one K = 16 slice (kk) of a BK-wide K block:
-// K-major: rows of 2 BK bytes (swizzle span), 8-row groups kKSbo apart, slice
-// kk starts 32 bytes further inside the swizzle atom; MN-major: 64-element MN
-// chunks one box apart (LBO), 8-row K groups 1 KB apart (SBO), slice kk starts
-// 16 rows = 2 KB further.
+// K-major: 128-byte rows (swizzle span), 8-row groups kKSbo apart, the K
+// chunks of 64 elements one 128-row atom column (kAtomBytes) apart, slice kk
+// 32 bytes further into its chunk; MN-major: 64-element MN chunks kMnLbo apart
+// (LBO), 8-row K groups 1 KB apart (SBO), slice kk starts 16 rows = 2 KB
+// further.
 template <class C>
 __device__ __forceinline__ uint64_t operand_desc(uint32_t base, int kk, bool mn) {
-    return mn ? ptx::sdesc(base + kk * 16 * 128, C::kBoxBytes, 1024, 2u)
-              : ptx::sdesc(base + kk * 32, 16, C::kKSbo, C::kKLayout);
+    return mn ? ptx::sdesc(base + kk * 16 * 128, C::kMnLbo, 1024, 2u)
+              : ptx::sdesc(base + (kk >> 2) * C::kAtomBytes + (kk & 3) * 32, 16, C::kKSbo, C::kKLayout);
 }
 
 // Split K, one part of a tile: this warp stores its 32 rows of the part's
