@@ -170,17 +170,22 @@ __device__ __forceinline__ bool split_partial_is_last(const GemmLaunch& p, const
 // Staged epilogue stores (CTA-pair kernel).  A TMEM load gives each lane one
 // row of a 32 x 32 chunk, so a lane's own 16-byte stores would touch 32 rows
 // per instruction, half a 32-byte sector each.  Instead the warp stages the
-// chunk in its own shared-memory buffer (rows kStageRow bytes apart: the
-// 16-byte row writes of any 8 lanes fall in 8 different bank groups) and
-// stores it as 8 rows x 64 bytes per instruction, or transposed (column c of
-// the chunk as a row of the output) as 8 columns x 64 bytes.
+// chunk in its own shared-memory buffer and stores it as 8 rows x 64 bytes per
+// instruction, or transposed (column c of the chunk as a row of the output) as
+// 8 columns x 64 bytes.  Rows are kStageRow bytes apart, so the 16-byte row
+// writes of any 8 consecutive lanes fall in 8 different bank groups; each
+// row's four 16-byte segments are rotated by row / 8, so that the column
+// reads, which take 4 rows 8 apart per instruction (the same banks at any
+// pitch that is a multiple of 16 bytes), fall in 4 different bank groups.
 constexpr int kStageRow = 80;
 constexpr int kStageWarpBytes = 32 * kStageRow;
 
+// Row r's 16-byte segment q lies at r * kStageRow + 16 ((q + r / 8) mod 4).
 __device__ __forceinline__ void stage_chunk(uint8_t* buf, int lane, const uint4 (&o)[4]) {
-    uint4* dst = reinterpret_cast<uint4*>(buf + lane * kStageRow);
+    uint8_t* row = buf + lane * kStageRow;
+    const int rot = lane >> 3;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) dst[q] = o[q];
+    for (int q = 0; q < 4; ++q) *reinterpret_cast<uint4*>(row + (((q + rot) & 3) << 4)) = o[q];
     __syncwarp();
 }
 
@@ -190,7 +195,7 @@ __device__ __forceinline__ void put_rows(const uint8_t* buf, int lane, uint16_t*
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         const int r = i * 8 + (lane >> 2);
-        const uint4 v = *reinterpret_cast<const uint4*>(buf + r * kStageRow + seg * 16);
+        const uint4 v = *reinterpret_cast<const uint4*>(buf + r * kStageRow + (((seg + i) & 3) << 4));  // r / 8 = i
         *reinterpret_cast<uint4*>(out + int64_t(r0 + r) * ld + c0 + seg * 8) = v;
     }
 }
@@ -201,7 +206,8 @@ __device__ __forceinline__ void put_cols(const uint8_t* buf, int lane, uint16_t*
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         const int c = i * 8 + (lane >> 2);
-        const uint8_t* src = buf + (seg * 8) * kStageRow + c * 2;
+        // rows seg * 8 .. + 7: rotated by seg
+        const uint8_t* src = buf + (seg * 8) * kStageRow + ((c * 2 + (seg << 4)) & 63);
         uint32_t w[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
@@ -223,7 +229,9 @@ __device__ __forceinline__ void get_rows(const uint16_t* src, int64_t ld, int r0
         v[i] = __ldcg(reinterpret_cast<const uint4*>(src + int64_t(r0 + i * 8 + (lane >> 2)) * ld + c0 + seg * 8));
 }
 
-// A chunk from get_rows, through the staging buffer, as this lane's row.
+// A chunk from get_rows, through the staging buffer, as this lane's row (in
+// the buffer's plain layout, without the rotation: both of its accesses
+// are row-wise and already spread over the bank groups).
 __device__ __forceinline__ void own_row(uint8_t* buf, int lane, const uint4 (&v)[4], uint4 (&row)[4]) {
     const int seg = lane & 3;
 #pragma unroll
