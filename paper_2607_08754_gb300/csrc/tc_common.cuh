@@ -112,6 +112,13 @@ __device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmI
     return pi;
 }
 
+// M is stored only in the 256 x 256 tiles the Poly computes (tile column >=
+// tile row; no mirrored copy): an Update tile of tile row tm reads its A
+// operand (rows of M) K-major where K block kb (128 wide) lies in a stored
+// tile, and elsewhere MN-major from the stored transpose, M[kb rows][tm
+// columns], which equals it because M is symmetric.
+__device__ __forceinline__ bool update_a_mn(const GemmItem& it, int kb) { return (kb >> 1) < int(it.tm); }
+
 // Symmetric products (Gram, Poly): only tiles holding some 128 x 128 block on
 // or above the diagonal are computed.  Tile (tm, tn) covers row blocks 2 tm,
 // 2 tm + 1 and column blocks 2 tn .. min(2 tn + 1, nb - 1) (nb = Ppad / 128),
@@ -378,13 +385,14 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
                 }
                 ow[j] = pack2<BF16>(lo, hi);
             }
-            // The output is symmetric and strictly-lower tiles are skipped:
-            // write the transpose of this 128 x 128 block (I, J), J > I, when
-            // the tile that holds (J, I) is not computed.  The mirrored copy
-            // uses the same rounded 16-bit values, so the stored matrix is
-            // exactly symmetric.
+            // The output is symmetric and strictly-lower tiles are skipped.
+            // Gram: write the transpose of this 128 x 128 block (I, J), J > I,
+            // when the tile that holds (J, I) is not computed; the mirrored
+            // copy uses the same rounded 16-bit values, so the stored matrix is
+            // exactly symmetric.  Poly: no mirror (the Update reads the
+            // missing blocks MN-major, update_a_mn).
             const int I = row0 / kBM, J = col0 / kBM;
-            const bool mirror = J > I && !sym_tile_computed(J / 2, I / 2, md.Ppad);
+            const bool mirror = !poly && J > I && !sym_tile_computed(J / 2, I / 2, md.Ppad);
             if constexpr (STAGED) {
                 stage_chunk(sbuf, lane, o);
                 put_rows(sbuf, lane, out, ld, row_w, col0);
