@@ -289,8 +289,8 @@ void split_gram_items(slorr_handle* h) {
 // Costs are in K blocks (64) of a 256 x 256 tile: the tile's K blocks, scaled
 // by its width (an N = 128 UMMA moves 3/4 of the bytes of an N = 256 one), plus
 // one block for its start and epilogue (overlapped with the next tile); Poly
-// tiles count 1.6 x (their epilogue reads A and writes M and its mirror:
-// measured 0.82 against 1.37 PFLOP/s of MMA work on ViT-L/16-shaped tiles);
+// tiles count 1.6 x (their epilogue reads A and writes M: measured 0.82
+// against 1.37 PFLOP/s of MMA work on ViT-L/16-shaped tiles);
 // the last part of a split tile adds the parts.  A dependency adds 4 blocks
 // (the last increments, the producer's wake-up, the first copies landing).
 constexpr double kDepLatency = 4.0;
@@ -513,8 +513,8 @@ void build_plan(slorr_handle* h) {
         xtile_base += xseq;
         // tensor-core tiles: msz x nsz with msz, nsz <= 256.  The Gram and
         // Poly outputs are symmetric: tiles lying strictly below the diagonal
-        // (in 128 x 128 blocks) are skipped; the kernel mirrors the blocks
-        // they need.
+        // (in 128 x 128 blocks) are skipped, and their readers take those
+        // blocks MN-major from the stored transpose.
         for (int ph = 0; ph < 3; ++ph) {
             const int N = ph == kUpdate ? g.Qpad : g.Ppad;
             for (int tm = 0; tm * 256 < g.Ppad; ++tm) {

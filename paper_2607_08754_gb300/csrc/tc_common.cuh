@@ -112,12 +112,14 @@ __device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmI
     return pi;
 }
 
-// M is stored only in the 256 x 256 tiles the Poly computes (tile column >=
-// tile row; no mirrored copy): an Update tile of tile row tm reads its A
-// operand (rows of M) K-major where K block kb (128 wide) lies in a stored
-// tile, and elsewhere MN-major from the stored transpose, M[kb rows][tm
-// columns], which equals it because M is symmetric.
-__device__ __forceinline__ bool update_a_mn(const GemmItem& it, int kb) { return (kb >> 1) < int(it.tm); }
+// A and M are stored only in the 256 x 256 tiles the Gram and the Poly
+// compute (tile column >= tile row; no mirrored copy).  A product operand made
+// of rows of A or M in tile row t reads K block kb (128 wide) K-major where it
+// lies in a stored tile, and elsewhere MN-major from the stored transpose
+// (rows kb, columns t), which equals it because A and M are symmetric: the
+// Update's A operand (rows of M, t = tm) and both Poly operands (rows of A,
+// t = tm and t = tn).  Both CTAs of a pair take the same choice.
+__device__ __forceinline__ bool sym_mn(int kb, int t) { return (kb >> 1) < t; }
 
 // Symmetric products (Gram, Poly): only tiles holding some 128 x 128 block on
 // or above the diagonal are computed.  Tile (tm, tn) covers row blocks 2 tm,
@@ -385,32 +387,19 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
                 }
                 ow[j] = pack2<BF16>(lo, hi);
             }
-            // The output is symmetric and strictly-lower tiles are skipped.
-            // Gram: write the transpose of this 128 x 128 block (I, J), J > I,
-            // when the tile that holds (J, I) is not computed; the mirrored
-            // copy uses the same rounded 16-bit values, so the stored matrix is
-            // exactly symmetric.  Poly: no mirror (the Update reads the
-            // missing blocks MN-major, update_a_mn).
-            const int I = row0 / kBM, J = col0 / kBM;
-            const bool mirror = !poly && J > I && !sym_tile_computed(J / 2, I / 2, md.Ppad);
+            // The output is symmetric and strictly-lower tiles are skipped,
+            // with no mirrored copy: its readers take the missing blocks
+            // MN-major from the stored ones (sym_mn).
+
             if constexpr (STAGED) {
                 stage_chunk(sbuf, lane, o);
                 put_rows(sbuf, lane, out, ld, row_w, col0);
-                if (mirror) put_cols(sbuf, lane, out, ld, row_w, col0);
                 __syncwarp();
                 continue;
             }
             uint4* dst = reinterpret_cast<uint4*>(out + off);
 #pragma unroll
             for (int q = 0; q < 4; ++q) dst[q] = o[q];
-            if (mirror) {
-                uint16_t* tdst = out + int64_t(col0) * ld + row;
-#pragma unroll
-                for (int j = 0; j < 16; ++j) {
-                    tdst[int64_t(2 * j) * ld] = uint16_t(ow[j] & 0xffffu);
-                    tdst[int64_t(2 * j + 1) * ld] = uint16_t(ow[j] >> 16);
-                }
-            }
         }
     }
 }
