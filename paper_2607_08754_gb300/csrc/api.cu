@@ -291,9 +291,11 @@ void split_gram_items(slorr_handle* h) {
 // one block for its start and epilogue (overlapped with the next tile); Poly
 // tiles count 1.6 x (their epilogue reads A and writes M: measured 0.82
 // against 1.37 PFLOP/s of MMA work on ViT-L/16-shaped tiles);
-// the last part of a split tile adds the parts.  A dependency adds 4 blocks
-// (the last increments, the producer's wake-up, the first copies landing).
-constexpr double kDepLatency = 4.0;
+// the last part of a split tile adds the parts.  A dependency adds 8 blocks
+// (the last increments, the producer's wake-up, the first copies landing;
+// 8 measured best on ViT-S, ViT-512 and ViT-B with the 64 KB-stage kernel,
+// 12 lengthens ViT-S's chain past the launch-mode threshold).
+constexpr double kDepLatency = 8.0;
 
 // Which launch a set gets by default.  Per tile the dataflow launch is a few
 // per cent slower than the phase-specialised per-phase kernels (8 epilogue

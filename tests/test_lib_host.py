@@ -370,6 +370,10 @@ def test_split_plan_items(lib):
         slorr._check(slorr.load_library().slorr_gemm_item_list(slorr.Regularizer(rn).handle, 0, None, 0))
 
 
+# the planner's dependency latency, in K blocks (written out again here)
+DEP = 8.0
+
+
 def _df_cost(shapes, phase, nsz, K):
     """The planner's cost of one item in K blocks (written out again here)."""
     kb = (K // 64) * (0.5 + 0.5 * nsz / 256.0)
@@ -428,7 +432,7 @@ def test_dataflow_plan(lib, name):
             c = _df_cost(shapes, ph, r[4], K) + (2.0 if r[6] > 1 else 0.0)
             total += T * c
             cost[(r[0], ph)] = max(cost.get((r[0], ph), 0.0), c)
-    chain = max(T * sum(cost[(m, ph)] + 4.0 for ph in range(3)) - 4.0 for m in range(len(shapes)))
+    chain = max(T * sum(cost[(m, ph)] + DEP for ph in range(3)) - DEP for m in range(len(shapes)))
     bound = max(total / 76, chain)
     assert bound <= makespan <= 1.15 * bound, (makespan, total / 76, chain)
 
