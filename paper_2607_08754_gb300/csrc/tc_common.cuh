@@ -121,15 +121,6 @@ __device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmI
 // t = tm and t = tn).  Both CTAs of a pair take the same choice.
 __device__ __forceinline__ bool sym_mn(int kb, int t) { return (kb >> 1) < t; }
 
-// Symmetric products (Gram, Poly): only tiles holding some 128 x 128 block on
-// or above the diagonal are computed.  Tile (tm, tn) covers row blocks 2 tm,
-// 2 tm + 1 and column blocks 2 tn .. min(2 tn + 1, nb - 1) (nb = Ppad / 128),
-// so it is computed iff its last column block reaches its first row block.
-__device__ __forceinline__ bool sym_tile_computed(int tm, int tn, int Ppad) {
-    const int last_col_block = min(2 * tn + 1, Ppad / 128 - 1);
-    return last_col_block >= 2 * tm;
-}
-
 // Shared-memory descriptor of one K = 16 slice (kk) of a BK-wide K block:
 // K-major: 128-byte rows (swizzle span), 8-row groups kKSbo apart, the K
 // chunks of 64 elements one 128-row atom column (kAtomBytes) apart, slice kk
@@ -257,8 +248,8 @@ __device__ __forceinline__ void own_row(uint8_t* buf, int lane, const uint4 (&v)
 //   Update: X' rows, stored in W's orientation (transposed iterates take one
 //           coalesced 64-byte segment per column);
 //   Gram / Poly: c * acc (+ b A + a I for Poly) into the Ppad x Ppad output,
-//           plus the transpose of every 128 x 128 block (I, J), J > I, whose
-//           mirror tile is skipped (tiles are 256 rows by 256 columns).
+//           the computed tile only (the skipped strictly-lower tiles are read
+//           as the transpose of these, sym_mn).
 // In the first step after the fused norm pass (p.fused_norm) the stored X_0
 // is W itself: the Gram scales acc by x0_scale^2 and the Update by x0_scale.
 // With split K (Gram), the accumulator is replaced by the sum, in part
