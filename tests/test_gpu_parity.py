@@ -144,6 +144,19 @@ def test_ragged_shapes(compute, variant):
     check(Ws, variant, compute, lam=0.7, grad_scale=2.0)
 
 
+@pytest.mark.parametrize("compute,variant", [("fp16", "hoyer"), ("fp16", "nuclear"), ("bf16", "hoyer"),
+                                             ("fp32", "hoyer")])
+def test_extreme_and_large_shapes(compute, variant):
+    """Shapes at the limits: rows of 65536 elements (the longest the library
+    takes; the Gram's K is 65536 and its tiles split K), the transposed case,
+    a P = 2048 matrix whose Poly and Update read most K blocks of A and M
+    MN-major from the stored transpose (8 tile rows), and a ragged transposed
+    matrix (P = 1500, Ppad = 1536)."""
+    shapes = [(64, 65536), (65536, 96), (2048, 6144), (3000, 1500)]
+    Ws = [workloads.random_matrix(s, seed=40 + i, std=0.02) for i, s in enumerate(shapes)]
+    check(Ws, variant, compute, lam=0.5)
+
+
 @pytest.mark.parametrize("compute", ["fp32", "fp16", "bf16"])
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 def test_flat_tiles_with_tails(compute, dtype):
