@@ -238,10 +238,9 @@ __device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, 
             // one 3-D box per operand half: 128 rows (y) of two 64-element
             // chunks (z) of each row.  K-major: rows are MN, chunks are K;
             // MN-major: rows are K, chunks are MN.
-            const bool sym = item_phase<PH>(it) != kGram;  // operands of rows of A or M
             if (load_a) {
                 const int mn = it.tm * (2 * kBM) + rank * kBM;
-                if (!(pi.a_mn || (sym && sym_mn(kb, it.tm))))
+                if (!a_mn_at<PH>(pi, it, kb))
                     ptx::tma_load_3d_pair(sa, pi.mapA, bar, 0, mn, k / 64);
                 else
                     ptx::tma_load_3d_pair(sa, pi.mapA, bar, 0, k, mn / 64);
@@ -250,7 +249,7 @@ __device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, 
             // takes the same box; the UMMA reads its first 64)
             if (load_b) {
                 const int mn = it.tn * kBNMax + rank * (it.nsz / 2);
-                if (!(pi.b_mn || (item_phase<PH>(it) == kPoly && sym_mn(kb, it.tn))))
+                if (!b_mn_at<PH>(pi, it, kb))
                     ptx::tma_load_3d_pair(sb, pi.mapB, bar, 0, mn, k / 64);
                 else
                     ptx::tma_load_3d_pair(sb, pi.mapB, bar, 0, k, mn / 64);
@@ -322,8 +321,6 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
          idx = next_running<PH>(p, idx + seq.stride, seq.end, seq.stride), ++local) {
         const GemmItem it = p.items[idx];
         const PhaseInfo pi = phase_info<C, PH>(p, it);
-        const bool sym = item_phase<PH>(it) != kGram;  // operands of rows of A or M (sym_mn)
-        const bool poly = item_phase<PH>(it) == kPoly;
         const int slot = local % C::kSlots;
         const uint32_t tphase = uint32_t(local / C::kSlots) & 1u;
         if (!ptx::mbar_wait<true>(&s.tempty[slot], tphase ^ 1u, s.abort, p.timeout_ns)) {
@@ -351,8 +348,8 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
             ptx::tc_fence_after();
             const uint32_t a0 = ptx::smem_u32(s.stages + size_t(stage) * C::kStageBytes);
             const uint32_t b0 = shared_operand<PH>(it) ? a0 : a0 + C::kABytes;
-            const bool a_mn = pi.a_mn || (sym && sym_mn(kb, it.tm));
-            const bool b_mn = pi.b_mn || (poly && sym_mn(kb, it.tn));
+            const bool a_mn = a_mn_at<PH>(pi, it, kb);
+            const bool b_mn = b_mn_at<PH>(pi, it, kb);
             const uint32_t id = ptx::idesc_f16(2 * kBM, it.nsz, BF16, a_mn, b_mn);
 #pragma unroll
             for (int kk = 0; kk < C::BK / 16; ++kk) {

@@ -121,6 +121,18 @@ __device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmI
 // t = tm and t = tn).  Both CTAs of a pair take the same choice.
 __device__ __forceinline__ bool sym_mn(int kb, int t) { return (kb >> 1) < t; }
 
+// The major-ness of a tile's A and B operand halves in K block kb: the
+// phase's own choice (phase_info), or MN-major for rows of A or M outside
+// the stored tiles.  The producer's copies and the MMA's descriptors use it.
+template <int PH>
+__device__ __forceinline__ bool a_mn_at(const PhaseInfo& pi, const GemmItem& it, int kb) {
+    return pi.a_mn || (item_phase<PH>(it) != kGram && sym_mn(kb, it.tm));
+}
+template <int PH>
+__device__ __forceinline__ bool b_mn_at(const PhaseInfo& pi, const GemmItem& it, int kb) {
+    return pi.b_mn || (item_phase<PH>(it) == kPoly && sym_mn(kb, it.tn));
+}
+
 // Shared-memory descriptor of one K = 16 slice (kk) of a BK-wide K block:
 // K-major: 128-byte rows (swizzle span), 8-row groups kKSbo apart, the K
 // chunks of 64 elements one 128-row atom column (kAtomBytes) apart, slice kk
