@@ -370,6 +370,31 @@ def test_split_plan_items(lib):
         slorr._check(slorr.load_library().slorr_gemm_item_list(slorr.Regularizer(rn).handle, 0, None, 0))
 
 
+def test_symmetric_reads_find_stored_tiles(lib):
+    """A and M are stored only in the 256 x 256 tiles the Gram and the Poly
+    compute.  The readers' rule (written out again here): an operand made of
+    rows of A or M in tile row t reads its 128-wide K block kb K-major from
+    tile (t, kb // 2) when kb // 2 >= t, else MN-major from tile (kb // 2, t).
+    Every such tile must be in the plan's item list of the phase that writes
+    it, for every padded size (ragged ones included)."""
+    for P in (64, 128, 200, 256, 320, 384, 640, 1000, 1024, 1536, 2048):
+        shapes = [(P, P + 64), (2 * P + 7, P)]
+        reg = slorr.Regularizer(shapes)
+        stored = {ph: {(r[0], r[1], r[2]) for r in slorr.slorr_gemm_item_list(reg.handle, ph).tolist()}
+                  for ph in (0, 1)}
+        Ppad = -(-P // 128) * 128
+        rows = -(-Ppad // 256)   # 256-row tiles
+        nkb = Ppad // 128
+        for mat in range(len(shapes)):
+            def tile_of(t, kb):
+                return (mat, t, kb // 2) if kb // 2 >= t else (mat, kb // 2, t)
+            for t in range(rows):
+                for kb in range(nkb):
+                    # the Update's A operand (rows of M) and both Poly operands (rows of A)
+                    assert tile_of(t, kb) in stored[1], (P, mat, t, kb)
+                    assert tile_of(t, kb) in stored[0], (P, mat, t, kb)
+
+
 # the planner's dependency latency, in K blocks (written out again here)
 DEP = 8.0
 
