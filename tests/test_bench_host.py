@@ -43,3 +43,23 @@ def test_traffic_scaling_is_consistent():
     sub = float(vals["dram_bytes_per_launch_subset"])
     scale = float(vals["scale_subset_to_vit_l16"])
     assert float(vals["dram_bytes_per_launch_scaled"]) == pytest.approx(sub * scale, rel=1e-3)
+
+
+def test_reference_arm_prints_the_contract_line():
+    """bench.py --impl reference (the fp64 oracle on the host cores) prints one
+    JSON line with the contract's keys, its own cpu_baseline and an e2e object
+    with no host<->device bytes."""
+    import json
+    import subprocess
+    out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--workload", "cfg1",
+                          "--steps", "1", "--warmup", "3"], capture_output=True, text=True, timeout=300, cwd=ROOT)
+    assert out.returncode == 0, out.stderr[-2000:]
+    line = json.loads(out.stdout.strip().splitlines()[-1])
+    for k in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better", "scaling",
+              "vs_baseline", "dtype", "data", "config", "impl", "cpu_baseline", "e2e"):
+        assert k in line, k
+    assert line["impl"] == "reference" and line["metric"] == bench.METRIC and line["steps"] == 1
+    assert line["value"] > 0 and line["cpu_baseline"]["value"] == line["value"]
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
+    assert line["e2e"]["value"] == line["value"] and line["e2e"]["unit"] == line["unit"]
