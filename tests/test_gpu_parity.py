@@ -315,6 +315,16 @@ def test_decoder_560m_mha_full_size_sampled_nuclear():
     full_set_sampled("decoder_560m_mha", (1, 5, 160), variant="nuclear")
 
 
+@pytest.mark.parametrize("variant", ["hoyer", "nuclear"])
+def test_vit_b16_full_size_sampled(variant):
+    """The ViT-B/16 set in the bench's configuration (fp16 operands; the plan
+    takes the dataflow launch for it): the first block's matrices, a middle
+    one and the last against the oracle."""
+    from paper_2607_08754_gb300.slorr import Regularizer, slorr_dataflow_items
+    slorr_dataflow_items(Regularizer(workloads.shapes("vit_b16")).handle)  # raises if per-phase
+    full_set_sampled("vit_b16", (0, 1, 2, 3, 25, 47), variant=variant)
+
+
 def test_vit_b16_full_size_sampled_bf16():
     full_set_sampled("vit_b16", (0, 1, 2, 3, 47), compute="bf16")
 
