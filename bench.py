@@ -223,8 +223,16 @@ class ClockSampler:
                 if v.strip().lower() == "active":
                     reasons.add(name)
         loaded = sorted(sm)[len(sm) // 2:] if sm else []
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        pw = [v for v in (num(r[3]) for r in rows) if v is not None]
         return {"sm_mhz": statistics.median(loaded) if loaded else None,
-                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons), "samples": len(rows)}
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons), "samples": len(rows),
+                "power_w_median": statistics.median(pw) if pw else None, "power_w_max": max(pw) if pw else None}
 
 
 def tc_source_hash() -> str:

@@ -63,3 +63,28 @@ def test_reference_arm_prints_the_contract_line():
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
     assert line["e2e"]["value"] == line["value"] and line["e2e"]["unit"] == line["unit"]
+
+
+def test_clock_sampler_summary(tmp_path):
+    """The clock record of a bench line: the median SM clock of the loaded
+    half of the samples, the throttle reasons seen, and the power draw."""
+    sampler = bench.ClockSampler(0)
+    sampler.path = str(tmp_path / "clocks.csv")
+    with open(sampler.path, "w") as f:
+        f.write("0, 1980, 2070, 1385.21, 0x4, Not Active, Not Active, Not Active, Active\n"
+                "0, 2070, 2070, 950.00, 0x0, Not Active, Not Active, Not Active, Not Active\n"
+                "0, 2010, 2070, [N/A], 0x0, Not Active, Not Active, Not Active, Not Active\n")
+
+    class _Done:
+        def terminate(self):
+            pass
+
+        def wait(self, timeout=None):
+            pass
+
+    sampler.proc = _Done()
+    sampler.out = open(os.devnull, "w")
+    rec = sampler.stop()
+    assert rec["sm_mhz"] == 2040.0 and rec["sm_max_mhz"] == 2070.0 and rec["samples"] == 3
+    assert rec["reasons"] == ["sw_power_cap"]
+    assert rec["power_w_median"] == pytest.approx((1385.21 + 950.0) / 2) and rec["power_w_max"] == 1385.21
