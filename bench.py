@@ -74,7 +74,7 @@ def parse():
                     help="only the first N matrices of the workload (a smaller case of the same shapes, "
                          "for profiling); 0: all")
     ap.add_argument("--variant", default="hoyer", choices=["hoyer", "nuclear"])
-    ap.add_argument("--compute", default="fp16", choices=["fp16", "bf16", "fp32"])
+    ap.add_argument("--compute", default="fp16", choices=["fp16", "bf16", "fp32", "bf16_split"])
     ap.add_argument("--dtype", default="f32", choices=["f32", "bf16"], help="storage of the weights and grads")
     ap.add_argument("--iters", type=int, default=6)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
@@ -243,10 +243,11 @@ def tc_source_hash() -> str:
     return h.hexdigest()
 
 
-def tc_traffic(workload: str, matrices: int, per_phase: bool):
+def tc_traffic(workload: str, matrices: int, per_phase: bool, compute: str = "fp16"):
     """dram bytes per launch of the tensor-core GEMM from the committed ncu
     summary, or None when the kernel source changed since it was taken, or when
-    this run's weight set, matrix count or launch mode is not the one captured."""
+    this run's weight set, matrix count, launch mode or operand mode is not the
+    one captured."""
     try:
         src = tc_source_hash()
         vals = {}
@@ -258,7 +259,8 @@ def tc_traffic(workload: str, matrices: int, per_phase: bool):
         if vals.get("source_sha256") != src:
             return None
         if (vals.get("workload") != workload or int(vals.get("matrices", -1)) != matrices
-                or vals.get("launch_mode") != ("per-phase" if per_phase else "dataflow")):
+                or vals.get("launch_mode") != ("per-phase" if per_phase else "dataflow")
+                or vals.get("compute") != compute):
             return None
         return float(vals["dram_bytes_per_launch_scaled"])
     except Exception:
@@ -456,7 +458,10 @@ def main():
         gemm_launches = sum(kt[k][1] for k in ("gram", "poly", "update", "gemm"))
         launches = sum(v[1] for v in kt.values())  # the same launches as the headline timed region
         per_launch_ms = gemm_ms / max(gemm_launches, 1)
-        flops_per_launch = flops_step * args.steps / max(gemm_launches, 1)
+        # bf16 hi/lo mode: three bf16 products per product, counted
+        split = args.compute == "bf16_split"
+        flops_gemm = 3 * flops_step if split else flops_step
+        flops_per_launch = flops_gemm * args.steps / max(gemm_launches, 1)
         achieved = flops_per_launch / (per_launch_ms * 1e-3) / 1e12
         peak = pk["bf16"]  # fp16 and bf16 share the dense tensor rate (nominal ratio 1)
         # CUDA-core GEMM (fp32 mode, or the 16-bit check path): bound by FP32
@@ -486,7 +491,7 @@ def main():
         xelems = sum(((max(m, n) + 127) // 128 * 128) * ((min(m, n) + 127) // 128 * 128) for m, n in shapes)
         comb = (2 * wsz + xsz) if descent else (3 * wsz + xsz)
         mem_bytes = {"sumsq": wsz * elems, "cast": wsz * elems + xsz * xelems,
-                     "normcast": wsz * elems + xsz * xelems, "dot": (wsz + xsz) * elems,
+                     "normcast": wsz * elems + (2 if split else 1) * xsz * xelems, "dot": (wsz + xsz) * elems,
                      "combine": comb * elems}
         memory_roofline = {}
         for k, b in mem_bytes.items():
@@ -503,7 +508,8 @@ def main():
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
             "scaling": "strong" if partition else "weak",
             "vs_baseline": None,
-            "dtype": {"fp16": "f16", "bf16": "bf16"}.get(args.compute, "tf32x3" if tf32 else "f32"),
+            "dtype": {"fp16": "f16", "bf16": "bf16", "bf16_split": "bf16 hi/lo"}.get(args.compute,
+                                                                                     "tf32x3" if tf32 else "f32"),
             "data": "synthetic",
             "config": {"workload": f"{name}{' (first %d matrices)' % len(set_shapes) if args.matrices else ''} "
                                    f"{args.variant}{' descent step' if descent else ''}: "
@@ -531,11 +537,13 @@ def main():
                                                         "1.1 / 2.25 PFLOP/s)" % TF32_RATIO}
                          if tf32 else
                          {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                          "frac": achieved / peak, "traffic": tc_traffic(args.workload, len(shapes), not kt["gemm"][1]),
+                          "frac": achieved / peak, "traffic": tc_traffic(args.workload, len(shapes), not kt["gemm"][1], args.compute),
                           "frac_of_sustained": achieved / pk["bf16_sustained"],
                           "kernel": "tc_pair_kernel (" + ("one dataflow launch per call: every Gram, Poly and "
                                                           "Update of the T steps" if kt["gemm"][1] else
-                                                          "Gram/Poly/Update launches") + ")",
+                                                          "Gram/Poly/Update launches") +
+                                    ("; bf16 hi/lo: three bf16 products per product, counted in "
+                                     "achieved" if split else "") + ")",
                           "peak_source": pk["source"] + " bf16 burst (fp16 dense rate equal)"}
                          if not simt else
                          {"bound": "alu", "achieved": achieved, "peak": alu_peak, "unit": "TFLOP/s",

@@ -71,10 +71,25 @@ typedef enum slorr_dtype {       /* storage type of the weights and of their gra
 typedef enum slorr_compute {     /* operand type of the Polar Express matrix products */
     SLORR_COMPUTE_FP16 = 0,      /* fp16 operands, fp32 accumulation (tensor cores)  */
     SLORR_COMPUTE_BF16 = 1,      /* bf16 operands, fp32 accumulation (tensor cores)  */
-    SLORR_COMPUTE_FP32 = 2       /* fp32 operands: three tf32 tensor-core products per
+    SLORR_COMPUTE_FP32 = 2,      /* fp32 operands: three tf32 tensor-core products per
                                     product, short-K fp32 accumulations added with
                                     compensated sums (CUDA cores, compensated dot
                                     products, with SLORR_FLAG_SIMT_GEMM)              */
+    SLORR_COMPUTE_BF16_SPLIT = 3 /* bf16 operands (App. C.1) with every product
+                                    operand -- the iterate X_t (X_0 included), A
+                                    and M -- carried as a bf16 pair hi = bf16(v),
+                                    lo = bf16(v - hi), and every product as three
+                                    bf16 tensor-core products (hi hi + lo hi +
+                                    hi lo, fp32 accumulation); the Poly's b A term
+                                    takes hi + lo; X_T is stored in fp16 for the
+                                    n_hat and gradient passes.  Three times the
+                                    tensor-core work of SLORR_COMPUTE_BF16, at the
+                                    bf16 rate; gradient errors of about 1e-3 against
+                                    the fp64 approximation, where plain bf16
+                                    operands lose up to 4e-2 on the Hoyer gradient.
+                                    Tensor cores only, per-phase launches:
+                                    SLORR_FLAG_SIMT_GEMM, SLORR_FLAG_SEPARATE_NORM
+                                    and SLORR_FLAG_DATAFLOW are rejected              */
 } slorr_compute;
 
 typedef struct slorr_shape {
@@ -221,8 +236,9 @@ SLORR_API slorr_status slorr_run_steps(slorr_handle* h, const void* const* weigh
  * an array in W's orientation -- rows x cols = m x n, row-major with leading
  * dimension ld >= n -- of element type elem (0 fp32, 1 fp16, 2 bf16).  The
  * Polar Express iterate X (P x Q, P = min(m,n)) is this array when m <= n and
- * its transpose when m > n (transposed = 1).  Also returns device pointers to
- * ||W_i||_F^2 (double) and n_hat_i (double). */
+ * its transpose when m > n (transposed = 1).  With SLORR_COMPUTE_BF16_SPLIT the
+ * array holds the hi parts (bf16) before step T and X_T in fp16 after it.  Also
+ * returns device pointers to ||W_i||_F^2 (double) and n_hat_i (double). */
 typedef struct slorr_matrix_view {
     const void*   x;
     int64_t       rows, cols, ld;

@@ -47,6 +47,7 @@ namespace {
 struct Geom {
     int m, n, P, Q, Ppad, Qpad, transposed, rows, ld;
     size_t off_x[2], off_a, off_b;
+    size_t off_xlo[2], off_alo, off_blo;  // bf16 hi/lo mode: the low parts of X_t, A and M
     size_t off_tf32[10];            // fp32 tensor-core mode: xg[2][2], xu[2][2], a lo, m lo
     int tile_base, tile_count;      // tiles of W (sumsq, dot, combine)
     int xtile_base, xtile_count;    // tiles of the padded iterate (cast, normcast)
@@ -117,8 +118,12 @@ namespace {
 // step (build_plan decides; see kDataflowMaxWork).
 bool dataflow(const slorr_handle* h) { return h->df; }
 
+// bf16 hi/lo mode (SLORR_COMPUTE_BF16_SPLIT): the iterates, A and M carried
+// as bf16 hi and lo parts, every product as three bf16 products.
+bool split16(const slorr_handle* h) { return h->opt.compute == SLORR_COMPUTE_BF16_SPLIT; }
+
 bool dataflow_possible(const slorr_handle* h) {
-    return h->opt.compute != SLORR_COMPUTE_FP32 &&
+    return h->opt.compute != SLORR_COMPUTE_FP32 && !split16(h) &&
            (h->opt.flags & (SLORR_FLAG_SIMT_GEMM | SLORR_FLAG_PHASE_LAUNCHES)) == 0;
 }
 
@@ -144,7 +149,7 @@ constexpr int32_t kKnownFlags = SLORR_FLAG_SIMT_GEMM | SLORR_FLAG_TEST_STALL | S
 
 bool valid_options(const slorr_options& o, std::string* why) {
     if (o.variant != SLORR_HOYER && o.variant != SLORR_NUCLEAR) return *why = "variant", false;
-    if (o.compute < SLORR_COMPUTE_FP16 || o.compute > SLORR_COMPUTE_FP32) return *why = "compute", false;
+    if (o.compute < SLORR_COMPUTE_FP16 || o.compute > SLORR_COMPUTE_BF16_SPLIT) return *why = "compute", false;
     if (o.dtype != SLORR_F32 && o.dtype != SLORR_BF16) return *why = "dtype", false;
     if (o.iters < 1 || o.iters > kMaxIters) return *why = "iters must be in [1, 16]", false;
     if (!(o.ell > 0.0 && o.ell < 1.0)) return *why = "ell must be in (0, 1)", false;
@@ -156,6 +161,11 @@ bool valid_options(const slorr_options& o, std::string* why) {
     if (o.flags & ~kKnownFlags) return *why = "flags holds a bit this build does not define", false;
     if ((o.flags & SLORR_FLAG_PHASE_LAUNCHES) && (o.flags & SLORR_FLAG_DATAFLOW))
         return *why = "SLORR_FLAG_PHASE_LAUNCHES and SLORR_FLAG_DATAFLOW exclude each other", false;
+    if (o.compute == SLORR_COMPUTE_BF16_SPLIT &&
+        (o.flags & (SLORR_FLAG_SIMT_GEMM | SLORR_FLAG_SEPARATE_NORM | SLORR_FLAG_DATAFLOW)))
+        return *why = "SLORR_COMPUTE_BF16_SPLIT runs on the tensor cores, after the fused norm pass, in per-phase "
+                      "launches (no SIMT_GEMM, SEPARATE_NORM or DATAFLOW flag)",
+               false;
     return true;
 }
 
@@ -659,6 +669,17 @@ void build_plan(slorr_handle* h) {
         off = align_up(off + pbytes, 1024);
         g.off_b = off;
         off = align_up(off + pbytes, 1024);
+        g.off_xlo[0] = g.off_xlo[1] = g.off_alo = g.off_blo = 0;
+        if (split16(h)) {
+            g.off_xlo[0] = off;
+            off = align_up(off + xbytes, 1024);
+            g.off_xlo[1] = off;
+            off = align_up(off + xbytes, 1024);
+            g.off_alo = off;
+            off = align_up(off + pbytes, 1024);
+            g.off_blo = off;
+            off = align_up(off + pbytes, 1024);
+        }
         if (tf32) {
             // xg[b][h] (Ppad x Qpad) and xu[b][h] (Qpad x Ppad), then the lo halves of A and M
             for (int k = 0; k < 8; ++k) {
@@ -764,6 +785,11 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
         md.x[1] = ws + g.off_x[1];
         md.a = ws + g.off_a;
         md.b = ws + g.off_b;
+        const bool lo = split16(h);
+        md.xlo[0] = lo ? ws + g.off_xlo[0] : nullptr;
+        md.xlo[1] = lo ? ws + g.off_xlo[1] : nullptr;
+        md.alo = lo ? ws + g.off_alo : nullptr;
+        md.blo = lo ? ws + g.off_blo : nullptr;
         md.m = g.m;
         md.n = g.n;
         md.P = g.P;
@@ -775,12 +801,17 @@ slorr_status prepare(slorr_handle* h, uint8_t* ws, cudaStream_t st) {
         md.ld = g.ld;
         md.pad_ = 0;
         if (tc) {
-            const bool bf = h->opt.compute == SLORR_COMPUTE_BF16;
+            const bool bf = h->opt.compute == SLORR_COMPUTE_BF16 || lo;
             CUtensorMap* mp = reinterpret_cast<CUtensorMap*>(maps.data() + size_t(i) * kMapsPerMatrix * 128);
             bool ok = true;
             for (int b = 0; b < 2; ++b) ok = ok && encode_map(mp + b, md.x[b], g.rows, g.ld, bf);
             ok = ok && encode_map(mp + 2, md.a, g.Ppad, g.Ppad, bf);
             ok = ok && encode_map(mp + 3, md.b, g.Ppad, g.Ppad, bf);
+            if (lo) {
+                for (int b = 0; b < 2; ++b) ok = ok && encode_map(mp + 4 + b, md.xlo[b], g.rows, g.ld, true);
+                ok = ok && encode_map(mp + 6, md.blo, g.Ppad, g.Ppad, true);
+                ok = ok && encode_map(mp + 7, md.alo, g.Ppad, g.Ppad, true);
+            }
             if (!ok) return fail(SLORR_ERR_CUDA, "cuTensorMapEncodeTiled failed");
         }
         if (tf32) {
@@ -1080,6 +1111,8 @@ slorr_status launch_all(slorr_handle* h, uint8_t* ws, float* loss, float* per, i
     g.coef = reinterpret_cast<const float*>(ws + h->off_coef);
     g.tf32 = reinterpret_cast<const MatTf32*>(ws + h->off_tf32_mats);
     g.tf32_maps = ws + h->off_tf32_maps;
+    g.split = split16(h) ? 1 : 0;
+    g.last_step = h->opt.iters - 1;
     if (use_tc && dataflow(h) && steps > 0) {
         // every phase of every step in one launch, ordered by completion counts
         g.items = reinterpret_cast<const GemmItem*>(ws + h->off_df_items);
@@ -1117,6 +1150,7 @@ slorr_status launch_all(slorr_handle* h, uint8_t* ws, float* loss, float* per, i
     }
     if (!finish) return SLORR_OK;
     MemLaunch dp = mem_params(h, ws, loss, per, steps & 1);
+    if (split16(h) && steps == h->opt.iters) dp.elem = kF16;  // the last Update stored X_T in fp16
     if (descent) {
         dp.out_mode = kOutDescent;
         dp.grad_scale = -eta * h->opt.grad_scale;  // alpha, beta then carry -eta * lambda * grad_scale
@@ -1203,7 +1237,7 @@ slorr_status slorr_create(slorr_handle** out, const slorr_shape* shapes, int32_t
         h->elem = kF32;
         h->esize = 4;
     } else {
-        h->elem = o.compute == SLORR_COMPUTE_BF16 ? kBF16 : kF16;
+        h->elem = (o.compute == SLORR_COMPUTE_BF16 || o.compute == SLORR_COMPUTE_BF16_SPLIT) ? kBF16 : kF16;
         h->esize = 2;
     }
     build_plan(h);
@@ -1229,7 +1263,9 @@ slorr_status slorr_executed_flops(const slorr_handle* h, double* out) {
             split_range(it, Kfull / kPairBK, &kb0, &kb1);
             const double K = it.ksplit ? double(kb1 - kb0) * kPairBK : double(Kfull);
             const double rows = (simt || tf32) ? double(it.msz) : 256.0;  // pair UMMAs are always M = 256
-            total += (tf32 ? 3.0 : 1.0) * 2.0 * rows * double(it.nsz) * K;  // tf32: three products
+            // three products per product: fp32 mode (tf32) and bf16 hi/lo mode
+            const bool three = tf32 || split16(h);
+            total += (three ? 3.0 : 1.0) * 2.0 * rows * double(it.nsz) * K;
         }
     }
     *out = total * double(h->opt.iters);
@@ -1371,7 +1407,8 @@ slorr_status slorr_iterate_view(const slorr_handle* h, const void* workspace, in
     out->rows = g.m;
     out->cols = g.n;
     out->ld = g.ld;
-    out->elem = h->elem;
+    // bf16 hi/lo mode: the high parts, and X_T (after the last step) in fp16
+    out->elem = (split16(h) && after_steps == h->opt.iters) ? kF16 : h->elem;
     out->transposed = g.transposed;
     const MatScalars* sc = reinterpret_cast<const MatScalars*>(ws + h->off_scalars) + i;
     out->frob_sq = &sc->frob_sq;

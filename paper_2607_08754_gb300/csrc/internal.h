@@ -42,6 +42,12 @@ struct MatDev {
     void* x[2];        // ping-pong iterate buffers, rows x ld in W's orientation
     void* a;           // A = X X^T, Ppad x Ppad
     void* b;           // M = a I + b A + c A^2, Ppad x Ppad
+    // bf16 hi/lo mode (SLORR_COMPUTE_BF16_SPLIT): x[], a and b hold bf16(v)
+    // and these the residuals bf16(v - bf16(v)) of the iterates, of A and of M
+    // (null in the other modes)
+    void* xlo[2];
+    void* alo;
+    void* blo;
     int32_t m, n;      // shape of W
     int32_t P, Q;      // min / max
     int32_t Ppad, Qpad;
@@ -173,11 +179,19 @@ struct GemmLaunch {
     // fp32 mode on the tensor cores: the hi/lo operand arrays and their maps
     const MatTf32* tf32;
     const void* tf32_maps;
+    // bf16 hi/lo mode: every product takes three bf16 products of the hi/lo
+    // parts of its operands (hi hi + lo hi + hi lo), the Gram and the Poly
+    // store A and M as hi and lo parts, and the Update stores X' so too,
+    // except in step last_step, which stores X_T in fp16 for the dot and
+    // combine passes
+    int32_t split;
+    int32_t last_step;
 };
 
-// Tensor maps per matrix: X0, X1, A, M (each read as K-major or MN-major
-// halves through the same 3-D map).
-constexpr int kMapsPerMatrix = 4;
+// Tensor maps per matrix: X0, X1, A, M, and in bf16 hi/lo mode the low
+// parts X0_lo, X1_lo, M_lo, A_lo (each read as K-major or MN-major halves
+// through the same 3-D map).
+constexpr int kMapsPerMatrix = 8;
 
 // Where the combine pass puts lambda * grad_scale * G_i.
 enum OutMode : int32_t {

@@ -182,6 +182,15 @@ __device__ __forceinline__ void store_x8(void* X, int64_t off, const F8& v) {
     }
 }
 
+// bf16 hi/lo mode: the residuals v - bf16(v) of eight values.
+__device__ __forceinline__ float bf_lo(float v) { return v - __bfloat162float(__float2bfloat16_rn(v)); }
+__device__ __forceinline__ F8 lo8(const F8& v) {
+    F8 r;
+    r.lo = make_float4(bf_lo(v.lo.x), bf_lo(v.lo.y), bf_lo(v.lo.z), bf_lo(v.lo.w));
+    r.hi = make_float4(bf_lo(v.hi.x), bf_lo(v.hi.y), bf_lo(v.hi.z), bf_lo(v.hi.w));
+    return r;
+}
+
 __device__ __forceinline__ float dot8(const F8& a, const F8& b, float acc) {
     acc = fmaf(a.lo.x, b.lo.x, acc);
     acc = fmaf(a.lo.y, b.lo.y, acc);
@@ -243,6 +252,8 @@ __device__ __forceinline__ float absmax8(const F8& a, float m) {
 // and below overflow when max |w| <= 2^15, and its subnormal spacing (2^-24)
 // costs no more than in the scaled X_0 when ||W||_F >= 1; bf16 has fp32's
 // exponent range.
+// bf16 keeps every unscaled copy (its exponent range is fp32's), so the
+// re-cast below, which writes no low parts, never runs in bf16 hi/lo mode.
 __device__ __forceinline__ bool unscaled_cast_ok(int elem, float maxabs, double frob) {
     return elem == kBF16 || maxabs == 0.f || (maxabs <= 32768.f && frob >= 1.0);
 }
@@ -326,6 +337,7 @@ __global__ void __launch_bounds__(kThreads, 6) sumsq_kernel(const MemLaunch p) {
 // sumsq and cast in one read of W (16-bit iterates).  Items tile the padded
 // buffer (rows x ld); the buffer receives W rounded to 16 bits, unscaled, and
 // zeros in the padding; one partial of ||W||^2 and one of max |w| per item.
+// In bf16 hi/lo mode (a low-part buffer xlo) the low parts w - bf16(w) too.
 template <typename TW, typename TX>
 __global__ void __launch_bounds__(kThreads, 4) normcast_kernel(const MemLaunch p) {
     ptx::griddep_wait();  // inputs come from the previous kernel (programmatic launch)
@@ -342,6 +354,14 @@ __global__ void __launch_bounds__(kThreads, 4) normcast_kernel(const MemLaunch p
 #pragma unroll
     for (int k = 0; k < kPasses; ++k)
         if (in_x(tc, md, k)) store_x8<TX>(X, x_off(tc, md, k), w[k]);
+    if constexpr (std::is_same<TX, __nv_bfloat16>::value) {
+        void* XL = md.xlo[p.cur];
+        if (XL != nullptr) {
+#pragma unroll
+            for (int k = 0; k < kPasses; ++k)
+                if (in_x(tc, md, k)) store_x8<TX>(XL, x_off(tc, md, k), lo8(w[k]));
+        }
+    }
     float acc = 0.f, mx = 0.f;
 #pragma unroll
     for (int k = 0; k < kPasses; ++k) {

@@ -64,10 +64,11 @@ namespace {
 
 using namespace tc;
 
-template <int STAGES_, int EPIW_>
+template <int STAGES_, int EPIW_, bool SPLIT_ = false>
 struct PairCfg {
     static constexpr int BK = kPairBK;                    // two 128-byte swizzle atoms of K
     static constexpr int STAGES = STAGES_;
+    static constexpr bool kSplit = SPLIT_;                // bf16 hi/lo operands (three-pass Update)
     static constexpr int kSlots = 2;                      // accumulators per CTA in TMEM
     static constexpr int kABytes = kBM * BK * 2;          // this CTA's 128 rows of A
     static constexpr int kBBytes = 128 * BK * 2;          // this CTA's half of B (a 128-row box, <= 128 used)
@@ -97,6 +98,11 @@ struct PairCfg {
 // polling warps slow the producer and MMA threads of the long-K phases).
 using PairCfg2 = PairCfg<SLORR_PAIR_STAGES, 4>;
 using PairCfg2Wide = PairCfg<SLORR_PAIR_STAGES, 8>;
+// bf16 hi/lo mode: the kernels that run three products per product and store
+// low parts.  The mode runs per-phase launches only (a dataflow kernel with
+// every phase's epilogue spills registers).
+using PairCfg2Split = PairCfg<SLORR_PAIR_STAGES, 4, true>;
+using PairCfg2WideSplit = PairCfg<SLORR_PAIR_STAGES, 8, true>;
 static_assert(PairCfg2Wide::kEpiWarps == kDataflowEpiWarps, "the dataflow plan counts 2 x 8 warps per item");
 
 struct PairSmem {
@@ -181,10 +187,12 @@ __device__ __forceinline__ bool wait_done(const GemmLaunch& p, const PairSmem& s
 // Diagonal tiles of the symmetric products (Gram A = X X^T, Poly A A): with
 // tm == tn and a full 256 x 256 tile, each CTA's A rows and B columns are the
 // same 128 rows of the same matrix, so they are copied once and both UMMA
-// operands read them (the B descriptor points at the A half).
-template <int PH>
+// operands read them (the B descriptor points at the A half).  Not in bf16
+// hi/lo mode, whose cross products take different parts for A and B.
+template <class C, int PH>
 __device__ __forceinline__ bool shared_operand(const GemmItem& it) {
-    return item_phase<PH>(it) != kUpdate && it.tm == it.tn && it.msz == 2 * kBM && it.nsz == kBNMax;
+    return !C::kSplit && item_phase<PH>(it) != kUpdate && it.tm == it.tn && it.msz == 2 * kBM &&
+           it.nsz == kBNMax;
 }
 
 // Bytes one CTA of the pair copies per stage of a tile: its A rows, unless they
@@ -193,7 +201,7 @@ __device__ __forceinline__ bool shared_operand(const GemmItem& it) {
 template <class C, int PH>
 __device__ __forceinline__ uint32_t pair_stage_bytes(const GemmItem& it, int rank) {
     const uint32_t a = rank * kBM < it.msz ? uint32_t(C::kABytes) : 0u;
-    return shared_operand<PH>(it) ? a : a + uint32_t(C::kBBytes);
+    return shared_operand<C, PH>(it) ? a : a + uint32_t(C::kBBytes);
 }
 
 template <class C, int PH>
@@ -223,7 +231,7 @@ __device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, 
         }
         const PhaseInfo pi = phase_info<C, PH>(p, it);
         const bool load_a = rank * kBM < it.msz;
-        const bool load_b = !shared_operand<PH>(it);
+        const bool load_b = !shared_operand<C, PH>(it);
         int kb_begin, kb_end;
         split_range(it, pi.nkb, &kb_begin, &kb_end);
         for (int kb = kb_begin; kb < kb_end; ++kb) {
@@ -233,26 +241,27 @@ __device__ void pair_producer(const GemmLaunch& p, const PairSmem& s, int rank, 
             }
             uint8_t* sa = s.stages + size_t(stage) * C::kStageBytes;
             uint8_t* sb = sa + C::kABytes;
-            const int k = kb * C::BK;
+            const KPass kp = k_pass<C>(pi, kb);
+            const int k = kp.kr * C::BK;
             const uint32_t bar = even_full + uint32_t(stage * 8);
             // one 3-D box per operand half: 128 rows (y) of two 64-element
             // chunks (z) of each row.  K-major: rows are MN, chunks are K;
             // MN-major: rows are K, chunks are MN.
             if (load_a) {
                 const int mn = it.tm * (2 * kBM) + rank * kBM;
-                if (!a_mn_at<PH>(pi, it, kb))
-                    ptx::tma_load_3d_pair(sa, pi.mapA, bar, 0, mn, k / 64);
+                if (!a_mn_at<PH>(pi, it, kp.kr))
+                    ptx::tma_load_3d_pair(sa, kp.mapA, bar, 0, mn, k / 64);
                 else
-                    ptx::tma_load_3d_pair(sa, pi.mapA, bar, 0, k, mn / 64);
+                    ptx::tma_load_3d_pair(sa, kp.mapA, bar, 0, k, mn / 64);
             }
             // B columns: this CTA's half, nsz / 2 = 64 or 128 (a 64-wide half
             // takes the same box; the UMMA reads its first 64)
             if (load_b) {
                 const int mn = it.tn * kBNMax + rank * (it.nsz / 2);
-                if (!b_mn_at<PH>(pi, it, kb))
-                    ptx::tma_load_3d_pair(sb, pi.mapB, bar, 0, mn, k / 64);
+                if (!b_mn_at<PH>(pi, it, kp.kr))
+                    ptx::tma_load_3d_pair(sb, kp.mapB, bar, 0, mn, k / 64);
                 else
-                    ptx::tma_load_3d_pair(sb, pi.mapB, bar, 0, k, mn / 64);
+                    ptx::tma_load_3d_pair(sb, kp.mapB, bar, 0, k, mn / 64);
             }
             if (++stage == C::STAGES) {
                 stage = 0;
@@ -347,9 +356,10 @@ __device__ void pair_mma(const GemmLaunch& p, const PairSmem& s, uint32_t tmem_b
             }
             ptx::tc_fence_after();
             const uint32_t a0 = ptx::smem_u32(s.stages + size_t(stage) * C::kStageBytes);
-            const uint32_t b0 = shared_operand<PH>(it) ? a0 : a0 + C::kABytes;
-            const bool a_mn = a_mn_at<PH>(pi, it, kb);
-            const bool b_mn = b_mn_at<PH>(pi, it, kb);
+            const uint32_t b0 = shared_operand<C, PH>(it) ? a0 : a0 + C::kABytes;
+            const int kr = k_pass<C>(pi, kb).kr;
+            const bool a_mn = a_mn_at<PH>(pi, it, kr);
+            const bool b_mn = b_mn_at<PH>(pi, it, kr);
             const uint32_t id = ptx::idesc_f16(2 * kBM, it.nsz, BF16, a_mn, b_mn);
 #pragma unroll
             for (int kk = 0; kk < C::BK / 16; ++kk) {
@@ -414,15 +424,16 @@ __device__ void pair_epilogue(const GemmLaunch& p, const PairSmem& s, uint32_t t
             const int per = it.nsz / 32 / ngroups;  // 32-column chunks per warp
             const int parts = it.ksplit >> 8;
             if (parts <= 1) {
-                store_rows<BF16, PH, true>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per, nullptr,
-                                           1, 0, sbuf);
+                store_rows<BF16, PH, true, C::kSplit>(p, it, md, row0, t_row, quad, lane, group * per,
+                                                      (group + 1) * per, nullptr, 1, 0, sbuf);
             } else if (PH != kPoly && PH != kUpdate &&
                        split_partial_is_last(p, it, rank, quad, group, lane, t_row, group * per, (group + 1) * per)) {
                 // split K (Gram): direct stores, since the last part's sum is a
                 // serial step, which the staging round trip lengthens (small
                 // sets, ResNet-18 Gram +7%)
-                store_rows<BF16, PH>(p, it, md, row0, t_row, quad, lane, group * per, (group + 1) * per,
-                                 p.split_part + size_t(it.sid) * 65536, parts, rank * kBM + quad * 32 + lane);
+                store_rows<BF16, PH, false, C::kSplit>(p, it, md, row0, t_row, quad, lane, group * per,
+                                                       (group + 1) * per, p.split_part + size_t(it.sid) * 65536,
+                                                       parts, rank * kBM + quad * 32 + lane);
             }
         }
         // The slot may be overwritten once this warp's TMEM loads are done
@@ -580,11 +591,24 @@ cudaError_t launch_pair_bf(const GemmLaunch& p, int num_sms, cudaStream_t st, in
     }
 }
 
+cudaError_t launch_pair_split(const GemmLaunch& p, int num_sms, cudaStream_t st, int phase, int npairs) {
+    switch (phase) {
+        case kGram: return launch_pair_cfg<true, PairCfg2Split, kGram>(p, num_sms, st, npairs);
+        case kPoly: return launch_pair_cfg<true, PairCfg2WideSplit, kPoly>(p, num_sms, st, npairs);
+        case kUpdate: return launch_pair_cfg<true, PairCfg2Split, kUpdate>(p, num_sms, st, npairs);
+        default: return cudaErrorInvalidValue;  // no dataflow launch in this mode
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_gemm_tc_pair(const GemmLaunch& p, int elem, int num_sms, cudaStream_t st, int phase,
                                 int npairs) {
     if (p.num_items == 0) return cudaSuccess;
+    if (p.split) {
+        if (elem != kBF16) return cudaErrorInvalidValue;  // hi/lo parts are bf16
+        return launch_pair_split(p, num_sms, st, phase, npairs);
+    }
     return elem == kBF16 ? launch_pair_bf<true>(p, num_sms, st, phase, npairs)
                          : launch_pair_bf<false>(p, num_sms, st, phase, npairs);
 }

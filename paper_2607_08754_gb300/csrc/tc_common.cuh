@@ -73,14 +73,18 @@ __device__ __forceinline__ int item_step(const GemmLaunch& p, const GemmItem& it
 struct PhaseInfo {
     const void* mapA;
     const void* mapB;
-    int nkb;
+    const void* mapAlo;  // bf16 hi/lo mode: the low parts of the A operand (else mapA)
+    const void* mapBlo;  // and of the B operand (else mapB)
+    int nkb;     // K blocks the tile's main loop runs (3 nkr in bf16 hi/lo mode)
+    int nkr;     // K blocks of the product's K
     bool a_mn;   // A operand MN-major (else K-major)
     bool b_mn;   // B operand MN-major (else K-major)
 };
 
 // Tensor maps per matrix (kMapsPerMatrix of them, 128 bytes each): X0, X1,
-// A, M.
+// A, M, X0_lo, X1_lo, M_lo, A_lo.
 __device__ __forceinline__ const void* xmap(const uint8_t* maps, int buf) { return maps + buf * 128; }
+__device__ __forceinline__ const void* xlo_map(const uint8_t* maps, int buf) { return maps + (4 + buf) * 128; }
 
 template <class C, int PH>
 __device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmItem& it) {
@@ -109,7 +113,49 @@ __device__ __forceinline__ PhaseInfo phase_info(const GemmLaunch& p, const GemmI
         pi.mapB = xmap(maps, cur);
         pi.nkb = md.Ppad / C::BK;
     }
+    pi.mapAlo = pi.mapA;
+    pi.mapBlo = pi.mapB;
+    pi.nkr = pi.nkb;
+    if constexpr (C::kSplit) {
+        if (phase == kGram) {
+            pi.mapAlo = xlo_map(maps, cur);
+            pi.mapBlo = pi.mapAlo;
+        } else if (phase == kPoly) {
+            pi.mapAlo = maps + 7 * 128;
+            pi.mapBlo = pi.mapAlo;
+        } else {
+            pi.mapAlo = maps + 6 * 128;
+            pi.mapBlo = xlo_map(maps, cur);
+        }
+        pi.nkb = 3 * pi.nkr;
+    }
     return pi;
+}
+
+// Main-loop K block kb of a tile: the operand maps it reads and its block kr
+// of the product's K.  In bf16 hi/lo mode every product runs three passes
+// over K into one accumulator, A_hi B_hi, then A_lo B_hi, then A_hi B_lo (the
+// product of the two low parts, 2^-16 relative, is left out); otherwise one.
+struct KPass {
+    const void* mapA;
+    const void* mapB;
+    int kr;
+};
+template <class C>
+__device__ __forceinline__ KPass k_pass(const PhaseInfo& pi, int kb) {
+    KPass k{pi.mapA, pi.mapB, kb};
+    if constexpr (C::kSplit) {
+        if (kb >= pi.nkr) {
+            if (kb < 2 * pi.nkr) {
+                k.mapA = pi.mapAlo;
+                k.kr = kb - pi.nkr;
+            } else {
+                k.mapB = pi.mapBlo;
+                k.kr = kb - 2 * pi.nkr;
+            }
+        }
+    }
+    return k;
 }
 
 // A and M are stored only in the 256 x 256 tiles the Gram and the Poly
@@ -254,6 +300,13 @@ __device__ __forceinline__ void own_row(uint8_t* buf, int lane, const uint4 (&v)
     __syncwarp();
 }
 
+// bf16 hi/lo mode: the low parts bf16(v - hi) of two values whose high parts
+// are packed in hi.
+__device__ __forceinline__ uint32_t lo_part2(float v0, float v1, uint32_t hi) {
+    const float2 h = unpack2<true>(hi);
+    return pack2<true>(v0 - h.x, v1 - h.y);
+}
+
 // Epilogue of one 128-row block of a finished tile: this warp's 32 TMEM lanes
 // (rows row0 + 32 quad + [0, 32)) and the tile's 32-column chunks
 // [ch_begin, ch_end) (chunk c: columns 256 tn + 32 c, TMEM columns t_row + 32 c).
@@ -267,12 +320,16 @@ __device__ __forceinline__ void own_row(uint8_t* buf, int lane, const uint4 (&v)
 // With split K (Gram), the accumulator is replaced by the sum, in part
 // order, of the `parts` fp32 partials at split_tile (row row_t of the tile;
 // this warp's own part among them).  STAGED: the stores go through the
-// warp's staging buffer sbuf (kStageWarpBytes of shared memory).
-template <bool BF16, int PH, bool STAGED = false>
+// warp's staging buffer sbuf (kStageWarpBytes of shared memory).  SPLIT
+// (bf16 hi/lo mode): the Gram and the Poly also store the low parts of A and
+// M (the Poly's b A term reads both parts of A), and the Update those of X',
+// except in the last step, which stores X_T in fp16 alone.
+template <bool BF16, int PH, bool STAGED = false, bool SPLIT = false>
 __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& it, const MatDev& md, int row0,
                                            uint32_t t_row, int quad, int lane, int ch_begin, int ch_end,
                                            const float* split_tile = nullptr, int parts = 1, int row_t = 0,
                                            uint8_t* sbuf = nullptr) {
+    static_assert(BF16 || !SPLIT, "hi/lo parts are bf16");
     const int row_w = row0 + quad * 32;  // the warp's first row
     const int row = row_w + lane;
     const int nch = ch_end;
@@ -280,54 +337,84 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
     const int phase = item_phase<PH>(it);
     const float xs = (p.fused_norm && t == 0) ? p.scalars[it.mat].x0_scale : 1.f;
     if (phase == kUpdate) {
-        uint16_t* out = reinterpret_cast<uint16_t*>(md.x[(t & 1) ^ 1]);
+        const int nb = (t & 1) ^ 1;
+        uint16_t* out = reinterpret_cast<uint16_t*>(md.x[nb]);
+        const bool f16_out = SPLIT && t == p.last_step;
+        uint16_t* out_lo = (SPLIT && !f16_out) ? reinterpret_cast<uint16_t*>(md.xlo[nb]) : nullptr;
         const int64_t ld = md.ld;
         for (int ch = ch_begin; ch < nch; ++ch) {
             uint32_t r[32];
             ptx::tmem_ld_32x32b_x32(t_row + uint32_t(ch * 32), r);
             ptx::tmem_ld_wait();
             const int col0 = it.tn * kBNMax + ch * 32;
-            if constexpr (STAGED) {
-                uint4 o[4];
-                uint32_t* ow = reinterpret_cast<uint32_t*>(o);
+            uint4 o[4], l[4];
+            uint32_t* ow = reinterpret_cast<uint32_t*>(o);
+            uint32_t* lw = reinterpret_cast<uint32_t*>(l);
 #pragma unroll
-                for (int j = 0; j < 16; ++j)
-                    ow[j] = pack2<BF16>(xs * __uint_as_float(r[2 * j]), xs * __uint_as_float(r[2 * j + 1]));
-                stage_chunk(sbuf, lane, o);
+            for (int j = 0; j < 16; ++j) {
+                const float v0 = xs * __uint_as_float(r[2 * j]), v1 = xs * __uint_as_float(r[2 * j + 1]);
+                if (f16_out) {
+                    ow[j] = pack2<false>(v0, v1);
+                } else {
+                    ow[j] = pack2<BF16>(v0, v1);
+                    if (out_lo) lw[j] = lo_part2(v0, v1, ow[j]);
+                }
+            }
+            if constexpr (STAGED) {
                 // transposed iterates: X^T[q][p], the chunk's columns are rows of the buffer
+                stage_chunk(sbuf, lane, o);
                 if (md.transposed)
                     put_cols(sbuf, lane, out, ld, row_w, col0);
                 else
                     put_rows(sbuf, lane, out, ld, row_w, col0);
                 __syncwarp();
+                if (out_lo) {
+                    stage_chunk(sbuf, lane, l);
+                    if (md.transposed)
+                        put_cols(sbuf, lane, out_lo, ld, row_w, col0);
+                    else
+                        put_rows(sbuf, lane, out_lo, ld, row_w, col0);
+                    __syncwarp();
+                }
             } else if (md.transposed) {
                 // X^T[q][p]: for each column the warp's 32 rows are contiguous
+                const uint16_t* oh = reinterpret_cast<const uint16_t*>(o);
                 uint16_t* dst = out + int64_t(col0) * ld + row;
 #pragma unroll
-                for (int j = 0; j < 32; ++j) dst[int64_t(j) * ld] = to16<BF16>(xs * __uint_as_float(r[j]));
-            } else {
-                uint4 o[4];
-                uint32_t* ow = reinterpret_cast<uint32_t*>(o);
+                for (int j = 0; j < 32; ++j) dst[int64_t(j) * ld] = oh[j];
+                if (out_lo) {
+                    const uint16_t* lh = reinterpret_cast<const uint16_t*>(l);
+                    uint16_t* dl = out_lo + int64_t(col0) * ld + row;
 #pragma unroll
-                for (int j = 0; j < 16; ++j)
-                    ow[j] = pack2<BF16>(xs * __uint_as_float(r[2 * j]), xs * __uint_as_float(r[2 * j + 1]));
+                    for (int j = 0; j < 32; ++j) dl[int64_t(j) * ld] = lh[j];
+                }
+            } else {
                 uint4* dst = reinterpret_cast<uint4*>(out + int64_t(row) * ld + col0);
 #pragma unroll
                 for (int v = 0; v < 4; ++v) dst[v] = o[v];
+                if (out_lo) {
+                    uint4* dl = reinterpret_cast<uint4*>(out_lo + int64_t(row) * ld + col0);
+#pragma unroll
+                    for (int v = 0; v < 4; ++v) dl[v] = l[v];
+                }
             }
         }
     } else {
         uint16_t* out = reinterpret_cast<uint16_t*>(phase == kGram ? md.a : md.b);
         const uint16_t* amat = reinterpret_cast<const uint16_t*>(md.a);
+        const uint16_t* amat_lo = SPLIT ? reinterpret_cast<const uint16_t*>(md.alo) : nullptr;
         const int64_t ld = md.Ppad;
         const bool poly = phase == kPoly;
+        uint16_t* out_lo = SPLIT ? reinterpret_cast<uint16_t*>(poly ? md.blo : md.alo) : nullptr;
         const float ca = poly ? p.coef[3 * t] : 0.f, cb = poly ? p.coef[3 * t + 1] : 0.f;
         const float cacc = poly ? p.coef[3 * t + 2] : xs * xs;
         // Poly reads b A at the output position: loads for the next chunk are
         // issued before the current chunk is processed (staged: coalesced
-        // loads, turned into this lane's row through the staging buffer).
+        // loads, turned into this lane's row through the staging buffer).  In
+        // bf16 hi/lo mode the main loop, three products long, leaves the
+        // epilogue time enough without the prefetch, and both parts are read.
         uint4 e_next[4];
-        if (poly) {
+        if (poly && !SPLIT) {
             if constexpr (STAGED) {
                 get_rows(amat, ld, row_w, it.tn * kBNMax + ch_begin * 32, lane, e_next);
             } else {
@@ -340,8 +427,22 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
         for (int ch = ch_begin; ch < nch; ++ch) {
             const int col0 = it.tn * kBNMax + ch * 32;
             const int64_t off = int64_t(row) * ld + col0;
-            uint4 e[4];
-            if (poly) {
+            uint4 e[4], el[4];
+            if (poly && SPLIT) {
+                if constexpr (STAGED) {
+                    uint4 v[4];
+                    get_rows(amat, ld, row_w, col0, lane, v);
+                    own_row(sbuf, lane, v, e);
+                    get_rows(amat_lo, ld, row_w, col0, lane, v);
+                    own_row(sbuf, lane, v, el);
+                } else {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        e[q] = __ldcg(reinterpret_cast<const uint4*>(amat + off) + q);
+                        el[q] = __ldcg(reinterpret_cast<const uint4*>(amat_lo + off) + q);
+                    }
+                }
+            } else if (poly) {
                 if constexpr (STAGED) {
                     own_row(sbuf, lane, e_next, e);
                     if (ch + 1 < nch) get_rows(amat, ld, row_w, col0 + 32, lane, e_next);
@@ -374,21 +475,29 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
                     for (int j = 0; j < 32; ++j) r[j] = __float_as_uint(__uint_as_float(r[j]) + a[j]);
                 }
             }
-            uint4 o[4];
+            uint4 o[4], l[4];
             uint32_t* ow = reinterpret_cast<uint32_t*>(o);
+            uint32_t* lw = reinterpret_cast<uint32_t*>(l);
             const int d = row - col0;  // diagonal element of this row, if in the chunk
             const uint32_t* ew = reinterpret_cast<const uint32_t*>(e);
+            const uint32_t* elw = reinterpret_cast<const uint32_t*>(el);
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
-                float lo = cacc * __uint_as_float(r[2 * j]);
-                float hi = cacc * __uint_as_float(r[2 * j + 1]);
+                float v0 = cacc * __uint_as_float(r[2 * j]);
+                float v1 = cacc * __uint_as_float(r[2 * j + 1]);
                 if (poly) {
                     // M = c A^2 + b A + a I
-                    const float2 x = unpack2<BF16>(ew[j]);
-                    lo = fmaf(cb, x.x, lo) + (2 * j == d ? ca : 0.f);
-                    hi = fmaf(cb, x.y, hi) + (2 * j + 1 == d ? ca : 0.f);
+                    float2 x = unpack2<BF16>(ew[j]);
+                    if (SPLIT) {
+                        const float2 xl = unpack2<BF16>(elw[j]);
+                        x.x += xl.x;
+                        x.y += xl.y;
+                    }
+                    v0 = fmaf(cb, x.x, v0) + (2 * j == d ? ca : 0.f);
+                    v1 = fmaf(cb, x.y, v1) + (2 * j + 1 == d ? ca : 0.f);
                 }
-                ow[j] = pack2<BF16>(lo, hi);
+                ow[j] = pack2<BF16>(v0, v1);
+                if (out_lo) lw[j] = lo_part2(v0, v1, ow[j]);
             }
             // The output is symmetric and strictly-lower tiles are skipped,
             // with no mirrored copy: its readers take the missing blocks
@@ -398,11 +507,21 @@ __device__ __forceinline__ void store_rows(const GemmLaunch& p, const GemmItem& 
                 stage_chunk(sbuf, lane, o);
                 put_rows(sbuf, lane, out, ld, row_w, col0);
                 __syncwarp();
+                if (out_lo) {
+                    stage_chunk(sbuf, lane, l);
+                    put_rows(sbuf, lane, out_lo, ld, row_w, col0);
+                    __syncwarp();
+                }
                 continue;
             }
             uint4* dst = reinterpret_cast<uint4*>(out + off);
 #pragma unroll
             for (int q = 0; q < 4; ++q) dst[q] = o[q];
+            if (out_lo) {
+                uint4* dl = reinterpret_cast<uint4*>(out_lo + off);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) dl[q] = l[q];
+            }
         }
     }
 }

@@ -22,7 +22,7 @@ SLORR_OK = 0
 STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "CUDA", 4: "WORKSPACE",
                 5: "TIMEOUT", 6: "NONFINITE"}
 VARIANTS = {"hoyer": 0, "nuclear": 1}
-COMPUTES = {"fp16": 0, "bf16": 1, "fp32": 2}
+COMPUTES = {"fp16": 0, "bf16": 1, "fp32": 2, "bf16_split": 3}
 DTYPES = {"f32": 0, "bf16": 1}
 FLAG_SIMT_GEMM = 1
 FLAG_TEST_STALL = 16

@@ -27,15 +27,17 @@ def test_traffic_only_for_the_captured_case():
     vals = _profile()
     fresh = vals["source_sha256"] == bench.tc_source_hash()
     wl, n = vals["workload"], int(vals["matrices"])
-    got = bench.tc_traffic(wl, n, vals["launch_mode"] == "per-phase")
+    got = bench.tc_traffic(wl, n, vals["launch_mode"] == "per-phase", vals["compute"])
     if fresh:
         assert got == pytest.approx(float(vals["dram_bytes_per_launch_scaled"]))
     else:
         assert got is None
-    # any other set, count or launch mode: no figure
-    assert bench.tc_traffic("resnet18", n, True) is None
-    assert bench.tc_traffic(wl, n // 2, True) is None
-    assert bench.tc_traffic(wl, n, vals["launch_mode"] != "per-phase") is None
+    # any other set, count, launch mode or operand mode: no figure
+    pp = vals["launch_mode"] == "per-phase"
+    assert bench.tc_traffic("resnet18", n, pp, vals["compute"]) is None
+    assert bench.tc_traffic(wl, n // 2, pp, vals["compute"]) is None
+    assert bench.tc_traffic(wl, n, not pp, vals["compute"]) is None
+    assert bench.tc_traffic(wl, n, pp, "bf16_split") is None
 
 
 def test_traffic_scaling_is_consistent():

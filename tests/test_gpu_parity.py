@@ -5,17 +5,19 @@ Tolerances (relative, on the loss and on each matrix's gradient in Frobenius
 norm), the stated targets:
 * fp32 compute mode: 1e-5;
 * fp16-operand mode (tensor cores, the default): 2e-2;
-* bf16-operand mode: 2e-2.
+* bf16-operand modes: 2e-2 (bf16, and bf16_split: every product operand
+  carried as a bf16 hi/lo pair, every product as three bf16 products).
 Weights and gradients stored in bf16 add one rounding of the stored gradient
 (2^-9 relative).
 
 One exception, which does NOT meet the 2e-2 target: the SLORR-Hoyer gradient
-with bf16 operands.  It is the difference of two nearly equal terms, and
-rounding the iterate to bf16 (8 significand bits) after every step leaves
+with plain bf16 operands.  It is the difference of two nearly equal terms,
+and rounding the iterate to bf16 (8 significand bits) after every step leaves
 2.1e-2 to 4.1e-2 on the paper-shaped sets (fp16, 11 bits, at the same tensor
 rate: 2.7e-3 to 5.1e-3).  Those gradients are held to BF16_HOYER_GRAD = 5e-2,
 their measured floor with margin, so that the option stays tested; the bf16
-loss and the bf16 SLORR-Nuc gradient are held to 2e-2.
+loss and the bf16 SLORR-Nuc gradient are held to 2e-2.  The bf16_split mode,
+whose hi/lo pairs remove that rounding, is held to 2e-2 everywhere.
 
 The Hoyer gradient is the difference of two terms, 2 reg P_hat / frob and
 2 reg n_hat W / frob^3 (Listing 1).  When they cancel almost completely (rank
@@ -33,7 +35,7 @@ import workloads
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
-TOL = {"fp32": (1e-5, 1e-5), "fp16": (2e-2, 2e-2), "bf16": (2e-2, 2e-2)}
+TOL = {"fp32": (1e-5, 1e-5), "fp16": (2e-2, 2e-2), "bf16": (2e-2, 2e-2), "bf16_split": (2e-2, 2e-2)}
 BF16_HOYER_GRAD = 5e-2   # outside the 2e-2 target: see the module docstring
 BF16_STORAGE = 2.0 ** -9  # one rounding of a gradient stored in bf16
 EPS = 1e-7
@@ -135,7 +137,7 @@ def test_cfg1_fp32_iterates_match_every_step():
         assert fsq == pytest.approx(float(np.sum(Ws[0].astype(np.float64) ** 2)), rel=1e-6)
 
 
-@pytest.mark.parametrize("compute", ["fp32", "fp16", "bf16"])
+@pytest.mark.parametrize("compute", ["fp32", "fp16", "bf16", "bf16_split"])
 @pytest.mark.parametrize("variant", ["hoyer", "nuclear"])
 def test_ragged_shapes(compute, variant):
     shapes = [(1, 1), (1, 7), (9, 1), (3, 5), (5, 3), (64, 147), (130, 70), (200, 333), (320, 1280),
@@ -145,7 +147,7 @@ def test_ragged_shapes(compute, variant):
 
 
 @pytest.mark.parametrize("compute,variant", [("fp16", "hoyer"), ("fp16", "nuclear"), ("bf16", "hoyer"),
-                                             ("fp32", "hoyer")])
+                                             ("fp32", "hoyer"), ("bf16_split", "hoyer")])
 def test_extreme_and_large_shapes(compute, variant):
     """Shapes at the limits: rows of 65536 elements (the longest the library
     takes; the Gram's K is 65536 and its tiles split K), the transposed case,
@@ -157,7 +159,7 @@ def test_extreme_and_large_shapes(compute, variant):
     check(Ws, variant, compute, lam=0.5)
 
 
-@pytest.mark.parametrize("compute", ["fp32", "fp16", "bf16"])
+@pytest.mark.parametrize("compute", ["fp32", "fp16", "bf16", "bf16_split"])
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 def test_flat_tiles_with_tails(compute, dtype):
     """Rows a multiple of 128 elements: the memory passes take flat runs of
@@ -172,9 +174,12 @@ def test_flat_tiles_with_tails(compute, dtype):
     check(Ws, "hoyer", compute, lam=0.3, dtype=dtype, grads0=G0 if dtype == "f32" else None)
 
 
-@pytest.mark.parametrize("compute", ["fp16", "bf16"])
+@pytest.mark.parametrize("compute", ["fp16", "bf16", "bf16_split"])
 @pytest.mark.parametrize("variant", ["hoyer", "nuclear"])
 def test_resnet18_weight_set(compute, variant):
+    """All 21 matrices of the ResNet-18 set; with bf16_split every gradient
+    within the 2e-2 target (plain bf16 operands miss it on this set's Hoyer
+    gradients)."""
     check(workloads.generate("resnet18"), variant, compute)
 
 
@@ -213,7 +218,7 @@ def test_tensor_core_iterates_match_simt(compute, flags):
 
 # ---- edge cases -------------------------------------------------------------------
 
-@pytest.mark.parametrize("compute", ["fp32", "fp16"])
+@pytest.mark.parametrize("compute", ["fp32", "fp16", "bf16_split"])
 def test_zero_matrix_and_accumulation(compute):
     Ws = [np.zeros((40, 70), np.float32), workloads.random_matrix((70, 40), 3, 0.1)]
     rng = np.random.default_rng(4)
@@ -343,9 +348,44 @@ def test_decoder_560m_full_size_sampled_bf16():
     full_set_sampled("decoder_560m", (0, 1, 2, 4, 6, 164), compute="bf16")
 
 
+# ---- bf16 hi/lo operands: the bf16 configurations within the 2e-2 target ---------
+
+@pytest.mark.parametrize("variant", ["hoyer", "nuclear"])
+def test_vit_l16_full_size_sampled_bf16_split(variant):
+    full_set_sampled("vit_l16", (0, 1, 2, 3, 95), variant=variant, compute="bf16_split")
+
+
+def test_decoder_560m_full_size_sampled_bf16_split():
+    full_set_sampled("decoder_560m", (0, 1, 2, 4, 6, 164), compute="bf16_split")
+
+
+def test_vit_b16_full_size_sampled_bf16_split():
+    full_set_sampled("vit_b16", (0, 1, 2, 3, 47), compute="bf16_split")
+
+
+def test_bf16_split_beats_bf16_on_resnet18_hoyer():
+    """The hi/lo pairs are what brings the bf16 Hoyer gradient inside the
+    target: on the ResNet-18 set the worst gradient error of bf16_split is
+    below 5e-3 and a tenth of plain bf16's (a CPU emulation of both roundings
+    gives 4e-4 against 4.0e-2)."""
+    Ws = workloads.generate("resnet18")
+    co = oracle.pe_coefficients(6)
+    worst = {}
+    for compute in ("bf16", "bf16_split"):
+        _, _, grads, status, _, w_used = run_gpu(Ws, "hoyer", compute)
+        assert status == 0
+        errs = []
+        for i, W in enumerate(w_used):
+            _, G, _, _ = oracle.reg_single(W, "hoyer", co, EPS)
+            errs.append(grad_err(grads[i], G, W, "hoyer", 1.0, 1.0))
+        worst[compute] = max(errs)
+    assert worst["bf16_split"] <= 5e-3 and worst["bf16_split"] < 0.1 * worst["bf16"], worst
+
+
 # ---- failure detection: a bounded device wait runs out -----------------------------
 
-def test_bounded_wait_timeout_reports_status_and_context_survives():
+@pytest.mark.parametrize("compute", ["fp16", "bf16_split"])
+def test_bounded_wait_timeout_reports_status_and_context_survives(compute):
     """SLORR_FLAG_TEST_STALL makes every tensor-core CTA wait on a barrier nothing
     arrives on; with timeout_s = 0.05 each wait gives up, the kernel records
     SLORR_ERR_TIMEOUT in the status word, drains and returns.  The same process
@@ -353,12 +393,12 @@ def test_bounded_wait_timeout_reports_status_and_context_survives():
     from paper_2607_08754_gb300.slorr import Regularizer, FLAG_TEST_STALL
     Ws = [workloads.random_matrix((256, 512), 21, 0.05), workloads.random_matrix((384, 128), 22, 0.05)]
     w = [torch.from_numpy(W).cuda() for W in Ws]
-    stall = Regularizer([W.shape for W in Ws], flags=FLAG_TEST_STALL, timeout_s=0.05)
+    stall = Regularizer([W.shape for W in Ws], compute=compute, flags=FLAG_TEST_STALL, timeout_s=0.05)
     stall.run_steps(w, 1)
     torch.cuda.synchronize()
     assert stall.status() == 5          # SLORR_ERR_TIMEOUT
     assert stall.status() == 0          # reading clears it
-    check(Ws, "hoyer", "fp16")          # the context is still usable
+    check(Ws, "hoyer", compute)         # the context is still usable
 
 
 # ---- decoupled variant (Alg. 1): write the pre-update gradient --------------------
@@ -394,6 +434,7 @@ def test_iteration_count_sweep(T):
     Ws = [workloads.random_matrix(s, seed=300 + i, std=0.03) for i, s in enumerate([(256, 640), (640, 384)])]
     check(Ws, "hoyer", "fp16", iters=T)
     check(Ws, "hoyer", "fp32", iters=T)
+    check(Ws, "hoyer", "bf16_split", iters=T)   # T = 1: the first step is also the last
 
 
 @pytest.mark.parametrize("name", ["vit_ladder_vit_ti", "vit_ladder_vit_256", "vit_ladder_vit_s"])

@@ -497,3 +497,32 @@ def test_launch_mode_is_chosen_by_set_shape(lib):
                 slorr.slorr_dataflow_items(r.handle)
         # the workspace holds the dataflow plan only when it is used
         assert (forced.workspace_bytes > r.workspace_bytes) == (not df)
+
+
+def test_bf16_split_mode_plan(lib):
+    """SLORR_COMPUTE_BF16_SPLIT (bf16 hi/lo operands): the same tiles as
+    bf16, per-phase launches only, a workspace with the low parts of X0, X1,
+    A and M besides bf16's buffers, executed work of three products per
+    product, and the flags it cannot serve rejected."""
+    import workloads
+    shapes = [(64, 147), (3072, 1024), (1024, 4096), (130, 700)]
+    bf = slorr.Regularizer(shapes, compute="bf16", flags=slorr.FLAG_PHASE_LAUNCHES)
+    sp = slorr.Regularizer(shapes, compute="bf16_split")
+    for ph in range(3):
+        assert np.array_equal(slorr.slorr_gemm_item_list(sp.handle, ph), slorr.slorr_gemm_item_list(bf.handle, ph))
+    lo = 0
+    for m, n in shapes:
+        P, Q = min(m, n), max(m, n)
+        Pp, Qp = -(-P // 128) * 128, -(-Q // 128) * 128
+        lo += 2 * (2 * Pp * Qp) + 2 * (2 * Pp * Pp)
+    assert sp.workspace_bytes - bf.workspace_bytes >= lo
+    assert slorr.slorr_executed_flops(sp.handle) == 3 * slorr.slorr_executed_flops(bf.handle)
+    # the dataflow launch is never planned, even for a set that takes it in bf16
+    vb = workloads.shapes("vit_b16")
+    slorr.slorr_dataflow_items(slorr.Regularizer(vb, compute="bf16").handle)
+    with pytest.raises(slorr.SlorrError):
+        slorr.slorr_dataflow_items(slorr.Regularizer(vb, compute="bf16_split").handle)
+    for flag in (slorr.FLAG_SIMT_GEMM, slorr.FLAG_SEPARATE_NORM, slorr.FLAG_DATAFLOW):
+        with pytest.raises(slorr.SlorrError) as e:
+            slorr.Regularizer([(256, 512)], compute="bf16_split", flags=flag)
+        assert e.value.status == 1
