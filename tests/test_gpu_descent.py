@@ -20,7 +20,7 @@ import workloads
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
-TOL = {"fp32": 1e-5, "fp16": 2e-2}
+TOL = {"fp32": 1e-5, "fp16": 2e-2, "bf16_split": 2e-2}
 EPS = 1e-7
 U24 = 2.0 ** -24
 
@@ -72,7 +72,7 @@ def _gpu_steps(Ws, eta, steps, compute="fp32", variant="hoyer", lam=1.0, grad_sc
     return traj, pers
 
 
-@pytest.mark.parametrize("compute", ["fp32", "fp16"])
+@pytest.mark.parametrize("compute", ["fp32", "fp16", "bf16_split"])
 @pytest.mark.parametrize("variant", ["hoyer", "nuclear"])
 def test_one_descent_step_matches_oracle(compute, variant):
     Ws = _set()

@@ -92,17 +92,18 @@ def test_pipeline_vit_b16_matches_oracle_sampled():
         assert np.linalg.norm(got - G) <= 2e-2 * np.linalg.norm(G), i
 
 
-@pytest.mark.parametrize("dtype,variant,flags", [("bf16", "hoyer", 0), ("f32", "nuclear", 0), ("f32", "hoyer", 32),
-                                                 ("bf16", "nuclear", 32)])
-def test_pipeline_options_equal_device_call(dtype, variant, flags):
-    """bf16 weight storage, the nuclear variant and SLORR_FLAG_WRITE_GRAD (32) go
-    through the pipeline unchanged: grads and per-matrix values equal the
-    device-resident call bit for bit."""
+@pytest.mark.parametrize("dtype,variant,flags,compute", [("bf16", "hoyer", 0, "fp16"), ("f32", "nuclear", 0, "fp16"),
+                                                         ("f32", "hoyer", 32, "fp16"), ("bf16", "nuclear", 32, "fp16"),
+                                                         ("f32", "hoyer", 0, "bf16_split")])
+def test_pipeline_options_equal_device_call(dtype, variant, flags, compute):
+    """bf16 weight storage, the nuclear variant, SLORR_FLAG_WRITE_GRAD (32) and
+    the bf16 hi/lo operand mode go through the pipeline unchanged: grads and
+    per-matrix values equal the device-resident call bit for bit."""
     from paper_2607_08754_gb300.slorr import Regularizer, Pipeline
     tdt = torch.float32 if dtype == "f32" else torch.bfloat16
     Ws = [torch.from_numpy(workloads.random_matrix(s, seed=700 + i, std=0.05)).to(tdt) for i, s in enumerate(SHAPES)]
     G0 = [torch.from_numpy(workloads.random_matrix(s, seed=800 + i, std=0.01)).to(tdt) for i, s in enumerate(SHAPES)]
-    kw = dict(variant=variant, dtype=dtype, flags=flags, lam=0.7)
+    kw = dict(variant=variant, dtype=dtype, flags=flags, lam=0.7, compute=compute)
     reg = Regularizer(SHAPES, **kw)
     w = [x.cuda() for x in Ws]
     g = [x.cuda() for x in G0]
