@@ -39,6 +39,7 @@ import argparse
 import hashlib
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -235,11 +236,20 @@ class ClockSampler:
                 "power_w_median": statistics.median(pw) if pw else None, "power_w_max": max(pw) if pw else None}
 
 
+def code_only(text: str) -> str:
+    """C/CUDA source without its comments, whitespace runs collapsed: what
+    the compiler sees, so that a comment edit keeps a capture current."""
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    return " ".join(text.split())
+
+
 def tc_source_hash() -> str:
-    """sha256 over the default tensor-core kernel's source files, in order."""
+    """sha256 over the code (comments stripped) of the tensor-core kernel's
+    source files, in order."""
     h = hashlib.sha256()
     for f in TC_SOURCES:
-        h.update(open(f, "rb").read())
+        h.update(code_only(open(f, encoding="utf-8").read()).encode())
     return h.hexdigest()
 
 

@@ -17,6 +17,12 @@
 //               the items it waits for (see build_dataflow in api.cu), and all
 //               pairs are resident, so the launch cannot deadlock.
 //
+// bf16 hi/lo operand mode (PairCfg<..., true>, per-phase launches): every
+// product runs three passes over K into the same accumulator -- the operands'
+// hi parts, then the A operand's lo part with B's hi part, then A's hi part
+// with B's lo part (k_pass picks the tensor maps of each K block) -- and the
+// epilogues store hi and lo parts of A, M and X'.
+//
 // A cluster of two CTAs on two SMs computes one 256 x 256 tile.  CTA r of the
 // pair holds rows [128 r, 128 r + 128) of the tile's A operand and columns
 // [nsz/2 r, nsz/2 (r + 1)) of its B operand in shared memory, and rows
@@ -68,7 +74,7 @@ template <int STAGES_, int EPIW_, bool SPLIT_ = false>
 struct PairCfg {
     static constexpr int BK = kPairBK;                    // two 128-byte swizzle atoms of K
     static constexpr int STAGES = STAGES_;
-    static constexpr bool kSplit = SPLIT_;                // bf16 hi/lo operands (three-pass Update)
+    static constexpr bool kSplit = SPLIT_;                // bf16 hi/lo operands: three passes over K
     static constexpr int kSlots = 2;                      // accumulators per CTA in TMEM
     static constexpr int kABytes = kBM * BK * 2;          // this CTA's 128 rows of A
     static constexpr int kBBytes = 128 * BK * 2;          // this CTA's half of B (a 128-row box, <= 128 used)

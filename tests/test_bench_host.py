@@ -90,3 +90,11 @@ def test_clock_sampler_summary(tmp_path):
     assert rec["sm_mhz"] == 2040.0 and rec["sm_max_mhz"] == 2070.0 and rec["samples"] == 3
     assert rec["reasons"] == ["sw_power_cap"]
     assert rec["power_w_median"] == pytest.approx((1385.21 + 950.0) / 2) and rec["power_w_max"] == 1385.21
+
+
+def test_code_hash_ignores_comments_only():
+    """The traffic figure is keyed on the kernel's code: comments and
+    whitespace do not change it, a changed token does."""
+    src = "int f(int x) {  // the /* inner */ comment\n  return x + 1; /* block\n comment */ }\n"
+    assert bench.code_only(src) == bench.code_only("int f(int x) {\n return x + 1; }")
+    assert bench.code_only(src) != bench.code_only("int f(int x) { return x + 2; }")
