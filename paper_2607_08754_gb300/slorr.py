@@ -480,18 +480,21 @@ class Pipeline:
     receives lambda * sum_i L_i.  Keyword options as for ``Regularizer``."""
 
     @staticmethod
-    def auto_groups(shapes, dtype: str = "f32") -> int:
+    def auto_groups(shapes, dtype: str = "f32", compute: str = "fp16") -> int:
         """About 64 MiB of weights per group, 1 to 16 groups: enough groups for the
         copies to overlap the kernels, few enough that a group's launches stay
-        cheap next to its copies."""
+        cheap next to its copies.  With bf16 hi/lo operands, whose kernels take
+        2.4 times as long, about 128 MiB (ViT-L/16 on GB300: 18.0 ms with 8
+        groups, 31.7 ms with 16)."""
         esz = 4 if dtype == "f32" else 2
         total = sum(int(m) * int(n) for m, n in shapes) * esz
-        return max(1, min(16, total // (64 << 20)))
+        per = (128 << 20) if compute == "bf16_split" else (64 << 20)
+        return max(1, min(16, total // per))
 
     def __init__(self, shapes, groups: int | None = None, **kw):
         self.shapes = [(int(m), int(n)) for m, n in shapes]
         if groups is None:
-            groups = self.auto_groups(self.shapes, kw.get("dtype", "f32"))
+            groups = self.auto_groups(self.shapes, kw.get("dtype", "f32"), kw.get("compute", "fp16"))
         self.groups = int(groups)
         self.options = make_options(**kw)
         self.handle = slorr_pipeline_create(self.shapes, self.options, groups)
