@@ -18,10 +18,11 @@
 //               pairs are resident, so the launch cannot deadlock.
 //
 // bf16 hi/lo operand mode (PairCfg<..., true>, per-phase launches): every
-// product runs three passes over K into the same accumulator -- the operands'
-// hi parts, then the A operand's lo part with B's hi part, then A's hi part
-// with B's lo part (k_pass picks the tensor maps of each K block) -- and the
-// epilogues store hi and lo parts of A, M and X'.
+// product takes three products into the same accumulator -- the operands' hi
+// parts, the A operand's lo part with B's hi part, A's hi part with B's lo
+// part, one after the other for each K block (k_pass picks the tensor maps of
+// each main-loop block) -- and the epilogues store hi and lo parts of A, M
+// and X'.
 //
 // A cluster of two CTAs on two SMs computes one 256 x 256 tile.  CTA r of the
 // pair holds rows [128 r, 128 r + 128) of the tile's A operand and columns
@@ -74,7 +75,7 @@ template <int STAGES_, int EPIW_, bool SPLIT_ = false>
 struct PairCfg {
     static constexpr int BK = kPairBK;                    // two 128-byte swizzle atoms of K
     static constexpr int STAGES = STAGES_;
-    static constexpr bool kSplit = SPLIT_;                // bf16 hi/lo operands: three passes over K
+    static constexpr bool kSplit = SPLIT_;                // bf16 hi/lo operands: three products per K block
     static constexpr int kSlots = 2;                      // accumulators per CTA in TMEM
     static constexpr int kABytes = kBM * BK * 2;          // this CTA's 128 rows of A
     static constexpr int kBBytes = 128 * BK * 2;          // this CTA's half of B (a 128-row box, <= 128 used)
