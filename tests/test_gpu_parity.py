@@ -310,6 +310,13 @@ def full_set_sampled(name, samples, variant="hoyer", compute="fp16"):
         assert grad_err(g[i].double().cpu().numpy(), G, W, variant, 1.0, 1.0) <= tg, (name, i)
 
 
+def test_vit_l16_full_size_every_matrix():
+    """The bench's own configuration (ViT-L/16 set, fp16 operands, Hoyer, one
+    call over all 96 matrices) with every matrix's value and gradient against
+    the oracle, not a sample."""
+    full_set_sampled("vit_l16", range(96))
+
+
 def test_decoder_560m_full_size_sampled():
     """The 560M decoder set (168 matrices, 417 M weights): q, k, o, gate and
     down projections of the first and last blocks."""
