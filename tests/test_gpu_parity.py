@@ -137,6 +137,26 @@ def test_cfg1_fp32_iterates_match_every_step():
         assert fsq == pytest.approx(float(np.sum(Ws[0].astype(np.float64) ** 2)), rel=1e-6)
 
 
+def test_bf16_split_iterates_every_step():
+    """bf16 hi/lo mode, step by step: the iterate's hi part after k < T steps
+    (bf16, at most 2^-9 relative rounding) and X_T (stored in fp16) against
+    the oracle's fp64 iterates, with W in both orientations (the view is the
+    P x Q iterate either way)."""
+    from paper_2607_08754_gb300.slorr import Regularizer
+    Ws = [workloads.random_matrix((256, 640), 51, 0.05), workloads.random_matrix((700, 300), 52, 0.05)]
+    reg = Regularizer([W.shape for W in Ws], compute="bf16_split")
+    w = [torch.from_numpy(W).cuda() for W in Ws]
+    co = oracle.pe_coefficients(6)
+    for k in range(7):
+        reg.run_steps(w, k)
+        torch.cuda.synchronize()
+        assert reg.status() == 0
+        for i, W in enumerate(Ws):
+            ref_steps, tr = oracle.polar_express_steps(W.astype(np.float64), co, EPS)
+            got = reg.iterate(i, k).double().cpu().numpy()   # P x Q, X_0 scaled
+            assert rel(got, ref_steps[k]) <= 5e-3, (k, i, rel(got, ref_steps[k]))
+
+
 @pytest.mark.parametrize("compute", ["fp32", "fp16", "bf16", "bf16_split"])
 @pytest.mark.parametrize("variant", ["hoyer", "nuclear"])
 def test_ragged_shapes(compute, variant):

@@ -526,3 +526,16 @@ def test_bf16_split_mode_plan(lib):
         with pytest.raises(slorr.SlorrError) as e:
             slorr.Regularizer([(256, 512)], compute="bf16_split", flags=flag)
         assert e.value.status == 1
+
+
+def test_pipeline_groups_by_operand_mode(lib):
+    """The host-buffer pipeline's default grouping: about 64 MiB of weights
+    per group (128 MiB with bf16 hi/lo operands, whose kernels take longer
+    than the copies), between 1 and 16 groups."""
+    import workloads
+    vl = workloads.shapes("vit_l16")          # 1.21 GB of fp32 weights
+    assert slorr.Pipeline.auto_groups(vl) == 16
+    assert slorr.Pipeline.auto_groups(vl, "f32", "bf16_split") == 9
+    assert slorr.Pipeline.auto_groups(vl, "bf16", "bf16_split") == 4
+    assert slorr.Pipeline.auto_groups([(64, 64)]) == 1
+    assert slorr.Pipeline.auto_groups(workloads.shapes("vit_b16"), "f32", "fp16") == 5
