@@ -364,7 +364,10 @@ class Regularizer:
 
     ``reg(weights, grads)`` enqueues the forward value and gradient of every
     matrix on the current CUDA stream, accumulating lambda * grad into
-    ``grads`` and returning the device loss tensor (lambda * sum_i L_i)."""
+    ``grads`` and returning the device loss tensor (lambda * sum_i L_i).
+    ``compute`` picks the operand mode of the products: "fp16" (default),
+    "bf16", "bf16_split" (bf16 hi/lo pairs, three products per product) or
+    "fp32" (three tf32 products per product)."""
 
     def __init__(self, shapes, variant: str = "hoyer", compute: str = "fp16", dtype: str = "f32",
                  iters: int = 6, lam: float = 1.0, eps: float = 1e-7, grad_scale: float = 1.0,
