@@ -23,12 +23,13 @@ def _need_gpu():
     slorr.load_library()
 
 
-def test_graph_replays_equal_direct_launches():
+@pytest.mark.parametrize("compute", ["fp16", "bf16_split"])
+def test_graph_replays_equal_direct_launches(compute):
     from paper_2607_08754_gb300.slorr import Regularizer, FLAG_GRAPH
     Ws = [workloads.random_matrix(s, seed=600 + i, std=0.05) for i, s in enumerate(SHAPES)]
     outs = []
     for flags in (0, FLAG_GRAPH):
-        reg = Regularizer(SHAPES, flags=flags, lam=0.5)
+        reg = Regularizer(SHAPES, compute=compute, flags=flags, lam=0.5)
         w = [torch.from_numpy(W).cuda() for W in Ws]
         g = [torch.zeros_like(x) for x in w]
         per = torch.empty(len(SHAPES), device="cuda")
