@@ -346,10 +346,11 @@ SLORR_API slorr_status slorr_gemm_pair_load(const slorr_handle* h, int32_t phase
 SLORR_API slorr_status slorr_set_timing(slorr_handle* h, int32_t enable);
 SLORR_API slorr_status slorr_read_timing(slorr_handle* h, double* ms, int64_t* launches, int32_t kinds);
 
-/* ||W||_F^2 of one matrix without any device allocation (the paper has no
- * counterpart: this exists for callers that cannot provide a workspace, e.g.
- * code running while a stream is captured, or under a framework that owns
- * all device memory).
+/* ||W||_F^2 of one matrix (the squared Frobenius norm of Listing 1 and Sec. 3
+ * "Computing the nuclear and Frobenius norms") without any device allocation.
+ * The allocation-free form has no counterpart in the paper: it exists for
+ * callers that cannot provide a workspace, e.g. code running while a stream
+ * is captured, or under a framework that owns all device memory.
  *   weight       device pointer, row-major m x n, of slorr_dtype `dtype`
  *   out_frob_sq  device pointer to one double, written with sum_ij W_ij^2
  * Enqueued on `stream`; deterministic (fixed-order partial sums).  Scratch is
